@@ -1,0 +1,207 @@
+/*
+ * efsparse.h — C ABI of the error-feedback (EF) gradient-sparsification step
+ * of "Rethinking gradient sparsification as total error minimization"
+ * (Sahu et al., NeurIPS 2021, arXiv:2108.00951).
+ *
+ * One call performs, for one worker i at one iteration t, the compression
+ * part of the distributed EF-SGD loop (Algorithm 1):
+ *
+ *     a       = e + gamma * g              (Algorithm 1, corrected update p_{i,t})
+ *     C(a)    = sum_{j in S(a)} a[j] u_j   (Sec. 4.2: a deterministic sparsifier
+ *                                           keeps the coordinates of a support S)
+ *     e      <- a - C(a)                   (Algorithm 1, error update)
+ *
+ * and emits C(a) as (uint32 index, fp32 value) pairs in ascending index order.
+ * The support S is either
+ *   - the hard-threshold support S_lambda(a) = { j : |a[j]| >= lambda }
+ *     (Sec. 1 and Sec. 4.2), the paper's proposed sparsifier, or
+ *   - the Top-k support, the k largest-magnitude coordinates (Lemma 2), the
+ *     baseline the paper compares against.
+ * sparse_aggregate() then sums n workers' sparse vectors into one dense vector
+ * (Algorithm 1, exchange-and-average step; the 1/n factor is left to the caller).
+ *
+ * Conventions shared by every entry point:
+ *   - All array pointers are DEVICE pointers (CUDA global memory) unless stated
+ *     otherwise. The caller allocates and owns every input and output buffer.
+ *   - Every call is asynchronous on `stream` (NULL = the legacy default stream).
+ *     No call synchronises with the host, except the one-time growth of the
+ *     library's internal workspace (see "Workspace" below). Outputs are valid
+ *     once the stream has been synchronised.
+ *   - Argument checks happen on the host before any launch; a failing check
+ *     returns EF_ERR_INVALID_ARG and launches nothing.
+ *   - A CUDA runtime failure (launch or allocation) returns EF_ERR_CUDA or
+ *     EF_ERR_NO_MEMORY.
+ *   - Errors found on the device (a bounded wait that ran out, malformed sparse
+ *     input) are latched in a per-stream device status word and reported by
+ *     ef_check_status(); they never fault, trap or hang the GPU.
+ *   - No C++ exception crosses this ABI.
+ *
+ * Numerical contract (identical to the CPU oracle, bit for bit):
+ *   - a[j] is ONE fused multiply-add, fmaf(gamma, g[j], e[j]), rounded once to
+ *     nearest-even; subnormals are kept (no flush to zero).
+ *   - A coordinate with a[j] == +-0 is never sent (sending it changes nothing
+ *     and the paper's data volume counts non-zeros, Sec. 6 "average density").
+ *   - The residual of a sent coordinate is +0.0f; of an unsent one it is a[j].
+ *     Hence a == C(a) + e' holds exactly for every finite a.
+ *   - NaN: never satisfies |a| >= lambda (not sent by hard-threshold); in the
+ *     Top-k order, magnitudes compare by IEEE-754 totalOrder of |a|, so NaN
+ *     ranks above +inf.
+ *   - Top-k ties go to the lowest index; exactly k pairs are emitted.
+ *
+ * Workspace: the library keeps one grow-only device workspace per (device,
+ * stream) pair (scan tile status, histograms, candidate buffers, offsets).
+ * Growing it synchronises `stream` once. Calls on DIFFERENT streams never
+ * share a workspace and may run concurrently; calls on the same stream are
+ * ordered by the stream. ef_workspace_release() frees all workspaces.
+ */
+#ifndef EFSPARSE_H
+#define EFSPARSE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A CUDA stream handle; the same type as cudaStream_t (struct CUstream_st*). */
+typedef struct CUstream_st* ef_stream_t;
+
+typedef enum {
+  EF_OK = 0,
+  EF_ERR_INVALID_ARG = 1, /* host-side argument check failed; nothing launched */
+  EF_ERR_CUDA = 2,        /* a CUDA runtime call or kernel launch failed */
+  EF_ERR_TIMEOUT = 3,     /* a bounded device-side wait ran out (latched) */
+  EF_ERR_BAD_INPUT = 4,   /* malformed sparse input detected on the device (latched) */
+  EF_ERR_NO_MEMORY = 5    /* workspace allocation failed */
+} ef_status;
+
+/*
+ * ef_hard_threshold — EF accumulate + hard-threshold sparsifier + compaction
+ * + residual, fused in one pass over the d coordinates.
+ *
+ * Defines: Algorithm 1 (p = e + gamma g; error update e <- p - Delta) with the
+ * hard-threshold sparsifier C_lambda, S_lambda(x) = { j : |x[j]| >= lambda }
+ * (Sec. 1; Sec. 4.2). The threshold is applied to a itself: lambda here equals
+ * gamma * lambda_paper of Algorithm 1's Delta = gamma C(p / gamma) (Remark 1),
+ * and the value sent is a[j] unchanged.
+ *
+ *   g          [in]  fp32[d], the stochastic gradient g_{i,t}. 4-byte aligned.
+ *   e          [in/out] fp32[d], the error memory e_{i,t}; overwritten with
+ *                    e_{i,t+1} = a - C(a). 4-byte aligned; 16-byte alignment of
+ *                    both g and e selects the vectorised path.
+ *   gamma      step size; must be finite.
+ *   lambda     threshold; must be >= 0 and not NaN (+inf sends only +-inf).
+ *   d          number of coordinates, 0 <= d <= 2^32 - 1.
+ *   idx_out    [out] uint32[capacity >= d]; idx_out[0..count) = the sent
+ *                    coordinates, strictly ascending.
+ *   val_out    [out] fp32[capacity >= d]; val_out[p] = a[idx_out[p]].
+ *   count_out  [out] one uint32 in device memory: the number of pairs
+ *                    (= ||C(a)||_0, the per-iteration k_t of Sec. 6).
+ *   Outputs must not overlap g or e. Entries of idx_out/val_out at positions
+ *   >= count are left untouched.
+ */
+ef_status ef_hard_threshold(const float* g, float* e, float gamma, float lambda,
+                            uint64_t d, uint32_t* idx_out, float* val_out,
+                            uint32_t* count_out, ef_stream_t stream);
+
+/*
+ * ef_hard_threshold_bf16 — as ef_hard_threshold, with the gradient stored as
+ * bfloat16 bit patterns (uint16_t[d], 2-byte aligned; 8-byte alignment of g
+ * and 16-byte alignment of e select the vectorised path). Each g[j] is widened
+ * exactly to fp32 (its 16 bits become the high half of the fp32 word) before
+ * the same fused multiply-add; all other semantics are identical.
+ */
+ef_status ef_hard_threshold_bf16(const uint16_t* g, float* e, float gamma,
+                                 float lambda, uint64_t d, uint32_t* idx_out,
+                                 float* val_out, uint32_t* count_out,
+                                 ef_stream_t stream);
+
+/*
+ * ef_topk — EF accumulate + Top-k sparsifier + compaction + residual.
+ *
+ * Defines: Algorithm 1 with C = Top-k, the k largest-magnitude coordinates of a
+ * (Lemma 1 / Lemma 2: the minimiser of ||a - C(a)||^2 over supports of size
+ * k). The paper assumes distinct magnitudes (Sec. 4.3); ties here go to the
+ * lowest index, and exactly k pairs are always emitted (zero-magnitude
+ * coordinates fill a short support, lowest index first).
+ *
+ *   g, e, gamma, d   as for ef_hard_threshold.
+ *   k          number of coordinates to send, 0 <= k <= d.
+ *   idx_out    [out] uint32[capacity >= k], strictly ascending.
+ *   val_out    [out] fp32[capacity >= k], val_out[p] = a[idx_out[p]].
+ *   count_out  [out] one uint32 in device memory; always equals k.
+ *   During the call e temporarily holds a; on completion it holds a - C(a).
+ */
+ef_status ef_topk(const float* g, float* e, float gamma, uint64_t k, uint64_t d,
+                  uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                  ef_stream_t stream);
+
+/* ef_topk_bf16 — ef_topk with a bfloat16 gradient, widened as in
+ * ef_hard_threshold_bf16. */
+ef_status ef_topk_bf16(const uint16_t* g, float* e, float gamma, uint64_t k,
+                       uint64_t d, uint32_t* idx_out, float* val_out,
+                       uint32_t* count_out, ef_stream_t stream);
+
+/*
+ * sparse_aggregate — decompress and sum n workers' sparse vectors.
+ *
+ * Defines: Algorithm 1's exchange step, Delta_bar = (1/n) sum_i Delta_{i,t},
+ * without the 1/n factor (the caller scales; exact for power-of-two n):
+ *
+ *     dense_out[j] = sum over i = 0..n-1 with j in S_i of val[i][p_i(j)],
+ *
+ * accumulated in fp32 in ascending worker order starting from +0.0f, so the
+ * result is bit-for-bit deterministic. Coordinates no worker sent are +0.0f.
+ *
+ *   n          number of workers, 1 <= n <= 256.
+ *   idx        HOST array of n DEVICE pointers; idx[i][0..counts[i]) must be
+ *              strictly ascending and < d (the form ef_hard_threshold and
+ *              ef_topk produce).
+ *   val        HOST array of n DEVICE pointers to fp32 values.
+ *   counts     DEVICE array of n uint32 pair counts; counts[i] must not exceed
+ *              the allocated length of idx[i] and val[i].
+ *   d          length of the dense output, d <= 2^32 - 1.
+ *   dense_out  [out] fp32[d], fully overwritten.
+ * An index outside [0, d) or an unsorted list never causes an out-of-bounds
+ * access: the offending pair is skipped and EF_ERR_BAD_INPUT is latched.
+ */
+ef_status sparse_aggregate(uint32_t n, const uint32_t* const* idx,
+                           const float* const* val, const uint32_t* counts,
+                           uint64_t d, float* dense_out, ef_stream_t stream);
+
+/*
+ * ef_check_status — synchronise `stream`, then return and clear the device-side
+ * error latched by earlier calls on that stream (EF_OK if none).
+ */
+ef_status ef_check_status(ef_stream_t stream);
+
+/* ef_status_string — static, human-readable name of a status code. */
+const char* ef_status_string(ef_status status);
+
+/*
+ * ef_workspace_release — synchronise the device and free every workspace the
+ * library holds on the current device. Later calls re-create them.
+ */
+ef_status ef_workspace_release(void);
+
+/*
+ * ef_kernel_launches — number of kernels this library has launched in this
+ * process (all devices, all streams). For accounting in benchmarks.
+ */
+uint64_t ef_kernel_launches(void);
+
+/*
+ * ef_test_set_lookback_fault — test hook for the bounded waits of the
+ * ordered-compaction scan. When withheld_tile >= 0, the next compaction
+ * launches on any stream make that tile never publish its count, so its
+ * successors' waits run out after about spin_limit_us microseconds; they then
+ * latch EF_ERR_TIMEOUT, skip their pair writes and finish. withheld_tile < 0
+ * restores normal operation (the default). Never needed in production.
+ */
+void ef_test_set_lookback_fault(int64_t withheld_tile, uint32_t spin_limit_us);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* EFSPARSE_H */

@@ -1,0 +1,181 @@
+/*
+ * oracle.c — plain, slow, single-threaded CPU oracle for the error-feedback
+ * (EF) sparsification step of "Rethinking gradient sparsification as total
+ * error minimization" (arXiv:2108.00951).
+ *
+ * TEST INFRASTRUCTURE ONLY. Nothing in the product path may call, link or
+ * load this file or the library built from it; only the tests, the smoke
+ * check and the CPU-baseline leg of the benchmark use it. It shares no code,
+ * header, table or helper with the CUDA library: every line here is written
+ * from the paper's definitions, in the paper's order, for a reader to check
+ * by eye.
+ *
+ * Build: gcc -O2 -std=c11 -ffp-contract=off -fno-fast-math -fPIC -shared
+ * (no contraction: the only fused operation is the explicit fmaf below).
+ *
+ * Readings of the paper taken here (the same ones the CUDA library follows):
+ *   R1 gamma placement: the threshold applies to a = e + gamma*g directly and
+ *      the value sent is a itself (Algorithm 1 with Delta = C(p), which
+ *      Remark 1 states is the same for the sparsifiers considered).
+ *   R2 rounding: a is one fused multiply-add, fmaf(gamma, g, e).
+ *   R3 the hard-threshold support uses >= (Sec. 1; Sec. 4.2).
+ *   R4 a coordinate equal to +-0 is never sent (it adds nothing to C(a) and
+ *      ||C(a)||_0 does not count it).
+ *   R5 Top-k ties go to the lowest index; exactly k pairs are sent.
+ *   R6 magnitude order = IEEE-754 totalOrder of |a| (NaN above +inf); the
+ *      hard-threshold test |a| >= lambda is false for NaN.
+ *   R7 the residual of a sent coordinate is +0.0f.
+ *   R9 aggregation returns the sum (the 1/n of Algorithm 1 is the caller's),
+ *      accumulated from +0.0f in ascending worker order.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+/* Widen a bfloat16 bit pattern to the fp32 value it denotes: the 16 stored
+ * bits are the high half of the fp32 encoding, the low half is zero. */
+static float bf16_bits_to_float(uint16_t bits) {
+  uint32_t w = ((uint32_t)bits) << 16;
+  float f;
+  memcpy(&f, &w, sizeof f);
+  return f;
+}
+
+/* ------------------------------------------------------------------------
+ * Hard-threshold (Algorithm 1 with C = C_lambda).
+ *   p_{i,t} = e_{i,t} + gamma g_{i,t}             (Algorithm 1, first step)
+ *   S_lambda(p) = { j : |p[j]| >= lambda }         (Sec. 1; Sec. 4.2)
+ *   Delta = sum_{j in S} p[j] u_j, sent as pairs   (Sec. 4.2 sparsifier form)
+ *   e_{i,t+1} = p - Delta                          (Algorithm 1, error update)
+ * ------------------------------------------------------------------------ */
+static int hard_threshold_core(const float* g_f32, const uint16_t* g_bf16,
+                               float* e, float gamma, float lambda, uint64_t d,
+                               uint32_t* idx, float* val, uint32_t* count) {
+  uint64_t c = 0;
+  for (uint64_t j = 0; j < d; ++j) {
+    float gj = g_f32 ? g_f32[j] : bf16_bits_to_float(g_bf16[j]);
+    float a = fmaf(gamma, gj, e[j]);                    /* R2 */
+    int in_support = (fabsf(a) >= lambda) && (a != 0.0f); /* R3, R4, R6 */
+    if (in_support) {
+      idx[c] = (uint32_t)j;
+      val[c] = a;
+      ++c;
+      e[j] = 0.0f;                                       /* R7 */
+    } else {
+      e[j] = a;
+    }
+  }
+  *count = (uint32_t)c;
+  return 0;
+}
+
+int oracle_ef_hard_threshold(const float* g, float* e, float gamma,
+                             float lambda, uint64_t d, uint32_t* idx,
+                             float* val, uint32_t* count) {
+  return hard_threshold_core(g, NULL, e, gamma, lambda, d, idx, val, count);
+}
+
+int oracle_ef_hard_threshold_bf16(const uint16_t* g, float* e, float gamma,
+                                  float lambda, uint64_t d, uint32_t* idx,
+                                  float* val, uint32_t* count) {
+  return hard_threshold_core(NULL, g, e, gamma, lambda, d, idx, val, count);
+}
+
+/* ------------------------------------------------------------------------
+ * Top-k (Algorithm 1 with C = Top-k; Lemma 1 / Lemma 2: keeping the k
+ * largest-magnitude entries minimises ||p - C(p)||^2 under ||C(p)||_0 <= k).
+ * ------------------------------------------------------------------------ */
+
+/* Magnitude order of R6: compare |x| and |y| under IEEE-754 totalOrder.
+ * For non-NaN values this is the ordinary order of fabsf; every NaN ranks
+ * above +inf, and two NaNs rank by their payloads. Returns -1, 0 or +1. */
+static int magnitude_cmp(float x, float y) {
+  float ax = fabsf(x), ay = fabsf(y);
+  int nx = isnan(ax), ny = isnan(ay);
+  if (nx || ny) {
+    if (!ny) return 1;
+    if (!nx) return -1;
+    uint32_t px, py;
+    memcpy(&px, &ax, sizeof px);
+    memcpy(&py, &ay, sizeof py);
+    return (px > py) - (px < py);
+  }
+  return (ax > ay) - (ax < ay);
+}
+
+static const float* g_sort_keys; /* single-threaded oracle: qsort context */
+
+/* Sort order for the Top-k selection: larger magnitude first; equal
+ * magnitudes by ascending index (R5). */
+static int topk_order(const void* pa, const void* pb) {
+  uint32_t ia = *(const uint32_t*)pa, ib = *(const uint32_t*)pb;
+  int m = magnitude_cmp(g_sort_keys[ia], g_sort_keys[ib]);
+  if (m != 0) return -m;
+  return (ia > ib) - (ia < ib);
+}
+
+static int ascending_u32(const void* pa, const void* pb) {
+  uint32_t a = *(const uint32_t*)pa, b = *(const uint32_t*)pb;
+  return (a > b) - (a < b);
+}
+
+static int topk_core(const float* g_f32, const uint16_t* g_bf16, float* e,
+                     float gamma, uint64_t k, uint64_t d, uint32_t* idx,
+                     float* val, uint32_t* count) {
+  if (k > d) return 1;
+  float* a = (float*)malloc((d ? d : 1) * sizeof(float));
+  uint32_t* order = (uint32_t*)malloc((d ? d : 1) * sizeof(uint32_t));
+  if (!a || !order) { free(a); free(order); return 2; }
+  /* corrected update p = e + gamma g (Algorithm 1), one fma each (R2) */
+  for (uint64_t j = 0; j < d; ++j) {
+    float gj = g_f32 ? g_f32[j] : bf16_bits_to_float(g_bf16[j]);
+    a[j] = fmaf(gamma, gj, e[j]);
+    order[j] = (uint32_t)j;
+  }
+  /* S = the first k coordinates in decreasing magnitude, ties by index */
+  g_sort_keys = a;
+  qsort(order, d, sizeof(uint32_t), topk_order);
+  /* emit S in ascending index order */
+  qsort(order, k, sizeof(uint32_t), ascending_u32);
+  for (uint64_t j = 0; j < d; ++j) e[j] = a[j];      /* e' = p on j not in S */
+  for (uint64_t p = 0; p < k; ++p) {
+    uint32_t j = order[p];
+    idx[p] = j;
+    val[p] = a[j];
+    e[j] = 0.0f;                                      /* R7 */
+  }
+  *count = (uint32_t)k;
+  free(a);
+  free(order);
+  return 0;
+}
+
+int oracle_ef_topk(const float* g, float* e, float gamma, uint64_t k,
+                   uint64_t d, uint32_t* idx, float* val, uint32_t* count) {
+  return topk_core(g, NULL, e, gamma, k, d, idx, val, count);
+}
+
+int oracle_ef_topk_bf16(const uint16_t* g, float* e, float gamma, uint64_t k,
+                        uint64_t d, uint32_t* idx, float* val,
+                        uint32_t* count) {
+  return topk_core(NULL, g, e, gamma, k, d, idx, val, count);
+}
+
+/* ------------------------------------------------------------------------
+ * Aggregation (Algorithm 1, exchange step): sum_i Delta_{i,t}, decompressed
+ * into a dense vector. Sum, not mean (R9); from +0.0f; workers in order.
+ * ------------------------------------------------------------------------ */
+int oracle_sparse_aggregate(uint32_t n, const uint32_t* const* idx,
+                            const float* const* val, const uint32_t* counts,
+                            uint64_t d, float* dense) {
+  for (uint64_t j = 0; j < d; ++j) dense[j] = 0.0f;
+  for (uint32_t i = 0; i < n; ++i) {
+    for (uint32_t p = 0; p < counts[i]; ++p) {
+      uint32_t j = idx[i][p];
+      if ((uint64_t)j >= d) return 1;
+      dense[j] += val[i][p];
+    }
+  }
+  return 0;
+}

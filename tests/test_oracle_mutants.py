@@ -1,0 +1,90 @@
+"""The pins catch plausible mistakes: each mutant of the oracle fails one.
+
+A mutant is a copy of oracle.c with one planted mistake (a dropped term, a
+wrong sign, a swapped operand, '>' for '>=', a reversed order or tie rule, a
+wrong residual), compiled to a temporary library. The pin tests run against
+it with the module's loaded library swapped; at least one must fail. CPU only.
+"""
+import contextlib
+import ctypes
+import os
+import subprocess
+
+import pytest
+
+import oracle
+import test_oracle_pins as pins
+
+_SRC = os.path.join(os.path.dirname(oracle.__file__), "oracle.c")
+
+MUTANTS = {
+    "two_step_rounding": [("fmaf(gamma, gj, e[j])", "gamma * gj + e[j]")],
+    "swapped_operands": [("fmaf(gamma, gj, e[j])", "fmaf(gamma, e[j], gj)")],
+    "dropped_error_term": [("fmaf(gamma, gj, e[j])", "fmaf(gamma, gj, 0.0f)")],
+    "wrong_sign": [("fmaf(gamma, gj, e[j])", "fmaf(-gamma, gj, e[j])")],
+    "strict_threshold": [("(fabsf(a) >= lambda)", "(fabsf(a) > lambda)")],
+    "sends_zeros": [("&& (a != 0.0f)", "")],
+    "residual_not_cleared": [("      e[j] = 0.0f;                                       /* R7 */",
+                              "      e[j] = a;")],
+    "topk_smallest_first": [("if (m != 0) return -m;", "if (m != 0) return m;")],
+    "topk_highest_index_ties": [("  return (ia > ib) - (ia < ib);", "  return (ia < ib) - (ia > ib);")],
+    "topk_residual_kept": [("    e[j] = 0.0f;                                      /* R7 */",
+                            "    e[j] = a[j];")],
+    "aggregate_reverse_order": [("for (uint32_t i = 0; i < n; ++i) {",
+                                 "for (uint32_t i = n; i-- > 0;) {")],
+    "nan_ranks_lowest": [("    if (!ny) return 1;\n    if (!nx) return -1;",
+                          "    if (!ny) return -1;\n    if (!nx) return 1;")],
+}
+
+PIN_TESTS = [
+    pins.test_accumulate_is_one_rounded_fma,
+    pins.test_accumulate_operand_roles,
+    pins.test_ht_threshold_is_inclusive,
+    pins.test_ht_lambda_zero_sends_exactly_the_nonzeros,
+    pins.test_ht_nan_and_inf,
+    lambda: pins.test_ht_reconstruction_and_absolute_bound(3001),
+    lambda: pins.test_topk_matches_bruteforce_optimum(0),
+    lambda: pins.test_topk_matches_bruteforce_optimum(1),
+    pins.test_topk_matches_stable_argsort_with_ties,
+    pins.test_topk_special_cases,
+    pins.test_topk_nan_inf_order,
+    pins.test_aggregate_sums_in_worker_order,
+    lambda: pins.test_error_feedback_conserves_mass("ht"),
+]
+
+
+@contextlib.contextmanager
+def _swapped_library(path):
+    oracle._load()
+    saved = oracle._lib
+    lib = ctypes.CDLL(path)
+    # reuse the argtypes of the real library
+    for name in ("oracle_ef_hard_threshold", "oracle_ef_hard_threshold_bf16",
+                 "oracle_ef_topk", "oracle_ef_topk_bf16", "oracle_sparse_aggregate"):
+        fn, ref = getattr(lib, name), getattr(saved, name)
+        fn.argtypes, fn.restype = ref.argtypes, ref.restype
+    oracle._lib = lib
+    try:
+        yield
+    finally:
+        oracle._lib = saved
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_is_caught(name, tmp_path):
+    src = open(_SRC).read()
+    for old, new in MUTANTS[name]:
+        assert old in src, (name, old)
+        src = src.replace(old, new)
+    c_path = tmp_path / "mutant.c"
+    c_path.write_text(src)
+    so_path = str(tmp_path / "libmutant.so")
+    subprocess.run(["gcc", *oracle._CFLAGS, "-o", so_path, str(c_path), "-lm"], check=True)
+    failures = 0
+    with _swapped_library(so_path):
+        for t in PIN_TESTS:
+            try:
+                t()
+            except AssertionError:
+                failures += 1
+    assert failures >= 1, "mutant %s survived every pin" % name

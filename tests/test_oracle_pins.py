@@ -1,0 +1,363 @@
+"""Pins of the CPU oracle to what the paper and the mathematics fix (no GPU).
+
+Each test checks the oracle against something other than itself: exact
+rational arithmetic, brute-force search over supports, closed-form special
+cases, bounds stated in the paper, or a library routine. Together they are
+chosen so that a dropped term, a wrong sign, a swapped operand, a '>' for
+'>=', a wrong tie rule or a wrong summation order each fails at least one.
+"""
+from fractions import Fraction
+import itertools
+import math
+
+import numpy as np
+import pytest
+
+import oracle
+from exact_fp32 import fma_f32, round_f32, to_frac, ulp_f32
+
+RNG = np.random.default_rng(2108)
+
+
+def _f32(x):
+    return np.asarray(x, dtype=np.float32)
+
+
+def _exact_a(g, e, gamma):
+    gamma = np.float32(gamma)           # the library takes gamma as fp32
+    return np.array([fma_f32(gamma, gj, ej) for gj, ej in zip(g, e)], dtype=np.float32)
+
+
+def _same_bits(x, y):
+    x = np.asarray(x, np.float32)
+    y = np.asarray(y, np.float32)
+    return x.shape == y.shape and np.array_equal(x.view(np.uint32), y.view(np.uint32))
+
+
+# --------------------------------------------------------------------------
+# a = e + gamma g (Algorithm 1, first step), one correctly rounded fma
+# --------------------------------------------------------------------------
+
+def _fma_sensitive_triples(count):
+    """Random (gamma, g, e) with wide exponents, plus cases where the product
+    must not be rounded before the addition (fma != mul-then-add)."""
+    gam = _f32(RNG.uniform(0.01, 2.0, count) * np.exp2(RNG.integers(-8, 4, count)))
+    g = _f32(RNG.standard_normal(count) * np.exp2(RNG.integers(-20, 6, count)))
+    e = _f32(RNG.standard_normal(count) * np.exp2(RNG.integers(-20, 6, count)))
+    # cancellation cases: e = -round(gamma*g), so a is the product's rounding error
+    c = count // 4
+    e[:c] = -(gam[:c] * g[:c])
+    return gam, g, e
+
+
+def test_accumulate_is_one_rounded_fma():
+    gam, g, e = _fma_sensitive_triples(4000)
+    mismatched_two_step = 0
+    for gm, gj, ej in zip(gam, g, e):
+        a_exact = fma_f32(gm, gj, ej)
+        two_step = np.float32(np.float32(gm) * np.float32(gj)) + np.float32(ej)
+        if not _same_bits(two_step, a_exact):
+            mismatched_two_step += 1
+        # lambda = inf sends nothing finite, so e' = a exactly
+        idx, val, e_new = oracle.ef_hard_threshold(_f32([gj]), _f32([ej]), float(gm), math.inf)
+        assert idx.size == 0
+        assert _same_bits(e_new, [a_exact]), (gm, gj, ej)
+    # the set really distinguishes a fused from a two-step evaluation
+    assert mismatched_two_step > 500
+
+
+def test_accumulate_operand_roles():
+    # a = e + gamma*g; swapping g and e, or the sign, gives a different value
+    g, e, gamma = _f32([3.0]), _f32([5.0]), 0.5
+    _, _, e_new = oracle.ef_hard_threshold(g, e, gamma, math.inf)
+    assert e_new[0] == 5.0 + 0.5 * 3.0
+
+
+# --------------------------------------------------------------------------
+# hard-threshold S_lambda(a) = {j : |a_j| >= lambda} (Sec. 1, Sec. 4.2)
+# --------------------------------------------------------------------------
+
+def test_ht_threshold_is_inclusive():
+    # |a| == lambda exactly must be sent (">=", Sec. 1); just below must not
+    lam = 0.25
+    below = np.nextafter(np.float32(lam), np.float32(0))
+    e = _f32([lam, -lam, below, -below, 1.0])
+    g = np.zeros(5, np.float32)
+    idx, val, e_new = oracle.ef_hard_threshold(g, e, 1.0, lam)
+    assert idx.tolist() == [0, 1, 4]
+    assert val.tolist() == [lam, -lam, 1.0]
+    assert _same_bits(e_new, [0.0, 0.0, below, -below, 0.0])
+
+
+def test_ht_lambda_zero_sends_exactly_the_nonzeros():
+    # special case lambda = 0: every non-zero coordinate is sent, e' = 0 there
+    tiny = np.float32(np.finfo(np.float32).smallest_subnormal)
+    e = _f32([0.0, -0.0, tiny, -tiny, 3.5, 0.0, -2.0])
+    g = np.zeros_like(e)
+    g[1] = -0.0            # (-0)*0.1 + (-0) = -0: a signed zero stays unsent
+    idx, val, e_new = oracle.ef_hard_threshold(g, e, 0.1, 0.0)
+    assert idx.tolist() == [2, 3, 4, 6]
+    assert _same_bits(val, [tiny, -tiny, 3.5, -2.0])
+    assert _same_bits(e_new, [0.0, -0.0, 0.0, 0.0, 0.0, 0.0, 0.0])
+
+
+def test_ht_lambda_above_max_sends_nothing():
+    g = _f32(RNG.standard_normal(1000))
+    e = _f32(RNG.standard_normal(1000))
+    a = _exact_a(g, e, 0.1)
+    lam = float(np.nextafter(np.max(np.abs(a)), np.float32(np.inf)))
+    idx, val, e_new = oracle.ef_hard_threshold(g, e, 0.1, lam)
+    assert idx.size == 0
+    assert _same_bits(e_new, a)
+
+
+def test_ht_nan_and_inf():
+    e = _f32([np.nan, np.inf, -np.inf, 1.0])
+    g = np.zeros(4, np.float32)
+    idx, val, e_new = oracle.ef_hard_threshold(g, e, 1.0, 0.5)
+    assert idx.tolist() == [1, 2, 3]
+    assert val.tolist() == [np.inf, -np.inf, 1.0]
+    assert np.isnan(e_new[0]) and e_new[1:].tolist() == [0.0, 0.0, 0.0]
+
+
+@pytest.mark.parametrize("d", [1, 7, 64, 3001])
+def test_ht_reconstruction_and_absolute_bound(d):
+    # a = C(a) + e' exactly (Algorithm 1 error update) and ||e'||_inf < lambda,
+    # hence ||e'||^2 <= d lambda^2 (absolute compressor, kappa^2 = d lambda^2)
+    g = _f32(RNG.standard_normal(d) * 0.01)
+    e = _f32(RNG.standard_normal(d) * 0.001)
+    gamma, lam = 0.1, 1.5e-3
+    a = _exact_a(g, e, gamma)
+    idx, val, e_new = oracle.ef_hard_threshold(g, e, gamma, lam)
+    assert np.all(np.diff(idx.astype(np.int64)) > 0)
+    dense = np.zeros(d, np.float32)
+    dense[idx] = val
+    assert _same_bits(dense + e_new, a)
+    assert np.all(np.abs(e_new) < lam)
+    assert float(np.sum(e_new.astype(np.float64) ** 2)) <= d * lam * lam
+    assert idx.size == int(np.sum((np.abs(a) >= lam) & (a != 0)))
+
+
+def test_ht_monotone_in_lambda():
+    g = _f32(RNG.standard_normal(2000))
+    e = np.zeros(2000, np.float32)
+    prev = None
+    for lam in [0.0, 0.1, 0.5, 1.0, 2.0, 3.0]:
+        idx, _, _ = oracle.ef_hard_threshold(g, e, 1.0, lam)
+        s = set(idx.tolist())
+        if prev is not None:
+            assert s <= prev
+        prev = s
+
+
+def test_ht_bf16_widening():
+    # a bf16 value denotes exactly the fp32 value with the same high 16 bits
+    torch = pytest.importorskip("torch")
+    x = torch.randn(5000, generator=torch.Generator().manual_seed(3)) * 0.01
+    gb = x.to(torch.bfloat16)
+    bits = gb.view(torch.int16).numpy().view(np.uint16)
+    widened = gb.to(torch.float32).numpy()
+    e = _f32(RNG.standard_normal(5000) * 1e-3)
+    r16 = oracle.ef_hard_threshold(bits, e, 0.1, 2e-3)
+    r32 = oracle.ef_hard_threshold(widened, e, 0.1, 2e-3)
+    for u, v in zip(r16, r32):
+        assert _same_bits(u, v) if u.dtype == np.float32 else np.array_equal(u, v)
+    t16 = oracle.ef_topk(bits, e, 0.1, 50)
+    t32 = oracle.ef_topk(widened, e, 0.1, 50)
+    for u, v in zip(t16, t32):
+        assert _same_bits(u, v) if u.dtype == np.float32 else np.array_equal(u, v)
+
+
+# --------------------------------------------------------------------------
+# Top-k (Lemma 1 / Lemma 2): the support of size k minimising ||a - C(a)||^2
+# --------------------------------------------------------------------------
+
+def _bruteforce_topk(a, k):
+    """All size-k supports minimising the exact squared error; the minimiser
+    with the lexicographically smallest ascending index tuple (lowest-index
+    tie rule)."""
+    d = len(a)
+    sq = [to_frac(x) ** 2 for x in a]
+    total = sum(sq, Fraction(0))
+    best, best_err = None, None
+    for s in itertools.combinations(range(d), k):
+        err = total - sum((sq[j] for j in s), Fraction(0))
+        if best_err is None or err < best_err:
+            best, best_err = s, err
+        # combinations() enumerates in lexicographic order, so the first
+        # minimiser found is the lexicographically smallest one
+    return list(best), best_err
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_topk_matches_bruteforce_optimum(seed):
+    rng = np.random.default_rng(seed)
+    d = int(rng.integers(1, 11))
+    if seed % 3 == 0:   # heavy ties, signed zeros
+        pool = _f32([0.0, -0.0, 1.0, -1.0, 0.5, -0.5, 2.0])
+        e = pool[rng.integers(0, len(pool), d)]
+    else:
+        e = _f32(rng.standard_normal(d))
+    g = np.zeros(d, np.float32)
+    a = _exact_a(g, e, 1.0)             # 1*0 + e, with (+0) + (-0) = +0
+    for k in range(d + 1):
+        idx, val, e_new = oracle.ef_topk(g, e, 1.0, k)
+        want, err = _bruteforce_topk(a.tolist(), k)
+        assert idx.tolist() == want, (e, k)
+        assert _same_bits(val, a[want])
+        assert sum((to_frac(x) ** 2 for x in e_new), Fraction(0)) == err
+        assert int(np.count_nonzero(np.isin(np.arange(d), idx))) == k
+
+
+def test_topk_matches_stable_argsort_with_ties():
+    # library cross-check: a stable sort by decreasing |a| takes the lowest
+    # index first among equal magnitudes
+    d, k = 20000, 777
+    e = _f32(np.round(RNG.standard_normal(d) * 4) / 4)   # many exact ties
+    g = np.zeros(d, np.float32)
+    idx, val, e_new = oracle.ef_topk(g, e, 1.0, k)
+    want = np.sort(np.argsort(-np.abs(e), kind="stable")[:k])
+    assert np.array_equal(idx, want.astype(np.uint32))
+
+
+def test_topk_special_cases():
+    g = _f32(RNG.standard_normal(500))
+    e = _f32(RNG.standard_normal(500))
+    a = _exact_a(g, e, 0.3)
+    idx, val, e_new = oracle.ef_topk(g, e, 0.3, 0)          # k = 0: nothing sent
+    assert idx.size == 0 and _same_bits(e_new, a)
+    idx, val, e_new = oracle.ef_topk(g, e, 0.3, 500)        # k = d: identity
+    assert idx.tolist() == list(range(500)) and _same_bits(val, a)
+    assert not np.any(e_new)
+    z = np.zeros(10, np.float32)                             # short support filled by zeros
+    z[7] = -3.0
+    idx, val, _ = oracle.ef_topk(np.zeros(10, np.float32), z, 1.0, 4)
+    assert idx.tolist() == [0, 1, 2, 7]
+
+
+@pytest.mark.parametrize("k", [1, 10, 100, 999])
+def test_topk_delta_contraction_bound(k):
+    # Top-k is a delta-contraction with delta = k/d (Sec. 4.4):
+    # ||a - C(a)||^2 <= (1 - k/d) ||a||^2
+    d = 1000
+    g = _f32(RNG.standard_normal(d))
+    e = _f32(RNG.standard_normal(d))
+    a = _exact_a(g, e, 0.2).astype(np.float64)
+    _, _, e_new = oracle.ef_topk(g, e, 0.2, k)
+    assert np.sum(e_new.astype(np.float64) ** 2) <= (1 - k / d) * np.sum(a ** 2) + 1e-12
+
+
+def test_topk_nan_inf_order():
+    e = _f32([1.0, np.inf, np.nan, -np.inf, 5.0, -0.0])
+    g = np.zeros(6, np.float32)
+    idx, _, _ = oracle.ef_topk(g, e, 1.0, 1)
+    assert idx.tolist() == [2]          # NaN ranks above +inf
+    idx, _, _ = oracle.ef_topk(g, e, 1.0, 3)
+    assert idx.tolist() == [1, 2, 3]    # +inf and -inf tie: lower index first
+    idx, _, _ = oracle.ef_topk(g, e, 1.0, 4)
+    assert idx.tolist() == [1, 2, 3, 4]
+
+
+def test_ht_at_kth_magnitude_selects_topk():
+    # Sec. 4.3 (Lemma 3 argument): with distinct magnitudes and
+    # lambda in (|a|_(k+1), |a|_(k)], C_lambda keeps exactly the Top-k set
+    for seed in range(5):
+        rng = np.random.default_rng(100 + seed)
+        d = 9
+        e = _f32(rng.permutation(np.arange(1, d + 1)) * rng.choice([-1, 1], d) / 8)
+        g = np.zeros(d, np.float32)
+        mags = np.sort(np.abs(e))[::-1]
+        for k in range(1, d + 1):
+            lam = float(mags[k - 1])
+            ht_idx, _, ht_e = oracle.ef_hard_threshold(g, e, 1.0, lam)
+            want, _ = _bruteforce_topk(e.tolist(), k)
+            assert ht_idx.tolist() == want
+            tk_idx, _, tk_e = oracle.ef_topk(g, e, 1.0, k)
+            assert tk_idx.tolist() == want and _same_bits(ht_e, tk_e)
+
+
+# --------------------------------------------------------------------------
+# aggregation (Algorithm 1, exchange step): ordered fp32 sum from +0.0
+# --------------------------------------------------------------------------
+
+def test_aggregate_single_worker_is_scatter():
+    d = 50
+    idx = np.array([0, 3, 17, 49], np.uint32)
+    val = _f32([1.5, -2.25, -0.0, 7.0])
+    dense = oracle.sparse_aggregate([idx], [val], d)
+    want = np.zeros(d, np.float32)
+    want[[0, 3, 49]] = [1.5, -2.25, 7.0]      # 0 + (-0) = +0
+    assert _same_bits(dense, want)
+
+
+def test_aggregate_disjoint_and_integer_sums_are_exact():
+    d = 1000
+    perm = RNG.permutation(d)
+    idx_list = [np.sort(perm[i::4][:100]).astype(np.uint32) for i in range(4)]
+    val_list = [_f32(RNG.integers(-1000, 1000, 100)) for _ in range(4)]
+    dense = oracle.sparse_aggregate(idx_list, val_list, d)
+    want = np.zeros(d, np.float64)
+    for i, v in zip(idx_list, val_list):
+        want[i] += v
+    assert np.array_equal(dense, want.astype(np.float32))
+    # overlapping supports with small integers: every partial sum is exact
+    idx_list = [np.arange(0, d, s, dtype=np.uint32) for s in (1, 2, 3)]
+    val_list = [_f32(RNG.integers(-50, 50, len(i))) for i in idx_list]
+    dense = oracle.sparse_aggregate(idx_list, val_list, d)
+    want = np.zeros(d, np.float64)
+    for i, v in zip(idx_list, val_list):
+        want[i] += v
+    assert np.array_equal(dense, want.astype(np.float32))
+
+
+def test_aggregate_sums_in_worker_order():
+    # fp32: (0 + 2^24) + 1 = 2^24 (tie to even), then - 2^24 = 0;
+    # any other order gives 1 or -2^24 + ... != 0
+    big = np.float32(2.0 ** 24)
+    idx = [np.array([5], np.uint32)] * 3
+    dense = oracle.sparse_aggregate(idx, [_f32([big]), _f32([1.0]), _f32([-big])], 8)
+    assert dense[5] == 0.0
+    dense = oracle.sparse_aggregate(idx, [_f32([-big]), _f32([1.0]), _f32([big])], 8)
+    assert dense[5] == 1.0
+
+
+def test_aggregate_rejects_out_of_range():
+    with pytest.raises(RuntimeError):
+        oracle.sparse_aggregate([np.array([10], np.uint32)], [_f32([1.0])], 10)
+
+
+# --------------------------------------------------------------------------
+# multi-iteration EF: Lemma 9 (virtual iterate) per worker
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("method", ["ht", "topk"])
+def test_error_feedback_conserves_mass(method):
+    # sum_t Delta_t + e_T = sum_t gamma g_t exactly, up to the single rounding
+    # of each fma: |gap_j| <= sum_t ulp(a_t[j]) / 2
+    d, T, gamma = 300, 12, 0.1
+    e = np.zeros(d, np.float32)
+    sent = [Fraction(0)] * d
+    target = [Fraction(0)] * d
+    slack = [Fraction(0)] * d
+    for t in range(T):
+        g = _f32(RNG.standard_normal(d) * 0.01)
+        a = _exact_a(g, e, gamma)
+        if method == "ht":
+            idx, val, e = oracle.ef_hard_threshold(g, e, gamma, 2e-3)
+        else:
+            idx, val, e = oracle.ef_topk(g, e, gamma, 15)
+        for j, v in zip(idx.tolist(), val.tolist()):
+            sent[j] += to_frac(v)
+        for j in range(d):
+            target[j] += to_frac(np.float32(gamma)) * to_frac(g[j])
+            slack[j] += ulp_f32(a[j]) / 2
+    for j in range(d):
+        gap = abs(sent[j] + to_frac(e[j]) - target[j])
+        assert gap <= slack[j], j
+
+
+def test_round_f32_helper_agrees_with_numpy_on_doubles():
+    # the exact helper itself: rounding a double to binary32 matches numpy
+    xs = RNG.standard_normal(2000) * np.exp2(RNG.integers(-140, 100, 2000))
+    for x in xs:
+        assert _same_bits([round_f32(Fraction(float(x)))], [np.float32(x)])
