@@ -1,0 +1,518 @@
+#!/usr/bin/env python3
+"""Benchmark of the error-feedback sparsification step (arXiv:2108.00951).
+
+One step = one error-feedback iteration of the n simulated workers of a
+workload, through the whole hot path:
+  - n x ef_hard_threshold (EF accumulate + hard-threshold + compaction +
+    residual), then sparse_aggregate of their n messages;
+  - n x ef_topk on the same gradients (separate error memories), then
+    sparse_aggregate of those messages.
+Gradients come from two pre-generated synthetic batches (alternating), so
+every step compresses different data; each step's working set (n workers x
+(g, e_ht, e_topk)) is far larger than the 126 MB L2.
+
+Headline (`value`): hard-threshold compress throughput in GB/s of
+algorithmic traffic, 12 B/coordinate (read g, read e, write e) + 8 B per sent
+pair, summed over all compress calls of the K timed steps and divided by
+their device time (CUDA events on the launching stream). Top-k and
+aggregation are reported as ms per iteration and as fractions of the same
+HBM roofline. `e2e` repeats the hard-threshold iteration through the public
+API with the n gradients copied host->device from pinned memory and the
+dense aggregate copied back, every step.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload resnet18]
+  python bench.py --impl reference ...   # the CPU oracle as the reference arm
+
+For N > 1 (one process per GPU under torch.distributed.run) every rank runs
+its own replica of the workload (weak scaling); ranks only meet in a barrier
+and in the max/sum reductions of the timing.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+PEAK_FALLBACK_GBS = 6800.0
+NOMINAL_HBM_GBS = 8000.0
+METRIC = "EF hard-threshold compress GB/s & elem/s vs HBM peak; Top-k and aggregate ms/iter"
+HT_KERNEL_SOURCES = ["paper_2108_00951_gb300/csrc/ht.cu", "paper_2108_00951_gb300/csrc/compact.cuh",
+                     "paper_2108_00951_gb300/csrc/common.cuh",
+                     "paper_2108_00951_gb300/csrc/gradient.cuh"]
+
+
+def parse_args(argv=None):
+    p = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default="resnet18")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=10.0,
+                   help="bound on the CPU-oracle sample of the cpu_baseline leg")
+    return p.parse_args(argv)
+
+
+# ------------------------------------------------------------ distributed
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def dist_init(backend):
+    import torch.distributed as dist
+    rank, world, _ = dist_env()
+    if world > 1 and not dist.is_initialized():
+        dist.init_process_group(backend=backend, rank=rank, world_size=world)
+    return dist if world > 1 else None
+
+
+def reduce_timing(dist, seconds: float, units: float, device=None):
+    """(max seconds over ranks, sum of units over ranks)."""
+    if dist is None:
+        return seconds, units
+    import torch
+    t = torch.tensor([seconds], dtype=torch.float64, device=device)
+    u = torch.tensor([units], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(u.item())
+
+
+def barrier(dist, device=None):
+    if dist is not None:
+        if device is not None and device.type == "cuda":
+            dist.barrier(device_ids=[device.index])
+        else:
+            dist.barrier()
+
+
+# ------------------------------------------------------------ peaks, clocks
+def measured_peak_gbs():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            v = float(json.load(f)["hbm_gbs"])
+        return v, "measured"
+    except Exception:
+        return PEAK_FALLBACK_GBS, "fallback"
+
+
+class ClockSampler:
+    """Samples the SM clock and clock-event reasons of one GPU every ~10 ms
+    through NVML (read-only queries), falling back to nvidia-smi."""
+
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, cuda_index: int):
+        self.samples = []
+        self.reasons = set()
+        self.max_mhz = None
+        self._stop = threading.Event()
+        self._thread = None
+        self._nvml = None
+        self._handle = None
+        self._smi_index = cuda_index
+        try:
+            import torch
+            lib = ctypes.CDLL("libnvidia-ml.so.1")
+            if lib.nvmlInit_v2() != 0:
+                raise OSError("nvmlInit failed")
+            handle = ctypes.c_void_p()
+            uuid = "GPU-" + str(torch.cuda.get_device_properties(cuda_index).uuid)
+            if lib.nvmlDeviceGetHandleByUUID(uuid.encode(), ctypes.byref(handle)) != 0:
+                raise OSError("no NVML handle")
+            mx = ctypes.c_uint()
+            if lib.nvmlDeviceGetMaxClockInfo(handle, 1, ctypes.byref(mx)) == 0:
+                self.max_mhz = mx.value
+            self._nvml, self._handle = lib, handle
+        except Exception:
+            self._nvml = None
+
+    def _poll_nvml(self):
+        clk = ctypes.c_uint()
+        rs = ctypes.c_ulonglong()
+        get_reasons = getattr(self._nvml, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            getattr(self._nvml, "nvmlDeviceGetCurrentClocksThrottleReasons")
+        while not self._stop.is_set():
+            if self._nvml.nvmlDeviceGetClockInfo(self._handle, 1, ctypes.byref(clk)) == 0:
+                self.samples.append(clk.value)
+            if get_reasons(self._handle, ctypes.byref(rs)) == 0:
+                for bit, name in self.REASONS.items():
+                    if rs.value & bit:
+                        self.reasons.add(name)
+            time.sleep(0.01)
+
+    def _poll_smi(self):
+        q = ("clocks.sm,clocks.max.sm,clocks_event_reasons.hw_slowdown,"
+             "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+             "clocks_event_reasons.sw_power_cap")
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        while not self._stop.is_set():
+            try:
+                out = subprocess.run(["nvidia-smi", "-i", str(self._smi_index),
+                                      "--query-gpu=" + q, "--format=csv,noheader,nounits"],
+                                     capture_output=True, text=True, timeout=5).stdout
+                f = [x.strip() for x in out.strip().split(",")]
+                self.samples.append(float(f[0]))
+                self.max_mhz = float(f[1])
+                for name, v in zip(names, f[2:]):
+                    if v.lower() == "active":
+                        self.reasons.add(name)
+            except Exception:
+                pass
+            time.sleep(0.05)
+
+    def start(self):
+        self._thread = threading.Thread(target=self._poll_nvml if self._nvml else self._poll_smi,
+                                        daemon=True)
+        self._thread.start()
+
+    def stop(self):
+        self._stop.set()
+        if self._thread:
+            self._thread.join()
+        return {"sm_mhz": statistics.median(self.samples) if self.samples else None,
+                "sm_max_mhz": self.max_mhz, "reasons": sorted(self.reasons),
+                "samples": len(self.samples), "source": "nvml" if self._nvml else "nvidia-smi"}
+
+
+def sources_hash(paths):
+    h = hashlib.sha256()
+    for p in paths:
+        with open(os.path.join(ROOT, p), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel_tag: str, workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel sources; else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            entry = json.load(f)[kernel_tag][workload]
+    except Exception:
+        return None
+    if entry.get("sources_sha256_16") != sources_hash(HT_KERNEL_SOURCES):
+        return None
+    return entry.get("dram_bytes_per_launch")
+
+
+# ------------------------------------------------------------ our arm
+def ht_bytes(d, count, g_bytes=4):
+    return (g_bytes + 8) * d + 8 * count
+
+
+def run_ours(args):
+    import torch
+    import paper_2108_00951_gb300 as efs
+    from paper_2108_00951_gb300 import workloads
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    dist = dist_init("nccl")
+    efs.load_library()
+
+    w = workloads.BY_NAME[args.workload]
+    d, n, gamma = w.d, w.n, w.gamma
+    k = w.topk_values()[0]
+    # every rank simulates its own n workers (replica); seeds differ per rank
+    wr = workloads.Workload(**{**w.__dict__, "seed": w.seed + 1000 * rank})
+    batches = [[workloads.gradient(wr, i, b, device=dev) for i in range(n)] for b in range(2)]
+    lam = (workloads.density_lambda(wr, batches[0][0], w.density) if w.density is not None
+           else w.lambdas[0])
+
+    def outputs(cap):
+        return ([torch.empty(cap, dtype=torch.int32, device=dev) for _ in range(n)],
+                [torch.empty(cap, dtype=torch.float32, device=dev) for _ in range(n)])
+
+    e_ht = [torch.zeros(d, device=dev) for _ in range(n)]
+    e_tk = [torch.zeros(d, device=dev) for _ in range(n)]
+    idx_ht, val_ht = outputs(d)
+    idx_tk, val_tk = outputs(k)
+    dense_ht = torch.empty(d, device=dev)
+    dense_tk = torch.empty(d, device=dev)
+    total = args.warmup + args.steps
+    cnt_ht = torch.zeros(total, n, dtype=torch.int32, device=dev)
+    cnt_tk = torch.zeros(total, n, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    marks = [[ev() for _ in range(5)] for _ in range(args.steps)]
+    call_ev = [[(ev(), ev()) for _ in range(n)] for _ in range(args.steps)]
+
+    def step(s, timed):
+        g = batches[s % 2]
+        m = marks[s - args.warmup] if timed else None
+        if m: m[0].record(stream)
+        for i in range(n):
+            if timed: call_ev[s - args.warmup][i][0].record(stream)
+            efs.ef_hard_threshold(g[i], e_ht[i], gamma, lam, idx_ht[i], val_ht[i],
+                                  cnt_ht[s, i:i + 1])
+            if timed: call_ev[s - args.warmup][i][1].record(stream)
+        if m: m[1].record(stream)
+        efs.sparse_aggregate(idx_ht, val_ht, cnt_ht[s], d, dense_ht)
+        if m: m[2].record(stream)
+        for i in range(n):
+            efs.ef_topk(g[i], e_tk[i], gamma, k, idx_tk[i], val_tk[i], cnt_tk[s, i:i + 1])
+        if m: m[3].record(stream)
+        efs.sparse_aggregate(idx_tk, val_tk, cnt_tk[s], d, dense_tk)
+        if m: m[4].record(stream)
+
+    for s in range(args.warmup):
+        step(s, False)
+    torch.cuda.synchronize()
+    if efs.ef_check_status() != efs.EF_OK:
+        raise RuntimeError("device error during warm-up")
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    launches0 = efs.ef_kernel_launches()
+    barrier(dist, dev)
+    torch.cuda.synchronize()
+    t0, t1 = ev(), ev()
+    t0.record(stream)
+    for s in range(args.warmup, total):
+        step(s, True)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    barrier(dist, dev)
+    launches = efs.ef_kernel_launches() - launches0
+    clocks = sampler.stop()
+    if efs.ef_check_status() != efs.EF_OK:
+        raise RuntimeError("device error during the timed steps")
+
+    step_s = t0.elapsed_time(t1) / 1e3
+    ht_s = sum(m[0].elapsed_time(m[1]) for m in marks) / 1e3
+    agg_ht_s = sum(m[1].elapsed_time(m[2]) for m in marks) / 1e3
+    tk_s = sum(m[2].elapsed_time(m[3]) for m in marks) / 1e3
+    agg_tk_s = sum(m[3].elapsed_time(m[4]) for m in marks) / 1e3
+    per_call = [a.elapsed_time(b) / 1e3 for row in call_ev for (a, b) in row]
+    counts_ht = cnt_ht[args.warmup:].double()
+    counts_tk = cnt_tk[args.warmup:].double()
+    bytes_ht = float(ht_bytes(d, 0) * n * args.steps + 8 * counts_ht.sum().item())
+    bytes_tk = float((12 * d + 8 * k) * n * args.steps)
+    bytes_agg_ht = float(8 * counts_ht.sum().item() + 4 * d * args.steps)
+    bytes_agg_tk = float(8 * counts_tk.sum().item() + 4 * d * args.steps)
+
+    ht_s_max, bytes_ht_all = reduce_timing(dist, ht_s, bytes_ht, dev)
+    step_s_max, _ = reduce_timing(dist, step_s, 0.0, dev)
+    value = bytes_ht_all / ht_s_max / 1e9
+    peak, peak_kind = measured_peak_gbs()
+    avg_launch = statistics.mean(per_call)
+    achieved = (ht_bytes(d, 0) + 8 * counts_ht.mean().item()) / avg_launch / 1e9
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, efs, torch, dev, dist, batches[0], d, n, gamma, lam, stream)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(args, [b.cpu().numpy() for b in batches[0][:2]], d, gamma, lam, k)
+
+    if rank != 0:
+        return None
+    density = counts_ht.mean().item() / d
+    return {
+        "metric": METRIC,
+        "value": round(value, 2),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(step_s_max / args.steps * 1e3, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32",
+        "data": "synthetic (seeded %s-shaped gradients; no dataset or trained model)" % w.name,
+        "config": {
+            "workload": "%s: d=%d in %d segments, n=%d simulated workers, gamma=%g, "
+                        "hard-threshold lambda=%.6g (first-iteration density %.4g%%), "
+                        "Top-k k=%d" % (w.name, d, len(w.segments), n, gamma, lam,
+                                        100 * (w.density or 0), k),
+            "global_batch": n,
+            "seq_len": None,
+            "parallelism": "replicas x%d (simulated workers on each GPU)" % world,
+            "l2": "inputs larger than L2: %.2f GB touched per step vs 126 MB L2"
+                  % (n * 12 * d / 1e9),
+            "value_scope": "n hard-threshold compress calls per step, device time",
+        },
+        "elem_per_s": round(n * d * args.steps * world / ht_s_max, 1),
+        "ht_density": round(density, 6),
+        "ht_ms_per_iter": round(ht_s / args.steps * 1e3, 4),
+        "topk_ms_per_iter": round(tk_s / args.steps * 1e3, 4),
+        "topk_gbs": round(bytes_tk / tk_s / 1e9, 2),
+        "topk_frac_of_peak": round(bytes_tk / tk_s / 1e9 / peak, 4),
+        "aggregate_ms_per_iter": round(agg_ht_s / args.steps * 1e3, 4),
+        "aggregate_gbs": round(bytes_agg_ht / agg_ht_s / 1e9, 2),
+        "aggregate_frac_of_peak": round(bytes_agg_ht / agg_ht_s / 1e9 / peak, 4),
+        "aggregate_topk_ms_per_iter": round(agg_tk_s / args.steps * 1e3, 4),
+        "frac_of_nominal_8tbs": round(value / NOMINAL_HBM_GBS, 4),
+        "roofline": {
+            "bound": "hbm",
+            "kernel": "ht_kernel (fused EF accumulate + hard-threshold + compaction + residual)",
+            "achieved": round(achieved, 2),
+            "peak": peak,
+            "peak_kind": peak_kind,
+            "unit": "GB/s",
+            "frac": round(achieved / peak, 4),
+            "avg_launch_us": round(avg_launch * 1e6, 3),
+            "algorithmic_bytes_per_launch": int(ht_bytes(d, 0) + 8 * counts_ht.mean().item()),
+            "traffic": profiled_traffic("ht_kernel", w.name),
+        },
+        "gpu_launches": int(launches),
+        "clocks": clocks,
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+    }
+
+
+def run_e2e(args, efs, torch, dev, dist, grads, d, n, gamma, lam, stream):
+    """The hard-threshold iteration through the public API with host data:
+    per step, H2D of the n gradients from pinned memory, n compress calls,
+    the aggregate, and D2H of the dense result."""
+    host_g = [g.cpu().pin_memory() for g in grads]
+    host_out = torch.empty(d, dtype=torch.float32).pin_memory()
+    dev_g = [torch.empty(d, device=dev) for _ in range(n)]
+    e = [torch.zeros(d, device=dev) for _ in range(n)]
+    idx = [torch.empty(d, dtype=torch.int32, device=dev) for _ in range(n)]
+    val = [torch.empty(d, dtype=torch.float32, device=dev) for _ in range(n)]
+    cnt = torch.zeros(args.steps + args.warmup, n, dtype=torch.int32, device=dev)
+    dense = torch.empty(d, device=dev)
+
+    def step(s):
+        for i in range(n):
+            dev_g[i].copy_(host_g[i], non_blocking=True)
+            efs.ef_hard_threshold(dev_g[i], e[i], gamma, lam, idx[i], val[i], cnt[s, i:i + 1])
+        efs.sparse_aggregate(idx, val, cnt[s], d, dense)
+        host_out.copy_(dense, non_blocking=True)
+
+    for s in range(args.warmup):
+        step(s)
+    torch.cuda.synchronize()
+    barrier(dist, dev)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for s in range(args.warmup, args.warmup + args.steps):
+        step(s)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    barrier(dist, dev)
+    secs = t0.elapsed_time(t1) / 1e3
+    byts = float(12 * d * n * args.steps + 8 * cnt[args.warmup:].double().sum().item())
+    secs, byts = reduce_timing(dist, secs, byts, dev)
+    return {"value": round(byts / secs / 1e9, 2), "unit": "GB/s",
+            "h2d_bytes_per_step": 4 * d * n, "d2h_bytes_per_step": 4 * d,
+            "ms_per_step": round(secs / args.steps * 1e3, 4)}
+
+
+# ------------------------------------------------------------ CPU oracle legs
+def cpu_baseline(args, grads, d, gamma, lam, k):
+    """The oracle as it stands, single-threaded on this host: hard-threshold
+    calls on the first workers' full-size gradients for about
+    args.cpu_seconds, in the same unit as the headline."""
+    import numpy as np
+    import oracle
+    e = np.zeros(d, np.float32)
+    calls, byts, t_start = 0, 0.0, time.perf_counter()
+    while True:
+        idx, _, e = oracle.ef_hard_threshold(grads[calls % len(grads)], e, gamma, lam)
+        calls += 1
+        byts += ht_bytes(d, idx.size)
+        el = time.perf_counter() - t_start
+        if el >= args.cpu_seconds:
+            break
+    return {"value": round(byts / el / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": "%d single-threaded oracle hard-threshold calls at full d=%d (%.1f s)"
+                      % (calls, d, el),
+            "host_cores_available": os.cpu_count()}
+
+
+def run_reference(args):
+    """The reference arm: the CPU oracle (there is no reference code for this
+    paper) on this host, timed over the same workload, metric and unit; each
+    step is one full-size hard-threshold call of one simulated worker."""
+    import numpy as np
+    import torch
+    import oracle
+    from paper_2108_00951_gb300 import workloads
+
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return None
+    w = workloads.BY_NAME[args.workload]
+    grads = [workloads.gradient(w, i, 0).numpy() for i in range(2)]
+    lam = (workloads.density_lambda(w, torch.from_numpy(grads[0]), w.density)
+           if w.density is not None else w.lambdas[0])
+    e = np.zeros(w.d, np.float32)
+    for s in range(args.warmup):
+        _, _, e = oracle.ef_hard_threshold(grads[s % 2], e, w.gamma, lam)
+    byts, t0 = 0.0, time.perf_counter()
+    for s in range(args.steps):
+        idx, _, e = oracle.ef_hard_threshold(grads[s % 2], e, w.gamma, lam)
+        byts += ht_bytes(w.d, idx.size)
+    el = time.perf_counter() - t0
+    value = byts / el / 1e9
+    return {
+        "impl": "reference",
+        "metric": METRIC,
+        "value": round(value, 4),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(el / args.steps * 1e3, 3),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32",
+        "data": "synthetic (seeded %s-shaped gradients)" % w.name,
+        "config": {"workload": "%s: d=%d, one simulated worker's hard-threshold call per step"
+                               % (w.name, w.d), "global_batch": 1, "seq_len": None,
+                   "parallelism": "single CPU thread"},
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                         "sample": "%d full-size oracle hard-threshold calls" % args.steps},
+        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    if args.impl == "reference":
+        out = run_reference(args)
+    else:
+        out = run_ours(args)
+    if out is not None:
+        print(json.dumps(out), flush=True)
+    try:
+        import torch.distributed as dist
+        if dist.is_initialized():
+            dist.destroy_process_group()
+    except Exception:
+        pass
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

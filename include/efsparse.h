@@ -45,7 +45,8 @@
  *     Hence a == C(a) + e' holds exactly for every finite a.
  *   - NaN: never satisfies |a| >= lambda (not sent by hard-threshold); in the
  *     Top-k order, magnitudes compare by IEEE-754 totalOrder of |a|, so NaN
- *     ranks above +inf.
+ *     ranks above +inf. Every NaN the library writes (accumulator, residual,
+ *     sent value, aggregate sum) is the canonical quiet NaN 0x7fffffff.
  *   - Top-k ties go to the lowest index; exactly k pairs are emitted.
  *
  * Workspace: the library keeps one grow-only device workspace per (device,

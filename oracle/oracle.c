@@ -23,7 +23,10 @@
  *      ||C(a)||_0 does not count it).
  *   R5 Top-k ties go to the lowest index; exactly k pairs are sent.
  *   R6 magnitude order = IEEE-754 totalOrder of |a| (NaN above +inf); the
- *      hard-threshold test |a| >= lambda is false for NaN.
+ *      hard-threshold test |a| >= lambda is false for NaN. The paper is
+ *      silent on NaN; a NaN carries no value, so every NaN the step produces
+ *      (accumulator or aggregate sum) is written as the one canonical quiet
+ *      NaN, encoding 0x7fffffff.
  *   R7 the residual of a sent coordinate is +0.0f.
  *   R9 aggregation returns the sum (the 1/n of Algorithm 1 is the caller's),
  *      accumulated from +0.0f in ascending worker order.
@@ -32,6 +35,15 @@
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
+
+/* R6: the canonical encoding of a NaN result. */
+static float canonical_nan_if_nan(float x) {
+  if (!isnan(x)) return x;
+  uint32_t w = 0x7fffffffu;
+  float f;
+  memcpy(&f, &w, sizeof f);
+  return f;
+}
 
 /* Widen a bfloat16 bit pattern to the fp32 value it denotes: the 16 stored
  * bits are the high half of the fp32 encoding, the low half is zero. */
@@ -55,7 +67,7 @@ static int hard_threshold_core(const float* g_f32, const uint16_t* g_bf16,
   uint64_t c = 0;
   for (uint64_t j = 0; j < d; ++j) {
     float gj = g_f32 ? g_f32[j] : bf16_bits_to_float(g_bf16[j]);
-    float a = fmaf(gamma, gj, e[j]);                    /* R2 */
+    float a = canonical_nan_if_nan(fmaf(gamma, gj, e[j])); /* R2, R6 */
     int in_support = (fabsf(a) >= lambda) && (a != 0.0f); /* R3, R4, R6 */
     if (in_support) {
       idx[c] = (uint32_t)j;
@@ -130,7 +142,7 @@ static int topk_core(const float* g_f32, const uint16_t* g_bf16, float* e,
   /* corrected update p = e + gamma g (Algorithm 1), one fma each (R2) */
   for (uint64_t j = 0; j < d; ++j) {
     float gj = g_f32 ? g_f32[j] : bf16_bits_to_float(g_bf16[j]);
-    a[j] = fmaf(gamma, gj, e[j]);
+    a[j] = canonical_nan_if_nan(fmaf(gamma, gj, e[j]));    /* R6 */
     order[j] = (uint32_t)j;
   }
   /* S = the first k coordinates in decreasing magnitude, ties by index */
@@ -174,7 +186,7 @@ int oracle_sparse_aggregate(uint32_t n, const uint32_t* const* idx,
     for (uint32_t p = 0; p < counts[i]; ++p) {
       uint32_t j = idx[i][p];
       if ((uint64_t)j >= d) return 1;
-      dense[j] += val[i][p];
+      dense[j] = canonical_nan_if_nan(dense[j] + val[i][p]); /* R6 */
     }
   }
   return 0;

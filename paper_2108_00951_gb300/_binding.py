@@ -1,0 +1,180 @@
+"""ctypes binding of libefsparse.so — argument marshalling only.
+
+Every function here has the name of the C entry point it calls (declared in
+``include/efsparse.h``), takes torch CUDA tensors, checks their dtype, device,
+shape and contiguity, and passes raw device pointers and the current CUDA
+stream across the C ABI. All computation happens in the library's kernels;
+there is no fallback: if the library cannot be loaded, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import build as _build
+
+EF_OK = 0
+EF_ERR_INVALID_ARG = 1
+EF_ERR_CUDA = 2
+EF_ERR_TIMEOUT = 3
+EF_ERR_BAD_INPUT = 4
+EF_ERR_NO_MEMORY = 5
+
+
+class EfError(RuntimeError):
+    """A non-OK ef_status returned by the library."""
+
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__("%s: %s" % (where, status_string(status)))
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIBPATH
+
+
+def load_library(build_if_missing: bool = True):
+    """Load libefsparse.so (building it in-tree first if it is missing)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = _build.LIBPATH
+        if not os.path.exists(path) or not _build.up_to_date():
+            if not build_if_missing:
+                raise RuntimeError("libefsparse.so is not built: run __graft_entry__.build()")
+            _build.build()
+        lib = ctypes.CDLL(path)
+        vp, u64, f32, u32 = ctypes.c_void_p, ctypes.c_uint64, ctypes.c_float, ctypes.c_uint32
+        sig = {
+            "ef_hard_threshold": [vp, vp, f32, f32, u64, vp, vp, vp, vp],
+            "ef_hard_threshold_bf16": [vp, vp, f32, f32, u64, vp, vp, vp, vp],
+            "ef_topk": [vp, vp, f32, u64, u64, vp, vp, vp, vp],
+            "ef_topk_bf16": [vp, vp, f32, u64, u64, vp, vp, vp, vp],
+            "sparse_aggregate": [u32, ctypes.POINTER(vp), ctypes.POINTER(vp), vp, u64, vp, vp],
+            "ef_check_status": [vp],
+            "ef_workspace_release": [],
+        }
+        for name, args in sig.items():
+            fn = getattr(lib, name)
+            fn.argtypes = args
+            fn.restype = ctypes.c_int
+        lib.ef_status_string.argtypes = [ctypes.c_int]
+        lib.ef_status_string.restype = ctypes.c_char_p
+        lib.ef_kernel_launches.argtypes = []
+        lib.ef_kernel_launches.restype = ctypes.c_uint64
+        lib.ef_test_set_lookback_fault.argtypes = [ctypes.c_int64, ctypes.c_uint32]
+        lib.ef_test_set_lookback_fault.restype = None
+        _lib = lib
+        return lib
+
+
+def status_string(status: int) -> str:
+    return load_library().ef_status_string(int(status)).decode()
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def _check(status: int, where: str):
+    if status != EF_OK:
+        raise EfError(status, where)
+
+
+def _dev(t: torch.Tensor, name: str, dtype, numel=None):
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError("%s must be a CUDA tensor" % name)
+    if t.dtype != dtype:
+        raise TypeError("%s must be %s, got %s" % (name, dtype, t.dtype))
+    if not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % name)
+    if numel is not None and t.numel() < numel:
+        raise ValueError("%s holds %d elements, needs %d" % (name, t.numel(), numel))
+    return ctypes.c_void_p(t.data_ptr() if t.numel() else 0)
+
+
+def _gradient(g: torch.Tensor):
+    if g.dtype == torch.float32:
+        return False
+    if g.dtype == torch.bfloat16:
+        return True
+    raise TypeError("g must be float32 or bfloat16")
+
+
+def ef_hard_threshold(g, e, gamma, lam, idx_out, val_out, count_out, stream=None):
+    """EF accumulate + hard-threshold + compaction (``ef_hard_threshold[_bf16]``).
+
+    ``g`` float32 or bfloat16 [d]; ``e`` float32 [d], updated in place;
+    ``idx_out`` int32 [>= d] (uint32 bit patterns), ``val_out`` float32 [>= d],
+    ``count_out`` int32 [>= 1].
+    """
+    lib = load_library()
+    bf16 = _gradient(g)
+    d = e.numel()
+    if g.numel() != d:
+        raise ValueError("g and e differ in length")
+    args = (_dev(g, "g", g.dtype), _dev(e, "e", torch.float32), ctypes.c_float(gamma),
+            ctypes.c_float(lam), d, _dev(idx_out, "idx_out", torch.int32, d),
+            _dev(val_out, "val_out", torch.float32, d),
+            _dev(count_out, "count_out", torch.int32, 1), _stream(stream))
+    fn = lib.ef_hard_threshold_bf16 if bf16 else lib.ef_hard_threshold
+    _check(fn(*args), "ef_hard_threshold")
+
+
+def ef_topk(g, e, gamma, k, idx_out, val_out, count_out, stream=None):
+    """EF accumulate + Top-k + compaction (``ef_topk[_bf16]``); exactly k pairs."""
+    lib = load_library()
+    bf16 = _gradient(g)
+    d = e.numel()
+    if g.numel() != d:
+        raise ValueError("g and e differ in length")
+    args = (_dev(g, "g", g.dtype), _dev(e, "e", torch.float32), ctypes.c_float(gamma), int(k),
+            d, _dev(idx_out, "idx_out", torch.int32, k),
+            _dev(val_out, "val_out", torch.float32, k),
+            _dev(count_out, "count_out", torch.int32, 1), _stream(stream))
+    fn = lib.ef_topk_bf16 if bf16 else lib.ef_topk
+    _check(fn(*args), "ef_topk")
+
+
+def sparse_aggregate(idx_list, val_list, counts, d, dense_out, stream=None):
+    """Worker-ordered sum of n sparse vectors into ``dense_out`` (float32 [d]).
+
+    ``idx_list``/``val_list``: n int32 / float32 CUDA tensors; ``counts``: int32
+    CUDA tensor of n pair counts.
+    """
+    lib = load_library()
+    n = len(idx_list)
+    if n != len(val_list):
+        raise ValueError("idx_list and val_list differ in length")
+    idx_arr = (ctypes.c_void_p * max(n, 1))(*[_dev(t, "idx", torch.int32) for t in idx_list])
+    val_arr = (ctypes.c_void_p * max(n, 1))(*[_dev(t, "val", torch.float32) for t in val_list])
+    _check(lib.sparse_aggregate(n, idx_arr, val_arr, _dev(counts, "counts", torch.int32, n),
+                                int(d), _dev(dense_out, "dense_out", torch.float32, d),
+                                _stream(stream)), "sparse_aggregate")
+
+
+def ef_check_status(stream=None) -> int:
+    """Synchronise the stream; return (and clear) the latched device status."""
+    return int(load_library().ef_check_status(_stream(stream)))
+
+
+def ef_workspace_release():
+    _check(load_library().ef_workspace_release(), "ef_workspace_release")
+
+
+def ef_kernel_launches() -> int:
+    return int(load_library().ef_kernel_launches())
+
+
+def ef_test_set_lookback_fault(withheld_tile: int, spin_limit_us: int = 0):
+    load_library().ef_test_set_lookback_fault(int(withheld_tile), int(spin_limit_us))

@@ -1,0 +1,315 @@
+// api.cu — the extern "C" boundary declared in include/efsparse.h: host-side
+// argument checks, the per-(device, stream) workspaces, and status reporting.
+// Every compute step runs in the kernels of ht.cu, topk.cu and aggregate.cu.
+#include <atomic>
+#include <cmath>
+#include <cstring>
+#include <map>
+#include <mutex>
+#include <utility>
+
+#include "efsparse.h"
+#include "internal.h"
+
+namespace efs {
+namespace {
+
+std::mutex g_mu;
+std::map<std::pair<int, cudaStream_t>, Workspace*> g_workspaces;
+std::map<int, DeviceInfo> g_devices;
+std::atomic<uint64_t> g_launches{0};
+std::atomic<int64_t> g_withheld_tile{-1};
+std::atomic<uint64_t> g_wait_limit_ns{2000000000ull};  // 2 s per wait
+
+constexpr uint64_t kMaxD = 0xffffffffull;
+
+bool overlaps(const void* a, size_t na, const void* b, size_t nb) {
+  if (!a || !b || na == 0 || nb == 0) return false;
+  const uintptr_t x = reinterpret_cast<uintptr_t>(a), y = reinterpret_cast<uintptr_t>(b);
+  return x < y + nb && y < x + na;
+}
+
+bool aligned(const void* p, size_t a) { return reinterpret_cast<uintptr_t>(p) % a == 0; }
+
+ef_status device_info(int dev, DeviceInfo* out) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  auto it = g_devices.find(dev);
+  if (it == g_devices.end()) {
+    DeviceInfo info;
+    if (cudaDeviceGetAttribute(&info.sm_count, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return EF_ERR_CUDA;
+    const int per_sm = topk_refine_blocks_per_sm();
+    if (per_sm <= 0) return EF_ERR_CUDA;
+    info.refine_blocks = per_sm * info.sm_count;
+    it = g_devices.emplace(dev, info).first;
+  }
+  *out = it->second;
+  return EF_OK;
+}
+
+// Find or grow the workspace of (current device, stream). Growth
+// synchronises the stream once; the new header and tile-status array start
+// at zero.
+ef_status acquire_workspace(cudaStream_t stream, uint32_t tiles, uint32_t cand_cap,
+                            size_t offsets, Workspace** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
+  std::lock_guard<std::mutex> lk(g_mu);
+  Workspace*& ws = g_workspaces[std::make_pair(dev, stream)];
+  if (!ws) {
+    ws = new Workspace;
+    ws->device = dev;
+    ws->stream = stream;
+  }
+  if (!ws->base || tiles > ws->status_tiles || cand_cap > ws->cand_cap ||
+      offsets > ws->offsets_cap) {
+    const uint32_t new_tiles = tiles > ws->status_tiles ? tiles : ws->status_tiles;
+    const uint32_t new_cand = cand_cap > ws->cand_cap ? cand_cap : ws->cand_cap;
+    const size_t new_off = offsets > ws->offsets_cap ? offsets : ws->offsets_cap;
+    const size_t bytes = kHeaderBytes + sizeof(uint64_t) * (static_cast<size_t>(new_tiles) +
+                                                            2 * static_cast<size_t>(new_cand)) +
+                         sizeof(uint32_t) * new_off + 256;
+    if (ws->base) {
+      if (cudaStreamSynchronize(stream) != cudaSuccess) return EF_ERR_CUDA;
+      cudaFree(ws->base);
+      ws->base = nullptr;
+    }
+    void* p = nullptr;
+    if (cudaMalloc(&p, bytes) != cudaSuccess) {
+      cudaGetLastError();
+      ws->status_tiles = ws->cand_cap = 0;
+      ws->offsets_cap = 0;
+      return EF_ERR_NO_MEMORY;
+    }
+    ws->base = static_cast<char*>(p);
+    ws->bytes = bytes;
+    ws->status_tiles = new_tiles;
+    ws->cand_cap = new_cand;
+    ws->offsets_cap = new_off;
+    ws->dirty = true;
+  }
+  if (ws->dirty) {
+    const size_t clear = kHeaderBytes + sizeof(uint64_t) * ws->status_tiles;
+    if (cudaMemsetAsync(ws->base, 0, clear, stream) != cudaSuccess) return EF_ERR_CUDA;
+    ws->epoch = 0;
+    ws->dirty = false;
+  }
+  *out = ws;
+  return EF_OK;
+}
+
+ef_status finish_launch(cudaError_t err, Workspace* ws) {
+  if (err == cudaSuccess) return EF_OK;
+  ws->dirty = true;  // a partial launch may leave the dispenser or barrier mid-way
+  return EF_ERR_CUDA;
+}
+
+ef_status write_zero_count(uint32_t* count_out, cudaStream_t stream) {
+  return cudaMemsetAsync(count_out, 0, sizeof(uint32_t), stream) == cudaSuccess ? EF_OK
+                                                                                 : EF_ERR_CUDA;
+}
+
+ef_status hard_threshold_entry(const void* g, bool bf16, float* e, float gamma, float lambda,
+                               uint64_t d, uint32_t* idx_out, float* val_out,
+                               uint32_t* count_out, cudaStream_t stream) {
+  const size_t gsz = bf16 ? 2 : 4;
+  if (!count_out || !aligned(count_out, 4)) return EF_ERR_INVALID_ARG;
+  if (!std::isfinite(gamma) || !(lambda >= 0.0f)) return EF_ERR_INVALID_ARG;
+  if (d > kMaxD) return EF_ERR_INVALID_ARG;
+  if (d == 0) return write_zero_count(count_out, stream);
+  if (!g || !e || !idx_out || !val_out) return EF_ERR_INVALID_ARG;
+  if (!aligned(g, gsz) || !aligned(e, 4) || !aligned(idx_out, 4) || !aligned(val_out, 4))
+    return EF_ERR_INVALID_ARG;
+  const size_t nb = static_cast<size_t>(d) * 4;
+  const void* outs[3] = {idx_out, val_out, count_out};
+  const size_t out_n[3] = {nb, nb, 4};
+  for (int o = 0; o < 3; ++o) {
+    if (overlaps(outs[o], out_n[o], g, d * gsz) || overlaps(outs[o], out_n[o], e, nb))
+      return EF_ERR_INVALID_ARG;
+    for (int p = o + 1; p < 3; ++p)
+      if (overlaps(outs[o], out_n[o], outs[p], out_n[p])) return EF_ERR_INVALID_ARG;
+  }
+  if (overlaps(g, d * gsz, e, nb)) return EF_ERR_INVALID_ARG;
+  Workspace* ws = nullptr;
+  const ef_status st = acquire_workspace(stream, tiles_for(d), 0, 0, &ws);
+  if (st != EF_OK) return st;
+  return finish_launch(launch_hard_threshold(g, bf16, e, gamma, lambda, static_cast<uint32_t>(d),
+                                             idx_out, val_out, count_out, *ws),
+                       ws);
+}
+
+ef_status topk_entry(const void* g, bool bf16, float* e, float gamma, uint64_t k, uint64_t d,
+                     uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                     cudaStream_t stream) {
+  const size_t gsz = bf16 ? 2 : 4;
+  if (!count_out || !aligned(count_out, 4)) return EF_ERR_INVALID_ARG;
+  if (!std::isfinite(gamma)) return EF_ERR_INVALID_ARG;
+  if (d > kMaxD || k > d) return EF_ERR_INVALID_ARG;
+  if (d == 0) return write_zero_count(count_out, stream);
+  if (!g || !e || (k > 0 && (!idx_out || !val_out))) return EF_ERR_INVALID_ARG;
+  if (!aligned(g, gsz) || !aligned(e, 4) || !aligned(idx_out, 4) || !aligned(val_out, 4))
+    return EF_ERR_INVALID_ARG;
+  const size_t nb = static_cast<size_t>(d) * 4, kb = static_cast<size_t>(k) * 4;
+  const void* outs[3] = {idx_out, val_out, count_out};
+  const size_t out_n[3] = {kb, kb, 4};
+  for (int o = 0; o < 3; ++o) {
+    if (overlaps(outs[o], out_n[o], g, d * gsz) || overlaps(outs[o], out_n[o], e, nb))
+      return EF_ERR_INVALID_ARG;
+    for (int p = o + 1; p < 3; ++p)
+      if (overlaps(outs[o], out_n[o], outs[p], out_n[p])) return EF_ERR_INVALID_ARG;
+  }
+  if (overlaps(g, d * gsz, e, nb)) return EF_ERR_INVALID_ARG;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
+  DeviceInfo info;
+  ef_status st = device_info(dev, &info);
+  if (st != EF_OK) return st;
+  Workspace* ws = nullptr;
+  st = acquire_workspace(stream, tiles_for(d), topk_candidate_capacity(d), 0, &ws);
+  if (st != EF_OK) return st;
+  return finish_launch(launch_topk(g, bf16, e, gamma, static_cast<uint32_t>(k),
+                                   static_cast<uint32_t>(d), idx_out, val_out, count_out, *ws,
+                                   info),
+                       ws);
+}
+
+}  // namespace
+
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+uint64_t wait_limit_ns() { return g_wait_limit_ns.load(); }
+int64_t withheld_tile() { return g_withheld_tile.load(); }
+
+ScanCtx next_scan_ctx(Workspace& ws, uint32_t num_tiles) {
+  if (ws.epoch >= (1u << 30) - 1) {  // epoch wrap: old words must not match again
+    cudaMemsetAsync(ws.status(), 0, sizeof(uint64_t) * ws.status_tiles, ws.stream);
+    ws.epoch = 0;
+  }
+  ++ws.epoch;
+  ScanCtx c;
+  c.status = ws.status();
+  c.tile_counter = ws.u32(kOffTileCounter);
+  c.error = ws.u32(kOffError);
+  c.epoch = ws.epoch;
+  c.num_tiles = num_tiles;
+  c.withheld_tile = withheld_tile();
+  c.wait_limit_ns = wait_limit_ns();
+  return c;
+}
+
+}  // namespace efs
+
+using efs::Workspace;
+
+extern "C" {
+
+ef_status ef_hard_threshold(const float* g, float* e, float gamma, float lambda, uint64_t d,
+                            uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                            ef_stream_t stream) {
+  return efs::hard_threshold_entry(g, false, e, gamma, lambda, d, idx_out, val_out, count_out,
+                                   reinterpret_cast<cudaStream_t>(stream));
+}
+
+ef_status ef_hard_threshold_bf16(const uint16_t* g, float* e, float gamma, float lambda,
+                                 uint64_t d, uint32_t* idx_out, float* val_out,
+                                 uint32_t* count_out, ef_stream_t stream) {
+  return efs::hard_threshold_entry(g, true, e, gamma, lambda, d, idx_out, val_out, count_out,
+                                   reinterpret_cast<cudaStream_t>(stream));
+}
+
+ef_status ef_topk(const float* g, float* e, float gamma, uint64_t k, uint64_t d,
+                  uint32_t* idx_out, float* val_out, uint32_t* count_out, ef_stream_t stream) {
+  return efs::topk_entry(g, false, e, gamma, k, d, idx_out, val_out, count_out,
+                         reinterpret_cast<cudaStream_t>(stream));
+}
+
+ef_status ef_topk_bf16(const uint16_t* g, float* e, float gamma, uint64_t k, uint64_t d,
+                       uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                       ef_stream_t stream) {
+  return efs::topk_entry(g, true, e, gamma, k, d, idx_out, val_out, count_out,
+                         reinterpret_cast<cudaStream_t>(stream));
+}
+
+ef_status sparse_aggregate(uint32_t n, const uint32_t* const* idx, const float* const* val,
+                           const uint32_t* counts, uint64_t d, float* dense_out,
+                           ef_stream_t stream) {
+  if (n == 0 || n > efs::kMaxWorkers || !idx || !val || !counts) return EF_ERR_INVALID_ARG;
+  if (d > efs::kMaxD) return EF_ERR_INVALID_ARG;
+  if (d == 0) return EF_OK;
+  if (!dense_out || !efs::aligned(dense_out, 4) || !efs::aligned(counts, 4))
+    return EF_ERR_INVALID_ARG;
+  for (uint32_t i = 0; i < n; ++i)
+    if (!idx[i] || !val[i] || !efs::aligned(idx[i], 4) || !efs::aligned(val[i], 4))
+      return EF_ERR_INVALID_ARG;
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const uint32_t tiles = efs::agg_tiles_for(d);
+  Workspace* ws = nullptr;
+  const ef_status st = efs::acquire_workspace(
+      s, 0, 0, static_cast<size_t>(n) * (static_cast<size_t>(tiles) + 1), &ws);
+  if (st != EF_OK) return st;
+  return efs::finish_launch(
+      efs::launch_aggregate(n, idx, val, counts, static_cast<uint32_t>(d), dense_out, *ws), ws);
+}
+
+ef_status ef_check_status(ef_stream_t stream) {
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(s) != cudaSuccess) return EF_ERR_CUDA;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
+  Workspace* ws = nullptr;
+  {
+    std::lock_guard<std::mutex> lk(efs::g_mu);
+    auto it = efs::g_workspaces.find(std::make_pair(dev, s));
+    if (it == efs::g_workspaces.end() || !it->second->base) return EF_OK;
+    ws = it->second;
+  }
+  uint32_t bits = 0;
+  uint32_t* dev_err = ws->u32(efs::kOffError);
+  if (cudaMemcpyAsync(&bits, dev_err, sizeof bits, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return EF_ERR_CUDA;
+  if (bits == 0) return EF_OK;
+  if (cudaMemsetAsync(dev_err, 0, sizeof bits, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return EF_ERR_CUDA;
+  if (bits & efs::kDevErrTimeout) return EF_ERR_TIMEOUT;
+  return EF_ERR_BAD_INPUT;
+}
+
+const char* ef_status_string(ef_status status) {
+  switch (status) {
+    case EF_OK: return "EF_OK";
+    case EF_ERR_INVALID_ARG: return "EF_ERR_INVALID_ARG";
+    case EF_ERR_CUDA: return "EF_ERR_CUDA";
+    case EF_ERR_TIMEOUT: return "EF_ERR_TIMEOUT";
+    case EF_ERR_BAD_INPUT: return "EF_ERR_BAD_INPUT";
+    case EF_ERR_NO_MEMORY: return "EF_ERR_NO_MEMORY";
+  }
+  return "EF_ERR_UNKNOWN";
+}
+
+ef_status ef_workspace_release(void) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
+  if (cudaDeviceSynchronize() != cudaSuccess) return EF_ERR_CUDA;
+  std::lock_guard<std::mutex> lk(efs::g_mu);
+  for (auto it = efs::g_workspaces.begin(); it != efs::g_workspaces.end();) {
+    if (it->first.first == dev) {
+      if (it->second->base) cudaFree(it->second->base);
+      delete it->second;
+      it = efs::g_workspaces.erase(it);
+    } else {
+      ++it;
+    }
+  }
+  return EF_OK;
+}
+
+uint64_t ef_kernel_launches(void) { return efs::g_launches.load(); }
+
+void ef_test_set_lookback_fault(int64_t withheld_tile, uint32_t spin_limit_us) {
+  efs::g_withheld_tile.store(withheld_tile < 0 ? -1 : withheld_tile);
+  efs::g_wait_limit_ns.store(withheld_tile < 0 ? 2000000000ull
+                                               : static_cast<uint64_t>(spin_limit_us) * 1000ull);
+}
+
+}  // extern "C"

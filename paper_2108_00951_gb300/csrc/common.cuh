@@ -1,0 +1,174 @@
+// common.cuh — device-side building blocks shared by the efsparse kernels:
+// the tile geometry, the per-stream workspace view, bounded waits, and the
+// decoupled-lookback prefix used by the ordered compaction.
+//
+// The ordered compaction is a single-pass prefix scan with decoupled
+// look-back, implemented from the published method (Merrill & Garland,
+// "Single-pass Parallel Prefix Scan with Decoupled Look-back", NVIDIA
+// NVR-2016-002): every tile publishes its own count as soon as it is known,
+// then reads its predecessors' published counts until it meets an inclusive
+// prefix. Tile ids are taken from an atomic counter in launch order, so every
+// predecessor a tile waits for has already started; every wait is bounded
+// in both iterations and wall time and latches an error instead of hanging.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace efs {
+
+// ---------------------------------------------------------------- geometry
+constexpr int kThreads = 256;                 // threads per CTA
+constexpr int kWarps = kThreads / 32;         // 8
+constexpr int kUnits = 4;                     // 4-element units per thread per tile
+constexpr int kWarpElems = 32 * 4 * kUnits;   // 512 contiguous elements per warp
+constexpr int kTileElems = kWarps * kWarpElems;  // 4096 elements per tile
+
+// Latched device error bits (mapped to ef_status on the host).
+constexpr uint32_t kDevErrTimeout = 1u;
+constexpr uint32_t kDevErrBadInput = 2u;
+constexpr uint32_t kDevErrOverflow = 4u;  // a pair position fell outside the output
+
+// Tile status word: [63:34] epoch | [33:32] flag | [31:0] count.
+constexpr uint32_t kFlagNone = 0, kFlagAggregate = 1, kFlagPrefix = 2;
+
+// Everything a compaction launch needs from the per-stream workspace.
+struct ScanCtx {
+  uint64_t* status;        // one word per tile
+  uint32_t* tile_counter;  // dynamic tile-id dispenser; 0 between launches
+  uint32_t* error;         // latched kDevErr* bits
+  uint32_t epoch;          // tags this launch's status words (1 .. 2^30-1)
+  uint32_t num_tiles;
+  int64_t withheld_tile;   // test hook: this tile never publishes (-1: none)
+  uint64_t wait_limit_ns;  // bound on any single wait
+};
+
+// --------------------------------------------------------- memory helpers
+__device__ __forceinline__ void st_relaxed_u64(uint64_t* p, uint64_t v) {
+  asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+__device__ __forceinline__ uint64_t ld_relaxed_u64(const uint64_t* p) {
+  uint64_t v;
+  asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release_u32(uint32_t* p, uint32_t v) {
+  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ uint64_t global_timer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ uint32_t lanemask_lt() {
+  uint32_t m;
+  asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+  return m;
+}
+
+// Streaming loads/stores: data touched once per call should not evict the
+// small hot structures (tile status, histograms) from L2.
+__device__ __forceinline__ float4 ld_stream_f4(const float* p) {
+  float4 v;
+  asm volatile("ld.global.cs.v4.f32 {%0,%1,%2,%3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "l"(p));
+  return v;
+}
+__device__ __forceinline__ uint2 ld_stream_u2(const void* p) {
+  uint2 v;
+  asm volatile("ld.global.cs.v2.u32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "l"(p));
+  return v;
+}
+__device__ __forceinline__ void st_stream_f4(float* p, float4 v) {
+  asm volatile("st.global.cs.v4.f32 [%0], {%1,%2,%3,%4};" ::"l"(p), "f"(v.x), "f"(v.y),
+               "f"(v.z), "f"(v.w)
+               : "memory");
+}
+
+__device__ __forceinline__ float bf16_bits_to_f32(uint32_t bits16) {
+  return __uint_as_float(bits16 << 16);
+}
+
+__device__ __forceinline__ uint64_t pack_status(uint32_t epoch, uint32_t flag, uint32_t value) {
+  return (static_cast<uint64_t>(epoch) << 34) | (static_cast<uint64_t>(flag) << 32) | value;
+}
+
+__device__ __forceinline__ uint32_t warp_sum(uint32_t v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Take the next tile id in launch order (one thread). atomicInc wraps the
+// dispenser back to 0 after handing out num_tiles - 1, so it is ready for
+// the next launch on the stream without a reset; an id >= num_tiles (only
+// possible after an aborted launch left the counter mid-way) is returned as
+// is, and the caller latches an error and does nothing with it.
+__device__ __forceinline__ uint32_t take_tile(const ScanCtx& ctx) {
+  return atomicInc(ctx.tile_counter, ctx.num_tiles - 1);
+}
+
+// Publish this tile's status (one 64-bit store, so flag and count are seen
+// together). Called by one thread.
+__device__ __forceinline__ void publish(const ScanCtx& ctx, uint32_t tile, uint32_t flag,
+                                        uint32_t value) {
+  if (static_cast<int64_t>(tile) == ctx.withheld_tile) return;  // test hook
+  st_relaxed_u64(ctx.status + tile, pack_status(ctx.epoch, flag, value));
+}
+
+// Decoupled look-back, executed by one full warp: returns the number of
+// selected elements in all tiles before `tile`. Lane l inspects tile
+// (base - l); the window slides back 32 tiles at a time until it contains an
+// inclusive prefix. Only the lanes up to the nearest prefix must be ready.
+// On a wait that runs out, `timed_out` is set (uniformly) and the partial sum
+// is returned; the caller must not use it for addressing.
+__device__ __forceinline__ uint32_t lookback_exclusive(const ScanCtx& ctx, uint32_t tile,
+                                                      bool& timed_out) {
+  const int lane = threadIdx.x & 31;
+  uint32_t excl = 0;
+  int64_t base = static_cast<int64_t>(tile) - 1;
+  uint64_t t_start = 0;
+  uint32_t iters = 0;
+  timed_out = false;
+  while (true) {
+    const int64_t t = base - lane;
+    uint32_t flag = kFlagPrefix, value = 0;
+    if (t >= 0) {
+      const uint64_t w = ld_relaxed_u64(ctx.status + t);
+      if (static_cast<uint32_t>(w >> 34) == ctx.epoch) {
+        flag = static_cast<uint32_t>(w >> 32) & 3u;
+        value = static_cast<uint32_t>(w);
+      } else {
+        flag = kFlagNone;
+      }
+    }
+    const uint32_t prefix_mask = __ballot_sync(0xffffffffu, flag == kFlagPrefix);
+    const uint32_t ready_mask = __ballot_sync(0xffffffffu, flag != kFlagNone);
+    // lanes 0 .. (nearest prefix lane); all 32 lanes if there is none
+    const uint32_t need =
+        prefix_mask ? (((prefix_mask & (0u - prefix_mask)) << 1) - 1u) : 0xffffffffu;
+    if ((ready_mask & need) != need) {
+      uint64_t now = __shfl_sync(0xffffffffu, global_timer_ns(), 0);
+      if (iters == 0) t_start = now;
+      ++iters;
+      if (iters > (1u << 26) || now - t_start > ctx.wait_limit_ns) {
+        timed_out = true;
+        const uint32_t part = ((ready_mask & need) >> lane) & 1u ? value : 0u;
+        return excl + warp_sum(part);
+      }
+      __nanosleep(64);
+      continue;
+    }
+    excl += warp_sum(((need >> lane) & 1u) ? value : 0u);
+    if (prefix_mask) return excl;
+    base -= 32;
+  }
+}
+
+}  // namespace efs

@@ -1,0 +1,113 @@
+// ht.cu — the fused error-feedback + hard-threshold + compaction kernel.
+//
+// One pass over the d coordinates performs, per coordinate j (Algorithm 1
+// with the hard-threshold sparsifier of Sec. 1 / Sec. 4.2):
+//   a_j  = fmaf(gamma, g_j, e_j)                 corrected update p = e + gamma g
+//   s_j  = (|a_j| >= lambda) and (a_j != 0)      j in S_lambda(a)
+//   e_j <- s_j ? +0 : a_j                        error update e <- p - C(p)
+// and writes the selected (j, a_j) pairs in ascending j through the ordered
+// compaction. HBM traffic per coordinate is the algorithmic minimum: read g
+// (4 B, or 2 B for bf16) and e (4 B), write e (4 B); plus 8 B per sent pair.
+#include "compact.cuh"
+#include "gradient.cuh"
+#include "internal.h"
+
+namespace efs {
+namespace {
+
+__device__ __forceinline__ uint32_t in_support(float a, float lambda) {
+  return (fabsf(a) >= lambda && a != 0.0f) ? 1u : 0u;
+}
+
+template <typename GT, bool kVec>
+__global__ void __launch_bounds__(kThreads)
+    ht_kernel(const GT* __restrict__ g, float* __restrict__ e, float gamma, float lambda,
+              uint32_t d, uint32_t* __restrict__ idx_out, float* __restrict__ val_out,
+              uint32_t* __restrict__ count_out, ScanCtx ctx) {
+  __shared__ uint32_t s_tile;
+  if (threadIdx.x == 0) s_tile = take_tile(ctx);
+  __syncthreads();
+  const uint32_t tile = s_tile;
+  if (tile >= ctx.num_tiles) {  // stale dispenser: never touch memory with it
+    if (threadIdx.x == 0) atomicOr(ctx.error, kDevErrTimeout);
+    return;
+  }
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint64_t first = element_index(tile, warp, 0, lane, 0);
+
+  float a[kUnits][4];
+  uint32_t sel[kUnits];
+  const bool full_tile = static_cast<uint64_t>(tile + 1) * kTileElems <= d;
+
+  if (kVec && full_tile) {
+    GradVec<GT> gv[kUnits];
+    float4 ev[kUnits];
+#pragma unroll
+    for (int v = 0; v < kUnits; ++v) {  // all loads in flight before any use
+      gv[v].load(g + first + v * 128);
+      ev[v] = ld_stream_f4(e + first + v * 128);
+    }
+#pragma unroll
+    for (int v = 0; v < kUnits; ++v) {
+      a[v][0] = __fmaf_rn(gamma, gv[v][0], ev[v].x);
+      a[v][1] = __fmaf_rn(gamma, gv[v][1], ev[v].y);
+      a[v][2] = __fmaf_rn(gamma, gv[v][2], ev[v].z);
+      a[v][3] = __fmaf_rn(gamma, gv[v][3], ev[v].w);
+      sel[v] = in_support(a[v][0], lambda) | (in_support(a[v][1], lambda) << 1) |
+               (in_support(a[v][2], lambda) << 2) | (in_support(a[v][3], lambda) << 3);
+      const float4 r = make_float4((sel[v] & 1u) ? 0.0f : a[v][0], (sel[v] & 2u) ? 0.0f : a[v][1],
+                                   (sel[v] & 4u) ? 0.0f : a[v][2], (sel[v] & 8u) ? 0.0f : a[v][3]);
+      st_stream_f4(e + first + v * 128, r);
+    }
+  } else {
+#pragma unroll
+    for (int v = 0; v < kUnits; ++v) {
+      sel[v] = 0;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint64_t i = first + v * 128 + j;
+        a[v][j] = 0.0f;
+        if (i < d) {
+          const float x = __fmaf_rn(gamma, grad_scalar(g, i), e[i]);
+          const uint32_t s = in_support(x, lambda);
+          a[v][j] = x;
+          sel[v] |= s << j;
+          e[i] = s ? 0.0f : x;
+        }
+      }
+    }
+  }
+  compact_tile(ctx, tile, sel, a, idx_out, val_out, count_out, d);
+}
+
+template <typename GT>
+cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint32_t d,
+                         uint32_t* idx_out, float* val_out, uint32_t* count_out, Workspace& ws) {
+  const uint32_t tiles = tiles_for(d);
+  const ScanCtx ctx = next_scan_ctx(ws, tiles);
+  const uintptr_t ga = reinterpret_cast<uintptr_t>(g), ea = reinterpret_cast<uintptr_t>(e);
+  const bool vec = (ga % (4 * sizeof(GT)) == 0) && (ea % 16 == 0);
+  if (vec) {
+    ht_kernel<GT, true><<<tiles, kThreads, 0, ws.stream>>>(g, e, gamma, lambda, d, idx_out,
+                                                           val_out, count_out, ctx);
+  } else {
+    ht_kernel<GT, false><<<tiles, kThreads, 0, ws.stream>>>(g, e, gamma, lambda, d, idx_out,
+                                                            val_out, count_out, ctx);
+  }
+  count_launch();
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_hard_threshold(const void* g, bool g_bf16, float* e, float gamma,
+                                  float lambda, uint32_t d, uint32_t* idx_out, float* val_out,
+                                  uint32_t* count_out, Workspace& ws) {
+  if (g_bf16)
+    return launch_typed(static_cast<const uint16_t*>(g), e, gamma, lambda, d, idx_out, val_out,
+                        count_out, ws);
+  return launch_typed(static_cast<const float*>(g), e, gamma, lambda, d, idx_out, val_out,
+                      count_out, ws);
+}
+
+}  // namespace efs

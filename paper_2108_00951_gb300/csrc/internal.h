@@ -1,0 +1,85 @@
+// internal.h — host-side declarations shared by the efsparse translation
+// units: the per-stream workspace and the kernel launchers.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+
+namespace efs {
+
+// Layout of the workspace header (bytes from the workspace base).
+constexpr size_t kOffBarGen = 0;        // uint32: grid-barrier generation (never reset)
+constexpr size_t kOffTileCounter = 4;   // uint32: tile-id dispenser (0 between launches)
+constexpr size_t kOffError = 8;         // uint32: latched device error bits
+constexpr size_t kOffTopkReset = 16;    // start of the region cleared at each Top-k call
+constexpr size_t kOffBarArrive = 16;    // uint32
+constexpr size_t kOffCandCount = 20;    // uint32[6]
+constexpr size_t kOffThreshold = 48;    // uint64: Top-k composite-key threshold
+constexpr size_t kOffHist = 256;        // uint32[6][2048]
+constexpr int kHistLevels = 6;
+constexpr int kHistBins = 2048;
+constexpr size_t kHeaderBytes = kOffHist + sizeof(uint32_t) * kHistLevels * kHistBins;
+constexpr size_t kTopkResetBytes = kHeaderBytes - kOffTopkReset;
+
+struct Workspace {
+  int device = -1;
+  cudaStream_t stream = nullptr;
+  char* base = nullptr;
+  size_t bytes = 0;
+  uint32_t status_tiles = 0;   // capacity of the tile-status array
+  uint32_t cand_cap = 0;       // capacity of each Top-k candidate buffer
+  size_t offsets_cap = 0;      // capacity of the aggregation offsets (uint32)
+  uint32_t epoch = 0;          // last epoch handed to a compaction launch
+  bool dirty = false;          // a launch failed: header must be re-cleared
+
+  uint64_t* status() const { return reinterpret_cast<uint64_t*>(base + kHeaderBytes); }
+  uint64_t* cand(int i) const {
+    return reinterpret_cast<uint64_t*>(base + kHeaderBytes + sizeof(uint64_t) * status_tiles) +
+           static_cast<size_t>(i) * cand_cap;
+  }
+  uint32_t* offsets() const { return reinterpret_cast<uint32_t*>(cand(2)); }
+  uint32_t* u32(size_t off) const { return reinterpret_cast<uint32_t*>(base + off); }
+  uint64_t* u64(size_t off) const { return reinterpret_cast<uint64_t*>(base + off); }
+};
+
+// Per-device facts queried once.
+struct DeviceInfo {
+  int sm_count = 0;
+  int refine_blocks = 0;   // co-resident CTAs for the cooperative Top-k refine
+};
+
+// Launch bookkeeping.
+void count_launch();
+uint64_t wait_limit_ns();
+int64_t withheld_tile();
+ScanCtx next_scan_ctx(Workspace& ws, uint32_t num_tiles);
+
+// ---- launchers (return the launch's cudaError_t) ----
+cudaError_t launch_hard_threshold(const void* g, bool g_bf16, float* e, float gamma,
+                                  float lambda, uint32_t d, uint32_t* idx_out, float* val_out,
+                                  uint32_t* count_out, Workspace& ws);
+cudaError_t launch_topk(const void* g, bool g_bf16, float* e, float gamma, uint32_t k,
+                        uint32_t d, uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                        Workspace& ws, const DeviceInfo& dev);
+cudaError_t launch_aggregate(uint32_t n, const uint32_t* const* idx, const float* const* val,
+                             const uint32_t* counts, uint32_t d, float* dense_out,
+                             Workspace& ws);
+
+// Occupancy of the cooperative Top-k refine kernel (CTAs per SM).
+int topk_refine_blocks_per_sm();
+
+// Workspace sizing helpers.
+inline uint32_t tiles_for(uint64_t d) {
+  return static_cast<uint32_t>((d + kTileElems - 1) / kTileElems);
+}
+constexpr int kAggTile = 4096;             // dense elements per aggregation CTA
+constexpr uint32_t kMaxWorkers = 256;
+inline uint32_t agg_tiles_for(uint64_t d) {
+  return static_cast<uint32_t>((d + kAggTile - 1) / kAggTile);
+}
+uint32_t topk_candidate_capacity(uint64_t d);
+
+}  // namespace efs

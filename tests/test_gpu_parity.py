@@ -1,0 +1,277 @@
+"""GPU parity: the CUDA path against the CPU oracle, bit for bit.
+
+Masks, indices, counts, sent values and residuals must match exactly (same
+single fma, same tie rule); the aggregate must match exactly (same worker
+order). Small cases span several 4096-coordinate tiles with ragged tails;
+full-size cases use the benchmark's workloads and launch configuration.
+"""
+import zlib
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2108_00951_gb300 as efs
+from paper_2108_00951_gb300 import workloads
+
+pytestmark = pytest.mark.gpu
+if not torch.cuda.is_available():
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+import gpu_util as gu  # noqa: E402
+
+RAGGED = [1, 3, 4, 5, 127, 4095, 4096, 4097, 3 * 4096 + 17, 100_003]
+
+
+def _rng(*key):
+    return np.random.default_rng(zlib.crc32(repr(key).encode()))
+
+
+def _inputs(d, seed, gscale=1e-2, escale=1e-3, bf16=False):
+    rng = _rng("in", d, seed)
+    g = (rng.standard_normal(d) * gscale).astype(np.float32)
+    e = (rng.standard_normal(d) * escale).astype(np.float32)
+    if bf16:
+        g = torch.from_numpy(g).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    return g, e
+
+
+def _check_same(gpu, ref, what):
+    gi, gv, ge = gpu
+    ri, rv, re_ = ref
+    gu.assert_bits(gi, ri, what + " idx")
+    gu.assert_bits(gv, rv, what + " val")
+    gu.assert_bits(ge, re_, what + " e'")
+
+
+# ------------------------------------------------------------ hard-threshold
+@pytest.mark.parametrize("bf16", [False, True])
+@pytest.mark.parametrize("d", RAGGED)
+def test_ht_random(d, bf16):
+    g, e = _inputs(d, 1, bf16=bf16)
+    for lam in (0.0, 1e-3, 2e-3, 1.0):
+        _check_same(gu.ht(g, e, 0.1, lam), oracle.ef_hard_threshold(g, e, 0.1, lam),
+                    "d=%d lam=%g" % (d, lam))
+
+
+@pytest.mark.parametrize("offs", [(1, 0), (0, 1), (1, 1), (3, 2), (2, 0)])
+@pytest.mark.parametrize("bf16", [False, True])
+def test_ht_misaligned_bases(offs, bf16):
+    d = 2 * 4096 + 333
+    g, e = _inputs(d, 2, bf16=bf16)
+    _check_same(gu.ht(g, e, 0.1, 1.5e-3, g_off=offs[0], e_off=offs[1]),
+                oracle.ef_hard_threshold(g, e, 0.1, 1.5e-3), "offsets %s" % (offs,))
+
+
+def test_ht_adversarial_values():
+    d = 3 * 4096 + 5
+    rng = _rng("adv")
+    lam = np.float32(0.25)
+    pool = np.array([lam, -lam, np.nextafter(lam, np.float32(0)), 0.0, -0.0, np.nan, np.inf,
+                     -np.inf, np.finfo(np.float32).smallest_subnormal,
+                     -np.finfo(np.float32).tiny, 1e30, -3.0], dtype=np.float32)
+    e = pool[rng.integers(0, len(pool), d)]
+    g = np.zeros(d, np.float32)
+    g[rng.integers(0, d, 500)] = -0.0
+    for gamma, lam_ in ((1.0, float(lam)), (0.5, 0.0), (1.0, float("inf"))):
+        _check_same(gu.ht(g, e, gamma, lam_), oracle.ef_hard_threshold(g, e, gamma, lam_),
+                    "adversarial lam=%g" % lam_)
+
+
+def test_ht_fma_sensitive_values():
+    # e = -round(gamma*g): a is the product's rounding error, which only a
+    # single-rounding fma preserves
+    d = 50_000
+    rng = _rng("fma")
+    g = (rng.standard_normal(d) * np.exp2(rng.integers(-10, 10, d))).astype(np.float32)
+    gamma = np.float32(0.1)
+    e = -(gamma * g)
+    _check_same(gu.ht(g, e, float(gamma), 0.0), oracle.ef_hard_threshold(g, e, float(gamma), 0.0),
+                "fma")
+
+
+def test_ht_all_and_nothing_sent():
+    d = 5 * 4096 + 1
+    g, e = _inputs(d, 3)
+    i, v, en = gu.ht(g, e, 0.1, 0.0)            # every non-zero a is sent
+    assert i.size == d
+    _check_same((i, v, en), oracle.ef_hard_threshold(g, e, 0.1, 0.0), "all")
+    i, v, en = gu.ht(g, e, 0.1, 1e9)            # nothing is sent
+    assert i.size == 0
+    _check_same((i, v, en), oracle.ef_hard_threshold(g, e, 0.1, 1e9), "none")
+
+
+def test_ht_zero_length():
+    cnt = torch.full((1,), 7, dtype=torch.int32, device=gu.DEV)
+    z = torch.empty(0, device=gu.DEV)
+    zi = torch.empty(0, dtype=torch.int32, device=gu.DEV)
+    efs.ef_hard_threshold(z, z.clone(), 0.1, 1e-3, zi, z.clone(), cnt)
+    assert int(cnt.item()) == 0
+
+
+def test_ht_concurrent_streams():
+    # calls on different streams use different workspaces and may overlap
+    d = 300_000
+    g1, e1 = _inputs(d, 4)
+    g2, e2 = _inputs(d, 5)
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    outs = []
+    for (g, e), s in (((g1, e1), s1), ((g2, e2), s2)):
+        gd, ed = gu.to_dev(g), gu.to_dev(e)
+        idx = torch.empty(d, dtype=torch.int32, device=gu.DEV)
+        val = torch.empty(d, dtype=torch.float32, device=gu.DEV)
+        cnt = torch.empty(1, dtype=torch.int32, device=gu.DEV)
+        torch.cuda.synchronize()
+        for _ in range(3):
+            ed.copy_(torch.from_numpy(e))
+            with torch.cuda.stream(s):
+                efs.ef_hard_threshold(gd, ed, 0.1, 1e-3, idx, val, cnt)
+        outs.append((idx, val, cnt, ed))
+    torch.cuda.synchronize()
+    for (idx, val, cnt, ed), (g, e) in zip(outs, ((g1, e1), (g2, e2))):
+        c = int(cnt.item())
+        _check_same((idx[:c].cpu().numpy().view(np.uint32), val[:c].cpu().numpy(),
+                     ed.cpu().numpy()), oracle.ef_hard_threshold(g, e, 0.1, 1e-3), "stream")
+
+
+# ---------------------------------------------------------------------- Top-k
+@pytest.mark.parametrize("d", RAGGED)
+def test_topk_random(d):
+    g, e = _inputs(d, 11)
+    for k in sorted({0, 1, max(1, d // 100), d // 2, d}):
+        _check_same(gu.topk(g, e, 0.1, k), oracle.ef_topk(g, e, 0.1, k), "d=%d k=%d" % (d, k))
+
+
+def test_topk_bf16_and_misaligned():
+    d = 3 * 4096 + 77
+    g, e = _inputs(d, 12, bf16=True)
+    for offs in ((0, 0), (1, 1), (3, 0), (0, 2)):
+        _check_same(gu.topk(g, e, 0.1, 500, g_off=offs[0], e_off=offs[1]),
+                    oracle.ef_topk(g, e, 0.1, 500), "offs %s" % (offs,))
+
+
+def test_topk_heavy_ties():
+    d = 200_003
+    rng = _rng("ties")
+    pool = np.array([0.0, -0.0, 0.5, -0.5, 0.25, 1.0, -1.0, 2.0], np.float32)
+    e = pool[rng.integers(0, len(pool), d)]
+    g = np.zeros(d, np.float32)
+    for k in (1, 7, 1000, 25_000, 100_000, 199_999):
+        _check_same(gu.topk(g, e, 1.0, k), oracle.ef_topk(g, e, 1.0, k), "ties k=%d" % k)
+
+
+def test_topk_mostly_zero_like_lstm_embedding():
+    # ~62% exact zeros; k beyond the non-zeros forces the choice into the zero bucket
+    d = 400_000
+    rng = _rng("zeros")
+    g = (rng.standard_t(3, d) * 1e-3).astype(np.float32)
+    g[rng.random(d) < 0.62] = 0.0
+    e = np.zeros(d, np.float32)
+    nz = int(np.count_nonzero(g))
+    for k in (d // 100, nz - 1, nz, nz + 1, nz + 5000):
+        _check_same(gu.topk(g, e, 0.1, k), oracle.ef_topk(g, e, 0.1, k), "zeros k=%d" % k)
+
+
+def test_topk_all_equal_magnitude_large():
+    # all keys tie in the magnitude bits: the index digits decide, through
+    # full-array refine passes (the bucket exceeds the candidate buffer)
+    d = 3_000_017
+    e = np.full(d, 0.75, np.float32)
+    e[1::3] = -0.75
+    g = np.zeros(d, np.float32)
+    for k in (1, 1_000_000, 2_500_000):
+        gi, gv, ge = gu.topk(g, e, 1.0, k)
+        assert gi.size == k and np.array_equal(gi, np.arange(k, dtype=np.uint32))
+        gu.assert_bits(gv, e[:k], "vals")
+        want = e.copy()
+        want[:k] = 0.0
+        gu.assert_bits(ge, want, "e'")
+
+
+def test_topk_nan_inf():
+    d = 9000
+    g, e = _inputs(d, 13)
+    e[[5, 4097, 8000]] = [np.nan, np.inf, -np.inf]
+    for k in (1, 2, 3, 10):
+        _check_same(gu.topk(g, e, 0.1, k), oracle.ef_topk(g, e, 0.1, k), "nan k=%d" % k)
+
+
+# ---------------------------------------------------------------- aggregation
+def _sparse_lists(n, d, density, seed, integer=False):
+    rng = _rng("agg", n, d, seed)
+    idx, val = [], []
+    for _ in range(n):
+        m = rng.random(d) < density
+        i = np.nonzero(m)[0].astype(np.uint32)
+        v = (rng.integers(-9, 9, i.size) if integer else rng.standard_normal(i.size)).astype(np.float32)
+        idx.append(i)
+        val.append(v)
+    return idx, val
+
+
+@pytest.mark.parametrize("n", [1, 2, 4, 8, 16])
+@pytest.mark.parametrize("d", [5, 4096, 4097, 100_003])
+def test_aggregate_random(n, d):
+    for density in (0.001, 0.05, 1.0):
+        idx, val = _sparse_lists(n, d, density, 1)
+        gu.assert_bits(gu.aggregate(idx, val, d), oracle.sparse_aggregate(idx, val, d),
+                       "n=%d d=%d rho=%g" % (n, d, density))
+
+
+def test_aggregate_order_and_signed_zero():
+    big = np.float32(2.0 ** 24)
+    idx = [np.array([3, 4100], np.uint32)] * 3
+    val = [np.array([big, -0.0], np.float32), np.array([1.0, -0.0], np.float32),
+           np.array([-big, -0.0], np.float32)]
+    out = gu.aggregate(idx, val, 5000)
+    gu.assert_bits(out, oracle.sparse_aggregate(idx, val, 5000), "order")
+    assert out[3] == 0.0 and gu.bits(out[4100:4101])[0] == 0   # +0.0
+
+
+def test_aggregate_empty_lists_and_misaligned_output():
+    d = 20_001
+    idx, val = _sparse_lists(6, d, 0.01, 2)
+    idx[2], val[2] = idx[2][:0], val[2][:0]
+    idx[5], val[5] = idx[5][:0], val[5][:0]
+    for off in (0, 1, 3):
+        gu.assert_bits(gu.aggregate(idx, val, d, dense_off=off),
+                       oracle.sparse_aggregate(idx, val, d), "off=%d" % off)
+
+
+# ------------------------------------------------------- multi-iteration EF
+@pytest.mark.parametrize("method", ["ht", "topk"])
+def test_lr_workload_all_iterations(method):
+    """Configuration 0 (d = 100,000, n = 4, T = 10): every worker, every
+    iteration, and the aggregate of every iteration, each side on its own state."""
+    w = workloads.BY_NAME["lr"]
+    e_ref = [np.zeros(w.d, np.float32) for _ in range(w.n)]
+    e_gpu = [gu.to_dev(np.zeros(w.d, np.float32)) for _ in range(w.n)]
+    k, lam = w.topk_k[0], w.lambdas[0]
+    for t in range(w.T):
+        gi_all, gv_all, ri_all, rv_all = [], [], [], []
+        for i in range(w.n):
+            g = workloads.gradient(w, i, t)
+            idx = torch.empty(w.d, dtype=torch.int32, device=gu.DEV)
+            val = torch.empty(w.d, dtype=torch.float32, device=gu.DEV)
+            cnt = torch.empty(1, dtype=torch.int32, device=gu.DEV)
+            if method == "ht":
+                efs.ef_hard_threshold(g.to(gu.DEV), e_gpu[i], w.gamma, lam, idx, val, cnt)
+                ri, rv, e_ref[i] = oracle.ef_hard_threshold(g.numpy(), e_ref[i], w.gamma, lam)
+            else:
+                efs.ef_topk(g.to(gu.DEV), e_gpu[i], w.gamma, k, idx, val, cnt)
+                ri, rv, e_ref[i] = oracle.ef_topk(g.numpy(), e_ref[i], w.gamma, k)
+            c = int(cnt.item())
+            gu.assert_bits(idx[:c].cpu().numpy().view(np.uint32), ri, "t=%d i=%d idx" % (t, i))
+            gu.assert_bits(val[:c].cpu().numpy(), rv, "val")
+            gu.assert_bits(e_gpu[i].cpu().numpy(), e_ref[i], "e'")
+            gi_all.append(idx[:c])
+            gv_all.append(val[:c])
+            ri_all.append(ri)
+            rv_all.append(rv)
+        counts = torch.tensor([len(r) for r in ri_all], dtype=torch.int32, device=gu.DEV)
+        dense = torch.empty(w.d, dtype=torch.float32, device=gu.DEV)
+        efs.sparse_aggregate(gi_all, gv_all, counts, w.d, dense)
+        gu.assert_bits(dense.cpu().numpy(), oracle.sparse_aggregate(ri_all, rv_all, w.d),
+                       "aggregate t=%d" % t)
+    assert efs.ef_check_status() == efs.EF_OK

@@ -1,0 +1,102 @@
+"""The C-ABI library builds, loads and exports every declared entry point;
+host-side argument checks reject bad calls before any CUDA work (no GPU)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2108_00951_gb300 as efs
+from paper_2108_00951_gb300 import build
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))),
+                      "include", "efsparse.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return re.findall(r"^(?:ef_status|const char\s*\*|uint64_t|void)\s+(\w+)\s*\(", text, re.M)
+
+
+def test_header_declares_the_boundary():
+    names = set(declared_functions())
+    for required in ("ef_hard_threshold", "ef_hard_threshold_bf16", "ef_topk", "ef_topk_bf16",
+                     "sparse_aggregate", "ef_check_status", "ef_status_string"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol():
+    lib = ctypes.CDLL(build.build())
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_status_strings():
+    for code, name in [(0, "EF_OK"), (1, "EF_ERR_INVALID_ARG"), (2, "EF_ERR_CUDA"),
+                       (3, "EF_ERR_TIMEOUT"), (4, "EF_ERR_BAD_INPUT"), (5, "EF_ERR_NO_MEMORY")]:
+        assert efs.status_string(code) == name
+
+
+# Host-side checks run before any CUDA call, so they work without a GPU. The
+# pointers below are fake, 16-byte aligned, non-overlapping addresses; they
+# are never dereferenced because every call is rejected first.
+G, E, IDX, VAL, CNT = 0x10000000, 0x20000000, 0x30000000, 0x40000000, 0x50000000
+vp = ctypes.c_void_p
+
+
+def _ht(g=G, e=E, gamma=0.1, lam=1e-3, d=1000, idx=IDX, val=VAL, cnt=CNT, bf16=False):
+    lib = efs.load_library()
+    fn = lib.ef_hard_threshold_bf16 if bf16 else lib.ef_hard_threshold
+    return fn(vp(g), vp(e), ctypes.c_float(gamma), ctypes.c_float(lam), d, vp(idx), vp(val),
+              vp(cnt), vp(0))
+
+
+def _topk(g=G, e=E, gamma=0.1, k=10, d=1000, idx=IDX, val=VAL, cnt=CNT):
+    lib = efs.load_library()
+    return lib.ef_topk(vp(g), vp(e), ctypes.c_float(gamma), k, d, vp(idx), vp(val), vp(cnt),
+                       vp(0))
+
+
+@pytest.mark.parametrize("kwargs", [
+    dict(cnt=0), dict(g=0), dict(e=0), dict(idx=0), dict(val=0),
+    dict(lam=-1e-3), dict(lam=float("nan")), dict(gamma=float("inf")), dict(gamma=float("nan")),
+    dict(d=2 ** 32), dict(e=E + 2), dict(g=G + 1), dict(idx=IDX + 1), dict(cnt=CNT + 2),
+    dict(idx=E + 64), dict(val=G), dict(val=IDX + 100), dict(cnt=VAL + 8), dict(e=G + 400),
+])
+def test_hard_threshold_rejects(kwargs):
+    assert _ht(**kwargs) == efs.EF_ERR_INVALID_ARG
+
+
+def test_hard_threshold_bf16_alignment_rule():
+    assert _ht(g=G + 1, bf16=True) == efs.EF_ERR_INVALID_ARG      # bf16 needs 2-byte alignment
+
+
+@pytest.mark.parametrize("kwargs", [
+    dict(k=1001), dict(d=2 ** 32, k=1), dict(cnt=0), dict(g=0), dict(idx=0),
+    dict(gamma=float("nan")), dict(val=E), dict(e=E + 1),
+])
+def test_topk_rejects(kwargs):
+    assert _topk(**kwargs) == efs.EF_ERR_INVALID_ARG
+
+
+def test_aggregate_rejects():
+    lib = efs.load_library()
+    arr = (vp * 1)(vp(IDX))
+    varr = (vp * 1)(vp(VAL))
+    assert lib.sparse_aggregate(0, arr, varr, vp(CNT), 100, vp(G), vp(0)) == efs.EF_ERR_INVALID_ARG
+    assert lib.sparse_aggregate(257, arr, varr, vp(CNT), 100, vp(G), vp(0)) == efs.EF_ERR_INVALID_ARG
+    assert lib.sparse_aggregate(1, arr, varr, vp(0), 100, vp(G), vp(0)) == efs.EF_ERR_INVALID_ARG
+    assert lib.sparse_aggregate(1, arr, varr, vp(CNT), 100, vp(0), vp(0)) == efs.EF_ERR_INVALID_ARG
+    assert lib.sparse_aggregate(1, arr, varr, vp(CNT), 2 ** 32, vp(G), vp(0)) == efs.EF_ERR_INVALID_ARG
+    bad = (vp * 1)(vp(0))
+    assert lib.sparse_aggregate(1, bad, varr, vp(CNT), 100, vp(G), vp(0)) == efs.EF_ERR_INVALID_ARG
+    assert lib.sparse_aggregate(1, arr, varr, vp(CNT), 100, vp(G + 1), vp(0)) == efs.EF_ERR_INVALID_ARG
+
+
+def test_binding_fails_loudly_on_cpu_tensors():
+    torch = pytest.importorskip("torch")
+    x = torch.zeros(8)
+    i = torch.zeros(8, dtype=torch.int32)
+    with pytest.raises(TypeError):
+        efs.ef_hard_threshold(x, x.clone(), 0.1, 1e-3, i, x.clone(), i[:1])

@@ -18,7 +18,7 @@ import test_oracle_pins as pins
 _SRC = os.path.join(os.path.dirname(oracle.__file__), "oracle.c")
 
 MUTANTS = {
-    "two_step_rounding": [("fmaf(gamma, gj, e[j])", "gamma * gj + e[j]")],
+    "two_step_rounding": [("fmaf(gamma, gj, e[j])", "(gamma * gj + e[j])")],
     "swapped_operands": [("fmaf(gamma, gj, e[j])", "fmaf(gamma, e[j], gj)")],
     "dropped_error_term": [("fmaf(gamma, gj, e[j])", "fmaf(gamma, gj, 0.0f)")],
     "wrong_sign": [("fmaf(gamma, gj, e[j])", "fmaf(-gamma, gj, e[j])")],
@@ -30,6 +30,7 @@ MUTANTS = {
     "topk_highest_index_ties": [("  return (ia > ib) - (ia < ib);", "  return (ia < ib) - (ia > ib);")],
     "topk_residual_kept": [("    e[j] = 0.0f;                                      /* R7 */",
                             "    e[j] = a[j];")],
+    "nan_payload_kept": [("  if (!isnan(x)) return x;", "  return x;")],
     "aggregate_reverse_order": [("for (uint32_t i = 0; i < n; ++i) {",
                                  "for (uint32_t i = n; i-- > 0;) {")],
     "nan_ranks_lowest": [("    if (!ny) return 1;\n    if (!nx) return -1;",

@@ -111,13 +111,22 @@ def test_ht_lambda_above_max_sends_nothing():
     assert _same_bits(e_new, a)
 
 
+CANONICAL_NAN = 0x7FFFFFFF
+
+
 def test_ht_nan_and_inf():
-    e = _f32([np.nan, np.inf, -np.inf, 1.0])
-    g = np.zeros(4, np.float32)
+    # NaN never passes |a| >= lambda; +-inf does; 0 * inf is NaN (invalid)
+    e = _f32([np.nan, np.inf, -np.inf, 1.0, 5.0])
+    g = _f32([0.0, 0.0, 0.0, 0.0, np.inf])
     idx, val, e_new = oracle.ef_hard_threshold(g, e, 1.0, 0.5)
-    assert idx.tolist() == [1, 2, 3]
-    assert val.tolist() == [np.inf, -np.inf, 1.0]
-    assert np.isnan(e_new[0]) and e_new[1:].tolist() == [0.0, 0.0, 0.0]
+    assert idx.tolist() == [1, 2, 3, 4]
+    assert val.tolist() == [np.inf, -np.inf, 1.0, np.inf]
+    assert e_new[1:].tolist() == [0.0, 0.0, 0.0, 0.0]
+    # every NaN result carries the one canonical encoding (reading R6)
+    e = _f32([np.nan, 2.0])
+    e[0] = np.uint32(0x7FC00001).view(np.float32)        # a NaN with a payload
+    _, _, e_new = oracle.ef_hard_threshold(_f32([0.0, np.inf]), e, 0.0, 0.5)
+    assert e_new.view(np.uint32).tolist() == [CANONICAL_NAN, CANONICAL_NAN]
 
 
 @pytest.mark.parametrize("d", [1, 7, 64, 3001])
@@ -319,6 +328,13 @@ def test_aggregate_sums_in_worker_order():
     assert dense[5] == 0.0
     dense = oracle.sparse_aggregate(idx, [_f32([-big]), _f32([1.0]), _f32([big])], 8)
     assert dense[5] == 1.0
+
+
+def test_aggregate_nan_is_canonical():
+    nan = np.uint32(0x7FC00001).view(np.float32)
+    dense = oracle.sparse_aggregate([np.array([1], np.uint32), np.array([1], np.uint32)],
+                                    [_f32([nan]), _f32([1.0])], 3)
+    assert dense.view(np.uint32)[1] == CANONICAL_NAN
 
 
 def test_aggregate_rejects_out_of_range():
