@@ -41,6 +41,7 @@ ef_status device_info(int dev, DeviceInfo* out) {
     const int per_sm = topk_refine_blocks_per_sm();
     if (per_sm <= 0) return EF_ERR_CUDA;
     info.refine_blocks = per_sm * info.sm_count;
+    ht_init_device(info);
     it = g_devices.emplace(dev, info).first;
   }
   *out = it->second;
@@ -130,11 +131,16 @@ ef_status hard_threshold_entry(const void* g, bool bf16, float* e, float gamma, 
       if (overlaps(outs[o], out_n[o], outs[p], out_n[p])) return EF_ERR_INVALID_ARG;
   }
   if (overlaps(g, d * gsz, e, nb)) return EF_ERR_INVALID_ARG;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
+  DeviceInfo info;
+  ef_status st = device_info(dev, &info);
+  if (st != EF_OK) return st;
   Workspace* ws = nullptr;
-  const ef_status st = acquire_workspace(stream, tiles_for(d), 0, 0, &ws);
+  st = acquire_workspace(stream, tiles_for(d), 0, 0, &ws);
   if (st != EF_OK) return st;
   return finish_launch(launch_hard_threshold(g, bf16, e, gamma, lambda, static_cast<uint32_t>(d),
-                                             idx_out, val_out, count_out, *ws),
+                                             idx_out, val_out, count_out, *ws, info),
                        ws);
 }
 
@@ -187,7 +193,6 @@ ScanCtx next_scan_ctx(Workspace& ws, uint32_t num_tiles) {
   ++ws.epoch;
   ScanCtx c;
   c.status = ws.status();
-  c.tile_counter = ws.u32(kOffTileCounter);
   c.error = ws.u32(kOffError);
   c.epoch = ws.epoch;
   c.num_tiles = num_tiles;

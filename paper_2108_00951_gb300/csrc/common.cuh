@@ -7,9 +7,16 @@
 // "Single-pass Parallel Prefix Scan with Decoupled Look-back", NVIDIA
 // NVR-2016-002): every tile publishes its own count as soon as it is known,
 // then reads its predecessors' published counts until it meets an inclusive
-// prefix. Tile ids are taken from an atomic counter in launch order, so every
-// predecessor a tile waits for has already started; every wait is bounded
-// in both iterations and wall time and latches an error instead of hanging.
+// prefix. A tile's id is its CTA's linear index; CTAs of a one-dimensional
+// grid are dispatched in increasing index order, so every predecessor a tile
+// waits for has started before it. Every wait is bounded in iterations and
+// wall time and latches an error instead of hanging.
+//
+// Throughput of the scan: a tile can only finish once it sees an inclusive
+// prefix, so the set of resolved tiles grows by at most one look-back window
+// per L2 round trip. With a 32-tile window and 4096-element tiles that caps a
+// 12-byte-per-element pass near 2 TB/s on this GPU; each lane therefore reads
+// four status words, giving a 128-tile window.
 #pragma once
 
 #include <cstdint>
@@ -35,7 +42,6 @@ constexpr uint32_t kFlagNone = 0, kFlagAggregate = 1, kFlagPrefix = 2;
 // Everything a compaction launch needs from the per-stream workspace.
 struct ScanCtx {
   uint64_t* status;        // one word per tile
-  uint32_t* tile_counter;  // dynamic tile-id dispenser; 0 between launches
   uint32_t* error;         // latched kDevErr* bits
   uint32_t epoch;          // tags this launch's status words (1 .. 2^30-1)
   uint32_t num_tiles;
@@ -105,15 +111,6 @@ __device__ __forceinline__ uint32_t warp_sum(uint32_t v) {
   return v;
 }
 
-// Take the next tile id in launch order (one thread). atomicInc wraps the
-// dispenser back to 0 after handing out num_tiles - 1, so it is ready for
-// the next launch on the stream without a reset; an id >= num_tiles (only
-// possible after an aborted launch left the counter mid-way) is returned as
-// is, and the caller latches an error and does nothing with it.
-__device__ __forceinline__ uint32_t take_tile(const ScanCtx& ctx) {
-  return atomicInc(ctx.tile_counter, ctx.num_tiles - 1);
-}
-
 // Publish this tile's status (one 64-bit store, so flag and count are seen
 // together). Called by one thread.
 __device__ __forceinline__ void publish(const ScanCtx& ctx, uint32_t tile, uint32_t flag,
@@ -123,11 +120,15 @@ __device__ __forceinline__ void publish(const ScanCtx& ctx, uint32_t tile, uint3
 }
 
 // Decoupled look-back, executed by one full warp: returns the number of
-// selected elements in all tiles before `tile`. Lane l inspects tile
-// (base - l); the window slides back 32 tiles at a time until it contains an
-// inclusive prefix. Only the lanes up to the nearest prefix must be ready.
-// On a wait that runs out, `timed_out` is set (uniformly) and the partial sum
-// is returned; the caller must not use it for addressing.
+// selected elements in all tiles before `tile`. The window holds the 128
+// nearest unresolved predecessors: lane l inspects tiles base-4l .. base-4l-3
+// (nearest first). It slides back 128 tiles at a time until it contains an
+// inclusive prefix; only the positions up to the nearest prefix must be ready.
+// On a wait that runs out, `timed_out` is set (uniformly) and a partial sum is
+// returned; the caller must not use it for addressing.
+constexpr int kLookbackPerLane = 4;
+constexpr int kLookbackWindow = 32 * kLookbackPerLane;
+
 __device__ __forceinline__ uint32_t lookback_exclusive(const ScanCtx& ctx, uint32_t tile,
                                                       bool& timed_out) {
   const int lane = threadIdx.x & 31;
@@ -137,37 +138,51 @@ __device__ __forceinline__ uint32_t lookback_exclusive(const ScanCtx& ctx, uint3
   uint32_t iters = 0;
   timed_out = false;
   while (true) {
-    const int64_t t = base - lane;
-    uint32_t flag = kFlagPrefix, value = 0;
-    if (t >= 0) {
-      const uint64_t w = ld_relaxed_u64(ctx.status + t);
-      if (static_cast<uint32_t>(w >> 34) == ctx.epoch) {
-        flag = static_cast<uint32_t>(w >> 32) & 3u;
-        value = static_cast<uint32_t>(w);
-      } else {
-        flag = kFlagNone;
+    uint64_t word[kLookbackPerLane];
+#pragma unroll
+    for (int j = 0; j < kLookbackPerLane; ++j) {  // all loads in flight together
+      const int64_t t = base - (lane * kLookbackPerLane + j);
+      word[j] = t >= 0 ? ld_relaxed_u64(ctx.status + t)
+                       : pack_status(ctx.epoch, kFlagPrefix, 0);  // before tile 0: prefix 0
+    }
+    uint32_t flag[kLookbackPerLane], value[kLookbackPerLane];
+#pragma unroll
+    for (int j = 0; j < kLookbackPerLane; ++j) {
+      const bool current = static_cast<uint32_t>(word[j] >> 34) == ctx.epoch;
+      flag[j] = current ? (static_cast<uint32_t>(word[j] >> 32) & 3u) : kFlagNone;
+      value[j] = current ? static_cast<uint32_t>(word[j]) : 0u;
+    }
+    int jp = kLookbackPerLane;  // nearest prefix position within this lane
+#pragma unroll
+    for (int j = kLookbackPerLane - 1; j >= 0; --j)
+      if (flag[j] == kFlagPrefix) jp = j;
+    const uint32_t prefix_lanes = __ballot_sync(0xffffffffu, jp < kLookbackPerLane);
+    const int lp = prefix_lanes ? __ffs(prefix_lanes) - 1 : 32;  // lane of the nearest prefix
+    const int upto = lane < lp ? kLookbackPerLane - 1 : (lane == lp ? jp : -1);
+    bool ready = true;
+    uint32_t sum = 0, ready_sum = 0;
+#pragma unroll
+    for (int j = 0; j < kLookbackPerLane; ++j) {
+      if (j <= upto) {
+        ready = ready && flag[j] != kFlagNone;
+        sum += value[j];
+        if (flag[j] != kFlagNone) ready_sum += value[j];
       }
     }
-    const uint32_t prefix_mask = __ballot_sync(0xffffffffu, flag == kFlagPrefix);
-    const uint32_t ready_mask = __ballot_sync(0xffffffffu, flag != kFlagNone);
-    // lanes 0 .. (nearest prefix lane); all 32 lanes if there is none
-    const uint32_t need =
-        prefix_mask ? (((prefix_mask & (0u - prefix_mask)) << 1) - 1u) : 0xffffffffu;
-    if ((ready_mask & need) != need) {
-      uint64_t now = __shfl_sync(0xffffffffu, global_timer_ns(), 0);
+    if (!__all_sync(0xffffffffu, ready)) {
+      const uint64_t now = __shfl_sync(0xffffffffu, global_timer_ns(), 0);
       if (iters == 0) t_start = now;
       ++iters;
       if (iters > (1u << 26) || now - t_start > ctx.wait_limit_ns) {
         timed_out = true;
-        const uint32_t part = ((ready_mask & need) >> lane) & 1u ? value : 0u;
-        return excl + warp_sum(part);
+        return excl + warp_sum(ready_sum);
       }
-      __nanosleep(64);
+      __nanosleep(32);
       continue;
     }
-    excl += warp_sum(((need >> lane) & 1u) ? value : 0u);
-    if (prefix_mask) return excl;
-    base -= 32;
+    excl += warp_sum(sum);
+    if (prefix_lanes) return excl;
+    base -= kLookbackWindow;
   }
 }
 

@@ -11,6 +11,7 @@
 #include "compact.cuh"
 #include "gradient.cuh"
 #include "internal.h"
+#include "stream_compact.cuh"
 
 namespace efs {
 namespace {
@@ -24,14 +25,7 @@ __global__ void __launch_bounds__(kThreads)
     ht_kernel(const GT* __restrict__ g, float* __restrict__ e, float gamma, float lambda,
               uint32_t d, uint32_t* __restrict__ idx_out, float* __restrict__ val_out,
               uint32_t* __restrict__ count_out, ScanCtx ctx) {
-  __shared__ uint32_t s_tile;
-  if (threadIdx.x == 0) s_tile = take_tile(ctx);
-  __syncthreads();
-  const uint32_t tile = s_tile;
-  if (tile >= ctx.num_tiles) {  // stale dispenser: never touch memory with it
-    if (threadIdx.x == 0) atomicOr(ctx.error, kDevErrTimeout);
-    return;
-  }
+  const uint32_t tile = blockIdx.x;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const uint64_t first = element_index(tile, warp, 0, lane, 0);
 
@@ -80,12 +74,103 @@ __global__ void __launch_bounds__(kThreads)
   compact_tile(ctx, tile, sel, a, idx_out, val_out, count_out, d);
 }
 
+// The hard-threshold step as a streaming-compaction op: a stage holds a
+// tile of g followed by the same tile of e; the residual is written to e from
+// registers with streaming stores.
+template <typename GT>
+struct HtOp {
+  const GT* g;
+  float* e;
+  float gamma, lambda;
+  uint32_t d;
+  static constexpr uint32_t kGBytes = kTileElems * sizeof(GT);
+  static constexpr uint32_t kStageBytes = kGBytes + kTileElems * sizeof(float);
+
+  __device__ __forceinline__ void fill(unsigned char* stage, uint32_t t, uint64_t* bar,
+                                       uint64_t policy) const {
+    tma_load_1d(stage, g + static_cast<size_t>(t) * kTileElems, kGBytes, bar, policy);
+    tma_load_1d(stage + kGBytes, e + static_cast<size_t>(t) * kTileElems,
+                kTileElems * sizeof(float), bar, policy);
+  }
+
+  __device__ __forceinline__ void tile_smem(const unsigned char* stage, uint32_t t, int warp,
+                                            int lane, float (&a)[kUnits][4],
+                                            uint32_t (&sel)[kUnits]) const {
+    const GT* gs = reinterpret_cast<const GT*>(stage);
+    const float* es = reinterpret_cast<const float*>(stage + kGBytes);
+    const int local = warp * kWarpElems + lane * 4;
+    float* eg = e + element_index(t, warp, 0, lane, 0);
+#pragma unroll
+    for (int v = 0; v < kUnits; ++v) {
+      GradVec<GT> gv;
+      if constexpr (sizeof(GT) == 4)
+        gv.v = *reinterpret_cast<const float4*>(gs + local + v * 128);
+      else
+        gv.v = *reinterpret_cast<const uint2*>(gs + local + v * 128);
+      const float4 ev = *reinterpret_cast<const float4*>(es + local + v * 128);
+      a[v][0] = __fmaf_rn(gamma, gv[0], ev.x);
+      a[v][1] = __fmaf_rn(gamma, gv[1], ev.y);
+      a[v][2] = __fmaf_rn(gamma, gv[2], ev.z);
+      a[v][3] = __fmaf_rn(gamma, gv[3], ev.w);
+      sel[v] = in_support(a[v][0], lambda) | (in_support(a[v][1], lambda) << 1) |
+               (in_support(a[v][2], lambda) << 2) | (in_support(a[v][3], lambda) << 3);
+      st_stream_f4(eg + v * 128,
+                   make_float4((sel[v] & 1u) ? 0.0f : a[v][0], (sel[v] & 2u) ? 0.0f : a[v][1],
+                               (sel[v] & 4u) ? 0.0f : a[v][2], (sel[v] & 8u) ? 0.0f : a[v][3]));
+    }
+  }
+
+  __device__ __forceinline__ void tile_global(uint32_t t, int warp, int lane,
+                                              float (&a)[kUnits][4],
+                                              uint32_t (&sel)[kUnits]) const {
+    const uint64_t first = element_index(t, warp, 0, lane, 0);
+#pragma unroll
+    for (int v = 0; v < kUnits; ++v) {
+      sel[v] = 0;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint64_t i = first + v * 128 + j;
+        a[v][j] = 0.0f;
+        if (i < d) {
+          const float x = __fmaf_rn(gamma, grad_scalar(g, i), e[i]);
+          const uint32_t sj = in_support(x, lambda);
+          a[v][j] = x;
+          sel[v] |= sj << j;
+          e[i] = sj ? 0.0f : x;
+        }
+      }
+    }
+  }
+};
+
+constexpr int kHtStages = 4;
+
+template <typename GT>
+using HtStreamKernel = StreamLayout<HtOp<GT>, kHtStages>;
+
 template <typename GT>
 cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint32_t d,
-                         uint32_t* idx_out, float* val_out, uint32_t* count_out, Workspace& ws) {
+                         uint32_t* idx_out, float* val_out, uint32_t* count_out, Workspace& ws,
+                         const DeviceInfo& dev) {
   const uint32_t tiles = tiles_for(d);
   const ScanCtx ctx = next_scan_ctx(ws, tiles);
   const uintptr_t ga = reinterpret_cast<uintptr_t>(g), ea = reinterpret_cast<uintptr_t>(e);
+  const int per_sm = sizeof(GT) == 4 ? dev.ht_stream_per_sm_f32 : dev.ht_stream_per_sm_bf16;
+  if (ga % 16 == 0 && ea % 16 == 0 && per_sm > 0) {
+    // TMA-fed streaming compaction: one cooperative launch over all SMs
+    HtOp<GT> op{g, e, gamma, lambda, d};
+    uint32_t slots = static_cast<uint32_t>(per_sm * dev.sm_count);
+    if (slots > kMaxStreamGrid) slots = kMaxStreamGrid;
+    const uint32_t grid = tiles < slots ? tiles : slots;
+    uint32_t cap = d;
+    ScanCtx c = ctx;
+    void* params[] = {&op, &d, &idx_out, &val_out, &count_out, &cap, &c};
+    const cudaError_t err = cudaLaunchCooperativeKernel(
+        reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages>), dim3(grid),
+        dim3(kStreamThreads), params, HtStreamKernel<GT>::kSmem, ws.stream);
+    count_launch();
+    return err;
+  }
   const bool vec = (ga % (4 * sizeof(GT)) == 0) && (ea % 16 == 0);
   if (vec) {
     ht_kernel<GT, true><<<tiles, kThreads, 0, ws.stream>>>(g, e, gamma, lambda, d, idx_out,
@@ -98,16 +183,34 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
   return cudaGetLastError();
 }
 
+template <typename GT>
+int stream_blocks_per_sm() {
+  const void* fn = reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages>);
+  int n = 0;
+  if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           HtStreamKernel<GT>::kSmem) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, kStreamThreads,
+                                                    HtStreamKernel<GT>::kSmem) != cudaSuccess)
+    n = 0;
+  cudaGetLastError();
+  return n;
+}
+
 }  // namespace
+
+void ht_init_device(DeviceInfo& info) {
+  info.ht_stream_per_sm_f32 = stream_blocks_per_sm<float>();
+  info.ht_stream_per_sm_bf16 = stream_blocks_per_sm<uint16_t>();
+}
 
 cudaError_t launch_hard_threshold(const void* g, bool g_bf16, float* e, float gamma,
                                   float lambda, uint32_t d, uint32_t* idx_out, float* val_out,
-                                  uint32_t* count_out, Workspace& ws) {
+                                  uint32_t* count_out, Workspace& ws, const DeviceInfo& dev) {
   if (g_bf16)
     return launch_typed(static_cast<const uint16_t*>(g), e, gamma, lambda, d, idx_out, val_out,
-                        count_out, ws);
+                        count_out, ws, dev);
   return launch_typed(static_cast<const float*>(g), e, gamma, lambda, d, idx_out, val_out,
-                      count_out, ws);
+                      count_out, ws, dev);
 }
 
 }  // namespace efs

@@ -12,7 +12,6 @@ namespace efs {
 
 // Layout of the workspace header (bytes from the workspace base).
 constexpr size_t kOffBarGen = 0;        // uint32: grid-barrier generation (never reset)
-constexpr size_t kOffTileCounter = 4;   // uint32: tile-id dispenser (0 between launches)
 constexpr size_t kOffError = 8;         // uint32: latched device error bits
 constexpr size_t kOffTopkReset = 16;    // start of the region cleared at each Top-k call
 constexpr size_t kOffBarArrive = 16;    // uint32
@@ -48,8 +47,14 @@ struct Workspace {
 // Per-device facts queried once.
 struct DeviceInfo {
   int sm_count = 0;
-  int refine_blocks = 0;   // co-resident CTAs for the cooperative Top-k refine
+  int refine_blocks = 0;          // co-resident CTAs for the cooperative Top-k refine
+  int ht_stream_per_sm_f32 = 0;   // streaming hard-threshold CTAs per SM (0: unavailable)
+  int ht_stream_per_sm_bf16 = 0;
 };
+
+// Per-device set-up of the streaming hard-threshold kernels (opts them into
+// their shared-memory ring on the current device and records occupancy).
+void ht_init_device(DeviceInfo& info);
 
 // Launch bookkeeping.
 void count_launch();
@@ -60,7 +65,7 @@ ScanCtx next_scan_ctx(Workspace& ws, uint32_t num_tiles);
 // ---- launchers (return the launch's cudaError_t) ----
 cudaError_t launch_hard_threshold(const void* g, bool g_bf16, float* e, float gamma,
                                   float lambda, uint32_t d, uint32_t* idx_out, float* val_out,
-                                  uint32_t* count_out, Workspace& ws);
+                                  uint32_t* count_out, Workspace& ws, const DeviceInfo& dev);
 cudaError_t launch_topk(const void* g, bool g_bf16, float* e, float gamma, uint32_t k,
                         uint32_t d, uint32_t* idx_out, float* val_out, uint32_t* count_out,
                         Workspace& ws, const DeviceInfo& dev);

@@ -342,14 +342,7 @@ __global__ void __launch_bounds__(kThreads)
     topk_select_kernel(float* __restrict__ e, uint32_t d, const uint64_t* __restrict__ threshold,
                        uint32_t k, uint32_t* __restrict__ idx_out, float* __restrict__ val_out,
                        uint32_t* __restrict__ count_out, ScanCtx ctx) {
-  __shared__ uint32_t s_tile;
-  if (threadIdx.x == 0) s_tile = take_tile(ctx);
-  __syncthreads();
-  const uint32_t tile = s_tile;
-  if (tile >= ctx.num_tiles) {  // stale dispenser: never touch memory with it
-    if (threadIdx.x == 0) atomicOr(ctx.error, kDevErrTimeout);
-    return;
-  }
+  const uint32_t tile = blockIdx.x;
   const uint64_t thr = __ldcg(threshold);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const uint64_t first = element_index(tile, warp, 0, lane, 0);
