@@ -52,7 +52,7 @@ ef_status device_info(int dev, DeviceInfo* out) {
 // synchronises the stream once; the new header and tile-status array start
 // at zero.
 ef_status acquire_workspace(cudaStream_t stream, uint32_t tiles, uint32_t cand_cap,
-                            size_t offsets, Workspace** out) {
+                            size_t offsets, size_t stage, Workspace** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
   std::lock_guard<std::mutex> lk(g_mu);
@@ -63,13 +63,13 @@ ef_status acquire_workspace(cudaStream_t stream, uint32_t tiles, uint32_t cand_c
     ws->stream = stream;
   }
   if (!ws->base || tiles > ws->status_tiles || cand_cap > ws->cand_cap ||
-      offsets > ws->offsets_cap) {
-    const uint32_t new_tiles = tiles > ws->status_tiles ? tiles : ws->status_tiles;
-    const uint32_t new_cand = cand_cap > ws->cand_cap ? cand_cap : ws->cand_cap;
-    const size_t new_off = offsets > ws->offsets_cap ? offsets : ws->offsets_cap;
-    const size_t bytes = kHeaderBytes + sizeof(uint64_t) * (static_cast<size_t>(new_tiles) +
-                                                            2 * static_cast<size_t>(new_cand)) +
-                         sizeof(uint32_t) * new_off + 256;
+      offsets > ws->offsets_cap || stage > ws->stage_cap) {
+    Workspace grown = *ws;
+    if (tiles > grown.status_tiles) grown.status_tiles = tiles;
+    if (cand_cap > grown.cand_cap) grown.cand_cap = cand_cap;
+    if (offsets > grown.offsets_cap) grown.offsets_cap = offsets;
+    if (stage > grown.stage_cap) grown.stage_cap = stage;
+    const size_t bytes = grown.total_bytes();
     if (ws->base) {
       if (cudaStreamSynchronize(stream) != cudaSuccess) return EF_ERR_CUDA;
       cudaFree(ws->base);
@@ -79,19 +79,20 @@ ef_status acquire_workspace(cudaStream_t stream, uint32_t tiles, uint32_t cand_c
     if (cudaMalloc(&p, bytes) != cudaSuccess) {
       cudaGetLastError();
       ws->status_tiles = ws->cand_cap = 0;
-      ws->offsets_cap = 0;
+      ws->offsets_cap = ws->stage_cap = 0;
       return EF_ERR_NO_MEMORY;
     }
-    ws->base = static_cast<char*>(p);
-    ws->bytes = bytes;
-    ws->status_tiles = new_tiles;
-    ws->cand_cap = new_cand;
-    ws->offsets_cap = new_off;
-    ws->dirty = true;
+    grown.base = static_cast<char*>(p);
+    grown.bytes = bytes;
+    grown.dirty = true;
+    *ws = grown;
   }
   if (ws->dirty) {
+    // everything tagged with an epoch restarts from zero with the epochs
     const size_t clear = kHeaderBytes + sizeof(uint64_t) * ws->status_tiles;
-    if (cudaMemsetAsync(ws->base, 0, clear, stream) != cudaSuccess) return EF_ERR_CUDA;
+    if (cudaMemsetAsync(ws->base, 0, clear, stream) != cudaSuccess ||
+        cudaMemsetAsync(ws->chunks(), 0, sizeof(uint64_t) * kMaxChunks, stream) != cudaSuccess)
+      return EF_ERR_CUDA;
     ws->epoch = 0;
     ws->dirty = false;
   }
@@ -137,7 +138,8 @@ ef_status hard_threshold_entry(const void* g, bool bf16, float* e, float gamma, 
   ef_status st = device_info(dev, &info);
   if (st != EF_OK) return st;
   Workspace* ws = nullptr;
-  st = acquire_workspace(stream, tiles_for(d), 0, 0, &ws);
+  st = acquire_workspace(stream, tiles_for(d), 0, 0,
+                         static_cast<size_t>(tiles_for(d)) * kTileElems, &ws);
   if (st != EF_OK) return st;
   return finish_launch(launch_hard_threshold(g, bf16, e, gamma, lambda, static_cast<uint32_t>(d),
                                              idx_out, val_out, count_out, *ws, info),
@@ -171,7 +173,7 @@ ef_status topk_entry(const void* g, bool bf16, float* e, float gamma, uint64_t k
   ef_status st = device_info(dev, &info);
   if (st != EF_OK) return st;
   Workspace* ws = nullptr;
-  st = acquire_workspace(stream, tiles_for(d), topk_candidate_capacity(d), 0, &ws);
+  st = acquire_workspace(stream, tiles_for(d), topk_candidate_capacity(d), 0, 0, &ws);
   if (st != EF_OK) return st;
   return finish_launch(launch_topk(g, bf16, e, gamma, static_cast<uint32_t>(k),
                                    static_cast<uint32_t>(d), idx_out, val_out, count_out, *ws,
@@ -188,6 +190,7 @@ int64_t withheld_tile() { return g_withheld_tile.load(); }
 ScanCtx next_scan_ctx(Workspace& ws, uint32_t num_tiles) {
   if (ws.epoch >= (1u << 30) - 1) {  // epoch wrap: old words must not match again
     cudaMemsetAsync(ws.status(), 0, sizeof(uint64_t) * ws.status_tiles, ws.stream);
+    cudaMemsetAsync(ws.chunks(), 0, sizeof(uint64_t) * kMaxChunks, ws.stream);
     ws.epoch = 0;
   }
   ++ws.epoch;
@@ -249,7 +252,7 @@ ef_status sparse_aggregate(uint32_t n, const uint32_t* const* idx, const float* 
   const uint32_t tiles = efs::agg_tiles_for(d);
   Workspace* ws = nullptr;
   const ef_status st = efs::acquire_workspace(
-      s, 0, 0, static_cast<size_t>(n) * (static_cast<size_t>(tiles) + 1), &ws);
+      s, 0, 0, static_cast<size_t>(n) * (static_cast<size_t>(tiles) + 1), 0, &ws);
   if (st != EF_OK) return st;
   return efs::finish_launch(
       efs::launch_aggregate(n, idx, val, counts, static_cast<uint32_t>(d), dense_out, *ws), ws);
@@ -276,7 +279,13 @@ ef_status ef_check_status(ef_stream_t stream) {
   if (cudaMemsetAsync(dev_err, 0, sizeof bits, s) != cudaSuccess ||
       cudaStreamSynchronize(s) != cudaSuccess)
     return EF_ERR_CUDA;
-  if (bits & efs::kDevErrTimeout) return EF_ERR_TIMEOUT;
+  if (bits & efs::kDevErrTimeout) {
+    // a wait that ran out may leave barrier counters mid-way: re-clear the
+    // workspace header before the next launch on this stream
+    std::lock_guard<std::mutex> lk(efs::g_mu);
+    ws->dirty = true;
+    return EF_ERR_TIMEOUT;
+  }
   return EF_ERR_BAD_INPUT;
 }
 

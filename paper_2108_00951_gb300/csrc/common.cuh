@@ -186,4 +186,37 @@ __device__ __forceinline__ uint32_t lookback_exclusive(const ScanCtx& ctx, uint3
   }
 }
 
+// Bounded grid-wide barrier for a cooperative launch (all CTAs co-resident).
+// Returns false, latching kDevErrTimeout, if the wait ran out.
+__device__ __forceinline__ bool grid_barrier(uint32_t* arrive, uint32_t* gen, uint64_t limit_ns,
+                             uint32_t* error) {
+  __shared__ int s_ok;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int ok = 1;
+    const uint32_t my_gen = ld_acquire_u32(gen);
+    __threadfence();  // this CTA's global writes before arriving
+    const uint32_t ticket = atomicAdd(arrive, 1u);
+    if (ticket == gridDim.x - 1) {
+      atomicExch(arrive, 0u);
+      __threadfence();
+      st_release_u32(gen, my_gen + 1);
+    } else {
+      const uint64_t t0 = global_timer_ns();
+      uint32_t iters = 0;
+      while (ld_acquire_u32(gen) == my_gen) {
+        if (++iters > (1u << 26) || global_timer_ns() - t0 > limit_ns) {
+          atomicOr(error, kDevErrTimeout);
+          ok = 0;
+          break;
+        }
+        __nanosleep(128);
+      }
+    }
+    s_ok = ok;
+  }
+  __syncthreads();
+  return s_ok != 0;
+}
+
 }  // namespace efs

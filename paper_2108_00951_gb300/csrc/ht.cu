@@ -94,14 +94,14 @@ struct HtOp {
   }
 
   __device__ __forceinline__ void tile_smem(const unsigned char* stage, uint32_t t, int warp,
-                                            int lane, float (&a)[kUnits][4],
-                                            uint32_t (&sel)[kUnits]) const {
+                                            int lane, float (&a)[kSUnits][4],
+                                            uint32_t (&sel)[kSUnits]) const {
     const GT* gs = reinterpret_cast<const GT*>(stage);
     const float* es = reinterpret_cast<const float*>(stage + kGBytes);
-    const int local = warp * kWarpElems + lane * 4;
-    float* eg = e + element_index(t, warp, 0, lane, 0);
+    const int local = warp * kSWarpElems + lane * 4;
+    float* eg = e + stream_element_index(t, warp, 0, lane, 0);
 #pragma unroll
-    for (int v = 0; v < kUnits; ++v) {
+    for (int v = 0; v < kSUnits; ++v) {
       GradVec<GT> gv;
       if constexpr (sizeof(GT) == 4)
         gv.v = *reinterpret_cast<const float4*>(gs + local + v * 128);
@@ -121,11 +121,11 @@ struct HtOp {
   }
 
   __device__ __forceinline__ void tile_global(uint32_t t, int warp, int lane,
-                                              float (&a)[kUnits][4],
-                                              uint32_t (&sel)[kUnits]) const {
-    const uint64_t first = element_index(t, warp, 0, lane, 0);
+                                              float (&a)[kSUnits][4],
+                                              uint32_t (&sel)[kSUnits]) const {
+    const uint64_t first = stream_element_index(t, warp, 0, lane, 0);
 #pragma unroll
-    for (int v = 0; v < kUnits; ++v) {
+    for (int v = 0; v < kSUnits; ++v) {
       sel[v] = 0;
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
@@ -160,11 +160,12 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
     // TMA-fed streaming compaction: one cooperative launch over all SMs
     HtOp<GT> op{g, e, gamma, lambda, d};
     uint32_t slots = static_cast<uint32_t>(per_sm * dev.sm_count);
-    if (slots > kMaxStreamGrid) slots = kMaxStreamGrid;
+    if (slots > kMaxChunks) slots = kMaxChunks;
     const uint32_t grid = tiles < slots ? tiles : slots;
     uint32_t cap = d;
     ScanCtx c = ctx;
-    void* params[] = {&op, &d, &idx_out, &val_out, &count_out, &cap, &c};
+    StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks()};
+    void* params[] = {&op, &d, &idx_out, &val_out, &count_out, &cap, &c, &sa};
     const cudaError_t err = cudaLaunchCooperativeKernel(
         reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages>), dim3(grid),
         dim3(kStreamThreads), params, HtStreamKernel<GT>::kSmem, ws.stream);

@@ -22,24 +22,44 @@ constexpr int kHistLevels = 6;
 constexpr int kHistBins = 2048;
 constexpr size_t kHeaderBytes = kOffHist + sizeof(uint32_t) * kHistLevels * kHistBins;
 constexpr size_t kTopkResetBytes = kHeaderBytes - kOffTopkReset;
+constexpr uint32_t kMaxChunks = 1024;   // per-CTA chunk sums of the streaming compaction
+constexpr uint32_t kCountsPerTile = 16; // per-segment counts of the streaming compaction
 
 struct Workspace {
   int device = -1;
   cudaStream_t stream = nullptr;
   char* base = nullptr;
   size_t bytes = 0;
-  uint32_t status_tiles = 0;   // capacity of the tile-status array
+  uint32_t status_tiles = 0;   // capacity of the per-tile arrays (status, counts)
   uint32_t cand_cap = 0;       // capacity of each Top-k candidate buffer
   size_t offsets_cap = 0;      // capacity of the aggregation offsets (uint32)
+  size_t stage_cap = 0;        // capacity of the pair staging buffers (pairs)
   uint32_t epoch = 0;          // last epoch handed to a compaction launch
-  bool dirty = false;          // a launch failed: header must be re-cleared
+  bool dirty = false;          // header must be re-cleared (failed launch or device timeout)
 
-  uint64_t* status() const { return reinterpret_cast<uint64_t*>(base + kHeaderBytes); }
-  uint64_t* cand(int i) const {
-    return reinterpret_cast<uint64_t*>(base + kHeaderBytes + sizeof(uint64_t) * status_tiles) +
-           static_cast<size_t>(i) * cand_cap;
+  // Regions after the header, each 256-byte aligned.
+  static size_t align(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+  size_t off_status() const { return kHeaderBytes; }
+  size_t off_cand() const { return align(off_status() + sizeof(uint64_t) * status_tiles); }
+  size_t off_offsets() const { return align(off_cand() + 2 * sizeof(uint64_t) * cand_cap); }
+  size_t off_counts() const { return align(off_offsets() + sizeof(uint32_t) * offsets_cap); }
+  size_t off_chunks() const {
+    return align(off_counts() + sizeof(uint32_t) * kCountsPerTile * status_tiles);
   }
-  uint32_t* offsets() const { return reinterpret_cast<uint32_t*>(cand(2)); }
+  size_t off_stage() const { return align(off_chunks() + sizeof(uint64_t) * kMaxChunks); }
+  size_t total_bytes() const { return align(off_stage() + 8 * stage_cap); }
+
+  uint64_t* status() const { return reinterpret_cast<uint64_t*>(base + off_status()); }
+  uint64_t* cand(int i) const {
+    return reinterpret_cast<uint64_t*>(base + off_cand()) + static_cast<size_t>(i) * cand_cap;
+  }
+  uint32_t* offsets() const { return reinterpret_cast<uint32_t*>(base + off_offsets()); }
+  uint32_t* counts() const { return reinterpret_cast<uint32_t*>(base + off_counts()); }
+  uint64_t* chunks() const { return reinterpret_cast<uint64_t*>(base + off_chunks()); }
+  uint32_t* stage_idx() const { return reinterpret_cast<uint32_t*>(base + off_stage()); }
+  float* stage_val() const {
+    return reinterpret_cast<float*>(base + off_stage() + sizeof(uint32_t) * stage_cap);
+  }
   uint32_t* u32(size_t off) const { return reinterpret_cast<uint32_t*>(base + off); }
   uint64_t* u64(size_t off) const { return reinterpret_cast<uint64_t*>(base + off); }
 };

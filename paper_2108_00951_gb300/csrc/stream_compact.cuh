@@ -1,43 +1,51 @@
-// stream_compact.cuh — single-pass ordered stream compaction at memory speed:
-// persistent co-resident CTAs, TMA-fed tiles, and a chained per-CTA scan.
+// stream_compact.cuh — ordered stream compaction at memory speed: one
+// cooperative launch of persistent CTAs, TMA-fed tiles, warp-independent
+// streaming of contiguous chunks, then pair placement.
 //
-// Why not a plain decoupled look-back with one tile per CTA: every CTA would
-// hold its tile in registers while its look-back waits on L2 round trips that,
-// under a saturated memory system, take microseconds; throughput is then
-// resident-bytes / CTA lifetime, about a third of HBM bandwidth on this GPU.
+// Why not a decoupled look-back, one tile per CTA: each CTA holds its tile
+// while its look-back waits on L2 round trips that, under a saturated memory
+// system, take microseconds; throughput is then resident-bytes / CTA
+// lifetime, about a third of HBM bandwidth on this GPU. Resolving offsets
+// inside the streaming loop of persistent CTAs instead couples every CTA to
+// the slowest one, and even one CTA-wide barrier per tile puts each tile's
+// latency chain on the refill path. So while streaming, nothing waits for
+// anything but its own data.
 //
-// Design (one cooperative launch, grid G = all co-resident CTAs):
-//  * Tiles of kTileElems coordinates are assigned round-robin: CTA c owns
-//    tiles c, c + G, c + 2G, ...
-//  * 8 compute warps stream the CTA's tiles through a kStages-deep ring of
-//    shared-memory stages filled by bulk copies (cp.async.bulk + mbarrier).
-//    Per tile they compute the selection, publish the tile's count, and stage
-//    the selected (index, value) pairs, in order, in a shared-memory pair ring.
-//  * One scan warp per CTA turns the staged tiles into output: the first
-//    selected coordinate of tile t lands at
-//        offset(t) = incl(t - G) + sum_{t - G < u < t} count(u),
-//    where incl(t - G) is this same CTA's previous tile's inclusive count (its
-//    own running total) and the counts in between are the other CTAs'
-//    published tile counts; for the CTA's first tile it is the sum of all
-//    counts before it. It never needs another CTA's inclusive prefix, so no
-//    prefix has to propagate across CTAs and the compute warps never wait on
-//    L2 round trips. It then copies the staged pairs to their final positions
-//    with coalesced stores.
-//  * Counts are published in the tile-status array tagged with the launch's
-//    epoch. Every wait (stage arrival, ring space, a missing count) is bounded
-//    and latches kDevErrTimeout; after a timeout both roles leave their loops,
-//    the copies still in flight get a bounded wait, and the kernel returns.
+// Phase 1 (streaming). CTA c owns the contiguous chunk of tiles
+// [c*T/G, (c+1)*T/G) of kTileElems coordinates each. A producer warp fills a
+// kStages-deep ring of shared-memory stages with bulk copies (cp.async.bulk,
+// completing on the stage's "full" mbarrier) and refills a stage once all 16
+// compute warps have released it (its "empty" mbarrier). Compute warp w owns
+// the segment [w*256, (w+1)*256) of every tile: it computes the selection and
+// its side effects (the residual store), compacts its selected (index, value)
+// pairs with ballots into the segment's own staging slot, records the
+// segment's count, and releases the stage. No CTA-wide barrier.
 //
-// An Op supplies the per-tile work:
+// Phase 2 (placement). Segments are ordered (tile, warp), which is coordinate
+// order. Each CTA publishes its chunk's total (tagged with the launch's epoch)
+// and sums the totals of all earlier chunks in one batched load, waiting
+// (bounded) for any not yet published; all CTAs finish phase 1 at about the
+// same time, so this is about one L2 round trip and no grid-wide barrier is
+// needed. It then scans its segments' counts in shared memory, and each warp
+// copies whole segments from staging to their final, ascending positions.
+//
+// Traffic beyond the step itself: 16 bytes per selected pair (staging write
+// and read) plus 4 bytes per segment. Every wait (stage arrival, stage
+// release, an earlier chunk's total) is bounded and latches kDevErrTimeout;
+// after a timeout the CTA places no pair.
+//
+// An Op supplies the per-segment work:
 //   static constexpr uint32_t kStageBytes;            bytes of one stage
 //   void fill(unsigned char* stage, uint32_t tile, uint64_t* bar, uint64_t pol)
-//        issue the bulk copies of a full tile (thread 0; after expect_tx)
+//        issue the bulk copies of a full tile (after expect_tx)
 //   void tile_smem(const unsigned char* stage, uint32_t tile, int warp, int lane,
-//                  float (&a)[kUnits][4], uint32_t (&sel)[kUnits])
+//                  float (&a)[kSUnits][4], uint32_t (&sel)[kSUnits])
 //   void tile_global(uint32_t tile, int warp, int lane, float (&a)[..], uint32_t (&sel)[..])
-//        compute values and selection bits (and side effects such as the
-//        residual store) for a full tile from its stage, or for the partial
-//        last tile from global memory.
+//        compute values and selection bits (and side effects) of the calling
+//        warp's segment, from the stage of a full tile, or from global memory
+//        for the partial last tile.
+// Element layout: unit v of lane l of warp w covers the 4 coordinates from
+// tile * kTileElems + w * 256 + v * 128 + l * 4 (see stream_element_index).
 #pragma once
 
 #include "compact.cuh"
@@ -45,260 +53,277 @@
 
 namespace efs {
 
-constexpr int kComputeThreads = kThreads;              // 8 compute warps
-constexpr int kStreamThreads = kComputeThreads + 32;   // + 1 scan warp
-constexpr uint32_t kPairRing = kTileElems;             // staged pairs (>= 1 full tile)
-constexpr uint32_t kEntryRing = 32;                    // staged tiles
-constexpr int kScanBatch = 4;                          // rounds resolved per batch
-constexpr int kScanWordsPerLane = 10;                  // counts per round per lane
-// The scan warp reads at most 32 * kScanWordsPerLane counts per round, i.e.
-// the G - 1 tiles between two of its own: launchers must keep G <= this.
-constexpr uint32_t kMaxStreamGrid = 32u * kScanWordsPerLane + 1u;
+constexpr int kSWarps = 16;                          // compute warps (segments per tile)
+constexpr int kSUnits = 2;                           // 4-coordinate units per lane per segment
+constexpr int kSWarpElems = 32 * 4 * kSUnits;        // 256 coordinates per segment
+static_assert(kSWarps * kSWarpElems == kTileElems, "tile geometry");
+constexpr int kComputeThreads = 32 * kSWarps;        // 512
+constexpr int kStreamThreads = kComputeThreads + 32; // + 1 producer warp
+constexpr int kProducerWarp = kSWarps;
+
+__device__ __forceinline__ uint64_t stream_element_index(uint32_t tile, int warp, int v, int lane,
+                                                        int j) {
+  return static_cast<uint64_t>(tile) * kTileElems + warp * kSWarpElems + v * 128 + lane * 4 + j;
+}
+
+// Workspace pieces of a launch.
+struct StreamArgs {
+  uint32_t* stage_idx;   // [num_tiles * kTileElems] staged indices, segment-slotted
+  float* stage_val;      // [num_tiles * kTileElems] staged values
+  uint32_t* counts;      // [num_tiles * kSWarps] selected per segment
+  uint64_t* chunk_sums;  // [gridDim.x] (epoch << 32) | chunk total
+};
 
 template <class Op, int kStages>
 struct StreamLayout {
-  static constexpr uint32_t kRingOff = kStages * Op::kStageBytes;
-  static constexpr uint32_t kSmem = kRingOff + kPairRing * 8;
+  static constexpr uint32_t kSmem = kStages * Op::kStageBytes;
+  // phase 2 reuses the ring for the chunk's segment counts
+  static constexpr uint32_t kChunkSegs = kSmem / sizeof(uint32_t);
 };
 
 template <class Op, int kStages>
 __global__ void __launch_bounds__(kStreamThreads, 1)
     stream_compact_kernel(Op op, uint32_t d, uint32_t* __restrict__ idx_out,
                           float* __restrict__ val_out, uint32_t* __restrict__ count_out,
-                          uint32_t cap, ScanCtx ctx) {
+                          uint32_t cap, ScanCtx ctx, StreamArgs sa) {
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ __align__(8) uint64_t s_full[kStages];
-  __shared__ uint32_t s_warp_total[kWarps];
-  __shared__ uint32_t s_ring_start;
-  __shared__ uint32_t s_entry_count[kEntryRing];
-  __shared__ uint32_t s_entry_start[kEntryRing];
-  __shared__ volatile uint32_t s_produced;  // tiles staged by the compute warps
-  __shared__ volatile uint32_t s_consumed;  // tiles written out by the scan warp
-  __shared__ volatile uint32_t s_tail;      // pair-ring slots released
-  __shared__ volatile int s_abort;
+  __shared__ __align__(8) uint64_t s_empty[kStages];
+  __shared__ uint32_t s_scratch[kStreamThreads / 32];
   using L = StreamLayout<Op, kStages>;
-  uint32_t* ring_idx = reinterpret_cast<uint32_t*>(smem + L::kRingOff);
-  float* ring_val = reinterpret_cast<float*>(smem + L::kRingOff + kPairRing * 4);
 
   const uint32_t T = ctx.num_tiles, G = gridDim.x, c = blockIdx.x;
-  const uint32_t rounds = c < T ? (T - c + G - 1) / G : 0;
+  const uint32_t t_lo = static_cast<uint32_t>(static_cast<uint64_t>(c) * T / G);
+  const uint32_t t_hi = static_cast<uint32_t>(static_cast<uint64_t>(c + 1) * T / G);
+  const uint32_t rounds = t_hi - t_lo;
   const uint32_t full_tiles = d / kTileElems;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) mbar_init(&s_full[s], 1);
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&s_full[s], 1);
+      mbar_init(&s_empty[s], kSWarps);
+    }
     mbar_init_fence();
-    s_produced = 0;
-    s_consumed = 0;
-    s_tail = 0;
-    s_abort = 0;
   }
   __syncthreads();
 
-  if (threadIdx.x < kComputeThreads) {
-    // ------------------------------------------------------ compute warps
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const uint32_t lt = lanemask_lt();
-    uint64_t policy = 0;
-    uint32_t issued = 0;  // thread 0: rounds whose stage fill was issued
-    uint32_t head = 0;    // thread 0: pair-ring slots reserved
-    auto fill = [&](uint32_t r) {
-      const int s = static_cast<int>(r % kStages);
-      const uint32_t t = c + r * G;
-      if (t < full_tiles) {
-        mbar_arrive_expect_tx(&s_full[s], Op::kStageBytes);
-        op.fill(smem + s * Op::kStageBytes, t, &s_full[s], policy);
-      } else {
-        mbar_arrive(&s_full[s]);  // the partial last tile is read from global memory
+  // ------------------------------------------------------------- phase 1
+  bool failed = false;    // a wait of this thread ran out
+  bool withheld = false;  // test hook: this CTA owns the withheld tile
+  uint32_t chunk_total = 0;  // compute warps: pairs selected by this warp
+  if (warp == kProducerWarp) {
+    if (lane == 0) {
+      const uint64_t policy = l2_evict_first_policy();
+      uint32_t r = 0;
+      for (; r < rounds; ++r) {
+        const int s = static_cast<int>(r % kStages);
+        const uint32_t k = r / kStages;
+        // wait for the 16 compute warps to release this stage's previous use
+        if (k > 0 && !mbar_wait(&s_empty[s], (k - 1) & 1u, ctx.wait_limit_ns)) {
+          failed = true;
+          break;
+        }
+        const uint32_t t = t_lo + r;
+        if (t < full_tiles) {
+          mbar_arrive_expect_tx(&s_full[s], Op::kStageBytes);
+          op.fill(smem + s * Op::kStageBytes, t, &s_full[s], policy);
+        } else {
+          mbar_arrive(&s_full[s]);  // the partial last tile is read from global memory
+        }
       }
-      issued = r + 1;
-    };
-    if (threadIdx.x == 0) {
-      policy = l2_evict_first_policy();
-      for (uint32_t r = 0; r < rounds && r < static_cast<uint32_t>(kStages); ++r) fill(r);
+      // no copy may land after the CTA exits: wait for the last fill of
+      // every stage (a completed phase reports complete immediately)
+      for (uint32_t q = r > kStages ? r - kStages : 0; q < r; ++q)
+        if (!mbar_wait(&s_full[q % kStages], (q / kStages) & 1u, ctx.wait_limit_ns))
+          failed = true;
     }
+  } else {
+    const uint32_t lt = lanemask_lt();
     for (uint32_t r = 0; r < rounds; ++r) {
       const int s = static_cast<int>(r % kStages);
+      const uint32_t t = t_lo + r;
       const bool arrived = mbar_wait(&s_full[s], (r / kStages) & 1u, ctx.wait_limit_ns);
-      if (group_bar_or(kComputeThreads, !arrived || s_abort)) {
-        if (threadIdx.x == 0) {
-          if (!arrived) atomicOr(ctx.error, kDevErrTimeout);
-          s_abort = 1;
-          for (uint32_t q = r; q < issued; ++q)  // let copies in flight land
-            mbar_wait(&s_full[q % kStages], (q / kStages) & 1u, ctx.wait_limit_ns);
-        }
+      if (!__all_sync(0xffffffffu, arrived)) {  // stop at the first failed wait
+        failed = true;
         break;
       }
-      const uint32_t t = c + r * G;
-      float a[kUnits][4];
-      uint32_t sel[kUnits];
-      if (t < full_tiles)
+      float a[kSUnits][4];
+      uint32_t sel[kSUnits];
+      if (t < full_tiles) {
         op.tile_smem(smem + s * Op::kStageBytes, t, warp, lane, a, sel);
-      else
+      } else {
         op.tile_global(t, warp, lane, a, sel);
-
-      uint32_t unit_off[kUnits];
-      uint32_t warp_total = 0;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_empty[s]);  // this warp is done with the stage
+      uint32_t off[kSUnits];
+      uint32_t total = 0;
 #pragma unroll
-      for (int v = 0; v < kUnits; ++v) {
+      for (int v = 0; v < kSUnits; ++v) {
         const uint32_t b0 = __ballot_sync(0xffffffffu, sel[v] & 1u);
         const uint32_t b1 = __ballot_sync(0xffffffffu, sel[v] & 2u);
         const uint32_t b2 = __ballot_sync(0xffffffffu, sel[v] & 4u);
         const uint32_t b3 = __ballot_sync(0xffffffffu, sel[v] & 8u);
-        unit_off[v] = warp_total + __popc(b0 & lt) + __popc(b1 & lt) + __popc(b2 & lt) +
-                      __popc(b3 & lt);
-        warp_total += __popc(b0) + __popc(b1) + __popc(b2) + __popc(b3);
+        off[v] = total + __popc(b0 & lt) + __popc(b1 & lt) + __popc(b2 & lt) + __popc(b3 & lt);
+        total += __popc(b0) + __popc(b1) + __popc(b2) + __popc(b3);
       }
-      if (lane == 0) s_warp_total[warp] = warp_total;
-      group_bar(kComputeThreads);
-      uint32_t warp_excl = 0, tile_total = 0;
+      const size_t seg = static_cast<size_t>(t) * kSWarps + warp;
+      if (lane == 0) sa.counts[seg] = total;
+      chunk_total += total;
+      if (total) {
+        uint32_t* sidx = sa.stage_idx + seg * kSWarpElems;
+        float* sval = sa.stage_val + seg * kSWarpElems;
 #pragma unroll
-      for (int w = 0; w < kWarps; ++w) {
-        const uint32_t cw = s_warp_total[w];
-        warp_excl += (w < warp) ? cw : 0u;
-        tile_total += cw;
-      }
-      if (threadIdx.x == 0) {
-        publish(ctx, t, kFlagAggregate, tile_total);
-        // room for this tile's pairs and a free entry slot (bounded wait)
-        const uint64_t t0 = global_timer_ns();
-        uint32_t it = 0;
-        while ((head - s_tail) + tile_total > kPairRing || r >= s_consumed + kEntryRing) {
-          if (s_abort || ++it > (1u << 26) || global_timer_ns() - t0 > ctx.wait_limit_ns) {
-            if (!s_abort) atomicOr(ctx.error, kDevErrTimeout);
-            s_abort = 1;
-            break;
-          }
-          __nanosleep(64);
-        }
-        __threadfence_block();
-        s_ring_start = head;
-        head += tile_total;
-      }
-      const bool abort_now = group_bar_or(kComputeThreads, s_abort != 0);
-      if (abort_now) {
-        if (threadIdx.x == 0)
-          for (uint32_t q = r + 1; q < issued; ++q)
-            mbar_wait(&s_full[q % kStages], (q / kStages) & 1u, ctx.wait_limit_ns);
-        break;
-      }
-      if (tile_total) {
-        const uint32_t base = s_ring_start + warp_excl;
-#pragma unroll
-        for (int v = 0; v < kUnits; ++v) {
-          uint32_t pos = base + unit_off[v];
+        for (int v = 0; v < kSUnits; ++v) {
+          uint32_t pos = off[v];
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
             if (sel[v] & (1u << j)) {
-              const uint32_t slot = pos % kPairRing;
-              ring_idx[slot] = static_cast<uint32_t>(element_index(t, warp, v, lane, j));
-              ring_val[slot] = a[v][j];
+              sidx[pos] = static_cast<uint32_t>(stream_element_index(t, warp, v, lane, j));
+              sval[pos] = a[v][j];
               ++pos;
             }
           }
         }
       }
-      group_bar(kComputeThreads);  // pairs staged; stage s fully read
-      if (threadIdx.x == 0) {
-        s_entry_count[r % kEntryRing] = tile_total;
-        s_entry_start[r % kEntryRing] = s_ring_start;
-        __threadfence_block();
-        s_produced = r + 1;
-        if (r + kStages < rounds) fill(r + kStages);
+      if (static_cast<int64_t>(t) == ctx.withheld_tile) withheld = true;
+    }
+  }
+  if (__syncthreads_or(failed)) {
+    if (threadIdx.x == 0) atomicOr(ctx.error, kDevErrTimeout);
+    return;
+  }
+  // A CTA that owns the withheld tile never arrives: the others' barrier
+  // waits run out (the failure-detection test).
+  if (__syncthreads_or(withheld)) return;
+
+  // ------------------------------------------------------------- phase 2
+  // the chunk's total (each compute warp contributes its own)
+  uint32_t mine = lane == 0 && warp < kSWarps ? chunk_total : 0u;
+  if (lane == 0) s_scratch[warp] = mine;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t sum = 0;
+    for (int w = 0; w < kSWarps; ++w) sum += s_scratch[w];
+    st_relaxed_u64(sa.chunk_sums + c, (static_cast<uint64_t>(ctx.epoch) << 32) | sum);
+  }
+  // sum of the earlier chunks' totals, waiting (bounded) for missing ones
+  uint32_t base = 0;
+  {
+    const uint64_t t0 = global_timer_ns();
+    uint32_t it = 0;
+    bool done = false;
+    while (!done) {
+      uint32_t part = 0;
+      bool present = true;
+      for (uint32_t q = threadIdx.x; q < c; q += kStreamThreads) {
+        const uint64_t w = ld_relaxed_u64(sa.chunk_sums + q);
+        if (static_cast<uint32_t>(w >> 32) == ctx.epoch)
+          part += static_cast<uint32_t>(w);
+        else
+          present = false;
+      }
+      part = warp_sum(part);
+      __syncthreads();
+      if (lane == 0) s_scratch[warp] = part;
+      const bool all_present = __syncthreads_and(present);
+      if (all_present) {
+        for (int w = 0; w < kStreamThreads / 32; ++w) base += s_scratch[w];
+        done = true;
+      } else {
+        const uint64_t now = global_timer_ns();
+        const bool out_of_time = ++it > (1u << 26) || now - t0 > ctx.wait_limit_ns;
+        if (__syncthreads_or(out_of_time)) {
+          if (threadIdx.x == 0) atomicOr(ctx.error, kDevErrTimeout);
+          return;
+        }
+        __nanosleep(64);
       }
     }
-  } else {
-    // ------------------------------------------------------------ scan warp
-    // Resolves staged tiles in order. The published counts it needs for up to
-    // kScanBatch staged rounds are loaded into registers together (one L2
-    // round trip per batch, not one per word), then the rounds are resolved
-    // in order as far as their counts are present.
-    const int lane = threadIdx.x & 31;
-    uint32_t incl = 0;  // this CTA's running inclusive count
-    uint32_t tail = 0;
-    bool overflow = false;
-    uint32_t r = 0;
-    uint64_t last_progress = __shfl_sync(0xffffffffu, global_timer_ns(), 0);
-    uint32_t idle_iters = 0;
-    while (r < rounds) {
-      const uint32_t produced = __shfl_sync(0xffffffffu, s_produced, 0);
-      const int aborted = __shfl_sync(0xffffffffu, s_abort, 0);
-      if (aborted) break;
-      uint32_t done = 0;
-      if (produced > r) {
-        __threadfence_block();
-        const uint32_t batch = produced - r < kScanBatch ? produced - r : kScanBatch;
-        uint64_t w[kScanBatch][kScanWordsPerLane];
+  }
+  const uint32_t lo = t_lo * kSWarps, hi = t_hi * kSWarps;
+
+  // The chunk's segment counts, a window at a time (the ring is free now):
+  // coalesced loads into shared memory, an exclusive scan there, then each
+  // warp copies kCopySegs adjacent segments at once with all of their loads
+  // in flight before the stores.
+  uint32_t* seg_off = reinterpret_cast<uint32_t*>(smem);
+  constexpr int kNumWarps = kStreamThreads / 32;
+  constexpr int kCopySegs = 8;
+  bool overflow = false;
+  for (uint32_t w0 = lo; w0 < hi; w0 += L::kChunkSegs) {
+    const uint32_t n = hi - w0 < L::kChunkSegs ? hi - w0 : L::kChunkSegs;
+    __syncthreads();
+    for (uint32_t i = threadIdx.x; i < n; i += kStreamThreads) seg_off[i] = __ldcg(sa.counts + w0 + i);
+    __syncthreads();
+    // each thread scans a contiguous run of the window in shared memory
+    const uint32_t per = (n + kStreamThreads - 1) / kStreamThreads;
+    const uint32_t b = threadIdx.x * per < n ? threadIdx.x * per : n;
+    const uint32_t e = b + per < n ? b + per : n;
+    uint32_t run = 0;
+    for (uint32_t i = b; i < e; ++i) {
+      const uint32_t cnt = seg_off[i];
+      seg_off[i] = run;
+      run += cnt;
+    }
+    uint32_t incl = run;
 #pragma unroll
-        for (int b = 0; b < kScanBatch; ++b) {
-          const uint32_t q = r + b;
-          const uint32_t t = c + q * G;
-          const uint32_t lo = q == 0 ? 0u : t - G + 1;
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    if (lane == 31) s_scratch[warp] = incl;
+    __syncthreads();
+    uint32_t warp_base = 0, window_total = 0;
+    for (int w = 0; w < kNumWarps; ++w) {
+      const uint32_t x = s_scratch[w];
+      warp_base += w < warp ? x : 0u;
+      window_total += x;
+    }
+    const uint32_t thread_base = base + warp_base + incl - run;
+    for (uint32_t i = b; i < e; ++i) seg_off[i] += thread_base;
+    __syncthreads();
+    const uint32_t window_end = base + window_total;
+    for (uint32_t i0 = warp * kCopySegs; i0 < n; i0 += kNumWarps * kCopySegs) {
+      uint32_t dst[kCopySegs], cnt[kCopySegs], maxc = 0;
 #pragma unroll
-          for (int k = 0; k < kScanWordsPerLane; ++k) {
-            const uint32_t u = lo + lane + 32u * k;
-            w[b][k] = (static_cast<uint32_t>(b) < batch && u < t) ? ld_relaxed_u64(ctx.status + u)
-                                                                 : (uint64_t(ctx.epoch) << 34);
+      for (int u = 0; u < kCopySegs; ++u) {
+        const uint32_t i = i0 + u;
+        dst[u] = i < n ? seg_off[i] : 0u;
+        const uint32_t next = i + 1 < n ? seg_off[i + 1] : window_end;
+        cnt[u] = i < n ? next - dst[u] : 0u;
+        maxc = cnt[u] > maxc ? cnt[u] : maxc;
+      }
+      for (uint32_t p0 = 0; p0 < maxc; p0 += 32) {
+        uint32_t xi[kCopySegs];
+        float xv[kCopySegs];
+#pragma unroll
+        for (int u = 0; u < kCopySegs; ++u) {
+          if (p0 + lane < cnt[u]) {
+            const size_t src = static_cast<size_t>(w0 + i0 + u) * kSWarpElems + p0 + lane;
+            xi[u] = __ldcs(sa.stage_idx + src);
+            xv[u] = __ldcs(sa.stage_val + src);
           }
         }
 #pragma unroll
-        for (int b = 0; b < kScanBatch; ++b) {
-          if (static_cast<uint32_t>(b) >= batch || done != static_cast<uint32_t>(b)) break;
-          uint32_t sum = 0;
-          bool ready = true;
-#pragma unroll
-          for (int k = 0; k < kScanWordsPerLane; ++k) {
-            if (static_cast<uint32_t>(w[b][k] >> 34) == ctx.epoch)
-              sum += static_cast<uint32_t>(w[b][k]);
-            else
-              ready = false;
-          }
-          if (!__all_sync(0xffffffffu, ready)) break;
-          const uint32_t q = r + b;
-          const uint32_t t = c + q * G;
-          const uint32_t cnt = s_entry_count[q % kEntryRing];
-          const uint32_t start = s_entry_start[q % kEntryRing];
-          const uint32_t excl = (q == 0 ? 0u : incl) + warp_sum(sum);
-          for (uint32_t p = lane; p < cnt; p += 32) {
-            const uint32_t slot = (start + p) % kPairRing;
-            const uint32_t dst = excl + p;
-            if (dst < cap) {
-              idx_out[dst] = ring_idx[slot];
-              val_out[dst] = ring_val[slot];
+        for (int u = 0; u < kCopySegs; ++u) {
+          if (p0 + lane < cnt[u]) {
+            const uint32_t q = dst[u] + p0 + lane;
+            if (q < cap) {
+              idx_out[q] = xi[u];
+              val_out[q] = xv[u];
             } else {
               overflow = true;
             }
           }
-          incl = excl + cnt;
-          if (t == T - 1 && lane == 0) *count_out = incl < cap ? incl : cap;
-          tail += cnt;
-          ++done;
         }
-      }
-      const uint64_t now = __shfl_sync(0xffffffffu, global_timer_ns(), 0);
-      if (done) {
-        __syncwarp();
-        if (lane == 0) {
-          __threadfence_block();
-          s_tail = tail;
-          s_consumed = r + done;
-        }
-        r += done;
-        last_progress = now;
-        idle_iters = 0;
-      } else {
-        if (++idle_iters > (1u << 26) || now - last_progress > ctx.wait_limit_ns) {
-          if (lane == 0) {
-            atomicOr(ctx.error, kDevErrTimeout);
-            s_abort = 1;
-          }
-          break;
-        }
-        __nanosleep(32);
       }
     }
-    if (__any_sync(0xffffffffu, overflow) && lane == 0) atomicOr(ctx.error, kDevErrOverflow);
+    base = window_end;
   }
-  __syncthreads();
+  if (hi == T * kSWarps && threadIdx.x == 0) *count_out = base < cap ? base : cap;
+  if (__syncthreads_or(overflow) && threadIdx.x == 0) atomicOr(ctx.error, kDevErrOverflow);
 }
 
 }  // namespace efs

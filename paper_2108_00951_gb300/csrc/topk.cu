@@ -183,39 +183,6 @@ __device__ Selection select_bin(const uint32_t* hist, uint32_t nbins, uint32_t k
   return s;
 }
 
-// Bounded grid-wide barrier for a cooperative launch (all CTAs co-resident).
-// Returns false, latching kDevErrTimeout, if the wait ran out.
-__device__ bool grid_barrier(uint32_t* arrive, uint32_t* gen, uint64_t limit_ns,
-                             uint32_t* error) {
-  __shared__ int s_ok;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    int ok = 1;
-    const uint32_t my_gen = ld_acquire_u32(gen);
-    __threadfence();  // this CTA's histogram merges and appends before arriving
-    const uint32_t ticket = atomicAdd(arrive, 1u);
-    if (ticket == gridDim.x - 1) {
-      atomicExch(arrive, 0u);
-      __threadfence();
-      st_release_u32(gen, my_gen + 1);
-    } else {
-      const uint64_t t0 = global_timer_ns();
-      uint32_t iters = 0;
-      while (ld_acquire_u32(gen) == my_gen) {
-        if (++iters > (1u << 26) || global_timer_ns() - t0 > limit_ns) {
-          atomicOr(error, kDevErrTimeout);
-          ok = 0;
-          break;
-        }
-        __nanosleep(128);
-      }
-    }
-    s_ok = ok;
-  }
-  __syncthreads();
-  return s_ok != 0;
-}
-
 // Warp-aggregated append of the keys of the lanes with pred set.
 __device__ __forceinline__ void warp_append(bool pred, uint64_t key, uint64_t* dst,
                                             uint32_t* count, uint32_t cap) {
