@@ -171,6 +171,41 @@ ef_status sparse_aggregate(uint32_t n, const uint32_t* const* idx,
                            uint64_t d, float* dense_out, ef_stream_t stream);
 
 /*
+ * ef_hard_threshold_noalloc — ef_hard_threshold for callers that cannot
+ * allocate device memory. (An implementation convenience; the paper has no
+ * counterpart.)
+ *
+ * The other entry points grow a per-stream workspace with cudaMalloc, which
+ * also synchronises the stream once. Some callers cannot allow that: their
+ * device memory is owned entirely by their own allocator or a framework's
+ * caching pool, they run under a fixed device-memory budget, or they sit in a
+ * loop that must never block in cudaMalloc/cudaFree. This entry point computes
+ * exactly the same result as ef_hard_threshold (same arguments, same bits)
+ * with a fixed scratch array that is part of the library image; it calls no
+ * cudaMalloc, cudaFree or allocating library routine.
+ *
+ *   g, e, gamma, lambda, idx_out, val_out, count_out   as for ef_hard_threshold
+ *                (fp32 gradient only).
+ *   d          0 <= d <= 268,435,456 (2^28); larger d returns
+ *              EF_ERR_INVALID_ARG and launches nothing.
+ *   status_out [out, optional] one uint32 in device memory, or NULL: after
+ *              the call it holds the device-side error bits of this call
+ *              (0 = success; nonzero = a bounded wait ran out or an output
+ *              position overflowed). ef_check_status() does not see them.
+ *
+ * The scratch (512 KiB + 256 bytes) is held on every device that loads the
+ * library until the process exits. The first call on a device looks up the
+ * scratch's device address; make that first call before any stream capture.
+ * All calls on one device share the scratch: calls that overlap on the GPU
+ * (on different streams, or from host threads without ordering between them)
+ * race and must not be made.
+ */
+ef_status ef_hard_threshold_noalloc(const float* g, float* e, float gamma, float lambda,
+                                    uint64_t d, uint32_t* idx_out, float* val_out,
+                                    uint32_t* count_out, uint32_t* status_out,
+                                    ef_stream_t stream);
+
+/*
  * ef_check_status — synchronise `stream`, then return and clear the device-side
  * error latched by earlier calls on that stream (EF_OK if none).
  */

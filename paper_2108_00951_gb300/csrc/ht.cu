@@ -204,6 +204,25 @@ void ht_init_device(DeviceInfo& info) {
   info.ht_stream_per_sm_bf16 = stream_blocks_per_sm<uint16_t>();
 }
 
+// Launch the look-back kernel over caller-provided scratch (the tile-status
+// words and the error word named by ctx); used by the allocation-free entry.
+cudaError_t launch_hard_threshold_lookback(const float* g, float* e, float gamma, float lambda,
+                                           uint32_t d, uint32_t* idx_out, float* val_out,
+                                           uint32_t* count_out, const ScanCtx& ctx,
+                                           cudaStream_t stream) {
+  const uint32_t tiles = tiles_for(d);
+  const bool vec = reinterpret_cast<uintptr_t>(g) % 16 == 0 &&
+                   reinterpret_cast<uintptr_t>(e) % 16 == 0;
+  if (vec)
+    ht_kernel<float, true><<<tiles, kThreads, 0, stream>>>(g, e, gamma, lambda, d, idx_out,
+                                                           val_out, count_out, ctx);
+  else
+    ht_kernel<float, false><<<tiles, kThreads, 0, stream>>>(g, e, gamma, lambda, d, idx_out,
+                                                            val_out, count_out, ctx);
+  count_launch();
+  return cudaGetLastError();
+}
+
 cudaError_t launch_hard_threshold(const void* g, bool g_bf16, float* e, float gamma,
                                   float lambda, uint32_t d, uint32_t* idx_out, float* val_out,
                                   uint32_t* count_out, Workspace& ws, const DeviceInfo& dev) {

@@ -86,6 +86,10 @@ ScanCtx next_scan_ctx(Workspace& ws, uint32_t num_tiles);
 cudaError_t launch_hard_threshold(const void* g, bool g_bf16, float* e, float gamma,
                                   float lambda, uint32_t d, uint32_t* idx_out, float* val_out,
                                   uint32_t* count_out, Workspace& ws, const DeviceInfo& dev);
+cudaError_t launch_hard_threshold_lookback(const float* g, float* e, float gamma, float lambda,
+                                           uint32_t d, uint32_t* idx_out, float* val_out,
+                                           uint32_t* count_out, const ScanCtx& ctx,
+                                           cudaStream_t stream);
 cudaError_t launch_topk(const void* g, bool g_bf16, float* e, float gamma, uint32_t k,
                         uint32_t d, uint32_t* idx_out, float* val_out, uint32_t* count_out,
                         Workspace& ws, const DeviceInfo& dev);
