@@ -47,7 +47,10 @@ if ROOT not in sys.path:
 PEAK_FALLBACK_GBS = 6800.0
 NOMINAL_HBM_GBS = 8000.0
 METRIC = "EF hard-threshold compress GB/s & elem/s vs HBM peak; Top-k and aggregate ms/iter"
-HT_KERNEL_SOURCES = ["paper_2108_00951_gb300/csrc/ht.cu", "paper_2108_00951_gb300/csrc/compact.cuh",
+HT_KERNEL_SOURCES = ["paper_2108_00951_gb300/csrc/ht.cu",
+                     "paper_2108_00951_gb300/csrc/stream_compact.cuh",
+                     "paper_2108_00951_gb300/csrc/tma.cuh",
+                     "paper_2108_00951_gb300/csrc/compact.cuh",
                      "paper_2108_00951_gb300/csrc/common.cuh",
                      "paper_2108_00951_gb300/csrc/gradient.cuh"]
 
@@ -368,7 +371,8 @@ def run_ours(args):
         "frac_of_nominal_8tbs": round(value / NOMINAL_HBM_GBS, 4),
         "roofline": {
             "bound": "hbm",
-            "kernel": "ht_kernel (fused EF accumulate + hard-threshold + compaction + residual)",
+            "kernel": "stream_compact_kernel<HtOp> (fused EF accumulate + hard-threshold + "
+                      "compaction + residual)",
             "achieved": round(achieved, 2),
             "peak": peak,
             "peak_kind": peak_kind,
