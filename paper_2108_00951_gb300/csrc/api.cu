@@ -38,10 +38,9 @@ ef_status device_info(int dev, DeviceInfo* out) {
     DeviceInfo info;
     if (cudaDeviceGetAttribute(&info.sm_count, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
       return EF_ERR_CUDA;
-    const int per_sm = topk_refine_blocks_per_sm();
-    if (per_sm <= 0) return EF_ERR_CUDA;
-    info.refine_blocks = per_sm * info.sm_count;
     ht_init_device(info);
+    topk_init_device(info);
+    if (info.refine_blocks <= 0 || info.finalize_blocks <= 0) return EF_ERR_CUDA;
     it = g_devices.emplace(dev, info).first;
   }
   *out = it->second;
@@ -173,7 +172,8 @@ ef_status topk_entry(const void* g, bool bf16, float* e, float gamma, uint64_t k
   ef_status st = device_info(dev, &info);
   if (st != EF_OK) return st;
   Workspace* ws = nullptr;
-  st = acquire_workspace(stream, tiles_for(d), topk_candidate_capacity(d), 0, 0, &ws);
+  st = acquire_workspace(stream, tiles_for(d), topk_candidate_capacity(d), 0,
+                         static_cast<size_t>(tiles_for(d)) * kTileElems, &ws);
   if (st != EF_OK) return st;
   return finish_launch(launch_topk(g, bf16, e, gamma, static_cast<uint32_t>(k),
                                    static_cast<uint32_t>(d), idx_out, val_out, count_out, *ws,

@@ -85,6 +85,12 @@ struct HtOp {
   uint32_t d;
   static constexpr uint32_t kGBytes = kTileElems * sizeof(GT);
   static constexpr uint32_t kStageBytes = kGBytes + kTileElems * sizeof(float);
+  static constexpr bool kPrepass = false;
+  static constexpr int kSampleBins = 1;
+  __device__ void sample(const unsigned char*, uint32_t, int, int, uint32_t*) const {}
+  __device__ void merge(const uint32_t*) const {}
+  __device__ bool barrier(uint64_t, uint32_t*) const { return true; }
+  __device__ uint64_t choose() const { return 0; }
 
   __device__ __forceinline__ void fill(unsigned char* stage, uint32_t t, uint64_t* bar,
                                        uint64_t policy) const {
@@ -95,7 +101,7 @@ struct HtOp {
 
   __device__ __forceinline__ void tile_smem(const unsigned char* stage, uint32_t t, int warp,
                                             int lane, float (&a)[kSUnits][4],
-                                            uint32_t (&sel)[kSUnits]) const {
+                                            uint32_t (&sel)[kSUnits], uint64_t) const {
     const GT* gs = reinterpret_cast<const GT*>(stage);
     const float* es = reinterpret_cast<const float*>(stage + kGBytes);
     const int local = warp * kSWarpElems + lane * 4;
@@ -122,7 +128,7 @@ struct HtOp {
 
   __device__ __forceinline__ void tile_global(uint32_t t, int warp, int lane,
                                               float (&a)[kSUnits][4],
-                                              uint32_t (&sel)[kSUnits]) const {
+                                              uint32_t (&sel)[kSUnits], uint64_t) const {
     const uint64_t first = stream_element_index(t, warp, 0, lane, 0);
 #pragma unroll
     for (int v = 0; v < kSUnits; ++v) {

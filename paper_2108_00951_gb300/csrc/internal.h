@@ -14,13 +14,21 @@ namespace efs {
 constexpr size_t kOffBarGen = 0;        // uint32: grid-barrier generation (never reset)
 constexpr size_t kOffError = 8;         // uint32: latched device error bits
 constexpr size_t kOffTopkReset = 16;    // start of the region cleared at each Top-k call
-constexpr size_t kOffBarArrive = 16;    // uint32
-constexpr size_t kOffCandCount = 20;    // uint32[6]
+constexpr size_t kOffBarArrive = 16;    // uint32: grid-barrier arrivals
+constexpr size_t kOffCandCount = 20;    // uint32[6]: refine-level candidate counts
 constexpr size_t kOffThreshold = 48;    // uint64: Top-k composite-key threshold
-constexpr size_t kOffHist = 256;        // uint32[6][2048]
+constexpr size_t kOffTkLowerBound = 56; // uint64: sampled lower bound of the candidates' keys
+constexpr size_t kOffTkMode = 64;       // uint32: 0 candidates, 1 full array
+constexpr size_t kOffTkSampleDone = 68; // uint32: sampling CTAs finished
+constexpr size_t kOffTkListCount = 72;  // uint32: candidates emitted by the streaming pass
+constexpr size_t kOffTkListFlags = 76;  // uint32: that pass's latched bits (overflow, timeout)
+constexpr size_t kOffHist = 256;        // uint32[6][2048] refine levels 0..5, then the sample
 constexpr int kHistLevels = 6;
 constexpr int kHistBins = 2048;
-constexpr size_t kHeaderBytes = kOffHist + sizeof(uint32_t) * kHistLevels * kHistBins;
+constexpr int kSampleBits = 13;         // the sample histogram: top 13 bits of |a|
+constexpr int kSampleBins = 1 << kSampleBits;
+constexpr size_t kOffSampleHist = kOffHist + sizeof(uint32_t) * kHistLevels * kHistBins;
+constexpr size_t kHeaderBytes = kOffSampleHist + sizeof(uint32_t) * kSampleBins;
 constexpr size_t kTopkResetBytes = kHeaderBytes - kOffTopkReset;
 constexpr uint32_t kMaxChunks = 1024;   // per-CTA chunk sums of the streaming compaction
 constexpr uint32_t kCountsPerTile = 16; // per-segment counts of the streaming compaction
@@ -41,7 +49,8 @@ struct Workspace {
   static size_t align(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
   size_t off_status() const { return kHeaderBytes; }
   size_t off_cand() const { return align(off_status() + sizeof(uint64_t) * status_tiles); }
-  size_t off_offsets() const { return align(off_cand() + 2 * sizeof(uint64_t) * cand_cap); }
+  // three candidate buffers: the streamed (index, value) list and two key buffers
+  size_t off_offsets() const { return align(off_cand() + 3 * sizeof(uint64_t) * cand_cap); }
   size_t off_counts() const { return align(off_offsets() + sizeof(uint32_t) * offsets_cap); }
   size_t off_chunks() const {
     return align(off_counts() + sizeof(uint32_t) * kCountsPerTile * status_tiles);
@@ -68,9 +77,15 @@ struct Workspace {
 struct DeviceInfo {
   int sm_count = 0;
   int refine_blocks = 0;          // co-resident CTAs for the cooperative Top-k refine
+  int finalize_blocks = 0;        // co-resident CTAs for the Top-k finalize
   int ht_stream_per_sm_f32 = 0;   // streaming hard-threshold CTAs per SM (0: unavailable)
   int ht_stream_per_sm_bf16 = 0;
+  int tk_stream_per_sm_f32 = 0;   // streaming Top-k candidate pass CTAs per SM
+  int tk_stream_per_sm_bf16 = 0;
 };
+
+// Per-device set-up of the Top-k kernels (shared-memory opt-in, occupancy).
+void topk_init_device(DeviceInfo& info);
 
 // Per-device set-up of the streaming hard-threshold kernels (opts them into
 // their shared-memory ring on the current device and records occupancy).
@@ -97,8 +112,6 @@ cudaError_t launch_aggregate(uint32_t n, const uint32_t* const* idx, const float
                              const uint32_t* counts, uint32_t d, float* dense_out,
                              Workspace& ws);
 
-// Occupancy of the cooperative Top-k refine kernel (CTAs per SM).
-int topk_refine_blocks_per_sm();
 
 // Workspace sizing helpers.
 inline uint32_t tiles_for(uint64_t d) {

@@ -36,6 +36,7 @@
 //
 // An Op supplies the per-segment work:
 //   static constexpr uint32_t kStageBytes;            bytes of one stage
+//   static constexpr bool kPrepass;                   see below
 //   void fill(unsigned char* stage, uint32_t tile, uint64_t* bar, uint64_t pol)
 //        issue the bulk copies of a full tile (after expect_tx)
 //   void tile_smem(const unsigned char* stage, uint32_t tile, int warp, int lane,
@@ -44,6 +45,17 @@
 //        compute values and selection bits (and side effects) of the calling
 //        warp's segment, from the stage of a full tile, or from global memory
 //        for the partial last tile.
+//   (tile_smem and tile_global also receive `aux`, the pre-pass result or 0)
+// Optional pre-pass (kPrepass): before streaming, the compute warps hand the
+// first tile of their CTA's chunk, from its ring stage, to
+//   void sample(const unsigned char* stage, uint32_t tile, int warp, int lane,
+//               uint32_t* s_hist)       (accumulate a kSampleBins histogram)
+// the CTA merges its histogram with
+//   void merge(const uint32_t* s_hist)  (all threads)
+// and after a grid barrier every CTA computes the same value with
+//   uint64_t choose()                   (all threads; uniform result)
+// which becomes `aux`. The producer warp issues its first fills before the
+// pre-pass, so the ring is loading while the CTAs sample and synchronise.
 // Element layout: unit v of lane l of warp w covers the 4 coordinates from
 // tile * kTileElems + w * 256 + v * 128 + l * 4 (see stream_element_index).
 #pragma once
@@ -90,6 +102,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   __shared__ __align__(8) uint64_t s_full[kStages];
   __shared__ __align__(8) uint64_t s_empty[kStages];
   __shared__ uint32_t s_scratch[kStreamThreads / 32];
+  __shared__ uint32_t s_sample_hist[Op::kPrepass ? Op::kSampleBins : 1];
   using L = StreamLayout<Op, kStages>;
 
   const uint32_t T = ctx.num_tiles, G = gridDim.x, c = blockIdx.x;
@@ -112,25 +125,63 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   bool failed = false;    // a wait of this thread ran out
   bool withheld = false;  // test hook: this CTA owns the withheld tile
   uint32_t chunk_total = 0;  // compute warps: pairs selected by this warp
+  uint64_t policy = 0;       // producer lane
+  auto fill = [&](uint32_t r) {  // producer lane
+    const int s = static_cast<int>(r % kStages);
+    const uint32_t t = t_lo + r;
+    if (t < full_tiles) {
+      mbar_arrive_expect_tx(&s_full[s], Op::kStageBytes);
+      op.fill(smem + s * Op::kStageBytes, t, &s_full[s], policy);
+    } else {
+      mbar_arrive(&s_full[s]);  // the partial last tile is read from global memory
+    }
+  };
+  const bool producer = warp == kProducerWarp && lane == 0;
+  if (producer) {
+    policy = l2_evict_first_policy();
+    for (uint32_t r = 0; r < rounds && r < static_cast<uint32_t>(kStages); ++r) fill(r);
+  }
+
+  uint64_t aux = 0;
+  if constexpr (Op::kPrepass) {
+    for (int b = threadIdx.x; b < Op::kSampleBins; b += kStreamThreads) s_sample_hist[b] = 0;
+    __syncthreads();
+    if (warp < kSWarps && rounds > 0 && t_lo < full_tiles) {
+      if (!__all_sync(0xffffffffu, mbar_wait(&s_full[0], 0, ctx.wait_limit_ns)))
+        failed = true;
+      else
+        op.sample(smem, t_lo, warp, lane, s_sample_hist);
+    }
+    if (__syncthreads_or(failed)) {
+      if (threadIdx.x == 0) atomicOr(ctx.error, kDevErrTimeout);
+      if (producer)  // no copy may land after the CTA exits
+        for (uint32_t q = 0; q < rounds && q < static_cast<uint32_t>(kStages); ++q)
+          mbar_wait(&s_full[q], 0, ctx.wait_limit_ns);
+      return;
+    }
+    op.merge(s_sample_hist);
+    const bool passed = op.barrier(ctx.wait_limit_ns, ctx.error);
+    if (!passed) {
+      if (producer)
+        for (uint32_t q = 0; q < rounds && q < static_cast<uint32_t>(kStages); ++q)
+          mbar_wait(&s_full[q], 0, ctx.wait_limit_ns);
+      return;
+    }
+    aux = op.choose();
+  }
+
   if (warp == kProducerWarp) {
     if (lane == 0) {
-      const uint64_t policy = l2_evict_first_policy();
-      uint32_t r = 0;
+      uint32_t r = rounds < static_cast<uint32_t>(kStages) ? rounds : kStages;
       for (; r < rounds; ++r) {
         const int s = static_cast<int>(r % kStages);
         const uint32_t k = r / kStages;
         // wait for the 16 compute warps to release this stage's previous use
-        if (k > 0 && !mbar_wait(&s_empty[s], (k - 1) & 1u, ctx.wait_limit_ns)) {
+        if (!mbar_wait(&s_empty[s], (k - 1) & 1u, ctx.wait_limit_ns)) {
           failed = true;
           break;
         }
-        const uint32_t t = t_lo + r;
-        if (t < full_tiles) {
-          mbar_arrive_expect_tx(&s_full[s], Op::kStageBytes);
-          op.fill(smem + s * Op::kStageBytes, t, &s_full[s], policy);
-        } else {
-          mbar_arrive(&s_full[s]);  // the partial last tile is read from global memory
-        }
+        fill(r);
       }
       // no copy may land after the CTA exits: wait for the last fill of
       // every stage (a completed phase reports complete immediately)
@@ -151,9 +202,9 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
       float a[kSUnits][4];
       uint32_t sel[kSUnits];
       if (t < full_tiles) {
-        op.tile_smem(smem + s * Op::kStageBytes, t, warp, lane, a, sel);
+        op.tile_smem(smem + s * Op::kStageBytes, t, warp, lane, a, sel, aux);
       } else {
-        op.tile_global(t, warp, lane, a, sel);
+        op.tile_global(t, warp, lane, a, sel, aux);
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&s_empty[s]);  // this warp is done with the stage

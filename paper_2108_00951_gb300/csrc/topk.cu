@@ -1,6 +1,6 @@
-// topk.cu — error-feedback + Top-k sparsifier (the paper's baseline, Lemma 2)
-// as a radix select on the magnitude bits, followed by the same ordered
-// compaction as the hard-threshold path.
+// topk.cu — error-feedback + Top-k sparsifier (the paper's baseline, Lemma 2):
+// one streaming pass over the coordinates, then an exact radix select and an
+// ordered compaction on a small candidate list.
 //
 // Order. Every coordinate j gets the 63-bit composite key
 //     K_j = (bits(|a_j|) << 32) | (~j & 0xffffffff),
@@ -10,26 +10,33 @@
 // magnitudes. All K_j are distinct, so the Top-k set is exactly
 // { j : K_j >= K_(k) } for the k-th largest key K_(k).
 //
-// Passes (launches per call: one memset of the small control block + 3):
-//   A  accumulate: a = fmaf(gamma, g, e) is written over e, and a histogram
-//      of the top 11 key bits (62..52) is built in shared memory and merged
-//      into global memory. 12 B/coordinate, the algorithmic traffic.
-//   R  refine (one cooperative launch, all CTAs co-resident): digit by digit
-//      (bits 51..42, 41..32, 31..21, 20..10, 9..0) histogram the coordinates
-//      whose key shares the bits fixed so far, pick the digit that contains
-//      the k-th key, until the remaining rank equals the bucket size. The
-//      first refine digit reads a (4 B/coordinate) and compacts the bucket's
-//      keys into a candidate buffer when it fits; later digits read only
-//      candidates. Every CTA selects redundantly from the merged histogram
-//      after a bounded grid barrier, so control flow is uniform.
-//   Z  select: the ordered compaction with predicate K_j >= threshold; e is
-//      zeroed at the selected coordinates (the residual a - C(a)).
-#include "compact.cuh"
+// Kernels of one call (after clearing the small control block):
+//  1 stream   the streaming compaction of stream_compact.cuh with a sampling
+//             pre-pass: every CTA histograms the top 11 key bits of the first
+//             tile of its chunk, the histograms are merged, and after a grid
+//             barrier every CTA derives the same lower bound B with about
+//             twice the needed mass above it (or, when the candidates would
+//             not fit, the full-array mode). Then a = fmaf(γ,g,e) is written
+//             over e (12 B per coordinate, the algorithmic bytes) and the
+//             coordinates with K_j >= B are emitted as an ordered (index,
+//             value) candidate list.
+//  2 select   radix select, digit by digit (11/10/10/11/11/10 bits), of the
+//             exact threshold K_(k) over the candidates — or over all of a
+//             when the candidates are short of k, overflowed, or were not
+//             gathered — then the ordered compaction of K_j >= K_(k), zeroing
+//             e at the selected coordinates. Up to 65,536 candidates one CTA
+//             does all of it; beyond, the whole grid does (merged histograms
+//             with bounded grid barriers; chunk counts, then positions).
+// The candidate path moves about 12 B per coordinate plus small amounts; the
+// full-array path adds a read of a per digit level and two for the output.
 #include "gradient.cuh"
 #include "internal.h"
+#include "stream_compact.cuh"
 
 namespace efs {
 namespace {
+
+constexpr uint64_t kSelectNone = 1ull << 63;  // above every composite key
 
 // LSB of each digit of the composite key; digit 0 is bits 62..52.
 __device__ __forceinline__ int digit_shift(int level) {
@@ -42,15 +49,24 @@ __device__ __forceinline__ uint64_t composite_key(float a, uint64_t j) {
 }
 
 struct TopkArgs {
-  uint32_t* hist;        // [kHistLevels][kHistBins]
-  uint64_t* cand0;
+  uint32_t* hist;        // [kHistLevels + 1][kHistBins]
+  uint64_t* cand0;       // key buffers of the refine levels
   uint64_t* cand1;
+  uint32_t* list_idx;    // ordered candidates from the streaming pass
+  float* list_val;
   uint32_t* cand_count;  // [kHistLevels]
   uint32_t cand_cap;
   uint64_t* threshold;
+  uint64_t* lower_bound;
+  uint32_t* mode;        // 0: candidates, 1: full array
+  uint32_t* sample_done;
+  uint32_t* list_count;
+  uint32_t* list_flags;
   uint32_t* bar_arrive;
   uint32_t* bar_gen;
   uint32_t* error;
+  uint64_t* chunk_sums;
+  uint32_t epoch;        // tags the finalize kernel's chunk totals
   uint64_t wait_limit_ns;
 };
 
@@ -62,111 +78,65 @@ __device__ __forceinline__ void hist_add_warp(uint32_t* h, uint32_t bin, bool va
     atomicAdd(&h[bin], static_cast<uint32_t>(__popc(peers)));
 }
 
-// ------------------------------------------------------------------ pass A
-template <typename GT, bool kVec>
-__global__ void __launch_bounds__(kThreads)
-    topk_accumulate_kernel(const GT* __restrict__ g, float* __restrict__ e, float gamma,
-                           uint32_t d, uint32_t num_tiles, uint32_t* __restrict__ hist0) {
-  __shared__ uint32_t s_hist[kHistBins];
-  for (int b = threadIdx.x; b < kHistBins; b += kThreads) s_hist[b] = 0;
-  __syncthreads();
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  for (uint32_t tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
-    const uint64_t first = element_index(tile, warp, 0, lane, 0);
-    const bool full_tile = static_cast<uint64_t>(tile + 1) * kTileElems <= d;
-    if (kVec && full_tile) {
-      GradVec<GT> gv[kUnits];
-      float4 ev[kUnits];
-#pragma unroll
-      for (int v = 0; v < kUnits; ++v) {
-        gv[v].load(g + first + v * 128);
-        ev[v] = ld_stream_f4(e + first + v * 128);
-      }
-#pragma unroll
-      for (int v = 0; v < kUnits; ++v) {
-        float4 a;
-        a.x = __fmaf_rn(gamma, gv[v][0], ev[v].x);
-        a.y = __fmaf_rn(gamma, gv[v][1], ev[v].y);
-        a.z = __fmaf_rn(gamma, gv[v][2], ev[v].z);
-        a.w = __fmaf_rn(gamma, gv[v][3], ev[v].w);
-        // default caching: the refine and select passes re-read a
-        *reinterpret_cast<float4*>(e + first + v * 128) = a;
-        hist_add_warp(s_hist, (__float_as_uint(a.x) & 0x7fffffffu) >> 20, true);
-        hist_add_warp(s_hist, (__float_as_uint(a.y) & 0x7fffffffu) >> 20, true);
-        hist_add_warp(s_hist, (__float_as_uint(a.z) & 0x7fffffffu) >> 20, true);
-        hist_add_warp(s_hist, (__float_as_uint(a.w) & 0x7fffffffu) >> 20, true);
-      }
-    } else {
-#pragma unroll
-      for (int v = 0; v < kUnits; ++v) {
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const uint64_t i = first + v * 128 + j;
-          const bool ok = i < d;
-          float x = 0.0f;
-          if (ok) {
-            x = __fmaf_rn(gamma, grad_scalar(g, i), e[i]);
-            e[i] = x;
-          }
-          hist_add_warp(s_hist, (__float_as_uint(x) & 0x7fffffffu) >> 20, ok);
-        }
-      }
-    }
-  }
-  __syncthreads();
-  for (int b = threadIdx.x; b < kHistBins; b += kThreads)
-    if (s_hist[b]) atomicAdd(&hist0[b], s_hist[b]);
-}
-
-// ------------------------------------------------------------------ pass R
 struct Selection {
   uint32_t bin, k_rem, n_in, found;
 };
 
+// Exclusive suffix sum over the threads of the CTA (the sum of v over every
+// higher thread index) and the block total. Whole CTA; blockDim.x a multiple
+// of 32; s_w holds blockDim.x / 32 words.
+__device__ __forceinline__ uint32_t block_suffix_exclusive(uint32_t v, uint32_t& total,
+                                                           uint32_t* s_w) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nw = static_cast<int>(blockDim.x >> 5);
+  uint32_t incl = v;  // v summed over this lane and the higher lanes
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t x = __shfl_down_sync(0xffffffffu, incl, o);
+    if (lane + o < 32) incl += x;
+  }
+  __syncthreads();  // a previous use of s_w is complete
+  if (lane == 0) s_w[warp] = incl;
+  __syncthreads();
+  uint32_t wsuf = lane < nw ? s_w[lane] : 0u;  // warp totals over warps >= lane
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t x = __shfl_down_sync(0xffffffffu, wsuf, o);
+    if (lane + o < 32) wsuf += x;
+  }
+  total = __shfl_sync(0xffffffffu, wsuf, 0);
+  const uint32_t higher = __shfl_sync(0xffffffffu, wsuf, (warp + 1) & 31);
+  return (warp + 1 < 32 ? higher : 0u) + incl - v;
+}
+
 // Find the bin holding the k_rem-th largest key of a histogram of nbins
-// (2048 or 1024) bins, scanning from the highest bin. Whole CTA; uniform.
-__device__ Selection select_bin(const uint32_t* hist, uint32_t nbins, uint32_t k_rem) {
-  __shared__ uint32_t s_part[kThreads];
+// (2048 or 1024) bins, scanning from the highest bin. Whole CTA of kBlock
+// threads (kBlock <= nbins); uniform result. kGlobal: the histogram is in
+// global memory (read through L2), else in shared memory. s_w holds
+// kBlock / 32 words.
+template <int kBlock, bool kGlobal>
+__device__ Selection select_bin(const uint32_t* hist, uint32_t nbins, uint32_t k_rem,
+                                uint32_t* s_w) {
+  constexpr int kMaxPer = kHistBins / kBlock;
   __shared__ Selection s_sel;
   const int t = threadIdx.x;
-  const uint32_t per = nbins / kThreads;  // 8 or 4 bins per thread
-  uint32_t c[8];
+  const uint32_t per = nbins / kBlock;
+  uint32_t c[kMaxPer];
   uint32_t sum = 0;
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    c[i] = (static_cast<uint32_t>(i) < per) ? __ldcg(hist + t * per + i) : 0u;
+  for (int i = 0; i < kMaxPer; ++i) {
+    c[i] = (static_cast<uint32_t>(i) < per)
+               ? (kGlobal ? __ldcg(hist + t * per + i) : hist[t * per + i]) : 0u;
     sum += c[i];
   }
   if (t == 0) s_sel = Selection{0, 0, 0, 0};
-  s_part[t] = sum;
-  __syncthreads();
-  if (t < 32) {  // exclusive suffix sums over the 256 per-thread totals
-    uint32_t loc[8], tot = 0;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      loc[i] = s_part[t * 8 + i];
-      tot += loc[i];
-    }
-    uint32_t incl = tot;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const uint32_t n = __shfl_down_sync(0xffffffffu, incl, o);
-      if (t + o < 32) incl += n;
-    }
-    uint32_t above = incl - tot;
-#pragma unroll
-    for (int i = 7; i >= 0; --i) {
-      s_part[t * 8 + i] = above;
-      above += loc[i];
-    }
-  }
-  __syncthreads();
-  const uint32_t above = s_part[t];
+  uint32_t total;
+  const uint32_t above = block_suffix_exclusive(sum, total, s_w);  // orders the reset
   if (above < k_rem && k_rem - above <= sum) {
     uint32_t r = k_rem - above;
     bool done = false;
 #pragma unroll
-    for (int i = 7; i >= 0; --i) {
+    for (int i = kMaxPer - 1; i >= 0; --i) {
       if (!done && static_cast<uint32_t>(i) < per) {
         if (c[i] >= r) {
           s_sel = Selection{t * per + i, r, c[i], 1u};
@@ -181,6 +151,262 @@ __device__ Selection select_bin(const uint32_t* hist, uint32_t nbins, uint32_t k
   const Selection s = s_sel;
   __syncthreads();
   return s;
+}
+
+// Exclusive block-wide prefix sum of one value per thread; also returns the
+// block total. Whole CTA of kBlock threads; s_w holds kBlock/32 words.
+template <int kBlock>
+__device__ __forceinline__ uint32_t block_exclusive(uint32_t v, uint32_t& total, uint32_t* s_w) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t incl = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t x = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += x;
+  }
+  __syncthreads();
+  if (lane == 31) s_w[warp] = incl;
+  __syncthreads();
+  uint32_t before = 0;
+  total = 0;
+  for (int w = 0; w < kBlock / 32; ++w) {
+    const uint32_t x = s_w[w];
+    before += w < warp ? x : 0u;
+    total += x;
+  }
+  return before + incl - v;
+}
+
+// ------------------------------------------------------------- 1 stream
+// The streaming pass as a stream_compact op. Pre-pass: every CTA histograms
+// the top 11 key bits of the first tile of its chunk (the tiles so sampled
+// are spread evenly over the vector), the histograms are merged, and after a
+// grid barrier every CTA derives the same lower bound B with about twice the
+// needed mass above it — or, when the candidates would not fit, chooses the
+// full-array mode and gathers none. Streaming: a = fmaf(γ,g,e) is written over
+// e and the coordinates with K_j >= B are selected (ordered candidates).
+template <typename GT>
+struct TopkCandOp {
+  const GT* g;
+  float* e;
+  float gamma;
+  uint32_t d, k, cand_cap;
+  uint32_t* hist;      // global sample histogram [kSampleBins]
+  uint32_t* bar_arrive;
+  uint32_t* bar_gen;
+  uint32_t* mode;      // published for the select kernel
+  uint64_t* lower_bound;
+  static constexpr uint32_t kGBytes = kTileElems * sizeof(GT);
+  static constexpr uint32_t kStageBytes = kGBytes + kTileElems * sizeof(float);
+  static constexpr bool kPrepass = true;
+  static constexpr int kSampleBins = efs::kSampleBins;
+  static constexpr int kSampleShift = 31 - kSampleBits;  // key bits below the sampled ones
+
+  __device__ __forceinline__ void fill(unsigned char* stage, uint32_t t, uint64_t* bar,
+                                       uint64_t policy) const {
+    tma_load_1d(stage, g + static_cast<size_t>(t) * kTileElems, kGBytes, bar, policy);
+    tma_load_1d(stage + kGBytes, e + static_cast<size_t>(t) * kTileElems,
+                kTileElems * sizeof(float), bar, policy);
+  }
+
+  __device__ __forceinline__ void accumulate(const unsigned char* stage, int warp, int lane, int v,
+                                             float (&x)[4]) const {
+    const GT* gs = reinterpret_cast<const GT*>(stage);
+    const float* es = reinterpret_cast<const float*>(stage + kGBytes);
+    const int local = warp * kSWarpElems + lane * 4 + v * 128;
+    GradVec<GT> gv;
+    if constexpr (sizeof(GT) == 4)
+      gv.v = *reinterpret_cast<const float4*>(gs + local);
+    else
+      gv.v = *reinterpret_cast<const uint2*>(gs + local);
+    const float4 ev = *reinterpret_cast<const float4*>(es + local);
+    x[0] = __fmaf_rn(gamma, gv[0], ev.x);
+    x[1] = __fmaf_rn(gamma, gv[1], ev.y);
+    x[2] = __fmaf_rn(gamma, gv[2], ev.z);
+    x[3] = __fmaf_rn(gamma, gv[3], ev.w);
+  }
+
+  __device__ void sample(const unsigned char* stage, uint32_t, int warp, int lane,
+                         uint32_t* s_hist) const {
+#pragma unroll
+    for (int v = 0; v < kSUnits; ++v) {
+      float x[4];
+      accumulate(stage, warp, lane, v, x);
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        hist_add_warp(s_hist, (__float_as_uint(x[j]) & 0x7fffffffu) >> kSampleShift, true);
+    }
+  }
+
+  __device__ void merge(const uint32_t* s_hist) const {
+    for (int b = threadIdx.x; b < kSampleBins; b += blockDim.x)
+      if (s_hist[b]) atomicAdd(&hist[b], s_hist[b]);
+  }
+
+  __device__ bool barrier(uint64_t limit_ns, uint32_t* error) const {
+    return grid_barrier(bar_arrive, bar_gen, limit_ns, error);
+  }
+
+  // Every CTA computes the same bound: each compute thread loads 16
+  // consecutive bins of the merged histogram (vector loads, all in flight
+  // together), a block suffix scan gives the sampled mass above each
+  // thread's bins, and the thread holding the target-th largest sample finds
+  // its bin; CTA 0 publishes the bound with the mode.
+  __device__ uint64_t choose() const {
+    constexpr int kPer = kSampleBins / kComputeThreads;
+    static_assert(kPer % 4 == 0 && kPer * kComputeThreads == kSampleBins, "sample bins");
+    __shared__ uint64_t s_bound;
+    __shared__ uint32_t s_bin, s_mass;
+    __shared__ uint32_t s_w[kStreamThreads / 32];
+    const int t = threadIdx.x;
+    uint32_t c[kPer];
+    uint32_t mine = 0;
+    if (t < kComputeThreads) {
+      const uint4* src = reinterpret_cast<const uint4*>(hist) + t * (kPer / 4);
+      uint4 v[kPer / 4];
+#pragma unroll
+      for (int q = 0; q < kPer / 4; ++q) v[q] = __ldcg(src + q);
+#pragma unroll
+      for (int q = 0; q < kPer / 4; ++q) {
+        c[4 * q] = v[q].x;
+        c[4 * q + 1] = v[q].y;
+        c[4 * q + 2] = v[q].z;
+        c[4 * q + 3] = v[q].w;
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < kPer; ++i) c[i] = 0;
+    }
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) mine += c[i];
+    if (t == 0) s_bin = 0xffffffffu;
+    uint32_t sampled;
+    const uint32_t above = block_suffix_exclusive(mine, sampled, s_w);  // orders the reset
+    const bool everything = sampled == d;
+    uint32_t target = k;
+    if (!everything) {
+      // 1.5x the expected sampled count above the k-th key, plus 32: many
+      // standard deviations of sampling noise; a miss costs the exact
+      // full-array fallback, never a wrong result
+      const double x = 1.5 * static_cast<double>(k) * sampled / d + 32.0;
+      target = x >= sampled ? sampled + 1 : static_cast<uint32_t>(x);
+    }
+    // the bin holding the target-th largest sample, and the sampled mass at
+    // or above it
+    if (target <= sampled && above < target && target - above <= mine) {
+      uint32_t run = above;
+#pragma unroll
+      for (int i = kPer - 1; i >= 0; --i) {
+        run += c[i];
+        if (run >= target && run - c[i] < target) {
+          s_bin = t * kPer + i;
+          s_mass = run;
+        }
+      }
+    }
+    __syncthreads();
+    if (t == 0) {
+      const bool found = s_bin != 0xffffffffu;
+      uint64_t bound = found ? static_cast<uint64_t>(s_bin) << (32 + kSampleShift) : 0ull;
+      const double expected =
+          found ? (everything ? s_mass : static_cast<double>(s_mass) * d / sampled)
+                : static_cast<double>(d);
+      uint32_t m = 0;
+      if (k == 0) {
+        bound = kSelectNone;
+      } else if (expected > 0.5 * cand_cap) {
+        m = 1;                // the candidates would not fit: full-array selection
+        bound = kSelectNone;  // and none gathered while streaming
+      }
+      s_bound = bound;
+      if (blockIdx.x == 0) {
+        *mode = m;
+        *lower_bound = bound;
+      }
+    }
+    __syncthreads();
+    return s_bound;
+  }
+
+  __device__ __forceinline__ void tile_smem(const unsigned char* stage, uint32_t t, int warp,
+                                            int lane, float (&a)[kSUnits][4],
+                                            uint32_t (&sel)[kSUnits], uint64_t bound) const {
+    const uint64_t first = stream_element_index(t, warp, 0, lane, 0);
+#pragma unroll
+    for (int v = 0; v < kSUnits; ++v) {
+      accumulate(stage, warp, lane, v, a[v]);
+      st_stream_f4(e + first + v * 128, make_float4(a[v][0], a[v][1], a[v][2], a[v][3]));
+      sel[v] = 0;
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        sel[v] |= (composite_key(a[v][j], first + v * 128 + j) >= bound ? 1u : 0u) << j;
+    }
+  }
+
+  __device__ __forceinline__ void tile_global(uint32_t t, int warp, int lane,
+                                              float (&a)[kSUnits][4],
+                                              uint32_t (&sel)[kSUnits], uint64_t bound) const {
+    const uint64_t first = stream_element_index(t, warp, 0, lane, 0);
+#pragma unroll
+    for (int v = 0; v < kSUnits; ++v) {
+      sel[v] = 0;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint64_t i = first + v * 128 + j;
+        a[v][j] = 0.0f;
+        if (i < d) {
+          const float x = __fmaf_rn(gamma, grad_scalar(g, i), e[i]);
+          e[i] = x;
+          a[v][j] = x;
+          sel[v] |= (composite_key(x, i) >= bound ? 1u : 0u) << j;
+        }
+      }
+    }
+  }
+};
+
+constexpr int kTkStages = 4;
+
+// Inputs the bulk copies cannot take (not 16-byte aligned): a = fmaf(γ,g,e)
+// written over e with plain loads, and the selection switched to the
+// full-array mode (block 0 runs after the sampling kernel on the stream).
+template <typename GT>
+__global__ void __launch_bounds__(kThreads)
+    topk_accumulate_plain_kernel(const GT* __restrict__ g, float* __restrict__ e, float gamma,
+                                 uint32_t d, TopkArgs args) {
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    *args.mode = 1;
+    *args.lower_bound = kSelectNone;
+  }
+  for (uint64_t i = static_cast<uint64_t>(blockIdx.x) * kThreads + threadIdx.x; i < d;
+       i += static_cast<uint64_t>(gridDim.x) * kThreads)
+    e[i] = __fmaf_rn(gamma, grad_scalar(g, i), e[i]);
+}
+
+// Reads the (mode, source length) a refine/finalize launch works on; the
+// streaming pass's flags decide whether the candidates are usable.
+struct SourceInfo {
+  uint32_t mode;   // 0: candidate list, 1: full array
+  uint32_t n;      // source length
+  bool failed;     // the streaming pass timed out: select nothing
+};
+
+__device__ __forceinline__ SourceInfo read_source(const TopkArgs& args, uint32_t d, uint32_t k) {
+  SourceInfo si;
+  const uint32_t flags = __ldcg(args.list_flags);
+  const uint32_t count = __ldcg(args.list_count);
+  si.failed = (flags & kDevErrTimeout) != 0;
+  si.mode = __ldcg(args.mode);
+  if (si.mode == 0 && ((flags & kDevErrOverflow) || count < k)) si.mode = 1;
+  si.n = si.mode == 0 ? count : d;
+  return si;
+}
+
+// Key of source element i: a candidate (index, value) or a coordinate of a.
+__device__ __forceinline__ uint64_t source_key(const TopkArgs& args, const float* a, uint32_t mode,
+                                               uint64_t i) {
+  if (mode == 0) return composite_key(__ldcg(args.list_val + i), __ldcg(args.list_idx + i));
+  return composite_key(__ldcg(a + i), i);
 }
 
 // Warp-aggregated append of the keys of the lanes with pred set.
@@ -199,88 +425,238 @@ __device__ __forceinline__ void warp_append(bool pred, uint64_t key, uint64_t* d
   }
 }
 
-__device__ __forceinline__ void refine_visit(uint64_t key, bool valid, uint64_t prefix,
-                                             int sh_prev, int sh, uint32_t nb, bool compact,
-                                             uint64_t* dst, uint32_t* dst_count,
-                                             uint32_t cap, uint32_t* s_hist) {
-  const bool match = valid && (key >> sh_prev) == prefix;
-  if (match) atomicAdd(&s_hist[(key >> sh) & (nb - 1)], 1u);
-  if (compact) warp_append(match, key, dst, dst_count, cap);
+// ------------------------------------------------------------- 2 select
+// Exact threshold by radix select, then the ordered compaction of K >= it.
+constexpr int kSelThreads = 1024;
+constexpr uint32_t kSmallCand = 48u * 1024u;  // magnitudes one CTA holds in shared memory
+constexpr uint32_t kSelSmem = kSmallCand * sizeof(uint32_t);
+
+// Writes the source elements [lo, hi) with key >= thr, in order, to the
+// outputs from position `base`, 4 consecutive elements per thread per block,
+// and zeroes the residual at each; returns the number written. Whole CTA.
+__device__ uint32_t write_selected(const TopkArgs& args, float* e, uint32_t mode, uint32_t lo,
+                                   uint32_t hi, uint64_t thr, uint32_t base, uint32_t k,
+                                   uint32_t* idx_out, float* val_out, bool& overflow,
+                                   uint32_t* s_w) {
+  const uint32_t start = base;
+  for (uint32_t b0 = lo; b0 < hi; b0 += 4 * kSelThreads) {
+    const uint32_t i0 = b0 + 4 * threadIdx.x;
+    uint32_t sel = 0, coord[4];
+    float val[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {  // all loads in flight before the scan
+      const bool in = i0 + j < hi;
+      coord[j] = in ? (mode == 0 ? __ldcg(args.list_idx + i0 + j) : i0 + j) : 0u;
+      val[j] = in ? (mode == 0 ? __ldcg(args.list_val + i0 + j) : __ldcg(e + i0 + j)) : 0.0f;
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (i0 + j < hi && composite_key(val[j], coord[j]) >= thr) sel |= 1u << j;
+    uint32_t block_total;
+    uint32_t pos = base + block_exclusive<kSelThreads>(__popc(sel), block_total, s_w);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      if (sel & (1u << j)) {
+        if (pos < k) {
+          idx_out[pos] = coord[j];
+          val_out[pos] = val[j];
+          e[coord[j]] = 0.0f;  // residual of a sent coordinate
+        } else {
+          overflow = true;
+        }
+        ++pos;
+      }
+    }
+    base += block_total;
+  }
+  return base - start;
 }
 
-template <bool kVec>
-__global__ void __launch_bounds__(kThreads)
-    topk_refine_kernel(const float* __restrict__ a, uint32_t d, uint32_t k, TopkArgs args) {
-  __shared__ uint32_t s_hist[kHistBins];
-  if (k == 0) {
-    if (blockIdx.x == 0 && threadIdx.x == 0) *args.threshold = 1ull << 63;  // selects nothing
+// One CTA resolves a short candidate list entirely in shared memory: the 31
+// magnitude bits of every candidate are loaded once; three digit levels
+// (bits 30..20, 19..10, 9..0) find the threshold magnitude T and how many of
+// the candidates equal to T are taken; equal magnitudes are taken in list
+// order, which is index order (the lowest-index tie rule); then the ordered
+// output is written.
+__device__ void select_small(const TopkArgs& args, float* e, uint32_t n, uint32_t k,
+                             uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                             uint32_t* s_mag, uint32_t* s_hist, uint32_t* s_w) {
+  __shared__ uint32_t s_last;
+  const int tid = threadIdx.x;
+  constexpr int kBatch = 8;  // loads in flight per thread
+  for (uint32_t i0 = tid; i0 < n; i0 += kBatch * kSelThreads) {
+    uint32_t v[kBatch];
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      const uint32_t i = i0 + j * kSelThreads;
+      v[j] = i < n ? __float_as_uint(__ldcg(args.list_val + i)) : 0u;
+    }
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      const uint32_t i = i0 + j * kSelThreads;
+      if (i < n) s_mag[i] = v[j] & 0x7fffffffu;
+    }
+  }
+  __syncthreads();
+  uint32_t prefix = 0, k_rem = k, n_in = n;
+  int shift = 31;
+  bool ok = true;
+  for (int l = 0; l < 3 && n_in != k_rem; ++l) {
+    const int sh = l == 0 ? 20 : l == 1 ? 10 : 0;
+    const uint32_t nb = 1u << (shift - sh);
+    for (uint32_t b = tid; b < nb; b += kSelThreads) s_hist[b] = 0;
+    __syncthreads();
+    // the magnitudes crowd into few bins: equal bins of a warp add once
+    for (uint32_t b0 = 0; b0 < n; b0 += 4 * kSelThreads) {  // uniform trip count
+      uint32_t m[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t i = b0 + j * kSelThreads + tid;
+        m[j] = i < n ? s_mag[i] : 0u;
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const bool in = b0 + j * kSelThreads + tid < n && (l == 0 || (m[j] >> shift) == prefix);
+        hist_add_warp(s_hist, (m[j] >> sh) & (nb - 1), in);
+      }
+    }
+    __syncthreads();
+    const Selection s = select_bin<kSelThreads, false>(s_hist, nb, k_rem, s_w);
+    if (!s.found) {
+      ok = false;
+      break;
+    }
+    prefix = (prefix << (shift - sh)) | s.bin;
+    k_rem = s.k_rem;
+    n_in = s.n_in;
+    shift = sh;
+  }
+  if (!ok) {
+    if (tid == 0) {
+      atomicOr(args.error, kDevErrBadInput);
+      *count_out = 0;
+    }
     return;
   }
-  Selection s = select_bin(args.hist, kHistBins, k);
-  bool ok = s.found != 0;
-  uint64_t prefix = s.bin;
-  uint32_t k_rem = s.k_rem, n_in = s.n_in;
-  int level = 0;
-  int src = -1;  // -1: scan all of a; 0/1: scan candidate buffer 0/1
-  uint32_t src_count = d;
+  // selection: magnitude above the final bucket, or in it; when the bucket
+  // (all 31 bits fixed) holds more equal magnitudes than are taken, only the
+  // first k_rem of them in list order, i.e. up to list position s_last
+  const bool ties = n_in != k_rem;
+  if (tid == 0) s_last = 0xffffffffu;
+  if (ties) {
+    const uint32_t per = (n + kSelThreads - 1) / kSelThreads;
+    const uint32_t lo = tid * per < n ? tid * per : n, hi = lo + per < n ? lo + per : n;
+    uint32_t cnt = 0;
+    for (uint32_t i = lo; i < hi; ++i) cnt += s_mag[i] == prefix ? 1u : 0u;
+    uint32_t total;
+    const uint32_t before = block_exclusive<kSelThreads>(cnt, total, s_w);
+    if (before < k_rem && k_rem <= before + cnt) {
+      uint32_t r = k_rem - before;
+      for (uint32_t i = lo; i < hi; ++i)
+        if (s_mag[i] == prefix && --r == 0) {
+          s_last = i;
+          break;
+        }
+    }
+  }
+  __syncthreads();
+  const uint32_t last = s_last;
+  bool overflow = false;
+  uint32_t base = 0;
+  for (uint32_t b0 = 0; b0 < n; b0 += 4 * kSelThreads) {
+    const uint32_t i0 = b0 + 4 * tid;
+    uint32_t coord[4], sel = 0;
+    float val[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {  // loads in flight before the scan
+      const bool in = i0 + j < n;
+      coord[j] = in ? __ldcg(args.list_idx + i0 + j) : 0u;
+      val[j] = in ? __ldcg(args.list_val + i0 + j) : 0.0f;
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      if (i0 + j >= n) continue;
+      const uint32_t m = s_mag[i0 + j];
+      const uint32_t top = m >> shift;
+      const bool take = top > prefix || (top == prefix && (!ties || i0 + j <= last));
+      sel |= (take ? 1u : 0u) << j;
+    }
+    uint32_t block_total;
+    uint32_t pos = base + block_exclusive<kSelThreads>(__popc(sel), block_total, s_w);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      if (sel & (1u << j)) {
+        if (pos < k) {
+          idx_out[pos] = coord[j];
+          val_out[pos] = val[j];
+          e[coord[j]] = 0.0f;  // residual of a sent coordinate
+        } else {
+          overflow = true;
+        }
+        ++pos;
+      }
+    }
+    base += block_total;
+  }
+  if (tid == 0) *count_out = base < k ? base : k;
+  if (__syncthreads_or(overflow) && tid == 0) atomicOr(args.error, kDevErrOverflow);
+}
 
-  while (ok && n_in != k_rem && level < kHistLevels - 1) {
+// Radix select of the k-th largest composite key of the source across the
+// grid: merged global histograms, bounded grid barriers, candidate compaction
+// into key buffers once a bucket fits.
+__device__ uint64_t radix_threshold_grid(const TopkArgs& args, const float* a,
+                                         const SourceInfo& si, uint32_t k, uint32_t* s_hist,
+                                         uint32_t* s_w, bool& ok) {
+  ok = true;
+  uint64_t prefix = 0;
+  uint32_t k_rem = k, n_in = si.n;
+  int level = -1;
+  int src = -1;  // -1: the source; 0/1: key buffer 0/1
+  uint32_t src_count = si.n;
+  Selection s{};
+  const uint64_t stride = static_cast<uint64_t>(gridDim.x) * kSelThreads;
+  do {
     ++level;
-    const int sh_prev = digit_shift(level - 1), sh = digit_shift(level);
+    const int sh = digit_shift(level);
+    const int sh_prev = level == 0 ? 63 : digit_shift(level - 1);
     const int bits = sh_prev - sh;
     const uint32_t nb = 1u << bits;
-    const bool compact = n_in <= args.cand_cap;
+    const bool compact = level > 0 && n_in <= args.cand_cap;
     const int dst = (src == 0) ? 1 : 0;
     uint64_t* dst_buf = dst ? args.cand1 : args.cand0;
     uint32_t* dst_count = args.cand_count + level;
-    for (uint32_t b = threadIdx.x; b < nb; b += kThreads) s_hist[b] = 0;
+    for (uint32_t b = threadIdx.x; b < nb; b += kSelThreads) s_hist[b] = 0;
     __syncthreads();
-
-    if (src < 0) {
-      const uint64_t units = (static_cast<uint64_t>(d) + 3) / 4;
-      const uint64_t full_units = d / 4;
-      for (uint64_t base = static_cast<uint64_t>(blockIdx.x) * kThreads; base < units;
-           base += static_cast<uint64_t>(gridDim.x) * kThreads) {
-        const uint64_t u = base + threadIdx.x;
-        float x[4];
-        bool valid[4];
-        if (kVec && u < full_units) {
-          const float4 q = __ldcg(reinterpret_cast<const float4*>(a) + u);
-          x[0] = q.x; x[1] = q.y; x[2] = q.z; x[3] = q.w;
-          valid[0] = valid[1] = valid[2] = valid[3] = true;
-        } else {
+    const uint64_t* keys = src == 0 ? args.cand0 : args.cand1;
+    constexpr int kBatch = 4;  // keys in flight per thread
+    for (uint64_t base = static_cast<uint64_t>(blockIdx.x) * kSelThreads; base < src_count;
+         base += kBatch * stride) {
+      uint64_t key[kBatch];
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const uint64_t i = u * 4 + j;
-            valid[j] = i < d;
-            x[j] = valid[j] ? __ldcg(a + i) : 0.0f;
-          }
-        }
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-          refine_visit(composite_key(x[j], u * 4 + j), valid[j], prefix, sh_prev, sh, nb,
-                       compact, dst_buf, dst_count, args.cand_cap, s_hist);
+      for (int j = 0; j < kBatch; ++j) {
+        const uint64_t i = base + j * stride + threadIdx.x;
+        key[j] = 0;
+        if (i < src_count) key[j] = src < 0 ? source_key(args, a, si.mode, i) : __ldcg(keys + i);
       }
-    } else {
-      const uint64_t* src_buf = src ? args.cand1 : args.cand0;
-      for (uint64_t base = static_cast<uint64_t>(blockIdx.x) * kThreads; base < src_count;
-           base += static_cast<uint64_t>(gridDim.x) * kThreads) {
-        const uint64_t i = base + threadIdx.x;
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const uint64_t i = base + j * stride + threadIdx.x;
         const bool valid = i < src_count;
-        const uint64_t key = valid ? __ldcg(src_buf + i) : 0ull;
-        refine_visit(key, valid, prefix, sh_prev, sh, nb, compact, dst_buf, dst_count,
-                     args.cand_cap, s_hist);
+        const bool match = valid && (level == 0 || (key[j] >> sh_prev) == prefix);
+        hist_add_warp(s_hist, static_cast<uint32_t>(key[j] >> sh) & (nb - 1), match);
+        if (compact) warp_append(match, key[j], dst_buf, dst_count, args.cand_cap);
       }
     }
     __syncthreads();
     uint32_t* gh = args.hist + level * kHistBins;
-    for (uint32_t b = threadIdx.x; b < nb; b += kThreads)
+    for (uint32_t b = threadIdx.x; b < nb; b += kSelThreads)
       if (s_hist[b]) atomicAdd(&gh[b], s_hist[b]);
     if (!grid_barrier(args.bar_arrive, args.bar_gen, args.wait_limit_ns, args.error)) {
       ok = false;
       break;
     }
-    s = select_bin(gh, nb, k_rem);
+    s = select_bin<kSelThreads, true>(gh, nb, k_rem, s_w);
     if (!s.found) {
       ok = false;
       break;
@@ -293,59 +669,109 @@ __global__ void __launch_bounds__(kThreads)
       src = dst;
       src_count = n_prev;
     }
+  } while (n_in != k_rem && level < kHistLevels - 1);
+  // an unfound bin or an unresolved rank means the histograms disagree with
+  // the data; a grid barrier latches its own timeout
+  if (!s.found || n_in != k_rem) {
+    if (threadIdx.x == 0 && blockIdx.x == 0) atomicOr(args.error, kDevErrBadInput);
+    ok = false;
   }
-  if (blockIdx.x == 0 && threadIdx.x == 0) {
-    // an unfound bin or an unresolved rank means the histograms disagree
-    // with the data (e changed during the call); the barrier latches its own
-    if (!s.found || n_in != k_rem) atomicOr(args.error, kDevErrBadInput);
-    ok = ok && n_in == k_rem;
-    *args.threshold = ok ? (prefix << digit_shift(level)) : (1ull << 63);
-  }
+  return prefix << digit_shift(level);
 }
 
-// ------------------------------------------------------------------ pass Z
-template <bool kVec>
-__global__ void __launch_bounds__(kThreads)
-    topk_select_kernel(float* __restrict__ e, uint32_t d, const uint64_t* __restrict__ threshold,
-                       uint32_t k, uint32_t* __restrict__ idx_out, float* __restrict__ val_out,
-                       uint32_t* __restrict__ count_out, ScanCtx ctx) {
-  const uint32_t tile = blockIdx.x;
-  const uint64_t thr = __ldcg(threshold);
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const uint64_t first = element_index(tile, warp, 0, lane, 0);
-  float a[kUnits][4];
-  uint32_t sel[kUnits];
-  const bool full_tile = static_cast<uint64_t>(tile + 1) * kTileElems <= d;
-  if (kVec && full_tile) {
-    float4 q[kUnits];
-#pragma unroll
-    for (int v = 0; v < kUnits; ++v) q[v] = __ldcg(reinterpret_cast<const float4*>(e + first + v * 128));
-#pragma unroll
-    for (int v = 0; v < kUnits; ++v) {
-      a[v][0] = q[v].x; a[v][1] = q[v].y; a[v][2] = q[v].z; a[v][3] = q[v].w;
+__global__ void __launch_bounds__(kSelThreads, 1)
+    topk_select_kernel(float* __restrict__ e, uint32_t d, uint32_t k,
+                       uint32_t* __restrict__ idx_out, float* __restrict__ val_out,
+                       uint32_t* __restrict__ count_out, TopkArgs args) {
+  extern __shared__ __align__(16) uint32_t s_mag[];
+  __shared__ uint32_t s_hist[kHistBins];
+  __shared__ uint32_t s_w[kSelThreads / 32];
+  const SourceInfo si = read_source(args, d, k);
+  if (k == 0 || si.failed) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+      if (si.failed) atomicOr(args.error, kDevErrTimeout);
+      *count_out = 0;
     }
-  } else {
-#pragma unroll
-    for (int v = 0; v < kUnits; ++v)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const uint64_t i = first + v * 128 + j;
-        a[v][j] = i < d ? __ldcg(e + i) : 0.0f;
-      }
+    return;
   }
+  if (si.mode == 0 && si.n <= kSmallCand) {
+    if (blockIdx.x == 0) select_small(args, e, si.n, k, idx_out, val_out, count_out, s_mag, s_hist, s_w);
+    return;
+  }
+  bool ok = true;
+  const uint64_t thr = radix_threshold_grid(args, e, si, k, s_hist, s_w, ok);
+  if (!ok) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) *count_out = 0;
+    return;
+  }
+  // ordered compaction across the grid: chunk counts, then positions
+  const uint32_t G = gridDim.x, c = blockIdx.x;
+  const uint32_t lo = static_cast<uint32_t>(static_cast<uint64_t>(c) * si.n / G);
+  const uint32_t hi = static_cast<uint32_t>(static_cast<uint64_t>(c + 1) * si.n / G);
+  uint32_t mine = 0;
+  for (uint32_t i0 = lo + threadIdx.x; i0 < hi; i0 += 4 * kSelThreads) {
+    uint64_t key[4];
 #pragma unroll
-  for (int v = 0; v < kUnits; ++v) {
-    sel[v] = 0;
+    for (int j = 0; j < 4; ++j) {  // loads in flight together
+      const uint32_t i = i0 + j * kSelThreads;
+      key[j] = i < hi ? source_key(args, e, si.mode, i) : 0ull;
+    }
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const uint64_t i = first + v * 128 + j;
-      if (i < d && composite_key(a[v][j], i) >= thr) {
-        sel[v] |= 1u << j;
-        e[i] = 0.0f;  // residual of a sent coordinate
+    for (int j = 0; j < 4; ++j) mine += (i0 + j * kSelThreads < hi && key[j] >= thr) ? 1u : 0u;
+  }
+  uint32_t total;
+  block_exclusive<kSelThreads>(mine, total, s_w);
+  if (threadIdx.x == 0)
+    st_relaxed_u64(args.chunk_sums + c, (static_cast<uint64_t>(args.epoch) << 32) | total);
+  uint32_t base = 0;
+  {
+    const uint64_t t0 = global_timer_ns();
+    uint32_t it = 0;
+    while (true) {
+      uint32_t part = 0;
+      bool present = true;
+      for (uint32_t q = threadIdx.x; q < c; q += kSelThreads) {
+        const uint64_t w = ld_relaxed_u64(args.chunk_sums + q);
+        if (static_cast<uint32_t>(w >> 32) == args.epoch)
+          part += static_cast<uint32_t>(w);
+        else
+          present = false;
       }
+      const bool all_present = __syncthreads_and(present);
+      uint32_t sum;
+      block_exclusive<kSelThreads>(part, sum, s_w);
+      if (all_present) {
+        base = sum;
+        break;
+      }
+      const bool out_of_time = ++it > (1u << 26) || global_timer_ns() - t0 > args.wait_limit_ns;
+      if (__syncthreads_or(out_of_time)) {
+        if (threadIdx.x == 0) atomicOr(args.error, kDevErrTimeout);
+        return;
+      }
+      __nanosleep(64);
     }
   }
-  compact_tile(ctx, tile, sel, a, idx_out, val_out, count_out, k);
+  bool overflow = false;
+  const uint32_t written =
+      write_selected(args, e, si.mode, lo, hi, thr, base, k, idx_out, val_out, overflow, s_w);
+  if (c == G - 1 && threadIdx.x == 0) {
+    const uint32_t end = base + written;
+    *count_out = end < k ? end : k;
+  }
+  if (__syncthreads_or(overflow) && threadIdx.x == 0) atomicOr(args.error, kDevErrOverflow);
+}
+
+template <typename GT>
+int tk_stream_blocks_per_sm() {
+  const void* fn = reinterpret_cast<const void*>(&stream_compact_kernel<TopkCandOp<GT>, kTkStages>);
+  const uint32_t smem = StreamLayout<TopkCandOp<GT>, kTkStages>::kSmem;
+  int n = 0;
+  if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, kStreamThreads, smem) != cudaSuccess)
+    n = 0;
+  cudaGetLastError();
+  return n;
 }
 
 template <typename GT>
@@ -356,56 +782,79 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
   cudaError_t err = cudaMemsetAsync(ws.base + kOffTopkReset, 0, kTopkResetBytes, ws.stream);
   if (err != cudaSuccess) return err;
 
-  const bool e_vec = reinterpret_cast<uintptr_t>(e) % 16 == 0;
-  const bool vec = e_vec && reinterpret_cast<uintptr_t>(g) % (4 * sizeof(GT)) == 0;
-  const uint32_t grid_a = static_cast<uint32_t>(
-      tiles < static_cast<uint32_t>(dev.sm_count * 4) ? tiles : dev.sm_count * 4);
-  uint32_t* hist = ws.u32(kOffHist);
-  if (vec)
-    topk_accumulate_kernel<GT, true><<<grid_a, kThreads, 0, ws.stream>>>(g, e, gamma, d, tiles, hist);
-  else
-    topk_accumulate_kernel<GT, false><<<grid_a, kThreads, 0, ws.stream>>>(g, e, gamma, d, tiles, hist);
-  count_launch();
-  if ((err = cudaGetLastError()) != cudaSuccess) return err;
-
   TopkArgs args;
-  args.hist = hist;
-  args.cand0 = ws.cand(0);
-  args.cand1 = ws.cand(1);
+  args.hist = ws.u32(kOffHist);
+  args.cand0 = ws.cand(1);
+  args.cand1 = ws.cand(2);
+  args.list_idx = reinterpret_cast<uint32_t*>(ws.cand(0));
+  args.list_val = reinterpret_cast<float*>(args.list_idx + ws.cand_cap);
   args.cand_count = ws.u32(kOffCandCount);
   args.cand_cap = ws.cand_cap;
   args.threshold = ws.u64(kOffThreshold);
+  args.lower_bound = ws.u64(kOffTkLowerBound);
+  args.mode = ws.u32(kOffTkMode);
+  args.sample_done = ws.u32(kOffTkSampleDone);
+  args.list_count = ws.u32(kOffTkListCount);
+  args.list_flags = ws.u32(kOffTkListFlags);
   args.bar_arrive = ws.u32(kOffBarArrive);
   args.bar_gen = ws.u32(kOffBarGen);
   args.error = ws.u32(kOffError);
+  args.chunk_sums = ws.chunks();
   args.wait_limit_ns = wait_limit_ns();
-  const float* a = e;
-  void* params[] = {(void*)&a, (void*)&d, (void*)&k, (void*)&args};
-  const void* fn = e_vec ? reinterpret_cast<const void*>(&topk_refine_kernel<true>)
-                         : reinterpret_cast<const void*>(&topk_refine_kernel<false>);
-  err = cudaLaunchCooperativeKernel(fn, dim3(dev.refine_blocks), dim3(kThreads), params, 0,
-                                    ws.stream);
-  count_launch();
-  if (err != cudaSuccess) return err;
 
-  const ScanCtx ctx = next_scan_ctx(ws, tiles);
-  if (e_vec)
-    topk_select_kernel<true><<<tiles, kThreads, 0, ws.stream>>>(e, d, args.threshold, k, idx_out,
-                                                                val_out, count_out, ctx);
-  else
-    topk_select_kernel<false><<<tiles, kThreads, 0, ws.stream>>>(e, d, args.threshold, k, idx_out,
-                                                                 val_out, count_out, ctx);
+  // 1 stream (sample pre-pass + candidates). The bulk copies need 16-byte
+  // aligned g and e; otherwise a plain pass writes a and the selection runs in
+  // the full-array mode.
+  ScanCtx ctx = next_scan_ctx(ws, tiles);
+  ctx.error = args.list_flags;
+  const int per_sm = sizeof(GT) == 4 ? dev.tk_stream_per_sm_f32 : dev.tk_stream_per_sm_bf16;
+  const bool streamable = reinterpret_cast<uintptr_t>(e) % 16 == 0 &&
+                          reinterpret_cast<uintptr_t>(g) % 16 == 0 && per_sm > 0;
+  if (streamable) {
+    TopkCandOp<GT> op{g, e, gamma, d, k, ws.cand_cap, ws.u32(kOffSampleHist),
+                      args.bar_arrive, args.bar_gen, args.mode, args.lower_bound};
+    uint32_t slots = static_cast<uint32_t>(per_sm * dev.sm_count);
+    if (slots > kMaxChunks) slots = kMaxChunks;
+    const uint32_t grid = tiles < slots ? tiles : slots;
+    uint32_t cap = ws.cand_cap;
+    StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks()};
+    void* params[] = {&op, &d, &args.list_idx, &args.list_val, &args.list_count, &cap, &ctx, &sa};
+    err = cudaLaunchCooperativeKernel(
+        reinterpret_cast<const void*>(&stream_compact_kernel<TopkCandOp<GT>, kTkStages>),
+        dim3(grid), dim3(kStreamThreads), params, StreamLayout<TopkCandOp<GT>, kTkStages>::kSmem,
+        ws.stream);
+    count_launch();
+    if (err != cudaSuccess) return err;
+  } else {
+    const uint32_t grid = tiles < static_cast<uint32_t>(dev.sm_count * 8)
+                              ? tiles : static_cast<uint32_t>(dev.sm_count * 8);
+    topk_accumulate_plain_kernel<GT><<<grid, kThreads, 0, ws.stream>>>(g, e, gamma, d, args);
+    count_launch();
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  }
+  // 2 select
+  args.epoch = next_scan_ctx(ws, 1).epoch;
+  void* params[] = {(void*)&e, (void*)&d, (void*)&k, (void*)&idx_out, (void*)&val_out,
+                    (void*)&count_out, (void*)&args};
+  uint32_t grid = static_cast<uint32_t>(dev.refine_blocks);
+  if (grid > kMaxChunks) grid = kMaxChunks;
+  err = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(&topk_select_kernel),
+                                    dim3(grid), dim3(kSelThreads), params, kSelSmem, ws.stream);
   count_launch();
-  return cudaGetLastError();
+  return err;
 }
 
 }  // namespace
 
-int topk_refine_blocks_per_sm() {
-  int a = 0, b = 0;
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&a, topk_refine_kernel<true>, kThreads, 0);
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, topk_refine_kernel<false>, kThreads, 0);
-  return a < b ? a : b;
+void topk_init_device(DeviceInfo& info) {
+  int a = 0;
+  cudaFuncSetAttribute(topk_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSelSmem);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&a, topk_select_kernel, kSelThreads, kSelSmem);
+  info.refine_blocks = a * info.sm_count;
+  info.finalize_blocks = info.refine_blocks;
+  info.tk_stream_per_sm_f32 = tk_stream_blocks_per_sm<float>();
+  info.tk_stream_per_sm_bf16 = tk_stream_blocks_per_sm<uint16_t>();
+  cudaGetLastError();
 }
 
 uint32_t topk_candidate_capacity(uint64_t d) {
