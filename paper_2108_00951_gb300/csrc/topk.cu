@@ -472,17 +472,20 @@ __device__ uint32_t write_selected(const TopkArgs& args, float* e, uint32_t mode
   return base - start;
 }
 
-// One CTA resolves a short candidate list entirely in shared memory: the 31
-// magnitude bits of every candidate are loaded once; three digit levels
-// (bits 30..20, 19..10, 9..0) find the threshold magnitude T and how many of
-// the candidates equal to T are taken; equal magnitudes are taken in list
-// order, which is index order (the lowest-index tie rule); then the ordered
-// output is written.
+// One CTA resolves a short candidate list entirely in shared memory: the
+// value bits of every candidate are loaded once; three digit levels of the
+// magnitude (bits 30..20, 19..10, 9..0) find the threshold magnitude T and
+// how many of the candidates equal to T are taken; equal magnitudes are taken
+// in list order, which is index order (the lowest-index tie rule); then the
+// ordered output is written.
+constexpr int kOutSlices = 8;  // list positions per thread per output round
+
 __device__ void select_small(const TopkArgs& args, float* e, uint32_t n, uint32_t k,
                              uint32_t* idx_out, float* val_out, uint32_t* count_out,
-                             uint32_t* s_mag, uint32_t* s_hist, uint32_t* s_w) {
+                             uint32_t* s_val, uint32_t* s_hist, uint32_t* s_w) {
   __shared__ uint32_t s_last;
-  const int tid = threadIdx.x;
+  __shared__ uint32_t s_cnt[kOutSlices * (kSelThreads / 32)];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int kBatch = 8;  // loads in flight per thread
   for (uint32_t i0 = tid; i0 < n; i0 += kBatch * kSelThreads) {
     uint32_t v[kBatch];
@@ -494,7 +497,7 @@ __device__ void select_small(const TopkArgs& args, float* e, uint32_t n, uint32_
 #pragma unroll
     for (int j = 0; j < kBatch; ++j) {
       const uint32_t i = i0 + j * kSelThreads;
-      if (i < n) s_mag[i] = v[j] & 0x7fffffffu;
+      if (i < n) s_val[i] = v[j];
     }
   }
   __syncthreads();
@@ -506,18 +509,32 @@ __device__ void select_small(const TopkArgs& args, float* e, uint32_t n, uint32_
     const uint32_t nb = 1u << (shift - sh);
     for (uint32_t b = tid; b < nb; b += kSelThreads) s_hist[b] = 0;
     __syncthreads();
-    // the magnitudes crowd into few bins: equal bins of a warp add once
-    for (uint32_t b0 = 0; b0 < n; b0 += 4 * kSelThreads) {  // uniform trip count
-      uint32_t m[4];
+    if (l == 0) {
+      // every candidate, crowded into few bins: equal bins of a warp add once
+      for (uint32_t b0 = 0; b0 < n; b0 += 4 * kSelThreads) {  // uniform trip count
+        uint32_t m[4];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const uint32_t i = b0 + j * kSelThreads + tid;
-        m[j] = i < n ? s_mag[i] : 0u;
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t i = b0 + j * kSelThreads + tid;
+          m[j] = i < n ? s_val[i] & 0x7fffffffu : 0u;
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          hist_add_warp(s_hist, (m[j] >> sh) & (nb - 1), b0 + j * kSelThreads + tid < n);
       }
+    } else {
+      // only the candidates in the chosen bin, spread over its sub-bins
+      for (uint32_t b0 = 0; b0 < n; b0 += 4 * kSelThreads) {
+        uint32_t m[4];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const bool in = b0 + j * kSelThreads + tid < n && (l == 0 || (m[j] >> shift) == prefix);
-        hist_add_warp(s_hist, (m[j] >> sh) & (nb - 1), in);
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t i = b0 + j * kSelThreads + tid;
+          m[j] = i < n ? s_val[i] & 0x7fffffffu : 0u;
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if (b0 + j * kSelThreads + tid < n && (m[j] >> shift) == prefix)
+            atomicAdd(&s_hist[(m[j] >> sh) & (nb - 1)], 1u);
       }
     }
     __syncthreads();
@@ -547,13 +564,13 @@ __device__ void select_small(const TopkArgs& args, float* e, uint32_t n, uint32_
     const uint32_t per = (n + kSelThreads - 1) / kSelThreads;
     const uint32_t lo = tid * per < n ? tid * per : n, hi = lo + per < n ? lo + per : n;
     uint32_t cnt = 0;
-    for (uint32_t i = lo; i < hi; ++i) cnt += s_mag[i] == prefix ? 1u : 0u;
+    for (uint32_t i = lo; i < hi; ++i) cnt += (s_val[i] & 0x7fffffffu) == prefix ? 1u : 0u;
     uint32_t total;
     const uint32_t before = block_exclusive<kSelThreads>(cnt, total, s_w);
     if (before < k_rem && k_rem <= before + cnt) {
       uint32_t r = k_rem - before;
       for (uint32_t i = lo; i < hi; ++i)
-        if (s_mag[i] == prefix && --r == 0) {
+        if ((s_val[i] & 0x7fffffffu) == prefix && --r == 0) {
           s_last = i;
           break;
         }
@@ -561,42 +578,58 @@ __device__ void select_small(const TopkArgs& args, float* e, uint32_t n, uint32_
   }
   __syncthreads();
   const uint32_t last = s_last;
+  // Output rounds of kOutSlices * kSelThreads list positions. Slice j of a
+  // round holds the positions b0 + j * kSelThreads + tid, so list order is
+  // (slice, warp, lane) order: one scan over the per-(slice, warp) counts
+  // gives every warp's offset, a ballot the lane's.
+  const uint32_t lt = lanemask_lt();
   bool overflow = false;
   uint32_t base = 0;
-  for (uint32_t b0 = 0; b0 < n; b0 += 4 * kSelThreads) {
-    const uint32_t i0 = b0 + 4 * tid;
-    uint32_t coord[4], sel = 0;
-    float val[4];
+  for (uint32_t b0 = 0; b0 < n; b0 += kOutSlices * kSelThreads) {  // uniform trip count
+    uint32_t sel = 0;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {  // loads in flight before the scan
-      const bool in = i0 + j < n;
-      coord[j] = in ? __ldcg(args.list_idx + i0 + j) : 0u;
-      val[j] = in ? __ldcg(args.list_val + i0 + j) : 0.0f;
+    for (int j = 0; j < kOutSlices; ++j) {
+      const uint32_t i = b0 + j * kSelThreads + tid;
+      if (i < n) {
+        const uint32_t m = s_val[i] & 0x7fffffffu;
+        const uint32_t top = m >> shift;
+        const bool take = top > prefix || (top == prefix && (!ties || i <= last));
+        sel |= (take ? 1u : 0u) << j;
+      }
     }
+    uint32_t coord[kOutSlices];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      if (i0 + j >= n) continue;
-      const uint32_t m = s_mag[i0 + j];
-      const uint32_t top = m >> shift;
-      const bool take = top > prefix || (top == prefix && (!ties || i0 + j <= last));
-      sel |= (take ? 1u : 0u) << j;
+    for (int j = 0; j < kOutSlices; ++j)  // the indices of the taken, all in flight
+      coord[j] = (sel >> j) & 1u ? __ldcg(args.list_idx + b0 + j * kSelThreads + tid) : 0u;
+#pragma unroll
+    for (int j = 0; j < kOutSlices; ++j) {
+      const uint32_t bal = __ballot_sync(0xffffffffu, (sel >> j) & 1u);
+      if (lane == 0) s_cnt[j * (kSelThreads / 32) + warp] = __popc(bal);
     }
-    uint32_t block_total;
-    uint32_t pos = base + block_exclusive<kSelThreads>(__popc(sel), block_total, s_w);
+    __syncthreads();
+    constexpr uint32_t kCnt = kOutSlices * (kSelThreads / 32);
+    static_assert(kCnt <= static_cast<uint32_t>(kSelThreads), "one count per thread");
+    const uint32_t mine = static_cast<uint32_t>(tid) < kCnt ? s_cnt[tid] : 0u;
+    uint32_t round_total;
+    const uint32_t off = block_exclusive<kSelThreads>(mine, round_total, s_w);
+    if (static_cast<uint32_t>(tid) < kCnt) s_cnt[tid] = off;
+    __syncthreads();
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      if (sel & (1u << j)) {
+    for (int j = 0; j < kOutSlices; ++j) {
+      const uint32_t bal = __ballot_sync(0xffffffffu, (sel >> j) & 1u);
+      if ((sel >> j) & 1u) {
+        const uint32_t pos = base + s_cnt[j * (kSelThreads / 32) + warp] + __popc(bal & lt);
         if (pos < k) {
           idx_out[pos] = coord[j];
-          val_out[pos] = val[j];
+          val_out[pos] = __uint_as_float(s_val[b0 + j * kSelThreads + tid]);
           e[coord[j]] = 0.0f;  // residual of a sent coordinate
         } else {
           overflow = true;
         }
-        ++pos;
       }
     }
-    base += block_total;
+    base += round_total;
+    __syncthreads();  // s_cnt is rewritten by the next round
   }
   if (tid == 0) *count_out = base < k ? base : k;
   if (__syncthreads_or(overflow) && tid == 0) atomicOr(args.error, kDevErrOverflow);
