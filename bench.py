@@ -97,6 +97,13 @@ def reduce_timing(dist, seconds: float, units: float, device=None):
     return float(t.item()), float(u.item())
 
 
+def replica_workload(w, rank: int):
+    """The workload a rank simulates: every rank runs its own n workers (a
+    replica), on gradients drawn from a seed of its own."""
+    from paper_2108_00951_gb300 import workloads
+    return workloads.Workload(**{**w.__dict__, "seed": w.seed + 1000 * rank})
+
+
 def barrier(dist, device=None):
     if dist is not None:
         if device is not None and device.type == "cuda":
@@ -237,8 +244,7 @@ def run_ours(args):
     w = workloads.BY_NAME[args.workload]
     d, n, gamma = w.d, w.n, w.gamma
     k = w.topk_values()[0]
-    # every rank simulates its own n workers (replica); seeds differ per rank
-    wr = workloads.Workload(**{**w.__dict__, "seed": w.seed + 1000 * rank})
+    wr = replica_workload(w, rank)
     batches = [[workloads.gradient(wr, i, b, device=dev) for i in range(n)] for b in range(2)]
     lam = (workloads.density_lambda(wr, batches[0][0], w.density) if w.density is not None
            else w.lambdas[0])
