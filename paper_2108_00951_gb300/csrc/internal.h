@@ -16,12 +16,11 @@ constexpr size_t kOffError = 8;         // uint32: latched device error bits
 constexpr size_t kOffTopkReset = 16;    // start of the region cleared at each Top-k call
 constexpr size_t kOffBarArrive = 16;    // uint32: grid-barrier arrivals
 constexpr size_t kOffCandCount = 20;    // uint32[6]: refine-level candidate counts
-constexpr size_t kOffThreshold = 48;    // uint64: Top-k composite-key threshold
 constexpr size_t kOffTkLowerBound = 56; // uint64: sampled lower bound of the candidates' keys
 constexpr size_t kOffTkMode = 64;       // uint32: 0 candidates, 1 full array
-constexpr size_t kOffTkSampleDone = 68; // uint32: sampling CTAs finished
 constexpr size_t kOffTkListCount = 72;  // uint32: candidates emitted by the streaming pass
 constexpr size_t kOffTkListFlags = 76;  // uint32: that pass's latched bits (overflow, timeout)
+constexpr size_t kOffTkSelect = 128;    // uint32[5]: short-list threshold published by CTA 0
 constexpr size_t kOffHist = 256;        // uint32[6][2048] refine levels 0..5, then the sample
 constexpr int kHistLevels = 6;
 constexpr int kHistBins = 2048;

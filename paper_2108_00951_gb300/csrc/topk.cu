@@ -56,10 +56,9 @@ struct TopkArgs {
   float* list_val;
   uint32_t* cand_count;  // [kHistLevels]
   uint32_t cand_cap;
-  uint64_t* threshold;
   uint64_t* lower_bound;
   uint32_t* mode;        // 0: candidates, 1: full array
-  uint32_t* sample_done;
+  uint32_t* sel;         // small-list threshold: flag (1 found, 2 failed), prefix, shift, ties, last
   uint32_t* list_count;
   uint32_t* list_flags;
   uint32_t* bar_arrive;
@@ -472,20 +471,31 @@ __device__ uint32_t write_selected(const TopkArgs& args, float* e, uint32_t mode
   return base - start;
 }
 
-// One CTA resolves a short candidate list entirely in shared memory: the
-// value bits of every candidate are loaded once; three digit levels of the
-// magnitude (bits 30..20, 19..10, 9..0) find the threshold magnitude T and
-// how many of the candidates equal to T are taken; equal magnitudes are taken
-// in list order, which is index order (the lowest-index tie rule); then the
-// ordered output is written.
-constexpr int kOutSlices = 8;  // list positions per thread per output round
+// A short candidate list (n <= kSmallCand) is resolved in two parts.
+// CTA 0 finds the threshold in shared memory: the magnitudes of every
+// candidate are loaded once; three digit levels (bits 30..20, 19..10, 9..0)
+// find the threshold magnitude T and how many of the candidates equal to T
+// are taken; equal magnitudes are taken in list order, which is index order
+// (the lowest-index tie rule), i.e. up to list position `last`. It publishes
+// (T's digits, ties, last) behind a flag. Then every slice CTA writes the
+// selected pairs of its kSliceElems-position slice of the list in order,
+// zeroing the residual at each: it loads its slice while CTA 0 works,
+// publishes its slice's count, and sums the earlier slices' counts.
+constexpr uint32_t kSliceElems = 4 * kSelThreads;  // list positions per slice CTA
 
-__device__ void select_small(const TopkArgs& args, float* e, uint32_t n, uint32_t k,
-                             uint32_t* idx_out, float* val_out, uint32_t* count_out,
-                             uint32_t* s_val, uint32_t* s_hist, uint32_t* s_w) {
+struct SmallSelection {
+  uint32_t prefix;  // the threshold's magnitude bits above `shift`
+  uint32_t shift;   // digits below it are free
+  uint32_t ties;    // 1: only the equal magnitudes up to `last` are taken
+  uint32_t last;    // list position of the last taken equal magnitude
+};
+
+// CTA 0: the threshold of the list; returns false when the histograms do
+// not find the rank (never for a well-formed list).
+__device__ bool small_threshold(const TopkArgs& args, uint32_t n, uint32_t k, uint32_t* s_mag,
+                                uint32_t* s_hist, uint32_t* s_w, SmallSelection& out) {
   __shared__ uint32_t s_last;
-  __shared__ uint32_t s_cnt[kOutSlices * (kSelThreads / 32)];
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int tid = threadIdx.x;
   constexpr int kBatch = 8;  // loads in flight per thread
   for (uint32_t i0 = tid; i0 < n; i0 += kBatch * kSelThreads) {
     uint32_t v[kBatch];
@@ -497,13 +507,12 @@ __device__ void select_small(const TopkArgs& args, float* e, uint32_t n, uint32_
 #pragma unroll
     for (int j = 0; j < kBatch; ++j) {
       const uint32_t i = i0 + j * kSelThreads;
-      if (i < n) s_val[i] = v[j];
+      if (i < n) s_mag[i] = v[j] & 0x7fffffffu;
     }
   }
   __syncthreads();
   uint32_t prefix = 0, k_rem = k, n_in = n;
   int shift = 31;
-  bool ok = true;
   for (int l = 0; l < 3 && n_in != k_rem; ++l) {
     const int sh = l == 0 ? 20 : l == 1 ? 10 : 0;
     const uint32_t nb = 1u << (shift - sh);
@@ -516,7 +525,7 @@ __device__ void select_small(const TopkArgs& args, float* e, uint32_t n, uint32_
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           const uint32_t i = b0 + j * kSelThreads + tid;
-          m[j] = i < n ? s_val[i] & 0x7fffffffu : 0u;
+          m[j] = i < n ? s_mag[i] : 0u;
         }
 #pragma unroll
         for (int j = 0; j < 4; ++j)
@@ -529,7 +538,7 @@ __device__ void select_small(const TopkArgs& args, float* e, uint32_t n, uint32_
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           const uint32_t i = b0 + j * kSelThreads + tid;
-          m[j] = i < n ? s_val[i] & 0x7fffffffu : 0u;
+          m[j] = i < n ? s_mag[i] : 0u;
         }
 #pragma unroll
         for (int j = 0; j < 4; ++j)
@@ -539,99 +548,153 @@ __device__ void select_small(const TopkArgs& args, float* e, uint32_t n, uint32_
     }
     __syncthreads();
     const Selection s = select_bin<kSelThreads, false>(s_hist, nb, k_rem, s_w);
-    if (!s.found) {
-      ok = false;
-      break;
-    }
+    if (!s.found) return false;
     prefix = (prefix << (shift - sh)) | s.bin;
     k_rem = s.k_rem;
     n_in = s.n_in;
     shift = sh;
   }
-  if (!ok) {
-    if (tid == 0) {
-      atomicOr(args.error, kDevErrBadInput);
-      *count_out = 0;
-    }
-    return;
-  }
-  // selection: magnitude above the final bucket, or in it; when the bucket
-  // (all 31 bits fixed) holds more equal magnitudes than are taken, only the
-  // first k_rem of them in list order, i.e. up to list position s_last
+  // when the bucket (all 31 bits fixed) holds more equal magnitudes than are
+  // taken, only the first k_rem of them in list order
   const bool ties = n_in != k_rem;
   if (tid == 0) s_last = 0xffffffffu;
   if (ties) {
     const uint32_t per = (n + kSelThreads - 1) / kSelThreads;
     const uint32_t lo = tid * per < n ? tid * per : n, hi = lo + per < n ? lo + per : n;
     uint32_t cnt = 0;
-    for (uint32_t i = lo; i < hi; ++i) cnt += (s_val[i] & 0x7fffffffu) == prefix ? 1u : 0u;
+    for (uint32_t i = lo; i < hi; ++i) cnt += s_mag[i] == prefix ? 1u : 0u;
     uint32_t total;
     const uint32_t before = block_exclusive<kSelThreads>(cnt, total, s_w);
     if (before < k_rem && k_rem <= before + cnt) {
       uint32_t r = k_rem - before;
       for (uint32_t i = lo; i < hi; ++i)
-        if ((s_val[i] & 0x7fffffffu) == prefix && --r == 0) {
+        if (s_mag[i] == prefix && --r == 0) {
           s_last = i;
           break;
         }
     }
   }
   __syncthreads();
-  const uint32_t last = s_last;
-  // Output rounds of kOutSlices * kSelThreads list positions. Slice j of a
-  // round holds the positions b0 + j * kSelThreads + tid, so list order is
-  // (slice, warp, lane) order: one scan over the per-(slice, warp) counts
-  // gives every warp's offset, a ballot the lane's.
+  out = SmallSelection{prefix, static_cast<uint32_t>(shift), ties ? 1u : 0u, s_last};
+  return true;
+}
+
+// Slice CTA c of Gs: the selected pairs of list positions [c, c+1) * n / Gs.
+__device__ void small_emit(const TopkArgs& args, float* e, uint32_t n, uint32_t k, uint32_t Gs,
+                           uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                           uint32_t* s_w) {
+  constexpr int kJ = kSliceElems / kSelThreads;  // positions per thread
+  constexpr int kWarps = kSelThreads / 32;
+  __shared__ SmallSelection s_sel;
+  __shared__ uint32_t s_cnt[kJ * kWarps];
+  __shared__ uint32_t s_flag;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const uint32_t c = blockIdx.x;
+  const uint32_t lo = static_cast<uint32_t>(static_cast<uint64_t>(c) * n / Gs);
+  const uint32_t hi = static_cast<uint32_t>(static_cast<uint64_t>(c + 1) * n / Gs);
+  // the slice's candidates (position lo + j * kSelThreads + tid), loaded
+  // before the threshold is known
+  uint32_t coord[kJ], vbits[kJ];
+#pragma unroll
+  for (int j = 0; j < kJ; ++j) {
+    const uint32_t i = lo + j * kSelThreads + tid;
+    coord[j] = i < hi ? __ldcg(args.list_idx + i) : 0u;
+    vbits[j] = i < hi ? __float_as_uint(__ldcg(args.list_val + i)) : 0u;
+  }
+  // the threshold CTA 0 published (bounded wait)
+  if (tid == 0) {
+    uint32_t f = ld_acquire_u32(args.sel);
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t it = 0; f == 0; ++it) {
+      if (it > (1u << 26) || global_timer_ns() - t0 > args.wait_limit_ns) {
+        atomicOr(args.error, kDevErrTimeout);
+        f = 2;
+        break;
+      }
+      __nanosleep(64);
+      f = ld_acquire_u32(args.sel);
+    }
+    s_flag = f;
+    if (f == 1) s_sel = SmallSelection{args.sel[1], args.sel[2], args.sel[3], args.sel[4]};
+  }
+  __syncthreads();
+  if (s_flag != 1) {  // no threshold: nothing is written
+    if (c == 0 && tid == 0) *count_out = 0;
+    return;
+  }
+  const SmallSelection sel = s_sel;
+  uint32_t bits = 0;
+#pragma unroll
+  for (int j = 0; j < kJ; ++j) {
+    const uint32_t i = lo + j * kSelThreads + tid;
+    const uint32_t top = (vbits[j] & 0x7fffffffu) >> sel.shift;
+    const bool take = i < hi && (top > sel.prefix ||
+                                 (top == sel.prefix && (!sel.ties || i <= sel.last)));
+    bits |= (take ? 1u : 0u) << j;
+  }
+  // per-(j, warp) counts in list order, then one scan over them
+#pragma unroll
+  for (int j = 0; j < kJ; ++j) {
+    const uint32_t bal = __ballot_sync(0xffffffffu, (bits >> j) & 1u);
+    if (lane == 0) s_cnt[j * kWarps + warp] = __popc(bal);
+  }
+  __syncthreads();
+  const uint32_t mine = tid < kJ * kWarps ? s_cnt[tid] : 0u;
+  uint32_t slice_total;
+  const uint32_t off = block_exclusive<kSelThreads>(mine, slice_total, s_w);
+  if (tid < kJ * kWarps) s_cnt[tid] = off;
+  // publish the slice's count; sum the earlier slices' counts (bounded wait)
+  if (tid == 0)
+    st_relaxed_u64(args.chunk_sums + c, (static_cast<uint64_t>(args.epoch) << 32) | slice_total);
+  uint32_t base = 0;
+  {
+    const uint64_t t0 = global_timer_ns();
+    uint32_t it = 0;
+    while (true) {
+      uint32_t part = 0;
+      bool present = true;
+      for (uint32_t q = tid; q < c; q += kSelThreads) {
+        const uint64_t w = ld_relaxed_u64(args.chunk_sums + q);
+        if (static_cast<uint32_t>(w >> 32) == args.epoch)
+          part += static_cast<uint32_t>(w);
+        else
+          present = false;
+      }
+      const bool all_present = __syncthreads_and(present);
+      uint32_t sum;
+      block_exclusive<kSelThreads>(part, sum, s_w);
+      if (all_present) {
+        base = sum;
+        break;
+      }
+      const bool out_of_time = ++it > (1u << 26) || global_timer_ns() - t0 > args.wait_limit_ns;
+      if (__syncthreads_or(out_of_time)) {
+        if (tid == 0) atomicOr(args.error, kDevErrTimeout);
+        return;
+      }
+      __nanosleep(64);
+    }
+  }
   const uint32_t lt = lanemask_lt();
   bool overflow = false;
-  uint32_t base = 0;
-  for (uint32_t b0 = 0; b0 < n; b0 += kOutSlices * kSelThreads) {  // uniform trip count
-    uint32_t sel = 0;
 #pragma unroll
-    for (int j = 0; j < kOutSlices; ++j) {
-      const uint32_t i = b0 + j * kSelThreads + tid;
-      if (i < n) {
-        const uint32_t m = s_val[i] & 0x7fffffffu;
-        const uint32_t top = m >> shift;
-        const bool take = top > prefix || (top == prefix && (!ties || i <= last));
-        sel |= (take ? 1u : 0u) << j;
+  for (int j = 0; j < kJ; ++j) {
+    const uint32_t bal = __ballot_sync(0xffffffffu, (bits >> j) & 1u);
+    if ((bits >> j) & 1u) {
+      const uint32_t pos = base + s_cnt[j * kWarps + warp] + __popc(bal & lt);
+      if (pos < k) {
+        idx_out[pos] = coord[j];
+        val_out[pos] = __uint_as_float(vbits[j]);
+        e[coord[j]] = 0.0f;  // residual of a sent coordinate
+      } else {
+        overflow = true;
       }
     }
-    uint32_t coord[kOutSlices];
-#pragma unroll
-    for (int j = 0; j < kOutSlices; ++j)  // the indices of the taken, all in flight
-      coord[j] = (sel >> j) & 1u ? __ldcg(args.list_idx + b0 + j * kSelThreads + tid) : 0u;
-#pragma unroll
-    for (int j = 0; j < kOutSlices; ++j) {
-      const uint32_t bal = __ballot_sync(0xffffffffu, (sel >> j) & 1u);
-      if (lane == 0) s_cnt[j * (kSelThreads / 32) + warp] = __popc(bal);
-    }
-    __syncthreads();
-    constexpr uint32_t kCnt = kOutSlices * (kSelThreads / 32);
-    static_assert(kCnt <= static_cast<uint32_t>(kSelThreads), "one count per thread");
-    const uint32_t mine = static_cast<uint32_t>(tid) < kCnt ? s_cnt[tid] : 0u;
-    uint32_t round_total;
-    const uint32_t off = block_exclusive<kSelThreads>(mine, round_total, s_w);
-    if (static_cast<uint32_t>(tid) < kCnt) s_cnt[tid] = off;
-    __syncthreads();
-#pragma unroll
-    for (int j = 0; j < kOutSlices; ++j) {
-      const uint32_t bal = __ballot_sync(0xffffffffu, (sel >> j) & 1u);
-      if ((sel >> j) & 1u) {
-        const uint32_t pos = base + s_cnt[j * (kSelThreads / 32) + warp] + __popc(bal & lt);
-        if (pos < k) {
-          idx_out[pos] = coord[j];
-          val_out[pos] = __uint_as_float(s_val[b0 + j * kSelThreads + tid]);
-          e[coord[j]] = 0.0f;  // residual of a sent coordinate
-        } else {
-          overflow = true;
-        }
-      }
-    }
-    base += round_total;
-    __syncthreads();  // s_cnt is rewritten by the next round
   }
-  if (tid == 0) *count_out = base < k ? base : k;
+  if (c == Gs - 1 && tid == 0) {
+    const uint32_t end = base + slice_total;
+    *count_out = end < k ? end : k;
+  }
   if (__syncthreads_or(overflow) && tid == 0) atomicOr(args.error, kDevErrOverflow);
 }
 
@@ -728,7 +791,25 @@ __global__ void __launch_bounds__(kSelThreads, 1)
     return;
   }
   if (si.mode == 0 && si.n <= kSmallCand) {
-    if (blockIdx.x == 0) select_small(args, e, si.n, k, idx_out, val_out, count_out, s_mag, s_hist, s_w);
+    const uint32_t Gs = min(gridDim.x, (si.n + kSliceElems - 1) / kSliceElems);
+    if (blockIdx.x >= Gs) return;
+    if (blockIdx.x == 0) {
+      SmallSelection sel;
+      const bool found = small_threshold(args, si.n, k, s_mag, s_hist, s_w, sel);
+      if (threadIdx.x == 0) {
+        if (found) {
+          args.sel[1] = sel.prefix;
+          args.sel[2] = sel.shift;
+          args.sel[3] = sel.ties;
+          args.sel[4] = sel.last;
+        } else {
+          atomicOr(args.error, kDevErrBadInput);
+        }
+        __threadfence();
+        st_release_u32(args.sel, found ? 1u : 2u);
+      }
+    }
+    small_emit(args, e, si.n, k, Gs, idx_out, val_out, count_out, s_w);
     return;
   }
   bool ok = true;
@@ -823,10 +904,9 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
   args.list_val = reinterpret_cast<float*>(args.list_idx + ws.cand_cap);
   args.cand_count = ws.u32(kOffCandCount);
   args.cand_cap = ws.cand_cap;
-  args.threshold = ws.u64(kOffThreshold);
   args.lower_bound = ws.u64(kOffTkLowerBound);
   args.mode = ws.u32(kOffTkMode);
-  args.sample_done = ws.u32(kOffTkSampleDone);
+  args.sel = ws.u32(kOffTkSelect);
   args.list_count = ws.u32(kOffTkListCount);
   args.list_flags = ws.u32(kOffTkListFlags);
   args.bar_arrive = ws.u32(kOffBarArrive);
