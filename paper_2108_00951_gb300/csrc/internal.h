@@ -20,7 +20,7 @@ constexpr size_t kOffTkLowerBound = 56; // uint64: sampled lower bound of the ca
 constexpr size_t kOffTkMode = 64;       // uint32: 0 candidates, 1 full array
 constexpr size_t kOffTkListCount = 72;  // uint32: candidates emitted by the streaming pass
 constexpr size_t kOffTkListFlags = 76;  // uint32: that pass's latched bits (overflow, timeout)
-constexpr size_t kOffTkSelect = 128;    // uint32[5]: short-list threshold published by CTA 0
+constexpr size_t kOffTkSelect = 128;    // uint32[4]: short-list threshold published by CTA 0
 constexpr size_t kOffHist = 256;        // uint32[6][2048] refine levels 0..5, then the sample
 constexpr int kHistLevels = 6;
 constexpr int kHistBins = 2048;

@@ -58,7 +58,7 @@ struct TopkArgs {
   uint32_t cand_cap;
   uint64_t* lower_bound;
   uint32_t* mode;        // 0: candidates, 1: full array
-  uint32_t* sel;         // small-list threshold: flag (1 found, 2 failed), prefix, shift, ties, last
+  uint32_t* sel;         // short-list threshold: flag (1 found, 2 failed), B, ties, last
   uint32_t* list_count;
   uint32_t* list_flags;
   uint32_t* bar_arrive;
@@ -472,31 +472,55 @@ __device__ uint32_t write_selected(const TopkArgs& args, float* e, uint32_t mode
 }
 
 // A short candidate list (n <= kSmallCand) is resolved in two parts.
-// CTA 0 finds the threshold in shared memory: the magnitudes of every
-// candidate are loaded once; three digit levels (bits 30..20, 19..10, 9..0)
-// find the threshold magnitude T and how many of the candidates equal to T
-// are taken; equal magnitudes are taken in list order, which is index order
-// (the lowest-index tie rule), i.e. up to list position `last`. It publishes
-// (T's digits, ties, last) behind a flag. Then every slice CTA writes the
-// selected pairs of its kSliceElems-position slice of the list in order,
-// zeroing the residual at each: it loads its slice while CTA 0 works,
-// publishes its slice's count, and sums the earlier slices' counts.
+// CTA 0 finds the threshold in shared memory. The magnitudes of every
+// candidate are loaded once, with their minimum and maximum. Digit levels
+// narrow a window [B, B + W) of magnitude bit patterns (monotone in |a|):
+// level 0 splits [min, max] into at most 2048 bins, each later level splits
+// the chosen bin into at most 2048 sub-bins. The levels stop when the window holds exactly the remaining rank, or is
+// one magnitude T wide; then equal magnitudes are taken in list order, which
+// is index order (the lowest-index tie rule), up to list position `last`.
+// The selection is |a| > B, or |a| == B at a position <= last. CTA 0
+// publishes (B, ties, last) behind a flag; every slice CTA, having loaded
+// its slice of kSliceElems positions meanwhile, publishes its slice's count,
+// sums the earlier slices' counts, and writes its selected pairs in order,
+// zeroing the residual at each.
 constexpr uint32_t kSliceElems = 4 * kSelThreads;  // list positions per slice CTA
 
 struct SmallSelection {
-  uint32_t prefix;  // the threshold's magnitude bits above `shift`
-  uint32_t shift;   // digits below it are free
-  uint32_t ties;    // 1: only the equal magnitudes up to `last` are taken
-  uint32_t last;    // list position of the last taken equal magnitude
+  uint32_t B;       // threshold magnitude bits
+  uint32_t ties;    // 1: magnitudes equal to B are taken only up to `last`
+  uint32_t last;    // list position of the last taken magnitude equal to B
 };
+
+// Histogram pass of a level over `cnt` magnitudes of `src`: those in the
+// window [B, B + W) (W == 0: all) add to bin (m - B) >> sh.
+__device__ __forceinline__ void window_hist(const uint32_t* src, uint32_t cnt, uint32_t B,
+                                            uint32_t W, int sh, uint32_t* s_hist) {
+  for (uint32_t b0 = threadIdx.x; b0 < cnt; b0 += 4 * kSelThreads) {
+    uint32_t m[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint32_t i = b0 + j * kSelThreads;
+      m[j] = i < cnt ? src[i] : 0u;
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint32_t off = m[j] - B;
+      if (b0 + j * kSelThreads < cnt && m[j] >= B && (W == 0 || off < W))
+        atomicAdd(&s_hist[off >> sh], 1u);
+    }
+  }
+}
 
 // CTA 0: the threshold of the list; returns false when the histograms do
 // not find the rank (never for a well-formed list).
 __device__ bool small_threshold(const TopkArgs& args, uint32_t n, uint32_t k, uint32_t* s_mag,
                                 uint32_t* s_hist, uint32_t* s_w, SmallSelection& out) {
   __shared__ uint32_t s_last;
-  const int tid = threadIdx.x;
+  __shared__ uint32_t s_lo[32], s_hi[32];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int kBatch = 8;  // loads in flight per thread
+  uint32_t lo = 0xffffffffu, hi = 0;
   for (uint32_t i0 = tid; i0 < n; i0 += kBatch * kSelThreads) {
     uint32_t v[kBatch];
 #pragma unroll
@@ -507,75 +531,74 @@ __device__ bool small_threshold(const TopkArgs& args, uint32_t n, uint32_t k, ui
 #pragma unroll
     for (int j = 0; j < kBatch; ++j) {
       const uint32_t i = i0 + j * kSelThreads;
-      if (i < n) s_mag[i] = v[j] & 0x7fffffffu;
+      if (i < n) {
+        const uint32_t m = v[j] & 0x7fffffffu;
+        s_mag[i] = m;
+        lo = m < lo ? m : lo;
+        hi = m > hi ? m : hi;
+      }
     }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    lo = min(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+    hi = max(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+  }
+  if (lane == 0) {
+    s_lo[warp] = lo;
+    s_hi[warp] = hi;
   }
   __syncthreads();
-  uint32_t prefix = 0, k_rem = k, n_in = n;
-  int shift = 31;
-  for (int l = 0; l < 3 && n_in != k_rem; ++l) {
-    const int sh = l == 0 ? 20 : l == 1 ? 10 : 0;
-    const uint32_t nb = 1u << (shift - sh);
-    for (uint32_t b = tid; b < nb; b += kSelThreads) s_hist[b] = 0;
+  lo = s_lo[lane];  // 32 warps
+  hi = s_hi[lane];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    lo = min(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+    hi = max(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+  }
+  // digit levels over the window [B, B + W); W == 0: the whole [lo, hi]
+  uint32_t B = lo, W = 0, k_rem = k, n_in = n;
+  int sh = 0;
+  while (((hi - lo) >> sh) >= static_cast<uint32_t>(kHistBins)) ++sh;
+  if (hi == lo) W = 1;  // every candidate has the same magnitude
+  while (W != 1 && n_in != k_rem) {
+    for (uint32_t b = tid; b < static_cast<uint32_t>(kHistBins); b += kSelThreads) s_hist[b] = 0;
     __syncthreads();
-    if (l == 0) {
-      // every candidate, crowded into few bins: equal bins of a warp add once
-      for (uint32_t b0 = 0; b0 < n; b0 += 4 * kSelThreads) {  // uniform trip count
-        uint32_t m[4];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const uint32_t i = b0 + j * kSelThreads + tid;
-          m[j] = i < n ? s_mag[i] : 0u;
-        }
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-          hist_add_warp(s_hist, (m[j] >> sh) & (nb - 1), b0 + j * kSelThreads + tid < n);
-      }
-    } else {
-      // only the candidates in the chosen bin, spread over its sub-bins
-      for (uint32_t b0 = 0; b0 < n; b0 += 4 * kSelThreads) {
-        uint32_t m[4];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const uint32_t i = b0 + j * kSelThreads + tid;
-          m[j] = i < n ? s_mag[i] : 0u;
-        }
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-          if (b0 + j * kSelThreads + tid < n && (m[j] >> shift) == prefix)
-            atomicAdd(&s_hist[(m[j] >> sh) & (nb - 1)], 1u);
-      }
-    }
+    window_hist(s_mag, n, B, W, sh, s_hist);
     __syncthreads();
-    const Selection s = select_bin<kSelThreads, false>(s_hist, nb, k_rem, s_w);
+    const Selection s = select_bin<kSelThreads, false>(s_hist, kHistBins, k_rem, s_w);
     if (!s.found) return false;
-    prefix = (prefix << (shift - sh)) | s.bin;
+    B += s.bin << sh;
+    W = 1u << sh;
     k_rem = s.k_rem;
     n_in = s.n_in;
-    shift = sh;
+    int bits = 0;
+    while ((1u << bits) < W) ++bits;
+    sh = bits > 11 ? bits - 11 : 0;
   }
-  // when the bucket (all 31 bits fixed) holds more equal magnitudes than are
-  // taken, only the first k_rem of them in list order
-  const bool ties = n_in != k_rem;
+  // at a one-wide threshold with more equal magnitudes than are taken, only
+  // the first k_rem of them in list order
+  const bool ties = W == 1 && n_in != k_rem;
   if (tid == 0) s_last = 0xffffffffu;
   if (ties) {
     const uint32_t per = (n + kSelThreads - 1) / kSelThreads;
-    const uint32_t lo = tid * per < n ? tid * per : n, hi = lo + per < n ? lo + per : n;
+    const uint32_t a0 = tid * per < n ? tid * per : n, a1 = a0 + per < n ? a0 + per : n;
     uint32_t cnt = 0;
-    for (uint32_t i = lo; i < hi; ++i) cnt += s_mag[i] == prefix ? 1u : 0u;
+    for (uint32_t i = a0; i < a1; ++i) cnt += s_mag[i] == B ? 1u : 0u;
     uint32_t total;
     const uint32_t before = block_exclusive<kSelThreads>(cnt, total, s_w);
     if (before < k_rem && k_rem <= before + cnt) {
       uint32_t r = k_rem - before;
-      for (uint32_t i = lo; i < hi; ++i)
-        if (s_mag[i] == prefix && --r == 0) {
+      for (uint32_t i = a0; i < a1; ++i)
+        if (s_mag[i] == B && --r == 0) {
           s_last = i;
           break;
         }
     }
   }
   __syncthreads();
-  out = SmallSelection{prefix, static_cast<uint32_t>(shift), ties ? 1u : 0u, s_last};
+  const uint32_t last = ties ? s_last : 0xffffffffu;
+  out = SmallSelection{B, ties ? 1u : 0u, last};
   return true;
 }
 
@@ -601,7 +624,7 @@ __device__ void small_emit(const TopkArgs& args, float* e, uint32_t n, uint32_t 
     coord[j] = i < hi ? __ldcg(args.list_idx + i) : 0u;
     vbits[j] = i < hi ? __float_as_uint(__ldcg(args.list_val + i)) : 0u;
   }
-  // the threshold CTA 0 published (bounded wait)
+  // the threshold and slice bases CTA 0 published (bounded wait)
   if (tid == 0) {
     uint32_t f = ld_acquire_u32(args.sel);
     const uint64_t t0 = global_timer_ns();
@@ -611,11 +634,10 @@ __device__ void small_emit(const TopkArgs& args, float* e, uint32_t n, uint32_t 
         f = 2;
         break;
       }
-      __nanosleep(64);
       f = ld_acquire_u32(args.sel);
     }
     s_flag = f;
-    if (f == 1) s_sel = SmallSelection{args.sel[1], args.sel[2], args.sel[3], args.sel[4]};
+    if (f == 1) s_sel = SmallSelection{args.sel[1], args.sel[2], args.sel[3]};
   }
   __syncthreads();
   if (s_flag != 1) {  // no threshold: nothing is written
@@ -627,9 +649,8 @@ __device__ void small_emit(const TopkArgs& args, float* e, uint32_t n, uint32_t 
 #pragma unroll
   for (int j = 0; j < kJ; ++j) {
     const uint32_t i = lo + j * kSelThreads + tid;
-    const uint32_t top = (vbits[j] & 0x7fffffffu) >> sel.shift;
-    const bool take = i < hi && (top > sel.prefix ||
-                                 (top == sel.prefix && (!sel.ties || i <= sel.last)));
+    const uint32_t m = vbits[j] & 0x7fffffffu;
+    const bool take = i < hi && (m > sel.B || (m == sel.B && (!sel.ties || i <= sel.last)));
     bits |= (take ? 1u : 0u) << j;
   }
   // per-(j, warp) counts in list order, then one scan over them
@@ -672,7 +693,6 @@ __device__ void small_emit(const TopkArgs& args, float* e, uint32_t n, uint32_t 
         if (tid == 0) atomicOr(args.error, kDevErrTimeout);
         return;
       }
-      __nanosleep(64);
     }
   }
   const uint32_t lt = lanemask_lt();
@@ -798,10 +818,9 @@ __global__ void __launch_bounds__(kSelThreads, 1)
       const bool found = small_threshold(args, si.n, k, s_mag, s_hist, s_w, sel);
       if (threadIdx.x == 0) {
         if (found) {
-          args.sel[1] = sel.prefix;
-          args.sel[2] = sel.shift;
-          args.sel[3] = sel.ties;
-          args.sel[4] = sel.last;
+          args.sel[1] = sel.B;
+          args.sel[2] = sel.ties;
+          args.sel[3] = sel.last;
         } else {
           atomicOr(args.error, kDevErrBadInput);
         }
