@@ -16,6 +16,7 @@ constexpr size_t kOffError = 8;         // uint32: latched device error bits
 constexpr size_t kOffTopkReset = 16;    // start of the region cleared at each Top-k call
 constexpr size_t kOffBarArrive = 16;    // uint32: grid-barrier arrivals
 constexpr size_t kOffCandCount = 20;    // uint32[6]: refine-level candidate counts
+constexpr size_t kOffTkStreamArrive = 44; // uint32: arrivals at the candidate stream's barrier
 constexpr size_t kOffTkLowerBound = 56; // uint64: sampled lower bound of the candidates' keys
 constexpr size_t kOffTkMode = 64;       // uint32: 0 candidates, 1 full array
 constexpr size_t kOffTkListCount = 72;  // uint32: candidates emitted by the streaming pass

@@ -191,8 +191,7 @@ struct TopkCandOp {
   float gamma;
   uint32_t d, k, cand_cap;
   uint32_t* hist;      // global sample histogram [kSampleBins]
-  uint32_t* bar_arrive;
-  uint32_t* bar_gen;
+  uint32_t* stream_arrive;  // arrivals at the pre-pass barrier (zero at the call's start)
   uint32_t* mode;      // published for the select kernel
   uint64_t* lower_bound;
   static constexpr uint32_t kGBytes = kTileElems * sizeof(GT);
@@ -242,8 +241,29 @@ struct TopkCandOp {
       if (s_hist[b]) atomicAdd(&hist[b], s_hist[b]);
   }
 
+  // One-shot grid barrier: the arrival counter starts at zero in every call
+  // (the per-call reset of the control block), so a CTA arrives once, after a
+  // fence that publishes its merged histogram, and waits (bounded) until all
+  // have arrived.
   __device__ bool barrier(uint64_t limit_ns, uint32_t* error) const {
-    return grid_barrier(bar_arrive, bar_gen, limit_ns, error);
+    __shared__ int s_ok;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      __threadfence();
+      atomicAdd(stream_arrive, 1u);
+      int ok = 1;
+      const uint64_t t0 = global_timer_ns();
+      for (uint32_t it = 0; ld_acquire_u32(stream_arrive) < gridDim.x; ++it) {
+        if (it > (1u << 26) || global_timer_ns() - t0 > limit_ns) {
+          atomicOr(error, kDevErrTimeout);
+          ok = 0;
+          break;
+        }
+      }
+      s_ok = ok;
+    }
+    __syncthreads();
+    return s_ok != 0;
   }
 
   // Every CTA computes the same bound: each compute thread loads 16
@@ -287,7 +307,8 @@ struct TopkCandOp {
       // 1.5x the expected sampled count above the k-th key, plus 32: many
       // standard deviations of sampling noise; a miss costs the exact
       // full-array fallback, never a wrong result
-      const double x = 1.5 * static_cast<double>(k) * sampled / d + 32.0;
+      // (integer arithmetic: the products stay below 2^56; FP64 is slow here)
+      const uint64_t x = 3ull * k * sampled / (2ull * d) + 32ull;
       target = x >= sampled ? sampled + 1 : static_cast<uint32_t>(x);
     }
     // the bin holding the target-th largest sample, and the sampled mass at
@@ -307,13 +328,16 @@ struct TopkCandOp {
     if (t == 0) {
       const bool found = s_bin != 0xffffffffu;
       uint64_t bound = found ? static_cast<uint64_t>(s_bin) << (32 + kSampleShift) : 0ull;
-      const double expected =
-          found ? (everything ? s_mass : static_cast<double>(s_mass) * d / sampled)
-                : static_cast<double>(d);
+      // expected candidates (the sampled mass scaled to d) above half the
+      // capacity: 2 * mass * d / sampled > cap, compared exactly
+      const bool too_many =
+          found ? (everything ? 2ull * s_mass > cand_cap
+                              : 2ull * s_mass * d > static_cast<uint64_t>(cand_cap) * sampled)
+                : 2ull * d > cand_cap;
       uint32_t m = 0;
       if (k == 0) {
         bound = kSelectNone;
-      } else if (expected > 0.5 * cand_cap) {
+      } else if (too_many) {
         m = 1;                // the candidates would not fit: full-array selection
         bound = kSelectNone;  // and none gathered while streaming
       }
@@ -944,7 +968,7 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
                           reinterpret_cast<uintptr_t>(g) % 16 == 0 && per_sm > 0;
   if (streamable) {
     TopkCandOp<GT> op{g, e, gamma, d, k, ws.cand_cap, ws.u32(kOffSampleHist),
-                      args.bar_arrive, args.bar_gen, args.mode, args.lower_bound};
+                      ws.u32(kOffTkStreamArrive), args.mode, args.lower_bound};
     uint32_t slots = static_cast<uint32_t>(per_sm * dev.sm_count);
     if (slots > kMaxChunks) slots = kMaxChunks;
     const uint32_t grid = tiles < slots ? tiles : slots;
