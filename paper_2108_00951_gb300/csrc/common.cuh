@@ -188,6 +188,14 @@ __device__ __forceinline__ uint32_t lookback_exclusive(const ScanCtx& ctx, uint3
 
 // Bounded grid-wide barrier for a cooperative launch (all CTAs co-resident).
 // Returns false, latching kDevErrTimeout, if the wait ran out.
+// Programmatic dependent launch: wait until the grids this one depends on
+// have completed and their memory is visible (a no-op when the launch did
+// not allow an early start), and let dependent grids be scheduled.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ bool grid_barrier(uint32_t* arrive, uint32_t* gen, uint64_t limit_ns,
                              uint32_t* error) {
   __shared__ int s_ok;

@@ -163,7 +163,7 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
   const uintptr_t ga = reinterpret_cast<uintptr_t>(g), ea = reinterpret_cast<uintptr_t>(e);
   const int per_sm = sizeof(GT) == 4 ? dev.ht_stream_per_sm_f32 : dev.ht_stream_per_sm_bf16;
   if (ga % 16 == 0 && ea % 16 == 0 && per_sm > 0) {
-    // TMA-fed streaming compaction: one cooperative launch over all SMs
+    // TMA-fed streaming compaction: one CTA per SM
     HtOp<GT> op{g, e, gamma, lambda, d};
     uint32_t slots = static_cast<uint32_t>(per_sm * dev.sm_count);
     if (slots > kMaxChunks) slots = kMaxChunks;
@@ -172,9 +172,21 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
     ScanCtx c = ctx;
     StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks()};
     void* params[] = {&op, &d, &idx_out, &val_out, &count_out, &cap, &c, &sa};
-    const cudaError_t err = cudaLaunchCooperativeKernel(
-        reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages>), dim3(grid),
-        dim3(kStreamThreads), params, HtStreamKernel<GT>::kSmem, ws.stream);
+    // A plain launch suffices: the only cross-CTA wait is on lower-numbered
+    // CTAs, which are scheduled first. It may start while the previous kernel
+    // on the stream finishes (the kernel waits for it before its first read).
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kStreamThreads);
+    cfg.dynamicSmemBytes = HtStreamKernel<GT>::kSmem;
+    cfg.stream = ws.stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const cudaError_t err = cudaLaunchKernelExC(
+        &cfg, reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages>), params);
     count_launch();
     return err;
   }

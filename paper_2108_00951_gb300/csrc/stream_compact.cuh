@@ -120,6 +120,9 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
     mbar_init_fence();
   }
   __syncthreads();
+  // a dependent launch may start early: everything the previous kernels on
+  // the stream wrote is read only after this
+  griddep_wait();
 
   // ------------------------------------------------------------- phase 1
   bool failed = false;    // a wait of this thread ran out
@@ -248,6 +251,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   // A CTA that owns the withheld tile never arrives: the others' barrier
   // waits run out (the failure-detection test).
   if (__syncthreads_or(withheld)) return;
+  griddep_launch_dependents();  // streaming is done: the next kernel may be scheduled
 
   // ------------------------------------------------------------- phase 2
   // the chunk's total (each compute warp contributes its own)
