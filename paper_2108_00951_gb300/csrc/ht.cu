@@ -89,6 +89,7 @@ struct HtOp {
   static constexpr int kSampleBins = 1;
   __device__ void sample(const unsigned char*, uint32_t, int, int, uint32_t*) const {}
   __device__ void merge(const uint32_t*) const {}
+  __device__ void prologue() const {}
   __device__ bool barrier(uint64_t, uint32_t*) const { return true; }
   __device__ uint64_t choose() const { return 0; }
 

@@ -13,23 +13,27 @@ namespace efs {
 // Layout of the workspace header (bytes from the workspace base).
 constexpr size_t kOffBarGen = 0;        // uint32: grid-barrier generation (never reset)
 constexpr size_t kOffError = 8;         // uint32: latched device error bits
-constexpr size_t kOffTopkReset = 16;    // start of the region cleared at each Top-k call
-constexpr size_t kOffBarArrive = 16;    // uint32: grid-barrier arrivals
-constexpr size_t kOffCandCount = 20;    // uint32[6]: refine-level candidate counts
-constexpr size_t kOffTkStreamArrive = 44; // uint32: arrivals at the candidate stream's barrier
+constexpr size_t kOffBarArrive = 16;    // uint32: grid-barrier arrivals (zero after each barrier)
 constexpr size_t kOffTkLowerBound = 56; // uint64: sampled lower bound of the candidates' keys
 constexpr size_t kOffTkMode = 64;       // uint32: 0 candidates, 1 full array
 constexpr size_t kOffTkListCount = 72;  // uint32: candidates emitted by the streaming pass
-constexpr size_t kOffTkListFlags = 76;  // uint32: that pass's latched bits (overflow, timeout)
-constexpr size_t kOffTkSelect = 128;    // uint32[4]: short-list threshold published by CTA 0
-constexpr size_t kOffHist = 256;        // uint32[6][2048] refine levels 0..5, then the sample
+// Per-call Top-k state that must start at zero, in two blocks used by
+// alternate calls on a workspace: a call's candidate stream zeroes the
+// other block (the previous call's, complete by then) for the next call.
+constexpr size_t kOffTkState = 256;
+constexpr size_t kStStreamArrive = 0;   // uint32: arrivals at the candidate stream's barrier
+constexpr size_t kStListFlags = 4;      // uint32: that pass's latched bits (overflow, timeout)
+constexpr size_t kStSelect = 16;        // uint32[4]: short-list threshold published by CTA 0
+constexpr size_t kStCandCount = 32;     // uint32[6]: refine-level candidate counts
+constexpr size_t kStHist = 256;         // uint32[6][2048]: refine-level histograms
 constexpr int kHistLevels = 6;
 constexpr int kHistBins = 2048;
 constexpr int kSampleBits = 13;         // the sample histogram: top 13 bits of |a|
 constexpr int kSampleBins = 1 << kSampleBits;
-constexpr size_t kOffSampleHist = kOffHist + sizeof(uint32_t) * kHistLevels * kHistBins;
-constexpr size_t kHeaderBytes = kOffSampleHist + sizeof(uint32_t) * kSampleBins;
-constexpr size_t kTopkResetBytes = kHeaderBytes - kOffTopkReset;
+constexpr size_t kStSampleHist = kStHist + sizeof(uint32_t) * kHistLevels * kHistBins;
+constexpr size_t kTkStateBytes = kStSampleHist + sizeof(uint32_t) * kSampleBins;
+static_assert(kTkStateBytes % 256 == 0, "state block alignment");
+constexpr size_t kHeaderBytes = kOffTkState + 2 * kTkStateBytes;
 constexpr uint32_t kMaxChunks = 1024;   // per-CTA chunk sums of the streaming compaction
 constexpr uint32_t kCountsPerTile = 16; // per-segment counts of the streaming compaction
 
@@ -43,6 +47,7 @@ struct Workspace {
   size_t offsets_cap = 0;      // capacity of the aggregation offsets (uint32)
   size_t stage_cap = 0;        // capacity of the pair staging buffers (pairs)
   uint32_t epoch = 0;          // last epoch handed to a compaction launch
+  uint32_t topk_calls = 0;     // Top-k calls so far: their parity picks the state block
   bool dirty = false;          // header must be re-cleared (failed launch or device timeout)
 
   // Regions after the header, each 256-byte aligned.
@@ -70,6 +75,9 @@ struct Workspace {
     return reinterpret_cast<float*>(base + off_stage() + sizeof(uint32_t) * stage_cap);
   }
   uint32_t* u32(size_t off) const { return reinterpret_cast<uint32_t*>(base + off); }
+  uint32_t* topk_state(uint32_t parity) const {
+    return u32(kOffTkState + (parity & 1u) * kTkStateBytes);
+  }
   uint64_t* u64(size_t off) const { return reinterpret_cast<uint64_t*>(base + off); }
 };
 

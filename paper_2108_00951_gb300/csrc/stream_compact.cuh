@@ -46,6 +46,7 @@
 //        warp's segment, from the stage of a full tile, or from global memory
 //        for the partial last tile.
 //   (tile_smem and tile_global also receive `aux`, the pre-pass result or 0)
+//   void prologue()                     every thread, once, at the start
 // Optional pre-pass (kPrepass): before streaming, the compute warps hand the
 // first tile of their CTA's chunk, from its ring stage, to
 //   void sample(const unsigned char* stage, uint32_t tile, int warp, int lane,
@@ -123,6 +124,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   // a dependent launch may start early: everything the previous kernels on
   // the stream wrote is read only after this
   griddep_wait();
+  op.prologue();
 
   // ------------------------------------------------------------- phase 1
   bool failed = false;    // a wait of this thread ran out

@@ -176,6 +176,15 @@ __device__ __forceinline__ uint32_t block_exclusive(uint32_t v, uint32_t& total,
   return before + incl - v;
 }
 
+// Zeroes a Top-k state block, the grid's threads striding over it (the
+// block belongs to the previous call on the workspace, which is complete).
+__device__ __forceinline__ void clear_state(uint32_t* block) {
+  constexpr uint32_t kWords = static_cast<uint32_t>(kTkStateBytes / sizeof(uint4));
+  uint4* b4 = reinterpret_cast<uint4*>(block);
+  for (uint32_t w = blockIdx.x * blockDim.x + threadIdx.x; w < kWords; w += gridDim.x * blockDim.x)
+    b4[w] = make_uint4(0u, 0u, 0u, 0u);
+}
+
 // ------------------------------------------------------------- 1 stream
 // The streaming pass as a stream_compact op. Pre-pass: every CTA histograms
 // the top 11 key bits of the first tile of its chunk (the tiles so sampled
@@ -194,6 +203,7 @@ struct TopkCandOp {
   uint32_t* stream_arrive;  // arrivals at the pre-pass barrier (zero at the call's start)
   uint32_t* mode;      // published for the select kernel
   uint64_t* lower_bound;
+  uint32_t* other_state;    // the other state block: zeroed here for the next call
   static constexpr uint32_t kGBytes = kTileElems * sizeof(GT);
   static constexpr uint32_t kStageBytes = kGBytes + kTileElems * sizeof(float);
   static constexpr bool kPrepass = true;
@@ -240,6 +250,9 @@ struct TopkCandOp {
     for (int b = threadIdx.x; b < kSampleBins; b += blockDim.x)
       if (s_hist[b]) atomicAdd(&hist[b], s_hist[b]);
   }
+
+  // every CTA, first thing, whatever happens later in the launch
+  __device__ void prologue() const { clear_state(other_state); }
 
   // One-shot grid barrier: the arrival counter starts at zero in every call
   // (the per-call reset of the control block), so a CTA arrives once, after a
@@ -396,7 +409,8 @@ constexpr int kTkStages = 4;
 template <typename GT>
 __global__ void __launch_bounds__(kThreads)
     topk_accumulate_plain_kernel(const GT* __restrict__ g, float* __restrict__ e, float gamma,
-                                 uint32_t d, TopkArgs args) {
+                                 uint32_t d, TopkArgs args, uint32_t* other_state) {
+  clear_state(other_state);
   if (blockIdx.x == 0 && threadIdx.x == 0) {
     *args.mode = 1;
     *args.lower_bound = kSelectNone;
@@ -936,22 +950,25 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
                          uint32_t* idx_out, float* val_out, uint32_t* count_out, Workspace& ws,
                          const DeviceInfo& dev) {
   const uint32_t tiles = tiles_for(d);
-  cudaError_t err = cudaMemsetAsync(ws.base + kOffTopkReset, 0, kTopkResetBytes, ws.stream);
-  if (err != cudaSuccess) return err;
+  cudaError_t err = cudaSuccess;
+  // this call's zeroed state block, and the other one, cleared for the next call
+  uint32_t* state = ws.topk_state(ws.topk_calls);
+  uint32_t* other = ws.topk_state(ws.topk_calls + 1);
+  ++ws.topk_calls;
 
   TopkArgs args;
-  args.hist = ws.u32(kOffHist);
+  args.hist = state + kStHist / 4;
   args.cand0 = ws.cand(1);
   args.cand1 = ws.cand(2);
   args.list_idx = reinterpret_cast<uint32_t*>(ws.cand(0));
   args.list_val = reinterpret_cast<float*>(args.list_idx + ws.cand_cap);
-  args.cand_count = ws.u32(kOffCandCount);
+  args.cand_count = state + kStCandCount / 4;
   args.cand_cap = ws.cand_cap;
   args.lower_bound = ws.u64(kOffTkLowerBound);
   args.mode = ws.u32(kOffTkMode);
-  args.sel = ws.u32(kOffTkSelect);
+  args.sel = state + kStSelect / 4;
   args.list_count = ws.u32(kOffTkListCount);
-  args.list_flags = ws.u32(kOffTkListFlags);
+  args.list_flags = state + kStListFlags / 4;
   args.bar_arrive = ws.u32(kOffBarArrive);
   args.bar_gen = ws.u32(kOffBarGen);
   args.error = ws.u32(kOffError);
@@ -967,8 +984,8 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
   const bool streamable = reinterpret_cast<uintptr_t>(e) % 16 == 0 &&
                           reinterpret_cast<uintptr_t>(g) % 16 == 0 && per_sm > 0;
   if (streamable) {
-    TopkCandOp<GT> op{g, e, gamma, d, k, ws.cand_cap, ws.u32(kOffSampleHist),
-                      ws.u32(kOffTkStreamArrive), args.mode, args.lower_bound};
+    TopkCandOp<GT> op{g, e, gamma, d, k, ws.cand_cap, state + kStSampleHist / 4,
+                      state + kStStreamArrive / 4, args.mode, args.lower_bound, other};
     uint32_t slots = static_cast<uint32_t>(per_sm * dev.sm_count);
     if (slots > kMaxChunks) slots = kMaxChunks;
     const uint32_t grid = tiles < slots ? tiles : slots;
@@ -984,7 +1001,8 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
   } else {
     const uint32_t grid = tiles < static_cast<uint32_t>(dev.sm_count * 8)
                               ? tiles : static_cast<uint32_t>(dev.sm_count * 8);
-    topk_accumulate_plain_kernel<GT><<<grid, kThreads, 0, ws.stream>>>(g, e, gamma, d, args);
+    topk_accumulate_plain_kernel<GT><<<grid, kThreads, 0, ws.stream>>>(g, e, gamma, d, args,
+                                                                       other);
     count_launch();
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
   }
