@@ -85,6 +85,7 @@ struct HtOp {
   uint32_t d;
   static constexpr uint32_t kGBytes = kTileElems * sizeof(GT);
   static constexpr uint32_t kStageBytes = kGBytes + kTileElems * sizeof(float);
+  static constexpr uint32_t kWarpStagePairs = 768;  // on-chip staged pairs per compute warp
   static constexpr bool kPrepass = false;
   static constexpr int kSampleBins = 1;
   __device__ void sample(const unsigned char*, uint32_t, int, int, uint32_t*) const {}

@@ -87,11 +87,24 @@ struct StreamArgs {
   uint64_t* chunk_sums;  // [gridDim.x] (epoch << 32) | chunk total
 };
 
+// A segment's count (<= 256: 9 bits) and its warp's earlier pairs in the
+// chunk, saturated to 23 bits, in one word.
+__device__ __forceinline__ uint32_t pack_count(uint32_t before, uint32_t count) {
+  return (before < (1u << 23) ? before : (1u << 23) - 1u) << 9 | count;
+}
+
 template <class Op, int kStages>
 struct StreamLayout {
-  static constexpr uint32_t kSmem = kStages * Op::kStageBytes;
-  // phase 2 reuses the ring for the chunk's segment counts
-  static constexpr uint32_t kChunkSegs = kSmem / sizeof(uint32_t);
+  static constexpr uint32_t kRing = kStages * Op::kStageBytes;
+  // each compute warp stages its first kWarpPairs pairs on chip, the rest in
+  // the global staging slots
+  static constexpr uint32_t kWarpPairs = Op::kWarpStagePairs;
+  static constexpr uint32_t kStaging = kSWarps * kWarpPairs * 8;
+  static constexpr uint32_t kSmem = kRing + kStaging;  // dynamic shared memory
+  // phase 2 reuses the ring: per segment of a window, its output offset and
+  // its warp's count of earlier pairs in the chunk
+  static constexpr uint32_t kChunkSegs = kRing / 8;
+  static_assert(kChunkSegs % kSWarps == 0, "whole tiles per window");
 };
 
 template <class Op, int kStages>
@@ -105,6 +118,8 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   __shared__ uint32_t s_scratch[kStreamThreads / 32];
   __shared__ uint32_t s_sample_hist[Op::kPrepass ? Op::kSampleBins : 1];
   using L = StreamLayout<Op, kStages>;
+  uint32_t* s_pair_idx = reinterpret_cast<uint32_t*>(smem + L::kRing);
+  float* s_pair_val = reinterpret_cast<float*>(smem + L::kRing + kSWarps * L::kWarpPairs * 4);
 
   const uint32_t T = ctx.num_tiles, G = gridDim.x, c = blockIdx.x;
   const uint32_t t_lo = static_cast<uint32_t>(static_cast<uint64_t>(c) * T / G);
@@ -225,11 +240,18 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
         total += __popc(b0) + __popc(b1) + __popc(b2) + __popc(b3);
       }
       const size_t seg = static_cast<size_t>(t) * kSWarps + warp;
-      if (lane == 0) sa.counts[seg] = total;
+      const uint32_t before = chunk_total;  // this warp's earlier pairs in the chunk
       chunk_total += total;
+      // the count with the warp's earlier pairs (saturated: only <= the
+      // on-chip share matters), which tells phase 2 where the pairs are
+      if (lane == 0) sa.counts[seg] = pack_count(before, total);
       if (total) {
-        uint32_t* sidx = sa.stage_idx + seg * kSWarpElems;
-        float* sval = sa.stage_val + seg * kSWarpElems;
+        // on chip while the warp's pairs fit, else the segment's global slot
+        const bool on_chip = chunk_total <= L::kWarpPairs;
+        uint32_t* sidx = on_chip ? s_pair_idx + warp * L::kWarpPairs + before
+                                 : sa.stage_idx + seg * kSWarpElems;
+        float* sval = on_chip ? s_pair_val + warp * L::kWarpPairs + before
+                              : sa.stage_val + seg * kSWarpElems;
 #pragma unroll
         for (int v = 0; v < kSUnits; ++v) {
           uint32_t pos = off[v];
@@ -301,18 +323,23 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   }
   const uint32_t lo = t_lo * kSWarps, hi = t_hi * kSWarps;
 
-  // The chunk's segment counts, a window at a time (the ring is free now):
-  // coalesced loads into shared memory, an exclusive scan there, then each
-  // warp copies kCopySegs adjacent segments at once with all of their loads
-  // in flight before the stores.
+  // The chunk's segments, a window at a time (the ring is free now): their
+  // counts and their warps' earlier pairs (coalesced loads; a segment was
+  // staged on chip iff the two add up to at most the warp's share), an
+  // exclusive scan of the counts into output offsets, then the copy.
   uint32_t* seg_off = reinterpret_cast<uint32_t*>(smem);
+  uint32_t* seg_pos = seg_off + L::kChunkSegs;  // the warp's earlier pairs
   constexpr int kNumWarps = kStreamThreads / 32;
   constexpr int kCopySegs = 8;
   bool overflow = false;
   for (uint32_t w0 = lo; w0 < hi; w0 += L::kChunkSegs) {
     const uint32_t n = hi - w0 < L::kChunkSegs ? hi - w0 : L::kChunkSegs;
     __syncthreads();
-    for (uint32_t i = threadIdx.x; i < n; i += kStreamThreads) seg_off[i] = __ldcg(sa.counts + w0 + i);
+    for (uint32_t i = threadIdx.x; i < n; i += kStreamThreads) {
+      const uint32_t packed = __ldcg(sa.counts + w0 + i);
+      seg_off[i] = packed & 0x1ffu;
+      seg_pos[i] = packed >> 9;
+    }
     __syncthreads();
     // each thread scans a contiguous run of the window in shared memory
     const uint32_t per = (n + kStreamThreads - 1) / kStreamThreads;
@@ -342,8 +369,12 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
     for (uint32_t i = b; i < e; ++i) seg_off[i] += thread_base;
     __syncthreads();
     const uint32_t window_end = base + window_total;
+    // each warp copies kCopySegs adjacent segments at once, all of their
+    // loads (shared memory for segments staged on chip) before the stores
     for (uint32_t i0 = warp * kCopySegs; i0 < n; i0 += kNumWarps * kCopySegs) {
       uint32_t dst[kCopySegs], cnt[kCopySegs], maxc = 0;
+      const uint32_t* src_i[kCopySegs];
+      const float* src_v[kCopySegs];
 #pragma unroll
       for (int u = 0; u < kCopySegs; ++u) {
         const uint32_t i = i0 + u;
@@ -351,6 +382,15 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
         const uint32_t next = i + 1 < n ? seg_off[i + 1] : window_end;
         cnt[u] = i < n ? next - dst[u] : 0u;
         maxc = cnt[u] > maxc ? cnt[u] : maxc;
+        const uint32_t pos = i < n ? seg_pos[i] : 0u;
+        if (pos + cnt[u] <= L::kWarpPairs) {
+          const uint32_t w = i % kSWarps;  // the segment's warp
+          src_i[u] = s_pair_idx + w * L::kWarpPairs + pos;
+          src_v[u] = s_pair_val + w * L::kWarpPairs + pos;
+        } else {
+          src_i[u] = sa.stage_idx + static_cast<size_t>(w0 + i) * kSWarpElems;
+          src_v[u] = sa.stage_val + static_cast<size_t>(w0 + i) * kSWarpElems;
+        }
       }
       for (uint32_t p0 = 0; p0 < maxc; p0 += 32) {
         uint32_t xi[kCopySegs];
@@ -358,9 +398,8 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
 #pragma unroll
         for (int u = 0; u < kCopySegs; ++u) {
           if (p0 + lane < cnt[u]) {
-            const size_t src = static_cast<size_t>(w0 + i0 + u) * kSWarpElems + p0 + lane;
-            xi[u] = __ldcs(sa.stage_idx + src);
-            xv[u] = __ldcs(sa.stage_val + src);
+            xi[u] = src_i[u][p0 + lane];
+            xv[u] = src_v[u][p0 + lane];
           }
         }
 #pragma unroll

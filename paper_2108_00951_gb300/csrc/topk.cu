@@ -206,6 +206,7 @@ struct TopkCandOp {
   uint32_t* other_state;    // the other state block: zeroed here for the next call
   static constexpr uint32_t kGBytes = kTileElems * sizeof(GT);
   static constexpr uint32_t kStageBytes = kGBytes + kTileElems * sizeof(float);
+  static constexpr uint32_t kWarpStagePairs = 512;  // on-chip staged pairs per compute warp
   static constexpr bool kPrepass = true;
   static constexpr int kSampleBins = efs::kSampleBins;
   static constexpr int kSampleShift = 31 - kSampleBits;  // key bits below the sampled ones
