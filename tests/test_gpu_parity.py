@@ -136,6 +136,38 @@ def test_ht_concurrent_streams():
 
 
 # ---------------------------------------------------------------------- Top-k
+# ------------------------------------------- on-chip staging and its spill
+# The streaming compaction keeps each compute warp's first pairs of its CTA's
+# chunk in shared memory (768 per warp for the hard-threshold op, 512 for the
+# Top-k candidate op) and spills the rest to global slots. At this size every
+# CTA owns several tiles, so dense chunks spill and sparse ones do not.
+SPILL_D = 3 * 2**20 + 4099
+
+
+@pytest.mark.parametrize("bf16", [False, True])
+def test_ht_spill_everything_sent(bf16):
+    g, e = _inputs(SPILL_D, 21, bf16=bf16)
+    _check_same(gu.ht(g, e, 0.1, 0.0), oracle.ef_hard_threshold(g, e, 0.1, 0.0), "all sent")
+
+
+def test_ht_spill_mixed_density():
+    g, e = _inputs(SPILL_D, 22)
+    g[: SPILL_D // 4] *= 1000.0  # a dense quarter (~96 % sent), the rest sends nothing
+    i, v, en = gu.ht(g, e, 0.1, 0.05)
+    assert i.size > 0.9 * (SPILL_D // 4) and i.max() < SPILL_D // 4
+    _check_same((i, v, en), oracle.ef_hard_threshold(g, e, 0.1, 0.05), "mixed")
+
+
+@pytest.mark.parametrize("region,k", [(SPILL_D // 50, 20_000), (SPILL_D // 5, SPILL_D // 16)])
+def test_topk_spill_concentrated_candidates(region, k):
+    # all candidates in the first `region` coordinates: the few CTAs there
+    # stage more than their warps' on-chip share (short and long lists)
+    g, e = _inputs(SPILL_D, 23)
+    g[:region] *= 1000.0
+    _check_same(gu.topk(g, e, 0.1, k), oracle.ef_topk(g, e, 0.1, k),
+                "region=%d k=%d" % (region, k))
+
+
 @pytest.mark.parametrize("d", RAGGED)
 def test_topk_random(d):
     g, e = _inputs(d, 11)
