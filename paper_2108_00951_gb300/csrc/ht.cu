@@ -88,7 +88,7 @@ struct HtOp {
   static constexpr uint32_t kWarpStagePairs = 768;  // on-chip staged pairs per compute warp
   static constexpr bool kPrepass = false;
   static constexpr int kSampleBins = 1;
-  __device__ void sample(const unsigned char*, uint32_t, int, int, uint32_t*) const {}
+  __device__ void sample(uint32_t, uint32_t, int, uint32_t*) const {}
   __device__ void merge(const uint32_t*) const {}
   __device__ void prologue() const {}
   __device__ bool barrier(uint64_t, uint32_t*) const { return true; }

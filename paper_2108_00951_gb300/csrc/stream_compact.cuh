@@ -47,10 +47,10 @@
 //        for the partial last tile.
 //   (tile_smem and tile_global also receive `aux`, the pre-pass result or 0)
 //   void prologue()                     every thread, once, at the start
-// Optional pre-pass (kPrepass): before streaming, the compute warps hand the
-// first tile of their CTA's chunk, from its ring stage, to
-//   void sample(const unsigned char* stage, uint32_t tile, int warp, int lane,
-//               uint32_t* s_hist)       (accumulate a kSampleBins histogram)
+// Optional pre-pass (kPrepass): before streaming, the compute threads sample
+// their CTA's chunk of tiles [t_lo, t_hi) with
+//   void sample(uint32_t t_lo, uint32_t t_hi, int tid, uint32_t* s_hist)
+//                                       (accumulate a kSampleBins histogram)
 // the CTA merges its histogram with
 //   void merge(const uint32_t* s_hist)  (all threads)
 // and after a grid barrier every CTA computes the same value with
@@ -166,12 +166,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   if constexpr (Op::kPrepass) {
     for (int b = threadIdx.x; b < Op::kSampleBins; b += kStreamThreads) s_sample_hist[b] = 0;
     __syncthreads();
-    if (warp < kSWarps && rounds > 0 && t_lo < full_tiles) {
-      if (!__all_sync(0xffffffffu, mbar_wait(&s_full[0], 0, ctx.wait_limit_ns)))
-        failed = true;
-      else
-        op.sample(smem, t_lo, warp, lane, s_sample_hist);
-    }
+    if (warp < kSWarps && rounds > 0) op.sample(t_lo, t_hi, threadIdx.x, s_sample_hist);
     if (__syncthreads_or(failed)) {
       if (threadIdx.x == 0) atomicOr(ctx.error, kDevErrTimeout);
       if (producer)  // no copy may land after the CTA exits

@@ -10,23 +10,27 @@
 // magnitudes. All K_j are distinct, so the Top-k set is exactly
 // { j : K_j >= K_(k) } for the k-th largest key K_(k).
 //
-// Kernels of one call (after clearing the small control block):
+// Kernels of one call:
 //  1 stream   the streaming compaction of stream_compact.cuh with a sampling
-//             pre-pass: every CTA histograms the top 11 key bits of the first
-//             tile of its chunk, the histograms are merged, and after a grid
-//             barrier every CTA derives the same lower bound B with about
-//             twice the needed mass above it (or, when the candidates would
-//             not fit, the full-array mode). Then a = fmaf(γ,g,e) is written
-//             over e (12 B per coordinate, the algorithmic bytes) and the
-//             coordinates with K_j >= B are emitted as an ordered (index,
-//             value) candidate list.
-//  2 select   radix select, digit by digit (11/10/10/11/11/10 bits), of the
-//             exact threshold K_(k) over the candidates — or over all of a
-//             when the candidates are short of k, overflowed, or were not
+//             pre-pass: every CTA histograms the top 13 key bits of 2048
+//             coordinates spread over its chunk, the histograms are merged,
+//             and after a grid barrier every CTA derives the same lower bound
+//             B with about 1.5 times the needed mass above it (or, when the
+//             candidates would not fit, the full-array mode). Then
+//             a = fmaf(γ,g,e) is written over e (12 B per coordinate, the
+//             algorithmic bytes) and the coordinates with K_j >= B are
+//             emitted as an ordered (index, value) candidate list. This
+//             kernel also zeroes the other of the two per-call state blocks
+//             for the next call.
+//  2 select   the exact threshold K_(k) over the candidates — or over all of
+//             a when the candidates are short of k, overflowed, or were not
 //             gathered — then the ordered compaction of K_j >= K_(k), zeroing
-//             e at the selected coordinates. Up to 65,536 candidates one CTA
-//             does all of it; beyond, the whole grid does (merged histograms
-//             with bounded grid barriers; chunk counts, then positions).
+//             e at the selected coordinates. Up to 48 K candidates CTA 0
+//             finds the threshold in shared memory (digit levels over the
+//             candidates' own magnitude range) and slice CTAs write the pairs
+//             in parallel; beyond, the whole grid runs a radix select (merged
+//             histograms with bounded grid barriers; chunk counts, then
+//             positions).
 // The candidate path moves about 12 B per coordinate plus small amounts; the
 // full-array path adds a read of a per digit level and two for the output.
 #include "gradient.cuh"
@@ -187,10 +191,9 @@ __device__ __forceinline__ void clear_state(uint32_t* block) {
 
 // ------------------------------------------------------------- 1 stream
 // The streaming pass as a stream_compact op. Pre-pass: every CTA histograms
-// the top 11 key bits of the first tile of its chunk (the tiles so sampled
-// are spread evenly over the vector), the histograms are merged, and after a
-// grid barrier every CTA derives the same lower bound B with about twice the
-// needed mass above it — or, when the candidates would not fit, chooses the
+// the top 13 key bits of 2048 coordinates spread evenly over its chunk, the
+// histograms are merged, and after a grid barrier every CTA derives the same
+// lower bound B with about 1.5 times the needed mass above it — or, when the candidates would not fit, chooses the
 // full-array mode and gathers none. Streaming: a = fmaf(γ,g,e) is written over
 // e and the coordinates with K_j >= B are selected (ordered candidates).
 template <typename GT>
@@ -235,16 +238,38 @@ struct TopkCandOp {
     x[3] = __fmaf_rn(gamma, gv[3], ev.w);
   }
 
-  __device__ void sample(const unsigned char* stage, uint32_t, int warp, int lane,
-                         uint32_t* s_hist) const {
-#pragma unroll
-    for (int v = 0; v < kSUnits; ++v) {
-      float x[4];
-      accumulate(stage, warp, lane, v, x);
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        hist_add_warp(s_hist, (__float_as_uint(x[j]) & 0x7fffffffu) >> kSampleShift, true);
+  // The sample: each compute thread reads one aligned group of 4 coordinates
+  // of g and e straight from global memory (issued together with the ring's
+  // first fills), the groups spread evenly over the CTA's chunk.
+  __device__ void sample(uint32_t t_lo, uint32_t t_hi, int tid, uint32_t* s_hist) const {
+    const uint64_t lo = static_cast<uint64_t>(t_lo) * kTileElems;
+    const uint64_t end = static_cast<uint64_t>(t_hi) * kTileElems;
+    const uint64_t hi = end < d ? end : d;
+    const uint64_t groups = (hi - lo) / 4;  // whole groups of 4 inside [lo, hi)
+    const uint64_t grp = groups >= static_cast<uint64_t>(kComputeThreads)
+                             ? static_cast<uint64_t>(tid) * groups / kComputeThreads
+                             : static_cast<uint64_t>(tid);
+    const bool in = grp < groups;
+    GradVec<GT> gv;
+    float4 ev = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    if (in) {
+      const uint64_t p = lo + grp * 4;
+      if constexpr (sizeof(GT) == 4)
+        gv.v = __ldg(reinterpret_cast<const float4*>(g + p));
+      else
+        gv.v = __ldg(reinterpret_cast<const uint2*>(g + p));
+      ev = __ldg(reinterpret_cast<const float4*>(e + p));
     }
+    float x[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    if (in) {
+      x[0] = __fmaf_rn(gamma, gv[0], ev.x);
+      x[1] = __fmaf_rn(gamma, gv[1], ev.y);
+      x[2] = __fmaf_rn(gamma, gv[2], ev.z);
+      x[3] = __fmaf_rn(gamma, gv[3], ev.w);
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      hist_add_warp(s_hist, (__float_as_uint(x[j]) & 0x7fffffffu) >> kSampleShift, in);
   }
 
   __device__ void merge(const uint32_t* s_hist) const {
