@@ -226,6 +226,13 @@ def profiled_traffic(kernel_tag: str, workload: str):
 
 
 # ------------------------------------------------------------ our arm
+def percentiles(xs):
+    """[p10, p50, p90] of a list, rounded."""
+    xs = sorted(xs)
+    pick = lambda q: xs[min(len(xs) - 1, int(q * (len(xs) - 1) + 0.5))]  # noqa: E731
+    return [round(pick(0.1), 2), round(pick(0.5), 2), round(pick(0.9), 2)]
+
+
 def ht_bytes(d, count, g_bytes=4):
     return (g_bytes + 8) * d + 8 * count
 
@@ -307,6 +314,8 @@ def run_ours(args):
         raise RuntimeError("device error during the timed steps")
 
     step_s = t0.elapsed_time(t1) / 1e3
+    # per-iteration segment times (µs per call: the segment of n calls / n)
+    seg_us = [[m[a].elapsed_time(m[a + 1]) * 1e3 for m in marks] for a in range(4)]
     ht_s = sum(m[0].elapsed_time(m[1]) for m in marks) / 1e3
     agg_ht_s = sum(m[1].elapsed_time(m[2]) for m in marks) / 1e3
     tk_s = sum(m[2].elapsed_time(m[3]) for m in marks) / 1e3
@@ -374,6 +383,12 @@ def run_ours(args):
         "aggregate_gbs": round(bytes_agg_ht / agg_ht_s / 1e9, 2),
         "aggregate_frac_of_peak": round(bytes_agg_ht / agg_ht_s / 1e9 / peak, 4),
         "aggregate_topk_ms_per_iter": round(agg_tk_s / args.steps * 1e3, 4),
+        "per_call_us_p10_p50_p90": {
+            "ht": percentiles([v / n for v in seg_us[0]]),
+            "topk": percentiles([v / n for v in seg_us[2]]),
+            "aggregate_ht": percentiles(seg_us[1]),
+            "aggregate_topk": percentiles(seg_us[3]),
+        },
         "frac_of_nominal_8tbs": round(value / NOMINAL_HBM_GBS, 4),
         "roofline": {
             "bound": "hbm",
