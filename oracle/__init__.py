@@ -12,6 +12,8 @@ passage behind every line):
 * ``ef_hard_threshold(g, e, gamma, lam)`` — hard-threshold sparsifier
   S_lambda = {j : |a_j| >= lambda} (Sec. 1, Sec. 4.2).
 * ``ef_topk(g, e, gamma, k)`` — Top-k sparsifier (Lemma 1, Lemma 2).
+* ``ef_topk_layerwise(g, e, gamma, seg_end, seg_k)`` — Top-k invoked on each
+  layer's tensor separately (Appendix, layer-wise sparsification).
 * ``sparse_aggregate(idx_list, val_list, d)`` — worker-ordered sum of the
   decompressed vectors (Algorithm 1, exchange step).
 
@@ -66,6 +68,13 @@ def _load():
                 fn = getattr(lib, name)
                 fn.argtypes = [gp, f32p, ctypes.c_float, ctypes.c_uint64, ctypes.c_uint64,
                                u32p, f32p, u32p]
+                fn.restype = ctypes.c_int
+            u64p = ctypes.POINTER(ctypes.c_uint64)
+            for name, gp in (("oracle_ef_topk_layerwise", f32p),
+                             ("oracle_ef_topk_layerwise_bf16", u16p)):
+                fn = getattr(lib, name)
+                fn.argtypes = [gp, f32p, ctypes.c_float, ctypes.c_uint32, u64p, u64p,
+                               ctypes.c_uint64, u32p, f32p, u32p]
                 fn.restype = ctypes.c_int
             lib.oracle_sparse_aggregate.argtypes = [
                 ctypes.c_uint32, ctypes.POINTER(u32p), ctypes.POINTER(f32p), u32p,
@@ -125,6 +134,33 @@ def ef_topk(g: np.ndarray, e: np.ndarray, gamma: float, k: int):
             _ptr(idx, ctypes.c_uint32), _ptr(val, ctypes.c_float), _ptr(cnt, ctypes.c_uint32))
     if rc != 0:
         raise RuntimeError("oracle_ef_topk failed (%d)" % rc)
+    c = int(cnt[0])
+    return idx[:c].copy(), val[:c].copy(), e_new
+
+
+def ef_topk_layerwise(g: np.ndarray, e: np.ndarray, gamma: float, seg_end, seg_k):
+    """One EF step with layer-wise Top-k: segment s = [seg_end[s-1], seg_end[s])
+    sends its seg_k[s] largest-magnitude coordinates; returns (idx, val, e_new)."""
+    lib = _load()
+    g, gctype, is_bf16 = _gradient(g)
+    e_new = np.array(e, dtype=np.float32, copy=True)
+    d = e_new.size
+    assert g.size == d
+    ends = np.ascontiguousarray(seg_end, dtype=np.uint64)
+    ks = np.ascontiguousarray(seg_k, dtype=np.uint64)
+    n_seg = ends.size
+    if n_seg < 1 or ks.size != n_seg:
+        raise ValueError("need one k per segment and at least one segment")
+    total = int(ks.sum())
+    idx = np.empty(max(total, 1), np.uint32)
+    val = np.empty(max(total, 1), np.float32)
+    cnt = np.zeros(1, np.uint32)
+    fn = lib.oracle_ef_topk_layerwise_bf16 if is_bf16 else lib.oracle_ef_topk_layerwise
+    rc = fn(_ptr(g, gctype), _ptr(e_new, ctypes.c_float), ctypes.c_float(gamma), n_seg,
+            _ptr(ends, ctypes.c_uint64), _ptr(ks, ctypes.c_uint64), d,
+            _ptr(idx, ctypes.c_uint32), _ptr(val, ctypes.c_float), _ptr(cnt, ctypes.c_uint32))
+    if rc != 0:
+        raise ValueError("oracle_ef_topk_layerwise rejected the segment table (%d)" % rc)
     c = int(cnt[0])
     return idx[:c].copy(), val[:c].copy(), e_new
 

@@ -175,6 +175,50 @@ int oracle_ef_topk_bf16(const uint16_t* g, float* e, float gamma, uint64_t k,
 }
 
 /* ------------------------------------------------------------------------
+ * Layer-wise Top-k (Appendix, "layer-wise or entire-model" sparsification:
+ * in layer-wise sparsification the sparsifier is invoked on each layer's
+ * tensor separately; the experiments use it for Top-k). The vector is the
+ * concatenation of n_seg tensors; segment s covers [seg_end[s-1], seg_end[s])
+ * (seg_end[-1] = 0, seg_end[n_seg-1] = d) and sends its k_s = seg_k[s]
+ * largest-magnitude coordinates under the Top-k rules above (R5, R6, R7).
+ * The pairs of all segments are emitted in ascending index order, so the
+ * message is the concatenation of the per-segment messages.
+ * ------------------------------------------------------------------------ */
+static int topk_layerwise_core(const float* g_f32, const uint16_t* g_bf16, float* e,
+                               float gamma, uint32_t n_seg, const uint64_t* seg_end,
+                               const uint64_t* seg_k, uint64_t d, uint32_t* idx,
+                               float* val, uint32_t* count) {
+  uint64_t lo = 0, sent = 0;
+  for (uint32_t s = 0; s < n_seg; ++s) {
+    uint64_t hi = seg_end[s];
+    if (hi < lo || hi > d || seg_k[s] > hi - lo) return 1;
+    uint32_t c = 0;
+    /* the Top-k sparsifier on this tensor alone: indices come out local */
+    int rc = topk_core(g_f32 ? g_f32 + lo : NULL, g_bf16 ? g_bf16 + lo : NULL, e + lo, gamma,
+                       seg_k[s], hi - lo, idx + sent, val + sent, &c);
+    if (rc != 0) return rc;
+    for (uint32_t p = 0; p < c; ++p) idx[sent + p] += (uint32_t)lo; /* to global indices */
+    sent += c;
+    lo = hi;
+  }
+  if (lo != d) return 1;
+  *count = (uint32_t)sent;
+  return 0;
+}
+
+int oracle_ef_topk_layerwise(const float* g, float* e, float gamma, uint32_t n_seg,
+                             const uint64_t* seg_end, const uint64_t* seg_k, uint64_t d,
+                             uint32_t* idx, float* val, uint32_t* count) {
+  return topk_layerwise_core(g, NULL, e, gamma, n_seg, seg_end, seg_k, d, idx, val, count);
+}
+
+int oracle_ef_topk_layerwise_bf16(const uint16_t* g, float* e, float gamma, uint32_t n_seg,
+                                  const uint64_t* seg_end, const uint64_t* seg_k, uint64_t d,
+                                  uint32_t* idx, float* val, uint32_t* count) {
+  return topk_layerwise_core(NULL, g, e, gamma, n_seg, seg_end, seg_k, d, idx, val, count);
+}
+
+/* ------------------------------------------------------------------------
  * Aggregation (Algorithm 1, exchange step): sum_i Delta_{i,t}, decompressed
  * into a dense vector. Sum, not mean (R9); from +0.0f; workers in order.
  * ------------------------------------------------------------------------ */

@@ -35,6 +35,10 @@ MUTANTS = {
                                  "for (uint32_t i = n; i-- > 0;) {")],
     "nan_ranks_lowest": [("    if (!ny) return 1;\n    if (!nx) return -1;",
                           "    if (!ny) return -1;\n    if (!nx) return 1;")],
+    "layerwise_local_indices": [("idx[sent + p] += (uint32_t)lo;", "idx[sent + p] += 0u;")],
+    "layerwise_first_k_everywhere": [("                       seg_k[s], hi - lo,",
+                                      "                       seg_k[0] < hi - lo ? seg_k[0] : hi - lo, hi - lo,")],
+    "layerwise_error_not_sliced": [("e + lo, gamma,", "e, gamma,")],
 }
 
 PIN_TESTS = [
@@ -51,6 +55,9 @@ PIN_TESTS = [
     pins.test_topk_nan_inf_order,
     pins.test_aggregate_sums_in_worker_order,
     lambda: pins.test_error_feedback_conserves_mass("ht"),
+    pins.test_topk_layerwise_hand_example,
+    lambda: pins.test_topk_layerwise_matches_bruteforce_per_segment(0),
+    lambda: pins.test_topk_layerwise_matches_bruteforce_per_segment(1),
 ]
 
 
@@ -61,7 +68,8 @@ def _swapped_library(path):
     lib = ctypes.CDLL(path)
     # reuse the argtypes of the real library
     for name in ("oracle_ef_hard_threshold", "oracle_ef_hard_threshold_bf16",
-                 "oracle_ef_topk", "oracle_ef_topk_bf16", "oracle_sparse_aggregate"):
+                 "oracle_ef_topk", "oracle_ef_topk_bf16", "oracle_ef_topk_layerwise",
+                 "oracle_ef_topk_layerwise_bf16", "oracle_sparse_aggregate"):
         fn, ref = getattr(lib, name), getattr(saved, name)
         fn.argtypes, fn.restype = ref.argtypes, ref.restype
     oracle._lib = lib

@@ -267,6 +267,107 @@ def test_topk_nan_inf_order():
     assert idx.tolist() == [1, 2, 3, 4]
 
 
+# --------------------------------------------------------------------------
+# Layer-wise Top-k (Appendix: in layer-wise sparsification the sparsifier is
+# invoked on each layer's tensor separately; hard-threshold is element-wise,
+# so for it layer-wise and entire-model coincide, while Top-k differs)
+# --------------------------------------------------------------------------
+
+def test_topk_layerwise_hand_example():
+    # tensors [1, -5, 2, 0.5] and [3, -1, 4] with k = (2, 1): the two largest
+    # magnitudes of the first are -5 (index 1) and 2 (index 2), the largest of
+    # the second is 4 (index 6); entire-model Top-3 takes -5, 3 and 4 instead
+    g = _f32([1, -5, 2, 0.5, 3, -1, 4])
+    e = np.zeros(7, np.float32)
+    idx, val, e_new = oracle.ef_topk_layerwise(g, e, 1.0, [4, 7], [2, 1])
+    assert idx.tolist() == [1, 2, 6]
+    assert val.tolist() == [-5.0, 2.0, 4.0]
+    assert e_new.tolist() == [1.0, 0.0, 0.0, 0.5, 3.0, -1.0, 0.0]
+    assert oracle.ef_topk(g, e, 1.0, 3)[0].tolist() == [1, 4, 6]
+
+
+def _random_table(rng, d):
+    """Segment ends (empty segments allowed) and k_s in [0, d_s]."""
+    cuts = np.sort(rng.integers(0, d + 1, int(rng.integers(0, 4))))
+    ends = [int(c) for c in cuts] + [d]
+    lo, ks = 0, []
+    for hi in ends:
+        ks.append(int(rng.integers(0, hi - lo + 1)))
+        lo = hi
+    return ends, ks
+
+
+@pytest.mark.parametrize("seed", range(10))
+def test_topk_layerwise_matches_bruteforce_per_segment(seed):
+    rng = np.random.default_rng(100 + seed)
+    d = int(rng.integers(1, 12))
+    pool = _f32([0.0, -0.0, 1.0, -1.0, 0.5, -2.0, 2.0])
+    e = pool[rng.integers(0, len(pool), d)] if seed % 2 else _f32(rng.standard_normal(d))
+    g = np.zeros(d, np.float32)
+    a = _exact_a(g, e, 1.0)
+    ends, ks = _random_table(rng, d)
+    idx, val, e_new = oracle.ef_topk_layerwise(g, e, 1.0, ends, ks)
+    want, err, lo = [], Fraction(0), 0
+    for hi, k in zip(ends, ks):   # each tensor's own optimum, at its offset
+        sel, seg_err = _bruteforce_topk(a[lo:hi].tolist(), k)
+        want += [lo + j for j in sel]
+        err += seg_err
+        lo = hi
+    assert idx.tolist() == want, (e, ends, ks)
+    assert _same_bits(val, a[want])
+    assert sum((to_frac(x) ** 2 for x in e_new), Fraction(0)) == err
+    rest = np.ones(d, bool)
+    rest[want] = False
+    assert _same_bits(e_new[rest], a[rest]) and not np.any(e_new[~rest])
+
+
+def test_topk_layerwise_one_segment_is_entire_model():
+    g = _f32(RNG.standard_normal(5000))
+    e = _f32(RNG.standard_normal(5000))
+    for k in (0, 1, 77, 5000):
+        got = oracle.ef_topk_layerwise(g, e, 0.4, [5000], [k])
+        ref = oracle.ef_topk(g, e, 0.4, k)
+        for x, y in zip(got, ref):
+            assert _same_bits(x, y) if x.dtype == np.float32 else np.array_equal(x, y)
+
+
+def test_ht_is_the_same_layerwise_and_entire_model():
+    # hard-threshold is element-wise: per-tensor calls, concatenated with
+    # their offsets, give the entire-model result
+    g = _f32(RNG.standard_normal(3000) * 0.01)
+    e = _f32(RNG.standard_normal(3000) * 0.001)
+    ref = oracle.ef_hard_threshold(g, e, 0.1, 2e-3)
+    parts, lo = [], 0
+    for hi in (700, 701, 2500, 3000):
+        i, v, en = oracle.ef_hard_threshold(g[lo:hi], e[lo:hi], 0.1, 2e-3)
+        parts.append((i + lo, v, en))
+        lo = hi
+    assert np.array_equal(np.concatenate([p[0] for p in parts]), ref[0])
+    assert _same_bits(np.concatenate([p[1] for p in parts]), ref[1])
+    assert _same_bits(np.concatenate([p[2] for p in parts]), ref[2])
+
+
+def test_topk_layerwise_bf16_is_the_widened_fp32():
+    g32 = _f32(RNG.standard_normal(4000))
+    g16 = (g32.view(np.uint32) >> 16).astype(np.uint16)     # truncation: exact bf16 values
+    gw = (g16.astype(np.uint32) << 16).view(np.float32)
+    e = _f32(RNG.standard_normal(4000))
+    got = oracle.ef_topk_layerwise(g16, e, 0.25, [1000, 1000, 4000], [10, 0, 300])
+    ref = oracle.ef_topk_layerwise(gw, e, 0.25, [1000, 1000, 4000], [10, 0, 300])
+    for x, y in zip(got, ref):
+        assert _same_bits(x, y) if x.dtype == np.float32 else np.array_equal(x, y)
+
+
+def test_topk_layerwise_rejects_bad_tables():
+    g = np.zeros(10, np.float32)
+    e = np.zeros(10, np.float32)
+    for ends, ks in (([5, 10], [6, 0]),      # k_s above the segment's length
+                     ([5, 9], [1, 1]),       # does not end at d
+                     ([6, 5, 10], [0, 0, 0])):  # decreasing ends
+        with pytest.raises(ValueError):
+            oracle.ef_topk_layerwise(g, e, 1.0, ends, ks)
+
+
 def test_ht_at_kth_magnitude_selects_topk():
     # Sec. 4.3 (Lemma 3 argument): with distinct magnitudes and
     # lambda in (|a|_(k+1), |a|_(k)], C_lambda keeps exactly the Top-k set
