@@ -144,6 +144,47 @@ ef_status ef_topk_bf16(const uint16_t* g, float* e, float gamma, uint64_t k,
                        uint32_t* count_out, ef_stream_t stream);
 
 /*
+ * ef_topk_layerwise — EF accumulate + layer-wise Top-k + compaction + residual.
+ *
+ * Defines: Algorithm 1 with C = Top-k applied to each tensor of the model on
+ * its own (the experiments of Sec. 6 compress layer by layer, with k_t a
+ * fraction of each layer; the Appendix section on layer-wise compression).
+ * The d coordinates form n_seg consecutive segments,
+ * segment s = [seg_end[s-1], seg_end[s]) (seg_end[-1] = 0), and segment s
+ * sends its seg_k[s] largest-magnitude coordinates with the ef_topk rules
+ * (ties to the lowest index, NaN above +inf, exactly seg_k[s] pairs). The
+ * hard-threshold sparsifier acts per coordinate, so it needs no layer-wise
+ * variant: ef_hard_threshold already gives it.
+ *
+ *   g, e, gamma, d   as for ef_topk.
+ *   n_seg      number of segments, 1 <= n_seg < 2^31.
+ *   seg_end    HOST array of n_seg uint64: the segments' exclusive ends,
+ *              non-decreasing, seg_end[n_seg-1] == d (empty segments allowed).
+ *   seg_k      HOST array of n_seg uint64: pairs sent by each segment,
+ *              0 <= seg_k[s] <= seg_end[s] - seg_end[s-1].
+ *   idx_out    [out] uint32[capacity >= K], K = sum of seg_k; segment s fills
+ *              positions [seg_k[0] + ... + seg_k[s-1], ... + seg_k[s]) in
+ *              ascending index, so the whole list is strictly ascending.
+ *   val_out    [out] fp32[capacity >= K], val_out[p] = a[idx_out[p]].
+ *   count_out  [out] one uint32 in device memory; always equals K.
+ *   The library copies the segment table to the device when it differs from
+ *   the previous call's on this stream (so a fixed table costs nothing after
+ *   the first call); growing that copy synchronises the stream once. Both
+ *   host arrays may be reused as soon as the call returns.
+ */
+ef_status ef_topk_layerwise(const float* g, float* e, float gamma, uint32_t n_seg,
+                            const uint64_t* seg_end, const uint64_t* seg_k, uint64_t d,
+                            uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                            ef_stream_t stream);
+
+/* ef_topk_layerwise_bf16 — ef_topk_layerwise with a bfloat16 gradient,
+ * widened as in ef_hard_threshold_bf16. */
+ef_status ef_topk_layerwise_bf16(const uint16_t* g, float* e, float gamma, uint32_t n_seg,
+                                 const uint64_t* seg_end, const uint64_t* seg_k, uint64_t d,
+                                 uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                                 ef_stream_t stream);
+
+/*
  * sparse_aggregate — decompress and sum n workers' sparse vectors.
  *
  * Defines: Algorithm 1's exchange step, Delta_bar = (1/n) sum_i Delta_{i,t},

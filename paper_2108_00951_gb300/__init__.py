@@ -21,6 +21,7 @@ from ._binding import (  # noqa: F401
     ef_kernel_launches,
     ef_test_set_lookback_fault,
     ef_topk,
+    ef_topk_layerwise,
     ef_workspace_release,
     library_path,
     load_library,

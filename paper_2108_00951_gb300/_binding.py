@@ -12,6 +12,7 @@ import ctypes
 import os
 import threading
 
+import numpy as np
 import torch
 
 from . import build as _build
@@ -58,6 +59,8 @@ def load_library(build_if_missing: bool = True):
             "ef_hard_threshold_bf16": [vp, vp, f32, f32, u64, vp, vp, vp, vp],
             "ef_topk": [vp, vp, f32, u64, u64, vp, vp, vp, vp],
             "ef_topk_bf16": [vp, vp, f32, u64, u64, vp, vp, vp, vp],
+            "ef_topk_layerwise": [vp, vp, f32, u32, vp, vp, u64, vp, vp, vp, vp],
+            "ef_topk_layerwise_bf16": [vp, vp, f32, u32, vp, vp, u64, vp, vp, vp, vp],
             "sparse_aggregate": [u32, ctypes.POINTER(vp), ctypes.POINTER(vp), vp, u64, vp, vp],
             "ef_check_status": [vp],
             "ef_workspace_release": [],
@@ -144,6 +147,32 @@ def ef_topk(g, e, gamma, k, idx_out, val_out, count_out, stream=None):
             _dev(count_out, "count_out", torch.int32, 1), _stream(stream))
     fn = lib.ef_topk_bf16 if bf16 else lib.ef_topk
     _check(fn(*args), "ef_topk")
+
+
+def ef_topk_layerwise(g, e, gamma, seg_end, seg_k, idx_out, val_out, count_out, stream=None):
+    """EF accumulate + layer-wise Top-k + compaction (``ef_topk_layerwise[_bf16]``).
+
+    ``seg_end``/``seg_k``: sequences of n_seg integers (host side): segment s
+    is ``[seg_end[s-1], seg_end[s])`` and sends its ``seg_k[s]`` largest
+    coordinates; exactly ``sum(seg_k)`` pairs are written.
+    """
+    lib = load_library()
+    bf16 = _gradient(g)
+    d = e.numel()
+    if g.numel() != d:
+        raise ValueError("g and e differ in length")
+    ends = np.ascontiguousarray(seg_end, dtype=np.uint64)
+    ks = np.ascontiguousarray(seg_k, dtype=np.uint64)
+    if ends.ndim != 1 or ks.shape != ends.shape:
+        raise ValueError("seg_end and seg_k must be 1-D of one length")
+    total = int(ks.sum()) if ks.size else 0
+    args = (_dev(g, "g", g.dtype), _dev(e, "e", torch.float32), ctypes.c_float(gamma),
+            ctypes.c_uint32(ends.size), ctypes.c_void_p(ends.ctypes.data),
+            ctypes.c_void_p(ks.ctypes.data), d, _dev(idx_out, "idx_out", torch.int32, total),
+            _dev(val_out, "val_out", torch.float32, total),
+            _dev(count_out, "count_out", torch.int32, 1), _stream(stream))
+    fn = lib.ef_topk_layerwise_bf16 if bf16 else lib.ef_topk_layerwise
+    _check(fn(*args), "ef_topk_layerwise")
 
 
 def sparse_aggregate(idx_list, val_list, counts, d, dense_out, stream=None):

@@ -1,6 +1,7 @@
 // api.cu — the extern "C" boundary declared in include/efsparse.h: host-side
 // argument checks, the per-(device, stream) workspaces, and status reporting.
-// Every compute step runs in the kernels of ht.cu, topk.cu and aggregate.cu.
+// Every compute step runs in the kernels of ht.cu, topk.cu, topk_layerwise.cu
+// and aggregate.cu.
 #include <atomic>
 #include <cmath>
 #include <cstring>
@@ -40,6 +41,7 @@ ef_status device_info(int dev, DeviceInfo* out) {
       return EF_ERR_CUDA;
     ht_init_device(info);
     topk_init_device(info);
+    topk_layerwise_init_device(info);
     if (info.refine_blocks <= 0 || info.finalize_blocks <= 0) return EF_ERR_CUDA;
     it = g_devices.emplace(dev, info).first;
   }
@@ -94,6 +96,7 @@ ef_status acquire_workspace(cudaStream_t stream, uint32_t tiles, uint32_t cand_c
       return EF_ERR_CUDA;
     ws->epoch = 0;
     ws->dirty = false;
+    if (ws->lw) ws->lw->valid = false;  // re-upload the tables, re-zero their counters
   }
   *out = ws;
   return EF_OK;
@@ -181,6 +184,53 @@ ef_status topk_entry(const void* g, bool bf16, float* e, float gamma, uint64_t k
                        ws);
 }
 
+ef_status topk_layerwise_entry(const void* g, bool bf16, float* e, float gamma, uint32_t n_seg,
+                               const uint64_t* seg_end, const uint64_t* seg_k, uint64_t d,
+                               uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                               cudaStream_t stream) {
+  const size_t gsz = bf16 ? 2 : 4;
+  if (!count_out || !aligned(count_out, 4)) return EF_ERR_INVALID_ARG;
+  if (!std::isfinite(gamma) || d > kMaxD) return EF_ERR_INVALID_ARG;
+  if (n_seg == 0 || n_seg >= (1u << 31) || !seg_end || !seg_k) return EF_ERR_INVALID_ARG;
+  uint64_t lo = 0, total_k = 0;
+  for (uint32_t s = 0; s < n_seg; ++s) {
+    if (seg_end[s] < lo || seg_end[s] > d || seg_k[s] > seg_end[s] - lo)
+      return EF_ERR_INVALID_ARG;
+    total_k += seg_k[s];
+    lo = seg_end[s];
+  }
+  if (lo != d) return EF_ERR_INVALID_ARG;
+  if (d == 0) return write_zero_count(count_out, stream);
+  if (!g || !e || (total_k > 0 && (!idx_out || !val_out))) return EF_ERR_INVALID_ARG;
+  if (!aligned(g, gsz) || !aligned(e, 4) || !aligned(idx_out, 4) || !aligned(val_out, 4))
+    return EF_ERR_INVALID_ARG;
+  const size_t nb = static_cast<size_t>(d) * 4, kb = static_cast<size_t>(total_k) * 4;
+  const void* outs[3] = {idx_out, val_out, count_out};
+  const size_t out_n[3] = {kb, kb, 4};
+  for (int o = 0; o < 3; ++o) {
+    if (overlaps(outs[o], out_n[o], g, d * gsz) || overlaps(outs[o], out_n[o], e, nb))
+      return EF_ERR_INVALID_ARG;
+    for (int p = o + 1; p < 3; ++p)
+      if (overlaps(outs[o], out_n[o], outs[p], out_n[p])) return EF_ERR_INVALID_ARG;
+  }
+  if (overlaps(g, d * gsz, e, nb)) return EF_ERR_INVALID_ARG;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
+  DeviceInfo info;
+  ef_status st = device_info(dev, &info);
+  if (st != EF_OK) return st;
+  Workspace* ws = nullptr;
+  st = acquire_workspace(stream, tiles_for(d), topk_candidate_capacity(d), 0,
+                         static_cast<size_t>(tiles_for(d)) * kTileElems, &ws);
+  if (st != EF_OK) return st;
+  const cudaError_t perr = lw_prepare(*ws, seg_end, seg_k, n_seg, d, info);
+  if (perr == cudaErrorMemoryAllocation) return EF_ERR_NO_MEMORY;
+  if (perr != cudaSuccess) return EF_ERR_CUDA;
+  return finish_launch(launch_topk_layerwise(g, bf16, e, gamma, static_cast<uint32_t>(d),
+                                             idx_out, val_out, count_out, *ws, info),
+                       ws);
+}
+
 }  // namespace
 
 void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
@@ -235,6 +285,22 @@ ef_status ef_topk_bf16(const uint16_t* g, float* e, float gamma, uint64_t k, uin
                        ef_stream_t stream) {
   return efs::topk_entry(g, true, e, gamma, k, d, idx_out, val_out, count_out,
                          reinterpret_cast<cudaStream_t>(stream));
+}
+
+ef_status ef_topk_layerwise(const float* g, float* e, float gamma, uint32_t n_seg,
+                            const uint64_t* seg_end, const uint64_t* seg_k, uint64_t d,
+                            uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                            ef_stream_t stream) {
+  return efs::topk_layerwise_entry(g, false, e, gamma, n_seg, seg_end, seg_k, d, idx_out,
+                                   val_out, count_out, reinterpret_cast<cudaStream_t>(stream));
+}
+
+ef_status ef_topk_layerwise_bf16(const uint16_t* g, float* e, float gamma, uint32_t n_seg,
+                                 const uint64_t* seg_end, const uint64_t* seg_k, uint64_t d,
+                                 uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                                 ef_stream_t stream) {
+  return efs::topk_layerwise_entry(g, true, e, gamma, n_seg, seg_end, seg_k, d, idx_out,
+                                   val_out, count_out, reinterpret_cast<cudaStream_t>(stream));
 }
 
 ef_status sparse_aggregate(uint32_t n, const uint32_t* const* idx, const float* const* val,
@@ -309,6 +375,10 @@ ef_status ef_workspace_release(void) {
   for (auto it = efs::g_workspaces.begin(); it != efs::g_workspaces.end();) {
     if (it->first.first == dev) {
       if (it->second->base) cudaFree(it->second->base);
+      if (it->second->lw) {
+        if (it->second->lw->dev) cudaFree(it->second->lw->dev);
+        delete it->second->lw;
+      }
       delete it->second;
       it = efs::g_workspaces.erase(it);
     } else {

@@ -4,6 +4,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <vector>
 #include <cuda_runtime.h>
 
 #include "common.cuh"
@@ -37,6 +38,46 @@ constexpr size_t kHeaderBytes = kOffTkState + 2 * kTkStateBytes;
 constexpr uint32_t kMaxChunks = 1024;   // per-CTA chunk sums of the streaming compaction
 constexpr uint32_t kCountsPerTile = 16; // per-segment counts of the streaming compaction
 
+// ---- layer-wise Top-k: one Top-k selection per segment of the vector.
+// Segment kinds: nothing sent (k = 0); the whole segment selected in one
+// CTA's shared memory; a sampled candidate bound, then a selection over the
+// candidates; every coordinate sent (k = d_s).
+constexpr uint32_t kLwNone = 0, kLwWhole = 1, kLwSampled = 2, kLwAll = 3;
+constexpr uint32_t kLwSmemElems = 48u * 1024u;  // values one select CTA holds in shared memory
+constexpr uint32_t kLwNoBound = 0xffffffffu;    // candidate bound that admits nothing
+constexpr uint32_t kLwTileUniform = 0x80000000u;  // tile_info: the tile lies in one segment
+constexpr uint32_t kLwSampleGroupsPerCta = 4096;  // sampled groups of 4 coordinates per CTA
+
+struct LwSeg {      // one segment (device and host layout)
+  uint32_t lo, hi;  // coordinates [lo, hi)
+  uint32_t k;       // pairs it sends
+  uint32_t out;     // output position of its first pair
+  uint32_t kind;    // kLw*
+  uint32_t slot;    // sampled: its histogram slot
+  uint32_t nblk;    // sampled: its sampling CTAs
+  uint32_t groups;  // sampled: its sampled groups of 4 consecutive coordinates
+};
+struct LwSample {   // one sampling CTA: groups [q0, q1) of segment seg
+  uint32_t seg, q0, q1, pad;
+};
+
+// The device tables of a segment table, rebuilt when the table changes.
+struct LwPlan {
+  std::vector<uint64_t> seg_end, seg_k;  // the host table this plan was built from
+  uint64_t d = 0;
+  bool valid = false;
+  uint32_t n_seg = 0, n_sampled = 0, n_sample_ctas = 0, n_select_ctas = 0, tiles = 0;
+  uint64_t total_k = 0;
+  std::vector<char> image;  // host image of the uploaded part
+  char* dev = nullptr;
+  size_t dev_bytes = 0;
+  // byte offsets in dev: uploaded tables, then zero-initialised counters
+  // and histograms (each user resets its own), then per-call outputs
+  size_t off_segs = 0, off_seg_end = 0, off_mbound = 0, off_tile_info = 0, off_samples = 0,
+         off_work_ptr = 0, off_work_seg = 0, off_done = 0, off_hist = 0, off_tile_base = 0,
+         total = 0;
+};
+
 struct Workspace {
   int device = -1;
   cudaStream_t stream = nullptr;
@@ -49,6 +90,7 @@ struct Workspace {
   uint32_t epoch = 0;          // last epoch handed to a compaction launch
   uint32_t topk_calls = 0;     // Top-k calls so far: their parity picks the state block
   bool dirty = false;          // header must be re-cleared (failed launch or device timeout)
+  LwPlan* lw = nullptr;        // layer-wise Top-k tables (created on first use)
 
   // Regions after the header, each 256-byte aligned.
   static size_t align(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
@@ -90,10 +132,15 @@ struct DeviceInfo {
   int ht_stream_per_sm_bf16 = 0;
   int tk_stream_per_sm_f32 = 0;   // streaming Top-k candidate pass CTAs per SM
   int tk_stream_per_sm_bf16 = 0;
+  int lw_stream_per_sm_f32 = 0;   // streaming layer-wise candidate pass CTAs per SM
+  int lw_stream_per_sm_bf16 = 0;
 };
 
 // Per-device set-up of the Top-k kernels (shared-memory opt-in, occupancy).
 void topk_init_device(DeviceInfo& info);
+
+// Per-device set-up of the layer-wise Top-k kernels.
+void topk_layerwise_init_device(DeviceInfo& info);
 
 // Per-device set-up of the streaming hard-threshold kernels (opts them into
 // their shared-memory ring on the current device and records occupancy).
@@ -116,6 +163,13 @@ cudaError_t launch_hard_threshold_lookback(const float* g, float* e, float gamma
 cudaError_t launch_topk(const void* g, bool g_bf16, float* e, float gamma, uint32_t k,
                         uint32_t d, uint32_t* idx_out, float* val_out, uint32_t* count_out,
                         Workspace& ws, const DeviceInfo& dev);
+// Layer-wise Top-k: lw_prepare builds and uploads the plan of a segment
+// table (a no-op when the workspace already holds that table's plan).
+cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* seg_k,
+                       uint32_t n_seg, uint64_t d, const DeviceInfo& dev);
+cudaError_t launch_topk_layerwise(const void* g, bool g_bf16, float* e, float gamma, uint32_t d,
+                                  uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                                  Workspace& ws, const DeviceInfo& dev);
 cudaError_t launch_aggregate(uint32_t n, const uint32_t* const* idx, const float* const* val,
                              const uint32_t* counts, uint32_t d, float* dense_out,
                              Workspace& ws);

@@ -85,6 +85,8 @@ struct StreamArgs {
   float* stage_val;      // [num_tiles * kTileElems] staged values
   uint32_t* counts;      // [num_tiles * kSWarps] selected per segment
   uint64_t* chunk_sums;  // [gridDim.x] (epoch << 32) | chunk total
+  uint32_t* tile_base;   // optional [num_tiles + 1]: output position of each tile's first
+                         // pair, and the total (untruncated), or null
 };
 
 // A segment's count (<= 256: 9 bits) and its warp's earlier pairs in the
@@ -361,7 +363,11 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
       window_total += x;
     }
     const uint32_t thread_base = base + warp_base + incl - run;
-    for (uint32_t i = b; i < e; ++i) seg_off[i] += thread_base;
+    for (uint32_t i = b; i < e; ++i) {
+      seg_off[i] += thread_base;
+      // windows start at whole tiles, so a tile's first segment has i % kSWarps == 0
+      if (sa.tile_base && i % kSWarps == 0) sa.tile_base[(w0 + i) / kSWarps] = seg_off[i];
+    }
     __syncthreads();
     const uint32_t window_end = base + window_total;
     // each warp copies kCopySegs adjacent segments at once, all of their
@@ -413,7 +419,10 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
     }
     base = window_end;
   }
-  if (hi == T * kSWarps && threadIdx.x == 0) *count_out = base < cap ? base : cap;
+  if (hi == T * kSWarps && threadIdx.x == 0) {
+    *count_out = base < cap ? base : cap;
+    if (sa.tile_base) sa.tile_base[T] = base;
+  }
   if (__syncthreads_or(overflow) && threadIdx.x == 0) atomicOr(ctx.error, kDevErrOverflow);
 }
 

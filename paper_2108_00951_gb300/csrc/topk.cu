@@ -35,6 +35,7 @@
 // full-array path adds a read of a per digit level and two for the output.
 #include "gradient.cuh"
 #include "internal.h"
+#include "select.cuh"
 #include "stream_compact.cuh"
 
 namespace efs {
@@ -72,122 +73,6 @@ struct TopkArgs {
   uint32_t epoch;        // tags the finalize kernel's chunk totals
   uint64_t wait_limit_ns;
 };
-
-// Lanes holding equal bins add once, with the number of lanes.
-__device__ __forceinline__ void hist_add_warp(uint32_t* h, uint32_t bin, bool valid) {
-  const uint32_t key = valid ? bin : 0xffffffffu;
-  const uint32_t peers = __match_any_sync(0xffffffffu, key);
-  if (valid && (__ffs(peers) - 1) == static_cast<int>(threadIdx.x & 31))
-    atomicAdd(&h[bin], static_cast<uint32_t>(__popc(peers)));
-}
-
-struct Selection {
-  uint32_t bin, k_rem, n_in, found;
-};
-
-// Exclusive suffix sum over the threads of the CTA (the sum of v over every
-// higher thread index) and the block total. Whole CTA; blockDim.x a multiple
-// of 32; s_w holds blockDim.x / 32 words.
-__device__ __forceinline__ uint32_t block_suffix_exclusive(uint32_t v, uint32_t& total,
-                                                           uint32_t* s_w) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int nw = static_cast<int>(blockDim.x >> 5);
-  uint32_t incl = v;  // v summed over this lane and the higher lanes
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const uint32_t x = __shfl_down_sync(0xffffffffu, incl, o);
-    if (lane + o < 32) incl += x;
-  }
-  __syncthreads();  // a previous use of s_w is complete
-  if (lane == 0) s_w[warp] = incl;
-  __syncthreads();
-  uint32_t wsuf = lane < nw ? s_w[lane] : 0u;  // warp totals over warps >= lane
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const uint32_t x = __shfl_down_sync(0xffffffffu, wsuf, o);
-    if (lane + o < 32) wsuf += x;
-  }
-  total = __shfl_sync(0xffffffffu, wsuf, 0);
-  const uint32_t higher = __shfl_sync(0xffffffffu, wsuf, (warp + 1) & 31);
-  return (warp + 1 < 32 ? higher : 0u) + incl - v;
-}
-
-// Find the bin holding the k_rem-th largest key of a histogram of nbins
-// (2048 or 1024) bins, scanning from the highest bin. Whole CTA of kBlock
-// threads (kBlock <= nbins); uniform result. kGlobal: the histogram is in
-// global memory (read through L2), else in shared memory. s_w holds
-// kBlock / 32 words.
-template <int kBlock, bool kGlobal>
-__device__ Selection select_bin(const uint32_t* hist, uint32_t nbins, uint32_t k_rem,
-                                uint32_t* s_w) {
-  constexpr int kMaxPer = kHistBins / kBlock;
-  __shared__ Selection s_sel;
-  const int t = threadIdx.x;
-  const uint32_t per = nbins / kBlock;
-  uint32_t c[kMaxPer];
-  uint32_t sum = 0;
-#pragma unroll
-  for (int i = 0; i < kMaxPer; ++i) {
-    c[i] = (static_cast<uint32_t>(i) < per)
-               ? (kGlobal ? __ldcg(hist + t * per + i) : hist[t * per + i]) : 0u;
-    sum += c[i];
-  }
-  if (t == 0) s_sel = Selection{0, 0, 0, 0};
-  uint32_t total;
-  const uint32_t above = block_suffix_exclusive(sum, total, s_w);  // orders the reset
-  if (above < k_rem && k_rem - above <= sum) {
-    uint32_t r = k_rem - above;
-    bool done = false;
-#pragma unroll
-    for (int i = kMaxPer - 1; i >= 0; --i) {
-      if (!done && static_cast<uint32_t>(i) < per) {
-        if (c[i] >= r) {
-          s_sel = Selection{t * per + i, r, c[i], 1u};
-          done = true;
-        } else {
-          r -= c[i];
-        }
-      }
-    }
-  }
-  __syncthreads();
-  const Selection s = s_sel;
-  __syncthreads();
-  return s;
-}
-
-// Exclusive block-wide prefix sum of one value per thread; also returns the
-// block total. Whole CTA of kBlock threads; s_w holds kBlock/32 words.
-template <int kBlock>
-__device__ __forceinline__ uint32_t block_exclusive(uint32_t v, uint32_t& total, uint32_t* s_w) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  uint32_t incl = v;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const uint32_t x = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += x;
-  }
-  __syncthreads();
-  if (lane == 31) s_w[warp] = incl;
-  __syncthreads();
-  uint32_t before = 0;
-  total = 0;
-  for (int w = 0; w < kBlock / 32; ++w) {
-    const uint32_t x = s_w[w];
-    before += w < warp ? x : 0u;
-    total += x;
-  }
-  return before + incl - v;
-}
-
-// Zeroes a Top-k state block, the grid's threads striding over it (the
-// block belongs to the previous call on the workspace, which is complete).
-__device__ __forceinline__ void clear_state(uint32_t* block) {
-  constexpr uint32_t kWords = static_cast<uint32_t>(kTkStateBytes / sizeof(uint4));
-  uint4* b4 = reinterpret_cast<uint4*>(block);
-  for (uint32_t w = blockIdx.x * blockDim.x + threadIdx.x; w < kWords; w += gridDim.x * blockDim.x)
-    b4[w] = make_uint4(0u, 0u, 0u, 0u);
-}
 
 // ------------------------------------------------------------- 1 stream
 // The streaming pass as a stream_compact op. Pre-pass: every CTA histograms
@@ -550,37 +435,10 @@ __device__ uint32_t write_selected(const TopkArgs& args, float* e, uint32_t mode
 // zeroing the residual at each.
 constexpr uint32_t kSliceElems = 4 * kSelThreads;  // list positions per slice CTA
 
-struct SmallSelection {
-  uint32_t B;       // threshold magnitude bits
-  uint32_t ties;    // 1: magnitudes equal to B are taken only up to `last`
-  uint32_t last;    // list position of the last taken magnitude equal to B
-};
-
-// Histogram pass of a level over `cnt` magnitudes of `src`: those in the
-// window [B, B + W) (W == 0: all) add to bin (m - B) >> sh.
-__device__ __forceinline__ void window_hist(const uint32_t* src, uint32_t cnt, uint32_t B,
-                                            uint32_t W, int sh, uint32_t* s_hist) {
-  for (uint32_t b0 = threadIdx.x; b0 < cnt; b0 += 4 * kSelThreads) {
-    uint32_t m[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const uint32_t i = b0 + j * kSelThreads;
-      m[j] = i < cnt ? src[i] : 0u;
-    }
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const uint32_t off = m[j] - B;
-      if (b0 + j * kSelThreads < cnt && m[j] >= B && (W == 0 || off < W))
-        atomicAdd(&s_hist[off >> sh], 1u);
-    }
-  }
-}
-
 // CTA 0: the threshold of the list; returns false when the histograms do
 // not find the rank (never for a well-formed list).
 __device__ bool small_threshold(const TopkArgs& args, uint32_t n, uint32_t k, uint32_t* s_mag,
                                 uint32_t* s_hist, uint32_t* s_w, SmallSelection& out) {
-  __shared__ uint32_t s_last;
   __shared__ uint32_t s_lo[32], s_hi[32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int kBatch = 8;  // loads in flight per thread
@@ -620,50 +478,7 @@ __device__ bool small_threshold(const TopkArgs& args, uint32_t n, uint32_t k, ui
     lo = min(lo, __shfl_xor_sync(0xffffffffu, lo, o));
     hi = max(hi, __shfl_xor_sync(0xffffffffu, hi, o));
   }
-  // digit levels over the window [B, B + W); W == 0: the whole [lo, hi]
-  uint32_t B = lo, W = 0, k_rem = k, n_in = n;
-  int sh = 0;
-  while (((hi - lo) >> sh) >= static_cast<uint32_t>(kHistBins)) ++sh;
-  if (hi == lo) W = 1;  // every candidate has the same magnitude
-  while (W != 1 && n_in != k_rem) {
-    for (uint32_t b = tid; b < static_cast<uint32_t>(kHistBins); b += kSelThreads) s_hist[b] = 0;
-    __syncthreads();
-    window_hist(s_mag, n, B, W, sh, s_hist);
-    __syncthreads();
-    const Selection s = select_bin<kSelThreads, false>(s_hist, kHistBins, k_rem, s_w);
-    if (!s.found) return false;
-    B += s.bin << sh;
-    W = 1u << sh;
-    k_rem = s.k_rem;
-    n_in = s.n_in;
-    int bits = 0;
-    while ((1u << bits) < W) ++bits;
-    sh = bits > 11 ? bits - 11 : 0;
-  }
-  // at a one-wide threshold with more equal magnitudes than are taken, only
-  // the first k_rem of them in list order
-  const bool ties = W == 1 && n_in != k_rem;
-  if (tid == 0) s_last = 0xffffffffu;
-  if (ties) {
-    const uint32_t per = (n + kSelThreads - 1) / kSelThreads;
-    const uint32_t a0 = tid * per < n ? tid * per : n, a1 = a0 + per < n ? a0 + per : n;
-    uint32_t cnt = 0;
-    for (uint32_t i = a0; i < a1; ++i) cnt += s_mag[i] == B ? 1u : 0u;
-    uint32_t total;
-    const uint32_t before = block_exclusive<kSelThreads>(cnt, total, s_w);
-    if (before < k_rem && k_rem <= before + cnt) {
-      uint32_t r = k_rem - before;
-      for (uint32_t i = a0; i < a1; ++i)
-        if (s_mag[i] == B && --r == 0) {
-          s_last = i;
-          break;
-        }
-    }
-  }
-  __syncthreads();
-  const uint32_t last = ties ? s_last : 0xffffffffu;
-  out = SmallSelection{B, ties ? 1u : 0u, last};
-  return true;
+  return threshold_levels<kSelThreads>(MagsShared{s_mag}, n, k, lo, hi, s_hist, s_w, out);
 }
 
 // Slice CTA c of Gs: the selected pairs of list positions [c, c+1) * n / Gs.

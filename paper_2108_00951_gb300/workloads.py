@@ -176,6 +176,22 @@ def gradient(w: Workload, worker: int, iteration: int, device="cpu",
     return g.to(dtype) if dtype != torch.float32 else g
 
 
+def segment_ends(w: Workload) -> List[int]:
+    """Exclusive end of each parameter tensor in the flattened vector."""
+    out, acc = [], 0
+    for n in w.segments:
+        acc += n
+        out.append(acc)
+    return out
+
+
+def layerwise_k(w: Workload, frac: float) -> List[int]:
+    """Per-tensor Top-k budgets k_s = max(1, floor(frac * d_s)) (0 for an
+    empty tensor): the layer-wise compression of the paper's experiments
+    keeps the same fraction of every layer."""
+    return [max(1, int(frac * n)) if n > 0 else 0 for n in w.segments]
+
+
 def density_lambda(w: Workload, g0: torch.Tensor, density: float) -> float:
     """lambda such that the first EF iteration (e = 0, so a = gamma g) sends
     about `density` of the coordinates: the ceil(density * d)-th largest

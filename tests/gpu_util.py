@@ -66,6 +66,18 @@ def topk(g, e, gamma, k, g_off=0, e_off=0):
     return idx[:c].cpu().numpy().view(np.uint32), val[:c].cpu().numpy(), ed.cpu().numpy()
 
 
+def topk_layerwise(g, e, gamma, seg_end, seg_k, g_off=0, e_off=0):
+    gd, ed = g_device(g, g_off), to_dev(e, e_off)
+    total = int(np.sum(np.asarray(seg_k, dtype=np.uint64)))
+    idx = torch.full((max(total, 1),), -1, dtype=torch.int32, device=DEV)
+    val = torch.empty(max(total, 1), dtype=torch.float32, device=DEV)
+    cnt = torch.full((1,), -1, dtype=torch.int32, device=DEV)
+    efs.ef_topk_layerwise(gd, ed, gamma, seg_end, seg_k, idx, val, cnt)
+    torch.cuda.synchronize()
+    c = int(cnt.item())
+    return idx[:c].cpu().numpy().view(np.uint32), val[:c].cpu().numpy(), ed.cpu().numpy()
+
+
 def aggregate(idx_list, val_list, d, dense_off=0):
     idx_t = [to_dev(np.asarray(i, np.uint32).view(np.int32)) if len(i) else
              torch.zeros(1, dtype=torch.int32, device=DEV) for i in idx_list]

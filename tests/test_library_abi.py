@@ -80,6 +80,30 @@ def test_topk_rejects(kwargs):
     assert _topk(**kwargs) == efs.EF_ERR_INVALID_ARG
 
 
+def _layerwise(g=G, e=E, gamma=0.1, ends=(600, 1000), ks=(6, 4), d=1000, idx=IDX, val=VAL,
+               cnt=CNT, n_seg=None):
+    import numpy as np
+    lib = efs.load_library()
+    ends_a = np.ascontiguousarray(ends, dtype=np.uint64)
+    ks_a = np.ascontiguousarray(ks, dtype=np.uint64)
+    n = len(ends) if n_seg is None else n_seg
+    return lib.ef_topk_layerwise(vp(g), vp(e), ctypes.c_float(gamma), ctypes.c_uint32(n),
+                                 vp(ends_a.ctypes.data if ends_a.size else 0),
+                                 vp(ks_a.ctypes.data if ks_a.size else 0), d, vp(idx), vp(val),
+                                 vp(cnt), vp(0))
+
+
+@pytest.mark.parametrize("kwargs", [
+    dict(n_seg=0), dict(ends=(600, 999)), dict(ends=(600, 1001)), dict(ends=(700, 600, 1000),
+                                                                        ks=(1, 0, 1)),
+    dict(ks=(601, 4)), dict(ks=(6, 401)), dict(d=2 ** 32, ends=(600, 2 ** 32)), dict(cnt=0),
+    dict(g=0), dict(idx=0), dict(gamma=float("inf")), dict(e=E + 2), dict(val=E),
+    dict(idx=VAL - 20),  # 10 pairs overlap val
+])
+def test_topk_layerwise_rejects(kwargs):
+    assert _layerwise(**kwargs) == efs.EF_ERR_INVALID_ARG
+
+
 def test_aggregate_rejects():
     lib = efs.load_library()
     arr = (vp * 1)(vp(IDX))
