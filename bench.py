@@ -6,6 +6,9 @@ workload, through the whole hot path:
   - n x ef_hard_threshold (EF accumulate + hard-threshold + compaction +
     residual), then sparse_aggregate of their n messages;
   - n x ef_topk on the same gradients (separate error memories), then
+    sparse_aggregate of those messages;
+  - n x ef_topk_layerwise (Top-k on each parameter tensor separately, the
+    same fraction of every tensor) on the same gradients, then
     sparse_aggregate of those messages.
 Gradients come from two pre-generated synthetic batches (alternating), so
 every step compresses different data; each step's working set (n workers x
@@ -251,6 +254,10 @@ def run_ours(args):
     w = workloads.BY_NAME[args.workload]
     d, n, gamma = w.d, w.n, w.gamma
     k = w.topk_values()[0]
+    frac = w.topk_fracs[0] if w.topk_fracs else k / d
+    seg_end = workloads.segment_ends(w)
+    seg_k = workloads.layerwise_k(w, frac)
+    k_lw = sum(seg_k)
     wr = replica_workload(w, rank)
     batches = [[workloads.gradient(wr, i, b, device=dev) for i in range(n)] for b in range(2)]
     lam = (workloads.density_lambda(wr, batches[0][0], w.density) if w.density is not None
@@ -262,17 +269,21 @@ def run_ours(args):
 
     e_ht = [torch.zeros(d, device=dev) for _ in range(n)]
     e_tk = [torch.zeros(d, device=dev) for _ in range(n)]
+    e_lw = [torch.zeros(d, device=dev) for _ in range(n)]
     idx_ht, val_ht = outputs(d)
     idx_tk, val_tk = outputs(k)
+    idx_lw, val_lw = outputs(k_lw)
     dense_ht = torch.empty(d, device=dev)
     dense_tk = torch.empty(d, device=dev)
+    dense_lw = torch.empty(d, device=dev)
     total = args.warmup + args.steps
     cnt_ht = torch.zeros(total, n, dtype=torch.int32, device=dev)
     cnt_tk = torch.zeros(total, n, dtype=torch.int32, device=dev)
+    cnt_lw = torch.zeros(total, n, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream()
 
     ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
-    marks = [[ev() for _ in range(5)] for _ in range(args.steps)]
+    marks = [[ev() for _ in range(7)] for _ in range(args.steps)]
 
     def step(s, timed):
         g = batches[s % 2]
@@ -289,6 +300,12 @@ def run_ours(args):
         if m: m[3].record(stream)
         efs.sparse_aggregate(idx_tk, val_tk, cnt_tk[s], d, dense_tk)
         if m: m[4].record(stream)
+        for i in range(n):
+            efs.ef_topk_layerwise(g[i], e_lw[i], gamma, seg_end, seg_k, idx_lw[i], val_lw[i],
+                                  cnt_lw[s, i:i + 1])
+        if m: m[5].record(stream)
+        efs.sparse_aggregate(idx_lw, val_lw, cnt_lw[s], d, dense_lw)
+        if m: m[6].record(stream)
 
     for s in range(args.warmup):
         step(s, False)
@@ -315,15 +332,18 @@ def run_ours(args):
 
     step_s = t0.elapsed_time(t1) / 1e3
     # per-iteration segment times (µs per call: the segment of n calls / n)
-    seg_us = [[m[a].elapsed_time(m[a + 1]) * 1e3 for m in marks] for a in range(4)]
+    seg_us = [[m[a].elapsed_time(m[a + 1]) * 1e3 for m in marks] for a in range(6)]
     ht_s = sum(m[0].elapsed_time(m[1]) for m in marks) / 1e3
     agg_ht_s = sum(m[1].elapsed_time(m[2]) for m in marks) / 1e3
     tk_s = sum(m[2].elapsed_time(m[3]) for m in marks) / 1e3
     agg_tk_s = sum(m[3].elapsed_time(m[4]) for m in marks) / 1e3
+    lw_s = sum(m[4].elapsed_time(m[5]) for m in marks) / 1e3
+    agg_lw_s = sum(m[5].elapsed_time(m[6]) for m in marks) / 1e3
     counts_ht = cnt_ht[args.warmup:].double()
     counts_tk = cnt_tk[args.warmup:].double()
     bytes_ht = float(ht_bytes(d, 0) * n * args.steps + 8 * counts_ht.sum().item())
     bytes_tk = float((12 * d + 8 * k) * n * args.steps)
+    bytes_lw = float((12 * d + 8 * k_lw) * n * args.steps)
     bytes_agg_ht = float(8 * counts_ht.sum().item() + 4 * d * args.steps)
     bytes_agg_tk = float(8 * counts_tk.sum().item() + 4 * d * args.steps)
 
@@ -383,11 +403,22 @@ def run_ours(args):
         "aggregate_gbs": round(bytes_agg_ht / agg_ht_s / 1e9, 2),
         "aggregate_frac_of_peak": round(bytes_agg_ht / agg_ht_s / 1e9 / peak, 4),
         "aggregate_topk_ms_per_iter": round(agg_tk_s / args.steps * 1e3, 4),
+        "topk_layerwise": {
+            "segments": len(seg_end),
+            "k_total": k_lw,
+            "k_rule": "k_s = max(1, floor(%g d_s))" % frac,
+            "ms_per_iter": round(lw_s / args.steps * 1e3, 4),
+            "gbs": round(bytes_lw / lw_s / 1e9, 2),
+            "frac_of_peak": round(bytes_lw / lw_s / 1e9 / peak, 4),
+            "aggregate_ms_per_iter": round(agg_lw_s / args.steps * 1e3, 4),
+        },
         "per_call_us_p10_p50_p90": {
             "ht": percentiles([v / n for v in seg_us[0]]),
             "topk": percentiles([v / n for v in seg_us[2]]),
+            "topk_layerwise": percentiles([v / n for v in seg_us[4]]),
             "aggregate_ht": percentiles(seg_us[1]),
             "aggregate_topk": percentiles(seg_us[3]),
+            "aggregate_topk_layerwise": percentiles(seg_us[5]),
         },
         "frac_of_nominal_8tbs": round(value / NOMINAL_HBM_GBS, 4),
         "roofline": {

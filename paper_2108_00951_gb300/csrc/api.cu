@@ -345,14 +345,14 @@ ef_status ef_check_status(ef_stream_t stream) {
   if (cudaMemsetAsync(dev_err, 0, sizeof bits, s) != cudaSuccess ||
       cudaStreamSynchronize(s) != cudaSuccess)
     return EF_ERR_CUDA;
-  if (bits & efs::kDevErrTimeout) {
-    // a wait that ran out may leave barrier counters mid-way: re-clear the
-    // workspace header before the next launch on this stream
+  {
+    // a wait that ran out, or a selection that stopped early, may leave
+    // barrier counters or histograms mid-way: re-clear the workspace before
+    // the next launch on this stream
     std::lock_guard<std::mutex> lk(efs::g_mu);
     ws->dirty = true;
-    return EF_ERR_TIMEOUT;
   }
-  return EF_ERR_BAD_INPUT;
+  return (bits & efs::kDevErrTimeout) ? EF_ERR_TIMEOUT : EF_ERR_BAD_INPUT;
 }
 
 const char* ef_status_string(ef_status status) {

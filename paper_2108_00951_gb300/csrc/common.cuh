@@ -196,8 +196,9 @@ __device__ __forceinline__ void griddep_launch_dependents() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
-__device__ __forceinline__ bool grid_barrier(uint32_t* arrive, uint32_t* gen, uint64_t limit_ns,
-                             uint32_t* error) {
+// Bounded barrier of `count` co-resident CTAs sharing the (arrive, gen) words.
+__device__ __forceinline__ bool group_barrier(uint32_t* arrive, uint32_t* gen, uint32_t count,
+                                              uint64_t limit_ns, uint32_t* error) {
   __shared__ int s_ok;
   __syncthreads();
   if (threadIdx.x == 0) {
@@ -205,7 +206,7 @@ __device__ __forceinline__ bool grid_barrier(uint32_t* arrive, uint32_t* gen, ui
     const uint32_t my_gen = ld_acquire_u32(gen);
     __threadfence();  // this CTA's global writes before arriving
     const uint32_t ticket = atomicAdd(arrive, 1u);
-    if (ticket == gridDim.x - 1) {
+    if (ticket == count - 1) {
       atomicExch(arrive, 0u);
       __threadfence();
       st_release_u32(gen, my_gen + 1);
@@ -225,6 +226,11 @@ __device__ __forceinline__ bool grid_barrier(uint32_t* arrive, uint32_t* gen, ui
   }
   __syncthreads();
   return s_ok != 0;
+}
+
+__device__ __forceinline__ bool grid_barrier(uint32_t* arrive, uint32_t* gen, uint64_t limit_ns,
+                                             uint32_t* error) {
+  return group_barrier(arrive, gen, gridDim.x, limit_ns, error);
 }
 
 }  // namespace efs

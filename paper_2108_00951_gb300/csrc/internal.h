@@ -39,34 +39,51 @@ constexpr uint32_t kMaxChunks = 1024;   // per-CTA chunk sums of the streaming c
 constexpr uint32_t kCountsPerTile = 16; // per-segment counts of the streaming compaction
 
 // ---- layer-wise Top-k: one Top-k selection per segment of the vector.
-// Segment kinds: nothing sent (k = 0); the whole segment selected in one
-// CTA's shared memory; a sampled candidate bound, then a selection over the
-// candidates; every coordinate sent (k = d_s).
+// Segment kinds: nothing sent (k = 0); a short segment selected from e in
+// one CTA's shared memory; a sampled candidate bound, then a selection over
+// the candidates; every coordinate sent (k = d_s).
 constexpr uint32_t kLwNone = 0, kLwWhole = 1, kLwSampled = 2, kLwAll = 3;
 constexpr uint32_t kLwSmemElems = 48u * 1024u;  // values one select CTA holds in shared memory
+constexpr uint32_t kLwWholeMax = 4096;          // segments at most this long: selected from e
+constexpr uint32_t kLwSampleGroups = 4096;      // groups of 4 coordinates sampled per segment
 constexpr uint32_t kLwNoBound = 0xffffffffu;    // candidate bound that admits nothing
 constexpr uint32_t kLwTileUniform = 0x80000000u;  // tile_info: the tile lies in one segment
-constexpr uint32_t kLwSampleGroupsPerCta = 4096;  // sampled groups of 4 coordinates per CTA
 
-struct LwSeg {      // one segment (device and host layout)
+struct LwSeg {      // one segment (device and host layout, 32 bytes)
+  uint64_t step;    // sampled: spacing of the groups, in aligned groups, 32.32 fixed point
   uint32_t lo, hi;  // coordinates [lo, hi)
   uint32_t k;       // pairs it sends
   uint32_t out;     // output position of its first pair
-  uint32_t kind;    // kLw*
-  uint32_t slot;    // sampled: its histogram slot
-  uint32_t nblk;    // sampled: its sampling CTAs
   uint32_t groups;  // sampled: its sampled groups of 4 consecutive coordinates
+  uint16_t kind;    // kLw*
+  uint16_t exact;   // sampled: the groups are every aligned group of the segment
 };
-struct LwSample {   // one sampling CTA: groups [q0, q1) of segment seg
-  uint32_t seg, q0, q1, pad;
+// A select CTA: either the segments work_seg[a, b) one after another
+// (team == kLwNoTeam), or member `rank` of a team of b CTAs that selects
+// segment a together (team = the team's index).
+constexpr uint32_t kLwNoTeam = 0xffffffffu;
+constexpr uint32_t kLwMaxTeam = 32;
+struct LwCta {
+  uint32_t team, a, b, rank;
 };
+// Per-team state of the select kernel: histograms of the three magnitude
+// digit levels and a barrier (zero at a call's start; the team's rank 0
+// clears the histograms at the end), and per-rank counts.
+struct LwTeamState {
+  uint32_t hist[3][2048];
+  uint32_t arrive, gen, last, pad0;
+  uint32_t cnt[kLwMaxTeam];
+  uint32_t tie_cnt[kLwMaxTeam];
+  uint32_t pad[60];
+};
+static_assert(sizeof(LwTeamState) % 256 == 0, "team state alignment");
 
 // The device tables of a segment table, rebuilt when the table changes.
 struct LwPlan {
   std::vector<uint64_t> seg_end, seg_k;  // the host table this plan was built from
   uint64_t d = 0;
   bool valid = false;
-  uint32_t n_seg = 0, n_sampled = 0, n_sample_ctas = 0, n_select_ctas = 0, tiles = 0;
+  uint32_t n_seg = 0, n_sampled = 0, n_select_ctas = 0, n_teams = 0, tiles = 0;
   uint64_t total_k = 0;
   std::vector<char> image;  // host image of the uploaded part
   char* dev = nullptr;
@@ -74,8 +91,7 @@ struct LwPlan {
   // byte offsets in dev: uploaded tables, then zero-initialised counters
   // and histograms (each user resets its own), then per-call outputs
   size_t off_segs = 0, off_seg_end = 0, off_mbound = 0, off_tile_info = 0, off_samples = 0,
-         off_work_ptr = 0, off_work_seg = 0, off_done = 0, off_hist = 0, off_tile_base = 0,
-         total = 0;
+         off_ctas = 0, off_work_seg = 0, off_teams = 0, off_tile_base = 0, total = 0;
 };
 
 struct Workspace {
@@ -134,6 +150,7 @@ struct DeviceInfo {
   int tk_stream_per_sm_bf16 = 0;
   int lw_stream_per_sm_f32 = 0;   // streaming layer-wise candidate pass CTAs per SM
   int lw_stream_per_sm_bf16 = 0;
+  int lw_select_per_sm = 0;       // co-resident layer-wise select CTAs per SM
 };
 
 // Per-device set-up of the Top-k kernels (shared-memory opt-in, occupancy).

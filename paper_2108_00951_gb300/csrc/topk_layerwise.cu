@@ -8,20 +8,20 @@
 // within each segment).
 //
 // Three launches, whatever the number of segments:
-//  1 sample   for each large segment (more than kLwSmemElems coordinates,
-//             0 < k_s < d_s), CTAs read groups of 4 consecutive coordinates
-//             spread evenly over it, histogram the top 13 magnitude bits of
-//             a = fmaf(γ,g,e), and merge into the segment's histogram; the
-//             last CTA of the segment to finish (an arrival counter) picks
-//             the candidate bound with about 1.5 times the needed mass above
-//             it, then clears the histogram and counter for the next call.
+//  1 sample   one CTA for each segment longer than kLwWholeMax with
+//             0 < k_s < d_s reads up to 4096 groups of 4 consecutive
+//             coordinates spread evenly over it (all of them when it holds no
+//             more), histograms the top 13 magnitude bits of a = fmaf(γ,g,e)
+//             in shared memory and picks the candidate bound: the bin holding
+//             k_s samples when every group was read, else about 1.5 times the
+//             needed mass above it.
 //  2 stream   the streaming compaction of stream_compact.cuh: a = fmaf(γ,g,e)
 //             is written over e (12 B per coordinate, the algorithmic bytes)
 //             and the coordinates at or above their segment's bound are
 //             emitted as one ordered candidate list, with the list position
 //             of each tile's first candidate.
 //  3 select   CTAs own groups of segments (balanced on the host). For each:
-//             a small segment is read into shared memory whole; a large one
+//             a short segment is read into shared memory whole; a longer one
 //             takes its candidates (located from the tile positions) into
 //             shared memory, or reads them (or, if the bound missed, the
 //             segment) from global memory level by level; the exact
@@ -43,7 +43,7 @@
 namespace efs {
 namespace {
 
-constexpr int kLwThreads = 1024;  // sample and select CTAs
+constexpr int kLwThreads = 1024;  // select CTAs
 constexpr uint32_t kLwSelectSmem = kLwSmemElems * sizeof(uint32_t);
 constexpr int kLwSampleShift = 31 - kSampleBits;  // magnitude bits below the sampled ones
 constexpr int kLwStages = 4;
@@ -51,73 +51,83 @@ constexpr int kLwStages = 4;
 __device__ __forceinline__ uint32_t mag_bits(float x) { return __float_as_uint(x) & 0x7fffffffu; }
 
 // ------------------------------------------------------------- 1 sample
+// One CTA per sampled segment, one round of loads: thread t reads groups
+// t, t + 1024, t + 2048, t + 3072 of the segment's G <= 4096 groups of 4
+// consecutive coordinates starting at multiples of 4 (one 16-byte load each
+// of e and of an fp32 g, 8 bytes of a bf16 g). Group q starts at
+// a0 + 4 floor(q step), a0 the first aligned coordinate inside the segment,
+// step = (A - 1) / (G - 1) rounded down in 32.32 fixed point and A the
+// aligned groups the segment holds (so the last group stays inside it);
+// G == A samples every one.
+//
+// Programmatic dependent launch: the loads and the histogram may run while
+// the previous kernel on the stream finishes (a sample read before that
+// kernel's writes only changes the bound, which is a filter); the bound is
+// written after the wait, so no earlier reader of it sees the new one.
+constexpr int kSampleThreads = 1024;
+
 template <typename GT>
-__global__ void __launch_bounds__(kLwThreads)
+__global__ void __launch_bounds__(kSampleThreads, 1)
     lw_sample_kernel(const GT* __restrict__ g, const float* __restrict__ e, float gamma,
-                     const LwSeg* __restrict__ segs, const LwSample* __restrict__ samples,
-                     uint32_t* hist, uint32_t* done, uint32_t* mbound, uint32_t cand_cap) {
+                     const LwSeg* __restrict__ segs, const uint32_t* __restrict__ sampled,
+                     uint32_t* mbound, uint32_t cand_cap) {
   __shared__ uint32_t s_hist[kSampleBins];
-  __shared__ uint32_t s_w[kLwThreads / 32];
-  __shared__ uint32_t s_last, s_bin, s_mass;
+  __shared__ uint32_t s_w[kSampleThreads / 32];
+  __shared__ uint32_t s_bin, s_mass;
   const int tid = threadIdx.x;
-  const LwSample sp = samples[blockIdx.x];
-  const LwSeg s = segs[sp.seg];
-  for (int b = tid; b < kSampleBins; b += kLwThreads) s_hist[b] = 0;
-  __syncthreads();
-  // group q starts at lo + q (d_s - 4) / (groups - 1): the groups spread
-  // evenly from the first to the last 4 coordinates of the segment
-  const uint64_t span = static_cast<uint64_t>(s.hi - s.lo) - 4u;
-  const uint64_t den = s.groups - 1u;
-  constexpr int kG = static_cast<int>(kLwSampleGroupsPerCta / kLwThreads);
-  float gv[kG][4], ev[kG][4];
+  griddep_launch_dependents();  // the stream pass may be scheduled (it waits for this grid)
+  const uint32_t si = sampled[blockIdx.x];
+  const LwSeg s = segs[si];
+  for (int b = tid; b < kSampleBins; b += kSampleThreads) s_hist[b] = 0;
+  const uint64_t a0 = (static_cast<uint64_t>(s.lo) + 3u) & ~static_cast<uint64_t>(3);
+  constexpr int kG = static_cast<int>(kLwSampleGroups / kSampleThreads);
+  GradVec<GT> gv[kG];
+  float4 ev[kG];
   bool in[kG];
 #pragma unroll
   for (int q = 0; q < kG; ++q) {  // every load in flight before any use
-    const uint32_t qq = sp.q0 + q * kLwThreads + tid;
-    in[q] = qq < sp.q1;
-    const uint64_t p = s.lo + (in[q] ? static_cast<uint64_t>(qq) * span / den : 0u);
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      gv[q][j] = in[q] ? grad_scalar(g, p + j) : 0.0f;
-      ev[q][j] = in[q] ? __ldg(e + p + j) : 0.0f;
+    const uint32_t qq = q * kSampleThreads + tid;
+    in[q] = qq < s.groups;
+    const uint64_t p = a0 + 4u * ((static_cast<uint64_t>(in[q] ? qq : 0u) * s.step) >> 32);
+    if (in[q]) {
+      if constexpr (sizeof(GT) == 4)
+        gv[q].v = __ldg(reinterpret_cast<const float4*>(g + p));
+      else
+        gv[q].v = __ldg(reinterpret_cast<const uint2*>(g + p));
+      ev[q] = __ldg(reinterpret_cast<const float4*>(e + p));
     }
   }
+  __syncthreads();
 #pragma unroll
-  for (int q = 0; q < kG; ++q)
+  for (int q = 0; q < kG; ++q) {
+    const float x[4] = {in[q] ? __fmaf_rn(gamma, gv[q][0], ev[q].x) : 0.0f,
+                        in[q] ? __fmaf_rn(gamma, gv[q][1], ev[q].y) : 0.0f,
+                        in[q] ? __fmaf_rn(gamma, gv[q][2], ev[q].z) : 0.0f,
+                        in[q] ? __fmaf_rn(gamma, gv[q][3], ev[q].w) : 0.0f};
 #pragma unroll
     for (int j = 0; j < 4; ++j)
-      hist_add_warp(s_hist, mag_bits(__fmaf_rn(gamma, gv[q][j], ev[q][j])) >> kLwSampleShift,
-                    in[q]);
-  __syncthreads();
-  uint32_t* h = hist + static_cast<size_t>(s.slot) * kSampleBins;
-  for (int b = tid; b < kSampleBins; b += kLwThreads)
-    if (s_hist[b]) atomicAdd(&h[b], s_hist[b]);
-  __threadfence();  // this CTA's histogram adds before its arrival
-  __syncthreads();
-  if (tid == 0) s_last = atomicAdd(done + sp.seg, 1u) == s.nblk - 1u ? 1u : 0u;
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();  // every arrival's adds are visible to the last CTA
-  // the segment's merged histogram: 8 consecutive bins per thread
-  constexpr int kPer = kSampleBins / kLwThreads;
-  static_assert(kPer == 8, "sample bins per thread");
-  uint32_t c[kPer];
-  {
-    const uint4 v0 = __ldcg(reinterpret_cast<const uint4*>(h) + 2 * tid);
-    const uint4 v1 = __ldcg(reinterpret_cast<const uint4*>(h) + 2 * tid + 1);
-    c[0] = v0.x; c[1] = v0.y; c[2] = v0.z; c[3] = v0.w;
-    c[4] = v1.x; c[5] = v1.y; c[6] = v1.z; c[7] = v1.w;
+      if (in[q]) atomicAdd(&s_hist[mag_bits(x[j]) >> kLwSampleShift], 1u);
   }
+  __syncthreads();
+  // kPer consecutive bins per thread
+  constexpr int kPer = kSampleBins / kSampleThreads;
+  uint32_t c[kPer];
   uint32_t mine = 0;
 #pragma unroll
-  for (int i = 0; i < kPer; ++i) mine += c[i];
+  for (int i = 0; i < kPer; ++i) {
+    c[i] = s_hist[tid * kPer + i];
+    mine += c[i];
+  }
   if (tid == 0) s_bin = 0xffffffffu;
   uint32_t m;  // sampled coordinates
   const uint32_t above = block_suffix_exclusive(mine, m, s_w);  // orders the reset
-  // 1.5x the expected sampled count above the k_s-th magnitude, plus 32
-  // (integer arithmetic; the products stay below 2^56)
   const uint64_t ds = s.hi - s.lo;
-  const uint64_t target = 3ull * s.k * m / (2ull * ds) + 32ull;
+  // Every sampled coordinate is a coordinate of the segment, so at least
+  // `target` coordinates lie at or above the bin found. With every group
+  // sampled, target = k_s is therefore enough; otherwise 1.5x the expected
+  // sampled count above the k_s-th magnitude, plus 32 (integer arithmetic;
+  // the products stay below 2^50).
+  const uint64_t target = s.exact ? s.k : 3ull * s.k * m / (2ull * ds) + 32ull;
   if (target <= m && above < target && target - above <= mine) {
     uint64_t run = above;
 #pragma unroll
@@ -130,9 +140,7 @@ __global__ void __launch_bounds__(kLwThreads)
     }
   }
   __syncthreads();
-  // clear the histogram for the next call: every read of it is complete
-  reinterpret_cast<uint4*>(h)[2 * tid] = make_uint4(0u, 0u, 0u, 0u);
-  reinterpret_cast<uint4*>(h)[2 * tid + 1] = make_uint4(0u, 0u, 0u, 0u);
+  griddep_wait();  // the previous kernel (which may read the bounds) is complete
   if (tid == 0) {
     uint32_t bound = kLwNoBound;
     // expected candidates (the sampled mass scaled to d_s) at most half the
@@ -140,8 +148,7 @@ __global__ void __launch_bounds__(kLwThreads)
     if (s_bin != 0xffffffffu &&
         2ull * s_mass * ds <= static_cast<uint64_t>(cand_cap) * m)
       bound = s_bin << kLwSampleShift;
-    mbound[sp.seg] = bound;
-    done[sp.seg] = 0;
+    mbound[si] = bound;
   }
 }
 
@@ -273,59 +280,80 @@ __global__ void __launch_bounds__(kThreads)
 struct LwArgs {
   const LwSeg* segs;
   const uint32_t* mbound;
-  const uint32_t* work_ptr;   // [grid + 1] each CTA's range of work_seg
-  const uint32_t* work_seg;   // segment ids, grouped by CTA
+  const LwCta* ctas;          // [grid] what each CTA selects
+  const uint32_t* work_seg;   // segment ids of the single CTAs, grouped by CTA
+  LwTeamState* teams;
   const uint32_t* tile_base;  // [tiles + 1] list position of each tile's first candidate
   const uint32_t* list_idx;   // ordered candidates of the streaming pass
   const float* list_val;
   const uint32_t* list_flags; // that pass's latched bits
   uint32_t* error;
   uint32_t* count_out;
+  uint64_t wait_limit_ns;
   uint32_t tiles, cap, use_list;
   uint32_t total_k;
 };
 
-// Number of list entries with index < x (x <= d): the list position of x's
-// tile, plus that tile's entries below x. ok = false when those entries were
-// cut off at the list's capacity. Whole CTA; uniform result.
-__device__ uint32_t list_position(const LwArgs& a, uint32_t x, bool& ok) {
-  const uint32_t t = x / kTileElems;
-  if (t >= a.tiles) return __ldcg(a.tile_base + a.tiles);
-  const uint32_t p0 = __ldcg(a.tile_base + t);
-  if (x % kTileElems == 0) return p0;
-  const uint32_t p1 = __ldcg(a.tile_base + t + 1);
-  if (p1 > a.cap) {
-    ok = false;
-    return p0;
+// The source a segment is selected from: its candidates [c0, c1) of the
+// list when they are complete and at least k_s, else its coordinates of a
+// (held in e after the stream). The list positions of lo and hi are the
+// positions of their tiles' first candidates plus those tiles' candidates
+// below them; all four tile positions are loaded at once, then both tiles
+// scanned together. Whole CTA; every CTA of a team decides alike.
+struct Source {
+  bool list;
+  uint32_t c0, n;
+};
+__device__ Source segment_source(const LwArgs& a, const LwSeg& s, uint32_t si) {
+  Source src{false, 0, s.hi - s.lo};
+  if (!a.use_list || __ldcg(a.mbound + si) == kLwNoBound) return src;
+  const uint32_t tl = s.lo / kTileElems, th = s.hi / kTileElems;  // tl < tiles, th <= tiles
+  const uint32_t p0 = __ldcg(a.tile_base + tl), p1 = __ldcg(a.tile_base + tl + 1);
+  const uint32_t q0 = __ldcg(a.tile_base + th);
+  const uint32_t q1 = th < a.tiles ? __ldcg(a.tile_base + th + 1) : q0;
+  // candidates of the partial tiles that lie below lo / hi (none to scan
+  // when lo / hi starts a tile); a tile cut off at the capacity disqualifies
+  const uint32_t e0 = s.lo % kTileElems ? p1 : p0, e1 = s.hi % kTileElems ? q1 : q0;
+  if (e0 > a.cap || e1 > a.cap) return src;
+  const uint32_t n0 = e0 - p0, n1 = e1 - q0, span = n0 > n1 ? n0 : n1;
+  uint32_t below0 = 0, below1 = 0;
+  for (uint32_t b = 0; b < span; b += kLwThreads) {
+    const uint32_t i = b + threadIdx.x;
+    const bool x0 = i < n0 && __ldcg(a.list_idx + p0 + i) < s.lo;
+    const bool x1 = i < n1 && __ldcg(a.list_idx + q0 + i) < s.hi;
+    below0 += __syncthreads_count(x0);
+    below1 += __syncthreads_count(x1);
   }
-  uint32_t below = 0;
-  for (uint32_t b = p0; b < p1; b += kLwThreads) {
-    const uint32_t p = b + threadIdx.x;
-    below += __syncthreads_count(p < p1 && __ldcg(a.list_idx + p) < x);
-  }
-  return p0 + below;
+  const uint32_t c0 = p0 + below0, c1 = q0 + below1;
+  if (c1 <= a.cap && c1 - c0 >= s.k) src = Source{true, c0, c1 - c0};
+  return src;
 }
 
 // Reads n fp32 values (8 loads in flight per thread), keeps their bits in
-// s_bits when it is given, and returns the minimum and maximum magnitude.
+// s_bits when it is given (and the coordinates idx[0, n) in s_idx when both
+// are given), and returns the minimum and maximum magnitude.
 __device__ void load_minmax(const float* src, uint32_t n, uint32_t* s_bits, uint32_t& lo,
-                            uint32_t& hi, uint32_t* s_lo, uint32_t* s_hi) {
+                            uint32_t& hi, uint32_t* s_lo, uint32_t* s_hi,
+                            const uint32_t* idx = nullptr, uint32_t* s_idx = nullptr) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int kBatch = 8;
   lo = 0xffffffffu;
   hi = 0;
+  const bool with_idx = idx && s_idx;
   for (uint32_t i0 = tid; i0 < n; i0 += kBatch * kLwThreads) {
-    uint32_t v[kBatch];
+    uint32_t v[kBatch], x[kBatch];
 #pragma unroll
     for (int j = 0; j < kBatch; ++j) {
       const uint32_t i = i0 + j * kLwThreads;
       v[j] = i < n ? __float_as_uint(__ldcg(src + i)) : 0u;
+      x[j] = with_idx && i < n ? __ldcg(idx + i) : 0u;
     }
 #pragma unroll
     for (int j = 0; j < kBatch; ++j) {
       const uint32_t i = i0 + j * kLwThreads;
       if (i < n) {
         if (s_bits) s_bits[i] = v[j];
+        if (with_idx) s_idx[i] = x[j];
         const uint32_t m = v[j] & 0x7fffffffu;
         lo = m < lo ? m : lo;
         hi = m > hi ? m : hi;
@@ -343,8 +371,8 @@ __device__ void load_minmax(const float* src, uint32_t n, uint32_t* s_bits, uint
     s_hi[warp] = hi;
   }
   __syncthreads();
-  lo = s_lo[lane];  // 32 warps
-  hi = s_hi[lane];
+  lo = lane < kLwThreads / 32 ? s_lo[lane] : 0xffffffffu;
+  hi = lane < kLwThreads / 32 ? s_hi[lane] : 0u;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     lo = min(lo, __shfl_xor_sync(0xffffffffu, lo, o));
@@ -352,71 +380,286 @@ __device__ void load_minmax(const float* src, uint32_t n, uint32_t* s_bits, uint
   }
 }
 
-// Sources of a selection: list position i has value bits bits(i) and
+// Sources of a selection: source position i has value bits bits(i) and
 // coordinate index(i).
-struct SrcSharedArray {  // a whole segment in shared memory
+struct SrcShared {  // values in shared memory; coordinates lo + i, or from a list
   const uint32_t* s_bits;
+  const uint32_t* idx;    // null: coordinates lo + i (or from s_idx)
+  const uint32_t* s_idx;  // the list's coordinates in shared memory, or null
   uint32_t lo;
   __device__ __forceinline__ uint32_t bits(uint32_t i) const { return s_bits[i]; }
-  __device__ __forceinline__ uint32_t index(uint32_t i) const { return lo + i; }
-};
-struct SrcSharedList {  // candidates' values in shared memory
-  const uint32_t* s_bits;
-  const uint32_t* idx;
-  __device__ __forceinline__ uint32_t bits(uint32_t i) const { return s_bits[i]; }
-  __device__ __forceinline__ uint32_t index(uint32_t i) const { return __ldcg(idx + i); }
-};
-struct SrcGlobalList {  // candidates in global memory
-  const float* val;
-  const uint32_t* idx;
-  __device__ __forceinline__ uint32_t bits(uint32_t i) const {
-    return __float_as_uint(__ldcg(val + i));
+  __device__ __forceinline__ uint32_t index(uint32_t i) const {
+    return s_idx ? s_idx[i] : idx ? __ldcg(idx + i) : lo + i;
   }
-  __device__ __forceinline__ uint32_t index(uint32_t i) const { return __ldcg(idx + i); }
 };
-struct SrcGlobalArray {  // a segment of a in global memory (e after the stream)
+struct SrcGlobal {  // values in global memory; coordinates lo + i, or from a list
   const float* val;
+  const uint32_t* idx;
   uint32_t lo;
   __device__ __forceinline__ uint32_t bits(uint32_t i) const {
     return __float_as_uint(__ldcg(val + i));
   }
-  __device__ __forceinline__ uint32_t index(uint32_t i) const { return lo + i; }
+  __device__ __forceinline__ uint32_t index(uint32_t i) const {
+    return idx ? __ldcg(idx + i) : lo + i;
+  }
 };
 
-// Writes the selected positions of [0, n), in order, as pairs at out[0, k)
-// and zeroes e at each; returns the number selected. Whole CTA.
-template <class Src>
-__device__ uint32_t emit_selected(const Src& src, uint32_t n, const SmallSelection& sel,
-                                  uint32_t k, uint32_t* idx_out, float* val_out, float* e,
-                                  bool& overflow, uint32_t* s_w) {
-  uint32_t base = 0;
-  for (uint32_t b0 = 0; b0 < n; b0 += 4 * kLwThreads) {
-    const uint32_t i0 = b0 + 4 * threadIdx.x;
-    uint32_t bits[4], take = 0;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) bits[j] = i0 + j < n ? src.bits(i0 + j) : 0u;
-#pragma unroll
-    for (int j = 0; j < 4; ++j)
-      if (i0 + j < n && selected(sel, bits[j] & 0x7fffffffu, i0 + j)) take |= 1u << j;
-    uint32_t total;
-    uint32_t pos = base + block_exclusive<kLwThreads>(__popc(take), total, s_w);
+// Ordered write-out of the selected source positions of [s0, s1), in two
+// passes. Warp w owns the contiguous part [s0 + w (s1-s0)/32, ...): it counts
+// its selected positions (coalesced loads, 4 in flight per lane); the CTA's
+// counts are scanned (plus `base`, the pairs of earlier CTAs of a team, which
+// `publish` supplies once it sees the CTA's total; 0xffffffff: none, write
+// nothing); then each warp writes its
+// pairs at ascending positions with ballots, zeroing e at each. Positions at
+// or past k are not written (overflow). Returns the CTA's count. Whole CTA.
+template <class Src, class Publish>
+__device__ uint32_t write_out(const Src& src, uint32_t s0, uint32_t s1, const SmallSelection& sel,
+                              uint32_t k, uint32_t* idx_out, float* val_out, float* e,
+                              bool& overflow, uint32_t* s_w, const Publish& publish) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  constexpr int kNumWarps = kLwThreads / 32;
+  const uint32_t len = s1 - s0;
+  const uint32_t w0 = s0 + static_cast<uint32_t>(static_cast<uint64_t>(warp) * len / kNumWarps);
+  const uint32_t w1 =
+      s0 + static_cast<uint32_t>(static_cast<uint64_t>(warp + 1) * len / kNumWarps);
+  uint32_t cnt = 0;
+  for (uint32_t i0 = w0; i0 < w1; i0 += 4 * 32) {
+    uint32_t b[4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      if (take & (1u << j)) {
-        if (pos < k) {
-          const uint32_t idx = src.index(i0 + j);
-          idx_out[pos] = idx;
-          val_out[pos] = __uint_as_float(bits[j]);
+      const uint32_t i = i0 + j * 32 + lane;
+      b[j] = i < w1 ? src.bits(i) : 0u;
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint32_t i = i0 + j * 32 + lane;
+      cnt += (i < w1 && selected(sel, b[j] & 0x7fffffffu, i)) ? 1u : 0u;
+    }
+  }
+  cnt = warp_sum(cnt);
+  __syncthreads();  // an earlier use of s_w is complete
+  if (lane == 0) s_w[warp] = cnt;
+  __syncthreads();
+  uint32_t before = 0, total = 0;
+  for (int w = 0; w < kNumWarps; ++w) {
+    const uint32_t x = s_w[w];
+    before += w < warp ? x : 0u;
+    total += x;
+  }
+  const uint32_t base = publish(total);
+  if (base == 0xffffffffu) return total;  // the team's counts are unknown: write nothing
+  const uint32_t lt = lanemask_lt();
+  uint32_t pos = base + before;
+  for (uint32_t i0 = w0; i0 < w1; i0 += 4 * 32) {
+    uint32_t b[4], ix[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {  // values and coordinates in flight together
+      const uint32_t i = i0 + j * 32 + lane;
+      b[j] = i < w1 ? src.bits(i) : 0u;
+      ix[j] = i < w1 ? src.index(i) : 0u;
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint32_t i = i0 + j * 32 + lane;
+      const bool take = i < w1 && selected(sel, b[j] & 0x7fffffffu, i);
+      const uint32_t bal = __ballot_sync(0xffffffffu, take);
+      if (take) {
+        const uint32_t q = pos + __popc(bal & lt);
+        if (q < k) {
+          const uint32_t idx = ix[j];
+          idx_out[q] = idx;
+          val_out[q] = __uint_as_float(b[j]);
           e[idx] = 0.0f;  // residual of a sent coordinate
         } else {
           overflow = true;
         }
-        ++pos;
+      }
+      pos += __popc(bal);
+    }
+  }
+  return total;
+}
+
+struct NoTeam {
+  __device__ uint32_t operator()(uint32_t) const { return 0; }
+};
+
+// One CTA selects segment s on its own. Returns false when the threshold
+// was not found or the count differs from k (never for well-formed data).
+__device__ bool select_single(const LwArgs& a, const LwSeg& s, uint32_t si, float* e,
+                              uint32_t* idx_out, float* val_out, bool& overflow,
+                              uint32_t* s_bits, uint32_t* s_hist, uint32_t* s_w, uint32_t* s_lo,
+                              uint32_t* s_hi) {
+  uint32_t* io = idx_out + s.out;
+  float* vo = val_out + s.out;
+  const uint32_t ds = s.hi - s.lo;
+  if (s.kind == kLwAll) {
+    for (uint32_t i = threadIdx.x; i < ds; i += kLwThreads) {
+      io[i] = s.lo + i;
+      vo[i] = __ldcg(e + s.lo + i);
+      e[s.lo + i] = 0.0f;
+    }
+    return true;
+  }
+  const Source src = s.kind == kLwWhole ? Source{false, 0, ds} : segment_source(a, s, si);
+  const float* vals = src.list ? a.list_val + src.c0 : e + s.lo;
+  const uint32_t* idxs = src.list ? a.list_idx + src.c0 : nullptr;
+  SmallSelection sel;
+  uint32_t lo, hi, got = 0;
+  bool found;
+  if (src.n <= kLwSmemElems) {
+    // a list of at most half the capacity keeps its coordinates on chip too
+    uint32_t* s_idx = idxs && src.n <= kLwSmemElems / 2 ? s_bits + kLwSmemElems / 2 : nullptr;
+    load_minmax(vals, src.n, s_bits, lo, hi, s_lo, s_hi, idxs, s_idx);
+    found = threshold_levels<kLwThreads>(MagsShared{s_bits}, src.n, s.k, lo, hi, s_hist, s_w, sel);
+    if (found)
+      got = write_out(SrcShared{s_bits, idxs, s_idx, s.lo}, 0, src.n, sel, s.k, io, vo, e,
+                      overflow, s_w, NoTeam{});
+  } else {
+    load_minmax(vals, src.n, nullptr, lo, hi, s_lo, s_hi);
+    found = threshold_levels<kLwThreads>(MagsGlobal{vals}, src.n, s.k, lo, hi, s_hist, s_w, sel);
+    if (found)
+      got = write_out(SrcGlobal{vals, idxs, s.lo}, 0, src.n, sel, s.k, io, vo, e, overflow, s_w,
+                      NoTeam{});
+  }
+  return found && got == s.k;
+}
+
+// A team of T co-resident CTAs selects segment s: CTA r owns the source
+// positions [r n / T, (r+1) n / T). The threshold is found by three digit
+// levels of the magnitude bits (30..20, 19..10, 9..0): each CTA histograms
+// the positions matching the prefix chosen so far into shared memory and adds
+// that into the team's level histogram; after a team barrier every CTA reads
+// the merged histogram and picks the same bin. The levels stop once the bin
+// holds exactly the remaining rank; otherwise equal magnitudes at the last
+// level are taken in position order (per-rank counts, a barrier, and the rank
+// holding the cut publishes its position). The write-out scans per-rank
+// counts behind one more barrier. Returns false on a barrier that ran out
+// (latched as a timeout) or an inconsistent histogram.
+__device__ bool select_team(const LwArgs& a, const LwSeg& s, uint32_t si, uint32_t T, uint32_t r,
+                            LwTeamState* st, float* e, uint32_t* idx_out, float* val_out,
+                            bool& overflow, bool& bad, uint32_t* s_hist, uint32_t* s_w) {
+  __shared__ uint32_t s_found, s_last;
+  const int tid = threadIdx.x;
+  const Source src = segment_source(a, s, si);
+  const float* vals = src.list ? a.list_val + src.c0 : e + s.lo;
+  const uint32_t* idxs = src.list ? a.list_idx + src.c0 : nullptr;
+  const MagsGlobal mag{vals};
+  const uint32_t n = src.n;
+  const uint32_t s0 = static_cast<uint32_t>(static_cast<uint64_t>(r) * n / T);
+  const uint32_t s1 = static_cast<uint32_t>(static_cast<uint64_t>(r + 1) * n / T);
+  auto barrier = [&]() {
+    return group_barrier(&st->arrive, &st->gen, T, a.wait_limit_ns, a.error);
+  };
+  uint32_t prefix = 0, k_rem = s.k, n_in = n;
+  int sh = 0;
+  for (int level = 0; level < 3; ++level) {
+    sh = level == 0 ? 20 : level == 1 ? 10 : 0;
+    const int width = level == 0 ? 11 : 10;
+    const uint32_t nb = 1u << width;
+    for (uint32_t b = tid; b < nb; b += kLwThreads) s_hist[b] = 0;
+    __syncthreads();
+    for (uint32_t b0 = s0; b0 < s1; b0 += 4 * kLwThreads) {
+      uint32_t m[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t i = b0 + j * kLwThreads + tid;
+        m[j] = i < s1 ? mag(i) : 0u;
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t i = b0 + j * kLwThreads + tid;
+        const bool match = i < s1 && (level == 0 || (m[j] >> (sh + width)) == prefix);
+        hist_add_warp(s_hist, (m[j] >> sh) & (nb - 1), match);
       }
     }
-    base += total;
+    __syncthreads();
+    for (uint32_t b = tid; b < nb; b += kLwThreads)
+      if (s_hist[b]) atomicAdd(&st->hist[level][b], s_hist[b]);
+    if (!barrier()) return false;
+    const Selection sl = select_bin<kLwThreads, true>(st->hist[level], nb, k_rem, s_w);
+    if (!sl.found) {
+      bad = true;
+      return false;
+    }
+    prefix = (prefix << width) | sl.bin;
+    k_rem = sl.k_rem;
+    n_in = sl.n_in;
+    if (n_in == k_rem) break;
   }
-  return base;
+  SmallSelection sel{prefix << sh, 0u, 0xffffffffu};
+  if (n_in != k_rem) {
+    // sh == 0: the magnitude is prefix itself; take its first k_rem
+    // occurrences in position order
+    sel.ties = 1u;
+    uint32_t c = 0;
+    for (uint32_t i = s0 + tid; i < s1; i += kLwThreads) c += mag(i) == sel.B ? 1u : 0u;
+    uint32_t mine;
+    block_exclusive<kLwThreads>(c, mine, s_w);
+    if (tid == 0) st->tie_cnt[r] = mine;
+    if (!barrier()) return false;
+    uint32_t before = 0;
+    for (uint32_t q = 0; q < r; ++q) before += __ldcg(&st->tie_cnt[q]);
+    if (before < k_rem && k_rem <= before + mine) {
+      // this rank holds the cut: find it in position order
+      uint32_t run = before;
+      if (tid == 0) s_found = 0;
+      for (uint32_t b0 = s0; b0 < s1; b0 += 4 * kLwThreads) {
+        const uint32_t i0 = b0 + 4 * tid;
+        uint32_t eq = 0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if (i0 + j < s1 && mag(i0 + j) == sel.B) eq |= 1u << j;
+        uint32_t blk;
+        uint32_t at = run + block_exclusive<kLwThreads>(__popc(eq), blk, s_w);
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if (eq & (1u << j)) {
+            if (++at == k_rem) {
+              s_last = i0 + j;
+              s_found = 1;
+            }
+          }
+        run += blk;
+        __syncthreads();
+        if (s_found) break;
+      }
+      if (tid == 0) st->last = s_last;
+    }
+    if (!barrier()) return false;
+    sel.last = __ldcg(&st->last);
+  }
+  uint32_t* io = idx_out + s.out;
+  float* vo = val_out + s.out;
+  __shared__ uint32_t s_base;
+  auto publish = [&](uint32_t total) -> uint32_t {
+    if (tid == 0) st->cnt[r] = total;
+    if (!barrier()) {
+      if (tid == 0) s_base = 0xffffffffu;
+      __syncthreads();
+      return 0xffffffffu;  // no position is below k: nothing is written
+    }
+    if (tid == 0) {
+      uint32_t before = 0, all = 0;
+      for (uint32_t q = 0; q < T; ++q) {
+        const uint32_t x = __ldcg(&st->cnt[q]);
+        before += q < r ? x : 0u;
+        all += x;
+      }
+      if (all != s.k) atomicOr(a.error, kDevErrBadInput);
+      s_base = before;
+    }
+    __syncthreads();
+    return s_base;
+  };
+  const SrcGlobal sg{vals, idxs, s.lo};
+  write_out(sg, s0, s1, sel, s.k, io, vo, e, overflow, s_w, publish);
+  if (s_base == 0xffffffffu) return false;
+  // every CTA has read the level histograms (before the write-out barrier):
+  // clear them for the next call
+  if (r == 0)
+    for (uint32_t b = tid; b < 3 * 2048; b += kLwThreads) (&st->hist[0][0])[b] = 0;
+  return true;
 }
 
 __global__ void __launch_bounds__(kLwThreads, 1)
@@ -427,6 +670,11 @@ __global__ void __launch_bounds__(kLwThreads, 1)
   __shared__ uint32_t s_w[kLwThreads / 32];
   __shared__ uint32_t s_lo[32], s_hi[32];
   const int tid = threadIdx.x;
+  // a dependent launch may start early: the stream pass's results are read
+  // only after this; the next call's sampling may then be scheduled (it
+  // writes nothing this kernel reads before waiting for it)
+  griddep_wait();
+  griddep_launch_dependents();
   const bool failed = (__ldcg(a.list_flags) & kDevErrTimeout) != 0;
   if (blockIdx.x == 0 && tid == 0) {
     *a.count_out = failed ? 0u : a.total_k;
@@ -434,64 +682,20 @@ __global__ void __launch_bounds__(kLwThreads, 1)
   }
   if (failed) return;  // a is incomplete: nothing is selected
   bool overflow = false, bad = false;
-  const uint32_t w_end = a.work_ptr[blockIdx.x + 1];
-  for (uint32_t w = a.work_ptr[blockIdx.x]; w < w_end; ++w) {
-    const uint32_t si = a.work_seg[w];
-    const LwSeg s = a.segs[si];
-    uint32_t* io = idx_out + s.out;
-    float* vo = val_out + s.out;
-    const uint32_t ds = s.hi - s.lo;
-    __syncthreads();  // the previous segment is done with shared memory
-    if (s.kind == kLwAll) {
-      for (uint32_t i = tid; i < ds; i += kLwThreads) {
-        io[i] = s.lo + i;
-        vo[i] = __ldcg(e + s.lo + i);
-        e[s.lo + i] = 0.0f;
-      }
-      continue;
+  const LwCta me = a.ctas[blockIdx.x];
+  if (me.team == kLwNoTeam) {
+    for (uint32_t w = me.a; w < me.b; ++w) {
+      const uint32_t si = a.work_seg[w];
+      const LwSeg s = a.segs[si];
+      __syncthreads();  // the previous segment is done with shared memory
+      if (!select_single(a, s, si, e, idx_out, val_out, overflow, s_bits, s_hist, s_w, s_lo,
+                         s_hi))
+        bad = true;
     }
-    SmallSelection sel;
-    uint32_t lo, hi, got = 0;
-    bool found = false;
-    if (s.kind == kLwWhole) {
-      load_minmax(e + s.lo, ds, s_bits, lo, hi, s_lo, s_hi);
-      found = threshold_levels<kLwThreads>(MagsShared{s_bits}, ds, s.k, lo, hi, s_hist, s_w, sel);
-      if (found)
-        got = emit_selected(SrcSharedArray{s_bits, s.lo}, ds, sel, s.k, io, vo, e, overflow, s_w);
-    } else {  // kLwSampled
-      bool use = a.use_list && __ldcg(a.mbound + si) != kLwNoBound;
-      uint32_t c0 = 0, c1 = 0;
-      if (use) {
-        bool ok = true;
-        c0 = list_position(a, s.lo, ok);
-        c1 = list_position(a, s.hi, ok);
-        use = ok && c1 <= a.cap && c1 - c0 >= s.k;
-      }
-      if (use && c1 - c0 <= kLwSmemElems) {
-        const uint32_t n = c1 - c0;
-        load_minmax(a.list_val + c0, n, s_bits, lo, hi, s_lo, s_hi);
-        found = threshold_levels<kLwThreads>(MagsShared{s_bits}, n, s.k, lo, hi, s_hist, s_w, sel);
-        if (found)
-          got = emit_selected(SrcSharedList{s_bits, a.list_idx + c0}, n, sel, s.k, io, vo, e,
-                              overflow, s_w);
-      } else if (use) {
-        const uint32_t n = c1 - c0;
-        load_minmax(a.list_val + c0, n, nullptr, lo, hi, s_lo, s_hi);
-        found = threshold_levels<kLwThreads>(MagsGlobal{a.list_val + c0}, n, s.k, lo, hi, s_hist,
-                                             s_w, sel);
-        if (found)
-          got = emit_selected(SrcGlobalList{a.list_val + c0, a.list_idx + c0}, n, sel, s.k, io,
-                              vo, e, overflow, s_w);
-      } else {
-        load_minmax(e + s.lo, ds, nullptr, lo, hi, s_lo, s_hi);
-        found = threshold_levels<kLwThreads>(MagsGlobal{e + s.lo}, ds, s.k, lo, hi, s_hist, s_w,
-                                             sel);
-        if (found)
-          got = emit_selected(SrcGlobalArray{e + s.lo, s.lo}, ds, sel, s.k, io, vo, e, overflow,
-                              s_w);
-      }
-    }
-    if (!found || got != s.k) bad = true;
+  } else {
+    const LwSeg s = a.segs[me.a];
+    select_team(a, s, me.a, me.b, me.rank, a.teams + me.team, e, idx_out, val_out, overflow, bad,
+                s_hist, s_w);
   }
   if (__syncthreads_or(overflow) && tid == 0) atomicOr(a.error, kDevErrOverflow);
   if (__syncthreads_or(bad) && tid == 0) atomicOr(a.error, kDevErrBadInput);
@@ -512,7 +716,27 @@ int lw_stream_blocks_per_sm() {
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
-// Work estimate of a segment's selection, in list positions handled.
+// A launch that may begin while the previous kernel on the stream finishes
+// (programmatic dependent launch; every kernel here waits for its
+// predecessor before reading what it wrote), optionally cooperative.
+cudaError_t launch_pdl(const void* fn, uint32_t grid, uint32_t block, uint32_t smem,
+                       cudaStream_t stream, void** params, bool cooperative) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(block);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeCooperative;
+  attr[1].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = cooperative ? 2 : 1;
+  return cudaLaunchKernelExC(&cfg, fn, params);
+}
+
+// Work estimate of a segment's selection by one CTA, in positions handled.
 uint64_t select_cost(const LwSeg& s) {
   const uint64_t ds = s.hi - s.lo;
   if (s.kind == kLwAll) return ds / 2 + 1024;
@@ -541,13 +765,15 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t d, uint32_
                           reinterpret_cast<uintptr_t>(g) % 16 == 0 && per_sm > 0;
   if (streamable) {
     // 1 sample
-    if (p.n_sample_ctas > 0) {
-      lw_sample_kernel<GT><<<p.n_sample_ctas, kLwThreads, 0, ws.stream>>>(
-          g, e, gamma, segs, reinterpret_cast<const LwSample*>(p.dev + p.off_samples),
-          reinterpret_cast<uint32_t*>(p.dev + p.off_hist),
-          reinterpret_cast<uint32_t*>(p.dev + p.off_done), mbound, ws.cand_cap);
+    if (p.n_sampled > 0) {
+      const uint32_t* sampled = reinterpret_cast<const uint32_t*>(p.dev + p.off_samples);
+      uint32_t cap = ws.cand_cap;
+      void* sp[] = {(void*)&g, (void*)&e, (void*)&gamma, (void*)&segs, (void*)&sampled,
+                    (void*)&mbound, (void*)&cap};
+      err = launch_pdl(reinterpret_cast<const void*>(&lw_sample_kernel<GT>), p.n_sampled,
+                       kSampleThreads, 0, ws.stream, sp, false);
       count_launch();
-      if ((err = cudaGetLastError()) != cudaSuccess) return err;
+      if (err != cudaSuccess) return err;
     }
     // 2 stream
     ScanCtx ctx = next_scan_ctx(ws, p.tiles);
@@ -562,16 +788,11 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t d, uint32_
     uint32_t* list_count = ws.u32(kOffTkListCount);
     StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks(), tile_base};
     void* params[] = {&op, &d, &list_idx, &list_val, &list_count, &cap, &ctx, &sa};
-    // a plain launch: the only cross-CTA wait is on lower-numbered CTAs,
+    // not cooperative: the only cross-CTA wait is on lower-numbered CTAs,
     // which are scheduled first
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(grid);
-    cfg.blockDim = dim3(kStreamThreads);
-    cfg.dynamicSmemBytes = StreamLayout<LwCandOp<GT>, kLwStages>::kSmem;
-    cfg.stream = ws.stream;
-    err = cudaLaunchKernelExC(
-        &cfg, reinterpret_cast<const void*>(&stream_compact_kernel<LwCandOp<GT>, kLwStages>),
-        params);
+    err = launch_pdl(
+        reinterpret_cast<const void*>(&stream_compact_kernel<LwCandOp<GT>, kLwStages>), grid,
+        kStreamThreads, StreamLayout<LwCandOp<GT>, kLwStages>::kSmem, ws.stream, params, false);
     count_launch();
     if (err != cudaSuccess) return err;
   } else {
@@ -581,33 +802,43 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t d, uint32_
     count_launch();
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
   }
-  // 3 select
+  // 3 select: a cooperative launch when there are teams, so that every
+  // team's CTAs are resident
   LwArgs a;
   a.segs = segs;
   a.mbound = mbound;
-  a.work_ptr = reinterpret_cast<const uint32_t*>(p.dev + p.off_work_ptr);
+  a.ctas = reinterpret_cast<const LwCta*>(p.dev + p.off_ctas);
   a.work_seg = reinterpret_cast<const uint32_t*>(p.dev + p.off_work_seg);
+  a.teams = reinterpret_cast<LwTeamState*>(p.dev + p.off_teams);
   a.tile_base = tile_base;
   a.list_idx = list_idx;
   a.list_val = list_val;
   a.list_flags = list_flags;
   a.error = ws.u32(kOffError);
   a.count_out = count_out;
+  a.wait_limit_ns = wait_limit_ns();
   a.tiles = p.tiles;
   a.cap = ws.cand_cap;
   a.use_list = streamable ? 1u : 0u;
   a.total_k = static_cast<uint32_t>(p.total_k);
-  lw_select_kernel<<<p.n_select_ctas, kLwThreads, kLwSelectSmem, ws.stream>>>(e, idx_out,
-                                                                              val_out, a);
+  void* params[] = {(void*)&e, (void*)&idx_out, (void*)&val_out, (void*)&a};
+  // (cooperative only when there are teams: nothing else waits on another CTA)
+  err = launch_pdl(reinterpret_cast<const void*>(&lw_select_kernel), p.n_select_ctas, kLwThreads,
+                   kLwSelectSmem, ws.stream, params, p.n_teams > 0);
   count_launch();
-  return cudaGetLastError();
+  return err;
 }
 
 }  // namespace
 
 void topk_layerwise_init_device(DeviceInfo& info) {
-  cudaFuncSetAttribute(lw_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                       kLwSelectSmem);
+  int n = 0;
+  if (cudaFuncSetAttribute(lw_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           kLwSelectSmem) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, lw_select_kernel, kLwThreads,
+                                                    kLwSelectSmem) != cudaSuccess)
+    n = 0;
+  info.lw_select_per_sm = n;
   info.lw_stream_per_sm_f32 = lw_stream_blocks_per_sm<float>();
   info.lw_stream_per_sm_bf16 = lw_stream_blocks_per_sm<uint16_t>();
   cudaGetLastError();
@@ -626,33 +857,32 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
   // segments, sampling CTAs
   std::vector<LwSeg> segs(n_seg);
   std::vector<uint32_t> ends(n_seg), mbound(n_seg, kLwNoBound);
-  std::vector<LwSample> samples;
+  std::vector<uint32_t> sampled;  // the sampled segments, one sampling CTA each
   uint32_t n_sampled = 0;
   uint64_t lo = 0, total_k = 0;
   for (uint32_t s = 0; s < n_seg; ++s) {
     const uint64_t hi = seg_end[s], ds = hi - lo, k = seg_k[s];
     LwSeg& x = segs[s];
-    x = LwSeg{static_cast<uint32_t>(lo), static_cast<uint32_t>(hi), static_cast<uint32_t>(k),
-              static_cast<uint32_t>(total_k), kLwNone, 0, 0, 0};
+    x = LwSeg{0, static_cast<uint32_t>(lo), static_cast<uint32_t>(hi), static_cast<uint32_t>(k),
+              static_cast<uint32_t>(total_k), 0, kLwNone, 0};
+    static_assert(sizeof(LwSeg) == 32, "segment record");
     if (k == 0 || ds == 0)
       x.kind = kLwNone;
     else if (k == ds)
       x.kind = kLwAll;
-    else if (ds <= kLwSmemElems)
+    else if (ds <= kLwWholeMax)
       x.kind = kLwWhole;
     else
       x.kind = kLwSampled;
     if (x.kind == kLwSampled) {
-      // about one group of 4 per 256 coordinates, 512 .. 65536 groups
-      const uint64_t gr = std::min<uint64_t>(std::max<uint64_t>(ds / 256, 512), 65536);
-      x.groups = static_cast<uint32_t>(gr);
-      x.slot = n_sampled++;
-      x.nblk = static_cast<uint32_t>((gr + kLwSampleGroupsPerCta - 1) / kLwSampleGroupsPerCta);
-      for (uint32_t b = 0; b < x.nblk; ++b) {
-        const uint32_t q0 = b * kLwSampleGroupsPerCta;
-        const uint32_t q1 = std::min<uint32_t>(x.groups, q0 + kLwSampleGroupsPerCta);
-        samples.push_back(LwSample{s, q0, q1, 0});
-      }
+      // every aligned group of 4 while there are at most kLwSampleGroups,
+      // else kLwSampleGroups of them spread evenly
+      const uint64_t avail = (hi - 4) / 4 - (lo + 3) / 4 + 1;
+      x.groups = static_cast<uint32_t>(std::min<uint64_t>(avail, kLwSampleGroups));
+      x.exact = x.groups == avail ? 1u : 0u;
+      x.step = ((avail - 1) << 32) / (x.groups - 1);  // a segment of > 4096 holds > 1000 groups
+      ++n_sampled;
+      sampled.push_back(s);
     }
     ends[s] = static_cast<uint32_t>(hi);
     total_k += k;
@@ -669,23 +899,69 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
       tile_info[t] = s | (ends[s] >= t1 ? kLwTileUniform : 0u);
     }
   }
-  // select work: the segments with pairs to write, longest first onto the
-  // least loaded CTA
-  std::vector<uint32_t> items;
-  for (uint32_t s = 0; s < n_seg; ++s)
-    if (segs[s].kind != kLwNone) items.push_back(s);
-  std::stable_sort(items.begin(), items.end(), [&](uint32_t x, uint32_t y) {
+  // Select work. A segment whose candidates may exceed one CTA's shared
+  // memory, or whose own length would make a selection from e slow for one
+  // CTA, gets a team of co-resident CTAs; the others go, longest first, onto
+  // the least loaded of the remaining CTAs. At most sm_count x (select CTAs
+  // per SM) CTAs in all, so that the cooperative launch is resident.
+  const uint32_t budget =
+      static_cast<uint32_t>(std::max(1, dev.sm_count * std::max(1, dev.lw_select_per_sm)));
+  std::vector<uint32_t> team_seg, team_size, singles;
+  for (uint32_t s = 0; s < n_seg; ++s) {
+    const LwSeg& x = segs[s];
+    if (x.kind == kLwNone) continue;
+    uint32_t t = 1;
+    if (x.kind == kLwSampled) {
+      // candidates the bound aims at: 1.5 k_s, plus 32 samples' worth
+      const uint64_t ds = x.hi - x.lo;
+      const uint64_t est = x.exact ? x.k + 2048 : 3ull * x.k / 2 + 32ull * ds / (4ull * x.groups);
+      uint64_t want = est > kLwSmemElems * 3ull / 4 ? (est + 24575) / 24576 : 1;
+      want = std::max<uint64_t>(want, (ds + (1u << 24) - 1) >> 24);
+      t = static_cast<uint32_t>(std::min<uint64_t>(want, kLwMaxTeam));
+    }
+    if (t > 1) {
+      team_seg.push_back(s);
+      team_size.push_back(t);
+    } else {
+      singles.push_back(s);
+    }
+  }
+  {
+    // shrink the teams until they leave at least one CTA for the singles
+    const uint32_t reserve = singles.empty() ? 0u : 1u;
+    uint64_t sum = 0;
+    for (uint32_t t : team_size) sum += t;
+    while (sum + reserve > budget) {
+      auto it = std::max_element(team_size.begin(), team_size.end());
+      if (*it <= 1) break;
+      --*it;
+      --sum;
+    }
+    for (size_t q = 0; q < team_seg.size();) {  // a team of one is a single
+      if (team_size[q] <= 1) {
+        singles.push_back(team_seg[q]);
+        team_seg.erase(team_seg.begin() + q);
+        team_size.erase(team_size.begin() + q);
+      } else {
+        ++q;
+      }
+    }
+  }
+  uint32_t team_ctas = 0;
+  for (uint32_t t : team_size) team_ctas += t;
+  std::stable_sort(singles.begin(), singles.end(), [&](uint32_t x, uint32_t y) {
     return select_cost(segs[x]) > select_cost(segs[y]);
   });
-  // at least one CTA: it also writes the count and reports a failed stream
-  const uint32_t n_ctas = static_cast<uint32_t>(std::max<size_t>(
-      1, std::min<size_t>(items.size(), static_cast<size_t>(dev.sm_count))));
-  std::vector<std::vector<uint32_t>> per(n_ctas);
+  const uint32_t room = budget > team_ctas ? budget - team_ctas : 1u;
+  // at least one CTA in all: it also writes the count and reports a failed stream
+  const uint32_t n_single = static_cast<uint32_t>(std::min<size_t>(
+      singles.size(), room)) + (singles.empty() && team_ctas == 0 ? 1u : 0u);
+  std::vector<std::vector<uint32_t>> per(n_single);
   {
     using Load = std::pair<uint64_t, uint32_t>;
     std::priority_queue<Load, std::vector<Load>, std::greater<Load>> heap;
-    for (uint32_t c = 0; c < n_ctas; ++c) heap.push(Load{0, c});
-    for (uint32_t s : items) {
+    for (uint32_t c = 0; c < n_single; ++c) heap.push(Load{0, c});
+    for (uint32_t s : singles) {
       Load l = heap.top();
       heap.pop();
       per[l.second].push_back(s);
@@ -693,12 +969,16 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
       heap.push(l);
     }
   }
-  std::vector<uint32_t> work_ptr(n_ctas + 1, 0), work_seg;
-  for (uint32_t c = 0; c < n_ctas; ++c) {
-    work_ptr[c] = static_cast<uint32_t>(work_seg.size());
+  std::vector<LwCta> ctas;
+  std::vector<uint32_t> work_seg;
+  for (uint32_t q = 0; q < team_seg.size(); ++q)  // teams first: the longest work
+    for (uint32_t r = 0; r < team_size[q]; ++r) ctas.push_back(LwCta{q, team_seg[q], team_size[q], r});
+  for (uint32_t c = 0; c < n_single; ++c) {
+    const uint32_t a = static_cast<uint32_t>(work_seg.size());
     work_seg.insert(work_seg.end(), per[c].begin(), per[c].end());
+    ctas.push_back(LwCta{kLwNoTeam, a, static_cast<uint32_t>(work_seg.size()), 0});
   }
-  work_ptr[n_ctas] = static_cast<uint32_t>(work_seg.size());
+  const uint32_t n_teams = static_cast<uint32_t>(team_seg.size());
 
   // device layout
   size_t off = 0;
@@ -711,12 +991,11 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
   p.off_seg_end = take(sizeof(uint32_t) * n_seg);
   p.off_mbound = take(sizeof(uint32_t) * n_seg);
   p.off_tile_info = take(sizeof(uint32_t) * tiles);
-  p.off_samples = take(sizeof(LwSample) * samples.size());
-  p.off_work_ptr = take(sizeof(uint32_t) * work_ptr.size());
+  p.off_samples = take(sizeof(uint32_t) * sampled.size());
+  p.off_ctas = take(sizeof(LwCta) * ctas.size());
   p.off_work_seg = take(sizeof(uint32_t) * work_seg.size());
   const size_t upload = off;
-  p.off_done = take(sizeof(uint32_t) * n_seg);
-  p.off_hist = take(sizeof(uint32_t) * kSampleBins * n_sampled);
+  p.off_teams = take(sizeof(LwTeamState) * n_teams);
   const size_t zero_end = off;
   p.off_tile_base = take(sizeof(uint32_t) * (tiles + 1));
   p.total = off;
@@ -729,8 +1008,8 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
   put(p.off_seg_end, ends.data(), sizeof(uint32_t) * n_seg);
   put(p.off_mbound, mbound.data(), sizeof(uint32_t) * n_seg);
   put(p.off_tile_info, tile_info.data(), sizeof(uint32_t) * tiles);
-  put(p.off_samples, samples.data(), sizeof(LwSample) * samples.size());
-  put(p.off_work_ptr, work_ptr.data(), sizeof(uint32_t) * work_ptr.size());
+  put(p.off_samples, sampled.data(), sizeof(uint32_t) * sampled.size());
+  put(p.off_ctas, ctas.data(), sizeof(LwCta) * ctas.size());
   put(p.off_work_seg, work_seg.data(), sizeof(uint32_t) * work_seg.size());
 
   cudaError_t err;
@@ -753,7 +1032,7 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
   if ((err = cudaMemcpyAsync(p.dev, p.image.data(), upload, cudaMemcpyHostToDevice,
                              ws.stream)) != cudaSuccess)
     return err;
-  if ((err = cudaMemsetAsync(p.dev + p.off_done, 0, zero_end - p.off_done, ws.stream)) !=
+  if ((err = cudaMemsetAsync(p.dev + p.off_teams, 0, zero_end - p.off_teams, ws.stream)) !=
       cudaSuccess)
     return err;
   p.seg_end.assign(seg_end, seg_end + n_seg);
@@ -761,8 +1040,8 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
   p.d = d;
   p.n_seg = n_seg;
   p.n_sampled = n_sampled;
-  p.n_sample_ctas = static_cast<uint32_t>(samples.size());
-  p.n_select_ctas = n_ctas;
+  p.n_select_ctas = static_cast<uint32_t>(ctas.size());
+  p.n_teams = n_teams;
   p.tiles = tiles;
   p.total_k = total_k;
   p.valid = true;

@@ -60,9 +60,11 @@ def _check(g, e, gamma, sizes, ks, what, g_off=0, e_off=0):
 
 
 # sizes and budgets that reach each kind of segment: empty, nothing sent,
-# everything sent, whole in shared memory (<= 49152), sampled (> 49152)
-KINDS_SIZES = [0, 5, 64, 4097, 49152, 49153, 100_003, 3 * 4096 + 17, 1, 200_000, 7, 65_536]
-KINDS_K = [0, 5, 3, 40, 491, 1, 1000, 0, 1, 2000, 6, 65_535]
+# everything sent, selected from e whole (<= 4096), sampled at every aligned
+# group (<= 65536), sampled sparsely (> 65536), at unaligned boundaries
+KINDS_SIZES = [0, 5, 64, 4097, 49152, 49153, 100_003, 3 * 4096 + 17, 1, 200_000, 7, 65_536,
+               4096, 65_537, 2]
+KINDS_K = [0, 5, 3, 40, 491, 1, 1000, 0, 1, 2000, 6, 65_535, 4095, 66, 1]
 
 
 @pytest.mark.parametrize("bf16", [False, True])
@@ -91,6 +93,20 @@ def test_layerwise_candidates_beyond_shared_memory():
     sizes, ks = [400_000, 70_000], [60_000, 700]
     g, e = _inputs(sum(sizes), 4)
     _check(g, e, 0.1, sizes, ks, "long candidate list")
+
+
+def test_layerwise_long_list_from_ties_one_cta():
+    # a modest k whose cut falls inside a block of 100,000 equal magnitudes:
+    # the candidates far exceed shared memory but the segment is not given a
+    # team, so one CTA selects from the list in global memory
+    rng = _rng("tieblock")
+    n = 200_000
+    e = (rng.standard_normal(n + 5000) * 1e-3).astype(np.float32)
+    e[:10_000] = (1.0 + np.arange(10_000, dtype=np.float32) * 1e-4)[rng.permutation(10_000)]
+    block = rng.permutation(np.arange(10_000, n))[:100_000]
+    e[block] = np.where(rng.random(100_000) < 0.5, 0.5, -0.5).astype(np.float32)
+    g = np.zeros(n + 5000, np.float32)
+    _check(g, e, 1.0, [n, 5000], [15_000, 5], "tie block")
 
 
 def test_layerwise_bound_admits_too_many():
