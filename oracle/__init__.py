@@ -16,6 +16,9 @@ passage behind every line):
   layer's tensor separately (Appendix, layer-wise sparsification).
 * ``sparse_aggregate(idx_list, val_list, d)`` — worker-ordered sum of the
   decompressed vectors (Algorithm 1, exchange step).
+* ``sparse_aggregate_apply(idx_list, val_list, d, alpha, x, m, mu, lr)`` —
+  that sum scaled by alpha, applied as Algorithm 1's model update, or as the
+  momentum update of the Appendix's gradient-compression EF SGD.
 
 Each compression function returns ``(idx, val, e_new)`` and leaves its inputs
 untouched; ``g`` may be float32 or bfloat16 bit patterns (uint16).
@@ -80,6 +83,10 @@ def _load():
                 ctypes.c_uint32, ctypes.POINTER(u32p), ctypes.POINTER(f32p), u32p,
                 ctypes.c_uint64, f32p]
             lib.oracle_sparse_aggregate.restype = ctypes.c_int
+            lib.oracle_sparse_aggregate_apply.argtypes = [
+                ctypes.c_uint32, ctypes.POINTER(u32p), ctypes.POINTER(f32p), u32p,
+                ctypes.c_uint64, ctypes.c_float, f32p, f32p, ctypes.c_float, ctypes.c_float]
+            lib.oracle_sparse_aggregate_apply.restype = ctypes.c_int
             _lib = lib
     return _lib
 
@@ -163,6 +170,49 @@ def ef_topk_layerwise(g: np.ndarray, e: np.ndarray, gamma: float, seg_end, seg_k
         raise ValueError("oracle_ef_topk_layerwise rejected the segment table (%d)" % rc)
     c = int(cnt[0])
     return idx[:c].copy(), val[:c].copy(), e_new
+
+
+def _lists(idx_list, val_list):
+    n = len(idx_list)
+    assert n == len(val_list) and n >= 1
+    idx_arrs = [np.ascontiguousarray(x, dtype=np.uint32) for x in idx_list]
+    val_arrs = [np.ascontiguousarray(v, dtype=np.float32) for v in val_list]
+    # keep zero-length lists addressable
+    idx_arrs = [a if a.size else np.zeros(1, np.uint32) for a in idx_arrs]
+    val_arrs = [v if v.size else np.zeros(1, np.float32) for v in val_arrs]
+    counts = np.array([len(x) for x in idx_list], dtype=np.uint32)
+    for i in range(n):
+        assert len(val_list[i]) == counts[i]
+    u32p = ctypes.POINTER(ctypes.c_uint32)
+    f32p = ctypes.POINTER(ctypes.c_float)
+    idx_ptrs = (u32p * n)(*[_ptr(a, ctypes.c_uint32) for a in idx_arrs])
+    val_ptrs = (f32p * n)(*[_ptr(v, ctypes.c_float) for v in val_arrs])
+    return n, idx_arrs, val_arrs, counts, idx_ptrs, val_ptrs
+
+
+def sparse_aggregate_apply(idx_list, val_list, d: int, alpha: float, x, m=None, mu: float = 0.0,
+                           lr: float = 0.0):
+    """Model update from the worker-ordered sum s of n sparse vectors:
+    Delta' = alpha * s; without ``m``: x <- x - Delta'; with ``m``:
+    m <- fmaf(mu, m, Delta'), x <- fmaf(-lr, Delta' + m, x). Returns
+    (x_new, m_new or None); the inputs are left untouched."""
+    lib = _load()
+    n, idx_arrs, val_arrs, counts, idx_ptrs, val_ptrs = _lists(idx_list, val_list)
+    x_new = np.array(x, dtype=np.float32, copy=True).reshape(-1)
+    assert x_new.size == d
+    m_new = None if m is None else np.array(m, dtype=np.float32, copy=True).reshape(-1)
+    if m_new is not None:
+        assert m_new.size == d
+    f32p = ctypes.POINTER(ctypes.c_float)
+    xb = x_new if d else np.zeros(1, np.float32)
+    mb = None if m_new is None else (m_new if d else np.zeros(1, np.float32))
+    rc = lib.oracle_sparse_aggregate_apply(
+        n, idx_ptrs, val_ptrs, _ptr(counts, ctypes.c_uint32), d, ctypes.c_float(alpha),
+        _ptr(xb, ctypes.c_float), ctypes.cast(None, f32p) if mb is None else _ptr(mb, ctypes.c_float),
+        ctypes.c_float(mu), ctypes.c_float(lr))
+    if rc != 0:
+        raise RuntimeError("oracle_sparse_aggregate_apply: index out of range")
+    return x_new, m_new
 
 
 def sparse_aggregate(idx_list, val_list, d: int) -> np.ndarray:

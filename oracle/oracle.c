@@ -30,6 +30,11 @@
  *   R7 the residual of a sent coordinate is +0.0f.
  *   R9 aggregation returns the sum (the 1/n of Algorithm 1 is the caller's),
  *      accumulated from +0.0f in ascending worker order.
+ *   R12 model update after aggregation (the paper is silent on rounding):
+ *      Delta'_j = alpha * s_j rounded once (alpha = 1/n gives the mean);
+ *      without momentum x_j <- x_j - Delta'_j; with momentum
+ *      m_j <- fmaf(mu, m_j, Delta'_j) and x_j <- fmaf(-lr, Delta'_j + m_j, x_j),
+ *      the sum Delta'_j + m_j rounded once.
  */
 #include <math.h>
 #include <stdint.h>
@@ -234,4 +239,36 @@ int oracle_sparse_aggregate(uint32_t n, const uint32_t* const* idx,
     }
   }
   return 0;
+}
+
+/* ------------------------------------------------------------------------
+ * Model update after the exchange step (R12).
+ *   Algorithm 1:  Delta_bar_t = (1/n) sum_i Delta_{i,t};  x_{t+1} = x_t - Delta_bar_t.
+ *   Appendix, distributed EF SGD with momentum by gradient compression (the
+ *   EF strategy of the experiments): Delta' = the aggregated compressed
+ *   vectors; m <- lambda m + Delta'; x <- x - gamma (Delta' + m), with the
+ *   momentum factor called mu and the learning rate lr here.
+ * m == NULL selects Algorithm 1's update; otherwise the momentum one.
+ * ------------------------------------------------------------------------ */
+int oracle_sparse_aggregate_apply(uint32_t n, const uint32_t* const* idx,
+                                  const float* const* val, const uint32_t* counts,
+                                  uint64_t d, float alpha, float* x, float* m, float mu,
+                                  float lr) {
+  float* s = (float*)malloc((d ? d : 1) * sizeof(float));
+  if (!s) return 2;
+  int rc = oracle_sparse_aggregate(n, idx, val, counts, d, s);
+  if (rc == 0) {
+    for (uint64_t j = 0; j < d; ++j) {
+      float delta = canonical_nan_if_nan(alpha * s[j]);          /* Delta'_j */
+      if (m) {
+        m[j] = canonical_nan_if_nan(fmaf(mu, m[j], delta));      /* m <- mu m + Delta' */
+        float u = canonical_nan_if_nan(delta + m[j]);            /* Delta' + m */
+        x[j] = canonical_nan_if_nan(fmaf(-lr, u, x[j]));         /* x <- x - lr (Delta' + m) */
+      } else {
+        x[j] = canonical_nan_if_nan(x[j] - delta);               /* x <- x - Delta_bar */
+      }
+    }
+  }
+  free(s);
+  return rc;
 }

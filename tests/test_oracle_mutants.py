@@ -39,6 +39,17 @@ MUTANTS = {
     "layerwise_first_k_everywhere": [("                       seg_k[s], hi - lo,",
                                       "                       seg_k[0] < hi - lo ? seg_k[0] : hi - lo, hi - lo,")],
     "layerwise_error_not_sliced": [("e + lo, gamma,", "e, gamma,")],
+    "update_uses_old_momentum": [
+        ("        m[j] = canonical_nan_if_nan(fmaf(mu, m[j], delta));      /* m <- mu m + Delta' */\n"
+         "        float u = canonical_nan_if_nan(delta + m[j]);            /* Delta' + m */",
+         "        float u = canonical_nan_if_nan(delta + m[j]);            /* Delta' + m */\n"
+         "        m[j] = canonical_nan_if_nan(fmaf(mu, m[j], delta));      /* m <- mu m + Delta' */")],
+    "update_alpha_dropped": [("float delta = canonical_nan_if_nan(alpha * s[j]);",
+                              "float delta = canonical_nan_if_nan(s[j]);")],
+    "update_momentum_two_step": [("fmaf(mu, m[j], delta)", "(mu * m[j] + delta)")],
+    "update_wrong_sign": [("fmaf(-lr, u, x[j])", "fmaf(lr, u, x[j])")],
+    "update_sgd_adds": [("x[j] = canonical_nan_if_nan(x[j] - delta);",
+                         "x[j] = canonical_nan_if_nan(x[j] + delta);")],
 }
 
 PIN_TESTS = [
@@ -58,6 +69,10 @@ PIN_TESTS = [
     pins.test_topk_layerwise_hand_example,
     lambda: pins.test_topk_layerwise_matches_bruteforce_per_segment(0),
     lambda: pins.test_topk_layerwise_matches_bruteforce_per_segment(1),
+    pins.test_update_algorithm1_subtracts_the_mean,
+    pins.test_update_momentum_closed_form,
+    pins.test_update_momentum_zero_factor,
+    pins.test_update_rounding_follows_r12,
 ]
 
 
@@ -69,7 +84,8 @@ def _swapped_library(path):
     # reuse the argtypes of the real library
     for name in ("oracle_ef_hard_threshold", "oracle_ef_hard_threshold_bf16",
                  "oracle_ef_topk", "oracle_ef_topk_bf16", "oracle_ef_topk_layerwise",
-                 "oracle_ef_topk_layerwise_bf16", "oracle_sparse_aggregate"):
+                 "oracle_ef_topk_layerwise_bf16", "oracle_sparse_aggregate",
+                 "oracle_sparse_aggregate_apply"):
         fn, ref = getattr(lib, name), getattr(saved, name)
         fn.argtypes, fn.restype = ref.argtypes, ref.restype
     oracle._lib = lib

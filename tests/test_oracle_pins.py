@@ -444,6 +444,96 @@ def test_aggregate_rejects_out_of_range():
 
 
 # --------------------------------------------------------------------------
+# model update after the exchange step: Algorithm 1 (x <- x - mean of the
+# Delta_i) and the Appendix's EF SGD with momentum by gradient compression
+# (m <- mu m + Delta', x <- x - lr (Delta' + m))
+# --------------------------------------------------------------------------
+def test_update_algorithm1_subtracts_the_mean():
+    # dyadic values keep every quantity exact, so the mean is a Fraction
+    rng = np.random.default_rng(11)
+    n, d = 4, 40
+    idx_list, val_list = [], []
+    for _ in range(n):
+        ix = np.sort(rng.choice(d, 12, replace=False)).astype(np.uint32)
+        idx_list.append(ix)
+        val_list.append(_f32(rng.integers(-64, 65, 12) / 64.0))
+    x0 = _f32(rng.integers(-32, 33, d) / 16.0)
+    x, m = oracle.sparse_aggregate_apply(idx_list, val_list, d, 1.0 / n, x0)
+    assert m is None
+    want = [Fraction(float(v)) for v in x0]
+    for ix, vv in zip(idx_list, val_list):
+        for j, v in zip(ix, vv):
+            want[j] -= Fraction(float(v)) / n
+    assert [Fraction(float(v)) for v in x] == want
+
+
+def test_update_momentum_closed_form():
+    # a constant aggregate Delta' = c: m_t = c (1 - mu^t) / (1 - mu) and
+    # x_t = x_{t-1} - lr (c + m_t); with mu = 1/2, lr = 1/4, c = 3/8 every
+    # value is dyadic and exact in fp32 over these iterations
+    mu, lr, c = Fraction(1, 2), Fraction(1, 4), Fraction(3, 8)
+    d = 6
+    idx = [np.array([1, 4], np.uint32), np.array([1, 4], np.uint32)]
+    val = [_f32([0.375, 0.375]), _f32([0.375, 0.375])]  # alpha = 1/2: Delta' = 3/8
+    x = _f32([0.5] * d)
+    m = np.zeros(d, np.float32)
+    xf, mf = Fraction(1, 2), Fraction(0)
+    for t in range(1, 13):
+        x, m = oracle.sparse_aggregate_apply(idx, val, d, 0.5, x, m, float(mu), float(lr))
+        mf = mu * mf + c
+        xf = xf - lr * (c + mf)
+        assert mf == c * (1 - mu ** t) / (1 - mu)
+        assert Fraction(float(m[1])) == mf and Fraction(float(m[4])) == mf
+        assert Fraction(float(x[1])) == xf and Fraction(float(x[4])) == xf
+        assert m[0] == 0.0 and x[0] == 0.5  # nothing sent: Delta' = 0, m stays 0
+
+
+def test_update_momentum_zero_factor():
+    # mu = 0: m = Delta' and x <- x - lr (Delta' + Delta'), as the algorithm is written
+    idx = [np.array([0, 2], np.uint32)]
+    val = [_f32([1.5, -2.0])]
+    x, m = oracle.sparse_aggregate_apply(idx, val, 3, 1.0, _f32([1.0, 1.0, 1.0]),
+                                         _f32([9.0, 9.0, 9.0]), 0.0, 0.25)
+    assert list(m) == [1.5, 0.0, -2.0]
+    assert list(x) == [1.0 - 0.25 * 3.0, 1.0, 1.0 + 0.25 * 4.0]
+
+
+def test_update_rounding_follows_r12():
+    # each step rounded as R12 states, predicted with exact rational arithmetic:
+    # Delta' = RN(alpha s), m' = RN(mu m + Delta'), u = RN(Delta' + m'),
+    # x' = RN(x - lr u); includes cases where a two-step mu m + Delta' differs
+    rng = np.random.default_rng(12)
+    d = 2000
+    s_vals = _f32(rng.standard_normal(d) * rng.choice([1e-3, 1.0, 1e3], d))
+    x0 = _f32(rng.standard_normal(d))
+    m0 = _f32(rng.standard_normal(d) * 0.1)
+    mu, lr, alpha = np.float32(0.9), np.float32(0.0123), np.float32(0.125)
+    idx = [np.arange(d, dtype=np.uint32)]
+    x, m = oracle.sparse_aggregate_apply(idx, [s_vals], d, float(alpha), x0, m0, float(mu),
+                                         float(lr))
+    differs = 0
+    for j in range(d):
+        delta = round_f32(to_frac(alpha) * to_frac(s_vals[j]))
+        mj = fma_f32(mu, m0[j], delta)
+        two_step = round_f32(to_frac(round_f32(to_frac(mu) * to_frac(m0[j]))) + to_frac(delta))
+        differs += two_step != mj
+        u = round_f32(to_frac(delta) + to_frac(mj))
+        xj = fma_f32(-lr, u, x0[j])
+        assert float(m[j]) == mj, j
+        assert float(x[j]) == xj, j
+    assert differs > 0
+
+
+def test_update_sums_workers_in_order():
+    # the update sees the worker-ordered sum: (0 + 2^24) + 1 - 2^24 = 0
+    big = np.float32(2.0 ** 24)
+    idx = [np.array([2], np.uint32)] * 3
+    x, _ = oracle.sparse_aggregate_apply(idx, [_f32([big]), _f32([1.0]), _f32([-big])], 4, 1.0,
+                                         _f32([5.0, 5.0, 5.0, 5.0]))
+    assert x[2] == 5.0
+
+
+# --------------------------------------------------------------------------
 # multi-iteration EF: Lemma 9 (virtual iterate) per worker
 # --------------------------------------------------------------------------
 
