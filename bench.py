@@ -9,7 +9,9 @@ workload, through the whole hot path:
     sparse_aggregate of those messages;
   - n x ef_topk_layerwise (Top-k on each parameter tensor separately, the
     same fraction of every tensor) on the same gradients, then
-    sparse_aggregate of those messages.
+    sparse_aggregate of those messages;
+  - sparse_aggregate_apply of the hard-threshold messages into a model and
+    momentum state (the momentum EF SGD update, fused with the exchange).
 Gradients come from two pre-generated synthetic batches (alternating), so
 every step compresses different data; each step's working set (n workers x
 (g, e_ht, e_topk)) is far larger than the 126 MB L2.
@@ -276,6 +278,8 @@ def run_ours(args):
     dense_ht = torch.empty(d, device=dev)
     dense_tk = torch.empty(d, device=dev)
     dense_lw = torch.empty(d, device=dev)
+    x_model = torch.zeros(d, device=dev)
+    m_model = torch.zeros(d, device=dev)
     total = args.warmup + args.steps
     cnt_ht = torch.zeros(total, n, dtype=torch.int32, device=dev)
     cnt_tk = torch.zeros(total, n, dtype=torch.int32, device=dev)
@@ -283,7 +287,7 @@ def run_ours(args):
     stream = torch.cuda.current_stream()
 
     ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
-    marks = [[ev() for _ in range(7)] for _ in range(args.steps)]
+    marks = [[ev() for _ in range(8)] for _ in range(args.steps)]
 
     def step(s, timed):
         g = batches[s % 2]
@@ -306,6 +310,9 @@ def run_ours(args):
         if m: m[5].record(stream)
         efs.sparse_aggregate(idx_lw, val_lw, cnt_lw[s], d, dense_lw)
         if m: m[6].record(stream)
+        efs.sparse_aggregate_apply(idx_ht, val_ht, cnt_ht[s], d, 1.0 / n, x_model, m_model, 0.9,
+                                   gamma)
+        if m: m[7].record(stream)
 
     for s in range(args.warmup):
         step(s, False)
@@ -332,13 +339,14 @@ def run_ours(args):
 
     step_s = t0.elapsed_time(t1) / 1e3
     # per-iteration segment times (µs per call: the segment of n calls / n)
-    seg_us = [[m[a].elapsed_time(m[a + 1]) * 1e3 for m in marks] for a in range(6)]
+    seg_us = [[m[a].elapsed_time(m[a + 1]) * 1e3 for m in marks] for a in range(7)]
     ht_s = sum(m[0].elapsed_time(m[1]) for m in marks) / 1e3
     agg_ht_s = sum(m[1].elapsed_time(m[2]) for m in marks) / 1e3
     tk_s = sum(m[2].elapsed_time(m[3]) for m in marks) / 1e3
     agg_tk_s = sum(m[3].elapsed_time(m[4]) for m in marks) / 1e3
     lw_s = sum(m[4].elapsed_time(m[5]) for m in marks) / 1e3
     agg_lw_s = sum(m[5].elapsed_time(m[6]) for m in marks) / 1e3
+    upd_s = sum(m[6].elapsed_time(m[7]) for m in marks) / 1e3
     counts_ht = cnt_ht[args.warmup:].double()
     counts_tk = cnt_tk[args.warmup:].double()
     bytes_ht = float(ht_bytes(d, 0) * n * args.steps + 8 * counts_ht.sum().item())
@@ -346,6 +354,7 @@ def run_ours(args):
     bytes_lw = float((12 * d + 8 * k_lw) * n * args.steps)
     bytes_agg_ht = float(8 * counts_ht.sum().item() + 4 * d * args.steps)
     bytes_agg_tk = float(8 * counts_tk.sum().item() + 4 * d * args.steps)
+    bytes_upd = float(8 * counts_ht.sum().item() + 16 * d * args.steps)
 
     ht_s_max, bytes_ht_all = reduce_timing(dist, ht_s, bytes_ht, dev)
     step_s_max, _ = reduce_timing(dist, step_s, 0.0, dev)
@@ -412,6 +421,12 @@ def run_ours(args):
             "frac_of_peak": round(bytes_lw / lw_s / 1e9 / peak, 4),
             "aggregate_ms_per_iter": round(agg_lw_s / args.steps * 1e3, 4),
         },
+        "aggregate_apply_momentum": {
+            "ms_per_iter": round(upd_s / args.steps * 1e3, 4),
+            "gbs": round(bytes_upd / upd_s / 1e9, 2),
+            "frac_of_peak": round(bytes_upd / upd_s / 1e9 / peak, 4),
+            "bytes": "8 per hard-threshold pair + 16 per coordinate (x, m read and written)",
+        },
         "per_call_us_p10_p50_p90": {
             "ht": percentiles([v / n for v in seg_us[0]]),
             "topk": percentiles([v / n for v in seg_us[2]]),
@@ -419,6 +434,7 @@ def run_ours(args):
             "aggregate_ht": percentiles(seg_us[1]),
             "aggregate_topk": percentiles(seg_us[3]),
             "aggregate_topk_layerwise": percentiles(seg_us[5]),
+            "aggregate_apply_momentum": percentiles(seg_us[6]),
         },
         "frac_of_nominal_8tbs": round(value / NOMINAL_HBM_GBS, 4),
         "roofline": {

@@ -212,6 +212,38 @@ ef_status sparse_aggregate(uint32_t n, const uint32_t* const* idx,
                            uint64_t d, float* dense_out, ef_stream_t stream);
 
 /*
+ * sparse_aggregate_apply — the exchange step followed by the model update,
+ * in one pass: the worker-ordered sum of sparse_aggregate is never written
+ * to memory.
+ *
+ * Defines: with s[j] the sum of sparse_aggregate and Delta'[j] = alpha * s[j]
+ * (rounded once; alpha = 1/n gives Algorithm 1's mean Delta_bar),
+ *   m == NULL:  x[j] <- x[j] - Delta'[j]
+ *               (Algorithm 1's model update x_{t+1} = x_t - Delta_bar_t);
+ *   m != NULL:  m[j] <- fmaf(momentum, m[j], Delta'[j]),
+ *               x[j] <- fmaf(-lr, Delta'[j] + m[j], x[j]), the sum rounded once
+ *               (the Appendix's distributed EF SGD with momentum by gradient
+ *               compression: m <- lambda m + Delta', x <- x - gamma (Delta' + m),
+ *               the EF strategy of the paper's experiments).
+ * The paper does not fix the rounding of these updates; these single
+ * roundings are the library's definition, bit-identical with the oracle.
+ *
+ *   n, idx, val, counts, d   as for sparse_aggregate.
+ *   alpha      scale of the sum, finite.
+ *   x          [in/out] fp32[d], the model parameters (DEVICE pointer, 4-byte
+ *              aligned; 16-byte alignment of x and m selects vector access).
+ *   m          [in/out] fp32[d], the momentum state, or NULL for Algorithm 1.
+ *   momentum   momentum factor (lambda of the Appendix algorithm), finite.
+ *   lr         learning rate (gamma of the Appendix algorithm), finite.
+ * x and m must not overlap each other or any idx/val list. Malformed lists
+ * behave as in sparse_aggregate (pair skipped, EF_ERR_BAD_INPUT latched).
+ */
+ef_status sparse_aggregate_apply(uint32_t n, const uint32_t* const* idx,
+                                 const float* const* val, const uint32_t* counts,
+                                 uint64_t d, float alpha, float* x, float* m,
+                                 float momentum, float lr, ef_stream_t stream);
+
+/*
  * ef_hard_threshold_noalloc — ef_hard_threshold for callers that cannot
  * allocate device memory. (An implementation convenience; the paper has no
  * counterpart.)

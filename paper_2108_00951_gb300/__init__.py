@@ -26,5 +26,6 @@ from ._binding import (  # noqa: F401
     library_path,
     load_library,
     sparse_aggregate,
+    sparse_aggregate_apply,
     status_string,
 )

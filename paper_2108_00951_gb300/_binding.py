@@ -62,6 +62,8 @@ def load_library(build_if_missing: bool = True):
             "ef_topk_layerwise": [vp, vp, f32, u32, vp, vp, u64, vp, vp, vp, vp],
             "ef_topk_layerwise_bf16": [vp, vp, f32, u32, vp, vp, u64, vp, vp, vp, vp],
             "sparse_aggregate": [u32, ctypes.POINTER(vp), ctypes.POINTER(vp), vp, u64, vp, vp],
+            "sparse_aggregate_apply": [u32, ctypes.POINTER(vp), ctypes.POINTER(vp), vp, u64, f32,
+                                       vp, vp, f32, f32, vp],
             "ef_check_status": [vp],
             "ef_workspace_release": [],
         }
@@ -190,6 +192,26 @@ def sparse_aggregate(idx_list, val_list, counts, d, dense_out, stream=None):
     _check(lib.sparse_aggregate(n, idx_arr, val_arr, _dev(counts, "counts", torch.int32, n),
                                 int(d), _dev(dense_out, "dense_out", torch.float32, d),
                                 _stream(stream)), "sparse_aggregate")
+
+
+def sparse_aggregate_apply(idx_list, val_list, counts, d, alpha, x, m=None, momentum=0.0, lr=0.0,
+                           stream=None):
+    """Worker-ordered sum of n sparse vectors, scaled by ``alpha``, applied to
+    the model ``x`` (float32 [d], in place): ``x -= Delta'`` without ``m``;
+    with ``m`` (float32 [d], in place) ``m = fmaf(momentum, m, Delta')`` and
+    ``x = fmaf(-lr, Delta' + m, x)``."""
+    lib = load_library()
+    n = len(idx_list)
+    if n != len(val_list):
+        raise ValueError("idx_list and val_list differ in length")
+    idx_arr = (ctypes.c_void_p * max(n, 1))(*[_dev(t, "idx", torch.int32) for t in idx_list])
+    val_arr = (ctypes.c_void_p * max(n, 1))(*[_dev(t, "val", torch.float32) for t in val_list])
+    m_ptr = ctypes.c_void_p(0) if m is None else _dev(m, "m", torch.float32, d)
+    _check(lib.sparse_aggregate_apply(n, idx_arr, val_arr, _dev(counts, "counts", torch.int32, n),
+                                      int(d), ctypes.c_float(alpha),
+                                      _dev(x, "x", torch.float32, d), m_ptr,
+                                      ctypes.c_float(momentum), ctypes.c_float(lr),
+                                      _stream(stream)), "sparse_aggregate_apply")
 
 
 def ef_check_status(stream=None) -> int:

@@ -324,6 +324,33 @@ ef_status sparse_aggregate(uint32_t n, const uint32_t* const* idx, const float* 
       efs::launch_aggregate(n, idx, val, counts, static_cast<uint32_t>(d), dense_out, *ws), ws);
 }
 
+ef_status sparse_aggregate_apply(uint32_t n, const uint32_t* const* idx, const float* const* val,
+                                 const uint32_t* counts, uint64_t d, float alpha, float* x,
+                                 float* m, float momentum, float lr, ef_stream_t stream) {
+  if (n == 0 || n > efs::kMaxWorkers || !idx || !val || !counts) return EF_ERR_INVALID_ARG;
+  if (d > efs::kMaxD) return EF_ERR_INVALID_ARG;
+  if (!std::isfinite(alpha) || !std::isfinite(momentum) || !std::isfinite(lr))
+    return EF_ERR_INVALID_ARG;
+  if (d == 0) return EF_OK;
+  if (!x || !efs::aligned(x, 4) || !efs::aligned(counts, 4) || (m && !efs::aligned(m, 4)))
+    return EF_ERR_INVALID_ARG;
+  if (m && efs::overlaps(x, static_cast<size_t>(d) * 4, m, static_cast<size_t>(d) * 4))
+    return EF_ERR_INVALID_ARG;
+  for (uint32_t i = 0; i < n; ++i)
+    if (!idx[i] || !val[i] || !efs::aligned(idx[i], 4) || !efs::aligned(val[i], 4))
+      return EF_ERR_INVALID_ARG;
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const uint32_t tiles = efs::agg_tiles_for(d);
+  Workspace* ws = nullptr;
+  const ef_status st = efs::acquire_workspace(
+      s, 0, 0, static_cast<size_t>(n) * (static_cast<size_t>(tiles) + 1), 0, &ws);
+  if (st != EF_OK) return st;
+  return efs::finish_launch(efs::launch_aggregate_apply(n, idx, val, counts,
+                                                        static_cast<uint32_t>(d), alpha, x, m,
+                                                        momentum, lr, *ws),
+                            ws);
+}
+
 ef_status ef_check_status(ef_stream_t stream) {
   const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (cudaStreamSynchronize(s) != cudaSuccess) return EF_ERR_CUDA;

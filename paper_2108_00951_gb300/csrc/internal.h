@@ -190,6 +190,10 @@ cudaError_t launch_topk_layerwise(const void* g, bool g_bf16, float* e, float ga
 cudaError_t launch_aggregate(uint32_t n, const uint32_t* const* idx, const float* const* val,
                              const uint32_t* counts, uint32_t d, float* dense_out,
                              Workspace& ws);
+cudaError_t launch_aggregate_apply(uint32_t n, const uint32_t* const* idx,
+                                   const float* const* val, const uint32_t* counts, uint32_t d,
+                                   float alpha, float* x, float* m, float mu, float lr,
+                                   Workspace& ws);
 
 
 // Workspace sizing helpers.

@@ -118,6 +118,21 @@ def test_aggregate_rejects():
     assert lib.sparse_aggregate(1, arr, varr, vp(CNT), 100, vp(G + 1), vp(0)) == efs.EF_ERR_INVALID_ARG
 
 
+def test_aggregate_apply_rejects():
+    lib = efs.load_library()
+    arr = (vp * 1)(vp(IDX))
+    varr = (vp * 1)(vp(VAL))
+    f = ctypes.c_float
+
+    def call(n=1, cnt=CNT, d=100, alpha=0.5, x=G, m=E, mu=0.9, lr=0.1):
+        return lib.sparse_aggregate_apply(n, arr, varr, vp(cnt), d, f(alpha), vp(x), vp(m), f(mu),
+                                          f(lr), vp(0))
+    for kwargs in (dict(n=0), dict(n=257), dict(cnt=0), dict(d=2 ** 32), dict(x=0),
+                   dict(x=G + 2), dict(m=E + 1), dict(m=G + 200), dict(alpha=float("nan")),
+                   dict(mu=float("inf")), dict(lr=float("nan"))):
+        assert call(**kwargs) == efs.EF_ERR_INVALID_ARG, kwargs
+
+
 def test_binding_fails_loudly_on_cpu_tensors():
     torch = pytest.importorskip("torch")
     x = torch.zeros(8)
