@@ -16,6 +16,7 @@ passage behind every line):
   layer's tensor separately (Appendix, layer-wise sparsification).
 * ``sparse_aggregate(idx_list, val_list, d)`` — worker-ordered sum of the
   decompressed vectors (Algorithm 1, exchange step).
+* ``error_norm_sq(e)`` — ||e||^2 in fp64, the per-step term of the total error.
 * ``sparse_aggregate_apply(idx_list, val_list, d, alpha, x, m, mu, lr)`` —
   that sum scaled by alpha, applied as Algorithm 1's model update, or as the
   momentum update of the Appendix's gradient-compression EF SGD.
@@ -87,6 +88,8 @@ def _load():
                 ctypes.c_uint32, ctypes.POINTER(u32p), ctypes.POINTER(f32p), u32p,
                 ctypes.c_uint64, ctypes.c_float, f32p, f32p, ctypes.c_float, ctypes.c_float]
             lib.oracle_sparse_aggregate_apply.restype = ctypes.c_int
+            lib.oracle_error_norm_sq.argtypes = [f32p, ctypes.c_uint64]
+            lib.oracle_error_norm_sq.restype = ctypes.c_double
             _lib = lib
     return _lib
 
@@ -213,6 +216,15 @@ def sparse_aggregate_apply(idx_list, val_list, d: int, alpha: float, x, m=None, 
     if rc != 0:
         raise RuntimeError("oracle_sparse_aggregate_apply: index out of range")
     return x_new, m_new
+
+
+def error_norm_sq(e) -> float:
+    """||e||^2 = sum_j e_j^2 in fp64, index order: the per-step error norm whose
+    sum over iterations is the paper's total error."""
+    lib = _load()
+    e = np.ascontiguousarray(e, dtype=np.float32).reshape(-1)
+    buf = e if e.size else np.zeros(1, np.float32)
+    return float(lib.oracle_error_norm_sq(_ptr(buf, ctypes.c_float), e.size))
 
 
 def sparse_aggregate(idx_list, val_list, d: int) -> np.ndarray:

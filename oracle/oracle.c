@@ -272,3 +272,15 @@ int oracle_sparse_aggregate_apply(uint32_t n, const uint32_t* const* idx,
   free(s);
   return rc;
 }
+
+/* ------------------------------------------------------------------------
+ * Squared error norm of one step, ||e_{t+1}||^2 = sum_j e'_j^2: the term
+ * whose sum over iterations is the total error (Sec. 1; the remark after
+ * the EF convergence theorem). Plain fp64: every fp32 square is exact in
+ * fp64, summed in index order.
+ * ------------------------------------------------------------------------ */
+double oracle_error_norm_sq(const float* e, uint64_t d) {
+  double s = 0.0;
+  for (uint64_t j = 0; j < d; ++j) s += (double)e[j] * (double)e[j];
+  return s;
+}

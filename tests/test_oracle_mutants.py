@@ -50,6 +50,8 @@ MUTANTS = {
     "update_wrong_sign": [("fmaf(-lr, u, x[j])", "fmaf(lr, u, x[j])")],
     "update_sgd_adds": [("x[j] = canonical_nan_if_nan(x[j] - delta);",
                          "x[j] = canonical_nan_if_nan(x[j] + delta);")],
+    "error_norm_fp32_square": [("s += (double)e[j] * (double)e[j];", "s += (double)(e[j] * e[j]);")],
+    "error_norm_abs": [("s += (double)e[j] * (double)e[j];", "s += fabs((double)e[j]);")],
 }
 
 PIN_TESTS = [
@@ -73,6 +75,8 @@ PIN_TESTS = [
     pins.test_update_momentum_closed_form,
     pins.test_update_momentum_zero_factor,
     pins.test_update_rounding_follows_r12,
+    pins.test_error_norm_hand_values_and_exactness,
+    pins.test_error_norm_bounds_of_the_sparsifiers,
 ]
 
 
@@ -85,7 +89,7 @@ def _swapped_library(path):
     for name in ("oracle_ef_hard_threshold", "oracle_ef_hard_threshold_bf16",
                  "oracle_ef_topk", "oracle_ef_topk_bf16", "oracle_ef_topk_layerwise",
                  "oracle_ef_topk_layerwise_bf16", "oracle_sparse_aggregate",
-                 "oracle_sparse_aggregate_apply"):
+                 "oracle_sparse_aggregate_apply", "oracle_error_norm_sq"):
         fn, ref = getattr(lib, name), getattr(saved, name)
         fn.argtypes, fn.restype = ref.argtypes, ref.restype
     oracle._lib = lib

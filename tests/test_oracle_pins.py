@@ -534,6 +534,39 @@ def test_update_sums_workers_in_order():
 
 
 # --------------------------------------------------------------------------
+# per-step error norm ||e_{t+1}||^2 (the total error is its sum over t)
+# --------------------------------------------------------------------------
+def test_error_norm_hand_values_and_exactness():
+    assert oracle.error_norm_sq(_f32([3.0, -4.0, 0.0])) == 25.0
+    assert oracle.error_norm_sq(_f32([])) == 0.0
+    # squares that fp32 cannot hold exactly are exact in fp64: (1 + 2^-23)^2
+    x = np.float32(1.0) + np.float32(2.0 ** -23)
+    assert oracle.error_norm_sq(_f32([x])) == float(Fraction(float(x)) ** 2)
+    # tiny and huge values are neither flushed nor overflowed
+    assert oracle.error_norm_sq(_f32([1e-30])) == float(np.float32(1e-30)) ** 2
+    assert oracle.error_norm_sq(_f32([1e30])) == float(np.float32(1e30)) ** 2
+
+
+def test_error_norm_bounds_of_the_sparsifiers():
+    # hard-threshold: ||e'||_inf < lambda, so ||e'||^2 <= d lambda^2 (Sec. 5,
+    # absolute compressor with kappa^2 = d lambda^2); Top-k: ||e'||^2 <=
+    # (1 - k/d) ||a||^2 (the delta-contraction with delta = k/d)
+    rng = np.random.default_rng(21)
+    d = 5000
+    g = _f32(rng.standard_normal(d))
+    e = _f32(rng.standard_normal(d) * 0.1)
+    for lam in (0.05, 0.2, 1.0):
+        _, _, e_new = oracle.ef_hard_threshold(g, e, 0.1, lam)
+        assert oracle.error_norm_sq(e_new) <= d * lam * lam
+    _, _, a = oracle.ef_hard_threshold(g, e, 0.1, float("inf"))
+    for k in (1, 50, 2500, 4999):
+        _, _, e_new = oracle.ef_topk(g, e, 0.1, k)
+        assert oracle.error_norm_sq(e_new) <= (1.0 - k / d) * oracle.error_norm_sq(a)
+    _, _, e_new = oracle.ef_topk(g, e, 0.1, d)
+    assert oracle.error_norm_sq(e_new) == 0.0
+
+
+# --------------------------------------------------------------------------
 # multi-iteration EF: Lemma 9 (virtual iterate) per worker
 # --------------------------------------------------------------------------
 
