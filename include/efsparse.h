@@ -67,6 +67,9 @@ extern "C" {
 /* A CUDA stream handle; the same type as cudaStream_t (struct CUstream_st*). */
 typedef struct CUstream_st* ef_stream_t;
 
+/* Storage type of a gradient passed through the _ex entry points. */
+typedef enum { EF_GRAD_F32 = 0, EF_GRAD_BF16 = 1 } ef_grad_type;
+
 typedef enum {
   EF_OK = 0,
   EF_ERR_INVALID_ARG = 1, /* host-side argument check failed; nothing launched */
@@ -183,6 +186,40 @@ ef_status ef_topk_layerwise_bf16(const uint16_t* g, float* e, float gamma, uint3
                                  const uint64_t* seg_end, const uint64_t* seg_k, uint64_t d,
                                  uint32_t* idx_out, float* val_out, uint32_t* count_out,
                                  ef_stream_t stream);
+
+/*
+ * ef_hard_threshold_ex, ef_topk_ex, ef_topk_layerwise_ex — the same steps as
+ * ef_hard_threshold[_bf16], ef_topk[_bf16] and ef_topk_layerwise[_bf16]
+ * (identical outputs), with the gradient's storage type as an argument and
+ * one optional output:
+ *
+ *   g_type      EF_GRAD_F32 (g is float[d]) or EF_GRAD_BF16 (uint16_t[d]).
+ *   err_sq_out  [out, optional] one double in device memory, 8-byte aligned,
+ *               or NULL: the squared error norm of this step,
+ *               ||e_{t+1}||^2 = sum_j e'_j^2. Summed over the iterations it
+ *               is the total error of Sec. 1 (the term that alone carries
+ *               the effect of compression in the EF convergence bound).
+ *
+ * Precision (the paper fixes none): squares are accumulated with fmaf in fp32
+ * in groups of at most 256 terms whose partial sums see at most 13 roundings,
+ * and the groups are added in fp64 in a fixed order. The result is within
+ * 1e-6 of the exact sum, relatively (nonnegative terms), plus the squares
+ * below the fp32 range (|e'_j| < 2^-75), which contribute 0; |e'_j| >= 2^64
+ * makes it +inf. It is bit-for-bit reproducible for a given device and input.
+ * The streaming kernels add it as they go; steps whose g or e are not
+ * 16-byte aligned compute it with one more pass over e'. After a step that
+ * failed on the device (a latched timeout) it holds a NaN.
+ */
+ef_status ef_hard_threshold_ex(const void* g, ef_grad_type g_type, float* e, float gamma,
+                               float lambda, uint64_t d, uint32_t* idx_out, float* val_out,
+                               uint32_t* count_out, double* err_sq_out, ef_stream_t stream);
+ef_status ef_topk_ex(const void* g, ef_grad_type g_type, float* e, float gamma, uint64_t k,
+                     uint64_t d, uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                     double* err_sq_out, ef_stream_t stream);
+ef_status ef_topk_layerwise_ex(const void* g, ef_grad_type g_type, float* e, float gamma,
+                               uint32_t n_seg, const uint64_t* seg_end, const uint64_t* seg_k,
+                               uint64_t d, uint32_t* idx_out, float* val_out,
+                               uint32_t* count_out, double* err_sq_out, ef_stream_t stream);
 
 /*
  * sparse_aggregate — decompress and sum n workers' sparse vectors.

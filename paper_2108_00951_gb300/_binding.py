@@ -61,6 +61,10 @@ def load_library(build_if_missing: bool = True):
             "ef_topk_bf16": [vp, vp, f32, u64, u64, vp, vp, vp, vp],
             "ef_topk_layerwise": [vp, vp, f32, u32, vp, vp, u64, vp, vp, vp, vp],
             "ef_topk_layerwise_bf16": [vp, vp, f32, u32, vp, vp, u64, vp, vp, vp, vp],
+            "ef_hard_threshold_ex": [vp, ctypes.c_int, vp, f32, f32, u64, vp, vp, vp, vp, vp],
+            "ef_topk_ex": [vp, ctypes.c_int, vp, f32, u64, u64, vp, vp, vp, vp, vp],
+            "ef_topk_layerwise_ex": [vp, ctypes.c_int, vp, f32, u32, vp, vp, u64, vp, vp, vp, vp,
+                                     vp],
             "sparse_aggregate": [u32, ctypes.POINTER(vp), ctypes.POINTER(vp), vp, u64, vp, vp],
             "sparse_aggregate_apply": [u32, ctypes.POINTER(vp), ctypes.POINTER(vp), vp, u64, f32,
                                        vp, vp, f32, f32, vp],
@@ -116,42 +120,61 @@ def _gradient(g: torch.Tensor):
     raise TypeError("g must be float32 or bfloat16")
 
 
-def ef_hard_threshold(g, e, gamma, lam, idx_out, val_out, count_out, stream=None):
-    """EF accumulate + hard-threshold + compaction (``ef_hard_threshold[_bf16]``).
+def _err(err_sq_out):
+    if err_sq_out is None:
+        return ctypes.c_void_p(0)
+    return _dev(err_sq_out, "err_sq_out", torch.float64, 1)
+
+
+def ef_hard_threshold(g, e, gamma, lam, idx_out, val_out, count_out, stream=None,
+                      err_sq_out=None):
+    """EF accumulate + hard-threshold + compaction (``ef_hard_threshold[_bf16]``;
+    ``ef_hard_threshold_ex`` when ``err_sq_out`` is given).
 
     ``g`` float32 or bfloat16 [d]; ``e`` float32 [d], updated in place;
     ``idx_out`` int32 [>= d] (uint32 bit patterns), ``val_out`` float32 [>= d],
-    ``count_out`` int32 [>= 1].
+    ``count_out`` int32 [>= 1]; ``err_sq_out`` optional float64 [>= 1]:
+    ||e'||^2 of the step.
     """
     lib = load_library()
     bf16 = _gradient(g)
     d = e.numel()
     if g.numel() != d:
         raise ValueError("g and e differ in length")
-    args = (_dev(g, "g", g.dtype), _dev(e, "e", torch.float32), ctypes.c_float(gamma),
+    head = (_dev(g, "g", g.dtype), _dev(e, "e", torch.float32), ctypes.c_float(gamma),
             ctypes.c_float(lam), d, _dev(idx_out, "idx_out", torch.int32, d),
             _dev(val_out, "val_out", torch.float32, d),
-            _dev(count_out, "count_out", torch.int32, 1), _stream(stream))
+            _dev(count_out, "count_out", torch.int32, 1))
+    if err_sq_out is not None:
+        _check(lib.ef_hard_threshold_ex(head[0], int(bf16), *head[1:], _err(err_sq_out),
+                                        _stream(stream)), "ef_hard_threshold_ex")
+        return
     fn = lib.ef_hard_threshold_bf16 if bf16 else lib.ef_hard_threshold
-    _check(fn(*args), "ef_hard_threshold")
+    _check(fn(*head, _stream(stream)), "ef_hard_threshold")
 
 
-def ef_topk(g, e, gamma, k, idx_out, val_out, count_out, stream=None):
-    """EF accumulate + Top-k + compaction (``ef_topk[_bf16]``); exactly k pairs."""
+def ef_topk(g, e, gamma, k, idx_out, val_out, count_out, stream=None, err_sq_out=None):
+    """EF accumulate + Top-k + compaction (``ef_topk[_bf16]``, ``ef_topk_ex`` with
+    ``err_sq_out``); exactly k pairs."""
     lib = load_library()
     bf16 = _gradient(g)
     d = e.numel()
     if g.numel() != d:
         raise ValueError("g and e differ in length")
-    args = (_dev(g, "g", g.dtype), _dev(e, "e", torch.float32), ctypes.c_float(gamma), int(k),
+    head = (_dev(g, "g", g.dtype), _dev(e, "e", torch.float32), ctypes.c_float(gamma), int(k),
             d, _dev(idx_out, "idx_out", torch.int32, k),
             _dev(val_out, "val_out", torch.float32, k),
-            _dev(count_out, "count_out", torch.int32, 1), _stream(stream))
+            _dev(count_out, "count_out", torch.int32, 1))
+    if err_sq_out is not None:
+        _check(lib.ef_topk_ex(head[0], int(bf16), *head[1:], _err(err_sq_out), _stream(stream)),
+               "ef_topk_ex")
+        return
     fn = lib.ef_topk_bf16 if bf16 else lib.ef_topk
-    _check(fn(*args), "ef_topk")
+    _check(fn(*head, _stream(stream)), "ef_topk")
 
 
-def ef_topk_layerwise(g, e, gamma, seg_end, seg_k, idx_out, val_out, count_out, stream=None):
+def ef_topk_layerwise(g, e, gamma, seg_end, seg_k, idx_out, val_out, count_out, stream=None,
+                      err_sq_out=None):
     """EF accumulate + layer-wise Top-k + compaction (``ef_topk_layerwise[_bf16]``).
 
     ``seg_end``/``seg_k``: sequences of n_seg integers (host side): segment s
@@ -168,13 +191,17 @@ def ef_topk_layerwise(g, e, gamma, seg_end, seg_k, idx_out, val_out, count_out, 
     if ends.ndim != 1 or ks.shape != ends.shape:
         raise ValueError("seg_end and seg_k must be 1-D of one length")
     total = int(ks.sum()) if ks.size else 0
-    args = (_dev(g, "g", g.dtype), _dev(e, "e", torch.float32), ctypes.c_float(gamma),
+    head = (_dev(g, "g", g.dtype), _dev(e, "e", torch.float32), ctypes.c_float(gamma),
             ctypes.c_uint32(ends.size), ctypes.c_void_p(ends.ctypes.data),
             ctypes.c_void_p(ks.ctypes.data), d, _dev(idx_out, "idx_out", torch.int32, total),
             _dev(val_out, "val_out", torch.float32, total),
-            _dev(count_out, "count_out", torch.int32, 1), _stream(stream))
+            _dev(count_out, "count_out", torch.int32, 1))
+    if err_sq_out is not None:
+        _check(lib.ef_topk_layerwise_ex(head[0], int(bf16), *head[1:], _err(err_sq_out),
+                                        _stream(stream)), "ef_topk_layerwise_ex")
+        return
     fn = lib.ef_topk_layerwise_bf16 if bf16 else lib.ef_topk_layerwise
-    _check(fn(*args), "ef_topk_layerwise")
+    _check(fn(*head, _stream(stream)), "ef_topk_layerwise")
 
 
 def sparse_aggregate(idx_list, val_list, counts, d, dense_out, stream=None):

@@ -113,14 +113,23 @@ ef_status write_zero_count(uint32_t* count_out, cudaStream_t stream) {
                                                                                  : EF_ERR_CUDA;
 }
 
+ef_status write_err_zero(double* err_out, cudaStream_t stream) {
+  if (!err_out) return EF_OK;
+  return cudaMemsetAsync(err_out, 0, sizeof(double), stream) == cudaSuccess ? EF_OK : EF_ERR_CUDA;
+}
+
 ef_status hard_threshold_entry(const void* g, bool bf16, float* e, float gamma, float lambda,
                                uint64_t d, uint32_t* idx_out, float* val_out,
-                               uint32_t* count_out, cudaStream_t stream) {
+                               uint32_t* count_out, double* err_out, cudaStream_t stream) {
   const size_t gsz = bf16 ? 2 : 4;
   if (!count_out || !aligned(count_out, 4)) return EF_ERR_INVALID_ARG;
   if (!std::isfinite(gamma) || !(lambda >= 0.0f)) return EF_ERR_INVALID_ARG;
   if (d > kMaxD) return EF_ERR_INVALID_ARG;
-  if (d == 0) return write_zero_count(count_out, stream);
+  if (err_out && !aligned(err_out, 8)) return EF_ERR_INVALID_ARG;
+  if (d == 0) {
+    const ef_status z = write_zero_count(count_out, stream);
+    return z != EF_OK ? z : write_err_zero(err_out, stream);
+  }
   if (!g || !e || !idx_out || !val_out) return EF_ERR_INVALID_ARG;
   if (!aligned(g, gsz) || !aligned(e, 4) || !aligned(idx_out, 4) || !aligned(val_out, 4))
     return EF_ERR_INVALID_ARG;
@@ -143,19 +152,27 @@ ef_status hard_threshold_entry(const void* g, bool bf16, float* e, float gamma, 
   st = acquire_workspace(stream, tiles_for(d), 0, 0,
                          static_cast<size_t>(tiles_for(d)) * kTileElems, &ws);
   if (st != EF_OK) return st;
+  if (err_out && (overlaps(err_out, 8, e, nb) || overlaps(err_out, 8, g, d * gsz) ||
+                  overlaps(err_out, 8, idx_out, nb) || overlaps(err_out, 8, val_out, nb) ||
+                  overlaps(err_out, 8, count_out, 4)))
+    return EF_ERR_INVALID_ARG;
   return finish_launch(launch_hard_threshold(g, bf16, e, gamma, lambda, static_cast<uint32_t>(d),
-                                             idx_out, val_out, count_out, *ws, info),
+                                             idx_out, val_out, count_out, err_out, *ws, info),
                        ws);
 }
 
 ef_status topk_entry(const void* g, bool bf16, float* e, float gamma, uint64_t k, uint64_t d,
-                     uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                     uint32_t* idx_out, float* val_out, uint32_t* count_out, double* err_out,
                      cudaStream_t stream) {
   const size_t gsz = bf16 ? 2 : 4;
   if (!count_out || !aligned(count_out, 4)) return EF_ERR_INVALID_ARG;
   if (!std::isfinite(gamma)) return EF_ERR_INVALID_ARG;
   if (d > kMaxD || k > d) return EF_ERR_INVALID_ARG;
-  if (d == 0) return write_zero_count(count_out, stream);
+  if (err_out && !aligned(err_out, 8)) return EF_ERR_INVALID_ARG;
+  if (d == 0) {
+    const ef_status z = write_zero_count(count_out, stream);
+    return z != EF_OK ? z : write_err_zero(err_out, stream);
+  }
   if (!g || !e || (k > 0 && (!idx_out || !val_out))) return EF_ERR_INVALID_ARG;
   if (!aligned(g, gsz) || !aligned(e, 4) || !aligned(idx_out, 4) || !aligned(val_out, 4))
     return EF_ERR_INVALID_ARG;
@@ -178,16 +195,20 @@ ef_status topk_entry(const void* g, bool bf16, float* e, float gamma, uint64_t k
   st = acquire_workspace(stream, tiles_for(d), topk_candidate_capacity(d), 0,
                          static_cast<size_t>(tiles_for(d)) * kTileElems, &ws);
   if (st != EF_OK) return st;
+  if (err_out && (overlaps(err_out, 8, e, nb) || overlaps(err_out, 8, g, d * gsz) ||
+                  overlaps(err_out, 8, idx_out, kb) || overlaps(err_out, 8, val_out, kb) ||
+                  overlaps(err_out, 8, count_out, 4)))
+    return EF_ERR_INVALID_ARG;
   return finish_launch(launch_topk(g, bf16, e, gamma, static_cast<uint32_t>(k),
-                                   static_cast<uint32_t>(d), idx_out, val_out, count_out, *ws,
-                                   info),
+                                   static_cast<uint32_t>(d), idx_out, val_out, count_out, err_out,
+                                   *ws, info),
                        ws);
 }
 
 ef_status topk_layerwise_entry(const void* g, bool bf16, float* e, float gamma, uint32_t n_seg,
                                const uint64_t* seg_end, const uint64_t* seg_k, uint64_t d,
                                uint32_t* idx_out, float* val_out, uint32_t* count_out,
-                               cudaStream_t stream) {
+                               double* err_out, cudaStream_t stream) {
   const size_t gsz = bf16 ? 2 : 4;
   if (!count_out || !aligned(count_out, 4)) return EF_ERR_INVALID_ARG;
   if (!std::isfinite(gamma) || d > kMaxD) return EF_ERR_INVALID_ARG;
@@ -200,7 +221,11 @@ ef_status topk_layerwise_entry(const void* g, bool bf16, float* e, float gamma, 
     lo = seg_end[s];
   }
   if (lo != d) return EF_ERR_INVALID_ARG;
-  if (d == 0) return write_zero_count(count_out, stream);
+  if (err_out && !aligned(err_out, 8)) return EF_ERR_INVALID_ARG;
+  if (d == 0) {
+    const ef_status z = write_zero_count(count_out, stream);
+    return z != EF_OK ? z : write_err_zero(err_out, stream);
+  }
   if (!g || !e || (total_k > 0 && (!idx_out || !val_out))) return EF_ERR_INVALID_ARG;
   if (!aligned(g, gsz) || !aligned(e, 4) || !aligned(idx_out, 4) || !aligned(val_out, 4))
     return EF_ERR_INVALID_ARG;
@@ -223,11 +248,15 @@ ef_status topk_layerwise_entry(const void* g, bool bf16, float* e, float gamma, 
   st = acquire_workspace(stream, tiles_for(d), topk_candidate_capacity(d), 0,
                          static_cast<size_t>(tiles_for(d)) * kTileElems, &ws);
   if (st != EF_OK) return st;
+  if (err_out && (overlaps(err_out, 8, e, nb) || overlaps(err_out, 8, g, d * gsz) ||
+                  overlaps(err_out, 8, idx_out, kb) || overlaps(err_out, 8, val_out, kb) ||
+                  overlaps(err_out, 8, count_out, 4)))
+    return EF_ERR_INVALID_ARG;
   const cudaError_t perr = lw_prepare(*ws, seg_end, seg_k, n_seg, d, info);
   if (perr == cudaErrorMemoryAllocation) return EF_ERR_NO_MEMORY;
   if (perr != cudaSuccess) return EF_ERR_CUDA;
   return finish_launch(launch_topk_layerwise(g, bf16, e, gamma, static_cast<uint32_t>(d),
-                                             idx_out, val_out, count_out, *ws, info),
+                                             idx_out, val_out, count_out, err_out, *ws, info),
                        ws);
 }
 
@@ -264,26 +293,26 @@ ef_status ef_hard_threshold(const float* g, float* e, float gamma, float lambda,
                             uint32_t* idx_out, float* val_out, uint32_t* count_out,
                             ef_stream_t stream) {
   return efs::hard_threshold_entry(g, false, e, gamma, lambda, d, idx_out, val_out, count_out,
-                                   reinterpret_cast<cudaStream_t>(stream));
+                                   nullptr, reinterpret_cast<cudaStream_t>(stream));
 }
 
 ef_status ef_hard_threshold_bf16(const uint16_t* g, float* e, float gamma, float lambda,
                                  uint64_t d, uint32_t* idx_out, float* val_out,
                                  uint32_t* count_out, ef_stream_t stream) {
   return efs::hard_threshold_entry(g, true, e, gamma, lambda, d, idx_out, val_out, count_out,
-                                   reinterpret_cast<cudaStream_t>(stream));
+                                   nullptr, reinterpret_cast<cudaStream_t>(stream));
 }
 
 ef_status ef_topk(const float* g, float* e, float gamma, uint64_t k, uint64_t d,
                   uint32_t* idx_out, float* val_out, uint32_t* count_out, ef_stream_t stream) {
-  return efs::topk_entry(g, false, e, gamma, k, d, idx_out, val_out, count_out,
+  return efs::topk_entry(g, false, e, gamma, k, d, idx_out, val_out, count_out, nullptr,
                          reinterpret_cast<cudaStream_t>(stream));
 }
 
 ef_status ef_topk_bf16(const uint16_t* g, float* e, float gamma, uint64_t k, uint64_t d,
                        uint32_t* idx_out, float* val_out, uint32_t* count_out,
                        ef_stream_t stream) {
-  return efs::topk_entry(g, true, e, gamma, k, d, idx_out, val_out, count_out,
+  return efs::topk_entry(g, true, e, gamma, k, d, idx_out, val_out, count_out, nullptr,
                          reinterpret_cast<cudaStream_t>(stream));
 }
 
@@ -292,7 +321,8 @@ ef_status ef_topk_layerwise(const float* g, float* e, float gamma, uint32_t n_se
                             uint32_t* idx_out, float* val_out, uint32_t* count_out,
                             ef_stream_t stream) {
   return efs::topk_layerwise_entry(g, false, e, gamma, n_seg, seg_end, seg_k, d, idx_out,
-                                   val_out, count_out, reinterpret_cast<cudaStream_t>(stream));
+                                   val_out, count_out, nullptr,
+                                   reinterpret_cast<cudaStream_t>(stream));
 }
 
 ef_status ef_topk_layerwise_bf16(const uint16_t* g, float* e, float gamma, uint32_t n_seg,
@@ -300,7 +330,35 @@ ef_status ef_topk_layerwise_bf16(const uint16_t* g, float* e, float gamma, uint3
                                  uint32_t* idx_out, float* val_out, uint32_t* count_out,
                                  ef_stream_t stream) {
   return efs::topk_layerwise_entry(g, true, e, gamma, n_seg, seg_end, seg_k, d, idx_out,
-                                   val_out, count_out, reinterpret_cast<cudaStream_t>(stream));
+                                   val_out, count_out, nullptr,
+                                   reinterpret_cast<cudaStream_t>(stream));
+}
+
+ef_status ef_hard_threshold_ex(const void* g, ef_grad_type g_type, float* e, float gamma,
+                               float lambda, uint64_t d, uint32_t* idx_out, float* val_out,
+                               uint32_t* count_out, double* err_sq_out, ef_stream_t stream) {
+  if (g_type != EF_GRAD_F32 && g_type != EF_GRAD_BF16) return EF_ERR_INVALID_ARG;
+  return efs::hard_threshold_entry(g, g_type == EF_GRAD_BF16, e, gamma, lambda, d, idx_out,
+                                   val_out, count_out, err_sq_out,
+                                   reinterpret_cast<cudaStream_t>(stream));
+}
+
+ef_status ef_topk_ex(const void* g, ef_grad_type g_type, float* e, float gamma, uint64_t k,
+                     uint64_t d, uint32_t* idx_out, float* val_out, uint32_t* count_out,
+                     double* err_sq_out, ef_stream_t stream) {
+  if (g_type != EF_GRAD_F32 && g_type != EF_GRAD_BF16) return EF_ERR_INVALID_ARG;
+  return efs::topk_entry(g, g_type == EF_GRAD_BF16, e, gamma, k, d, idx_out, val_out, count_out,
+                         err_sq_out, reinterpret_cast<cudaStream_t>(stream));
+}
+
+ef_status ef_topk_layerwise_ex(const void* g, ef_grad_type g_type, float* e, float gamma,
+                               uint32_t n_seg, const uint64_t* seg_end, const uint64_t* seg_k,
+                               uint64_t d, uint32_t* idx_out, float* val_out,
+                               uint32_t* count_out, double* err_sq_out, ef_stream_t stream) {
+  if (g_type != EF_GRAD_F32 && g_type != EF_GRAD_BF16) return EF_ERR_INVALID_ARG;
+  return efs::topk_layerwise_entry(g, g_type == EF_GRAD_BF16, e, gamma, n_seg, seg_end, seg_k,
+                                   d, idx_out, val_out, count_out, err_sq_out,
+                                   reinterpret_cast<cudaStream_t>(stream));
 }
 
 ef_status sparse_aggregate(uint32_t n, const uint32_t* const* idx, const float* const* val,

@@ -186,6 +186,49 @@ __device__ __forceinline__ uint32_t lookback_exclusive(const ScanCtx& ctx, uint3
   }
 }
 
+// ---------------------------------------------------------- error norm
+// Squared error norm ||e'||^2 = sum_j e'_j^2, deterministic for a given
+// launch shape: squares are accumulated with fmaf in fp32 in fixed groups of
+// at most 8 terms (a warp tree of 32 such groups in the streaming kernels),
+// and the groups are added in fp64 in a fixed order. Every fp32 partial sum
+// carries at most 13 roundings of nonnegative terms, so the result is within
+// 13 * 2^-24 (< 1e-6) of the exact sum, relatively, plus the squares below
+// the fp32 range (|e'_j| < 2^-75) that contribute 0. |e'_j| >= 2^64 squares
+// to +inf.
+// Written as ||e'||^2 when a failed step has none.
+__device__ __forceinline__ double err_invalid() { return __longlong_as_double(0x7ff8000000000000ll); }
+
+struct ErrAcc {
+  double total = 0.0;
+  float part = 0.0f;
+  int terms = 0;
+  __device__ __forceinline__ void add(float x) {
+    part = __fmaf_rn(x, x, part);
+    if (++terms == 8) flush();
+  }
+  __device__ __forceinline__ void flush() {
+    total += static_cast<double>(part);
+    part = 0.0f;
+    terms = 0;
+  }
+};
+
+// Sum of one double per thread over the CTA in a fixed order (warp trees,
+// then the warps in order); the result is valid in thread 0. s_d holds
+// blockDim.x / 32 doubles.
+__device__ __forceinline__ double block_sum_fixed(double v, double* s_d) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  __syncthreads();  // an earlier use of s_d is complete
+  if (lane == 0) s_d[warp] = v;
+  __syncthreads();
+  double t = 0.0;
+  if (threadIdx.x == 0)
+    for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) t += s_d[w];
+  return t;
+}
+
 // Bounded grid-wide barrier for a cooperative launch (all CTAs co-resident).
 // Returns false, latching kDevErrTimeout, if the wait ran out.
 // Programmatic dependent launch: wait until the grids this one depends on

@@ -18,12 +18,15 @@ constexpr size_t kOffBarArrive = 16;    // uint32: grid-barrier arrivals (zero a
 constexpr size_t kOffTkLowerBound = 56; // uint64: sampled lower bound of the candidates' keys
 constexpr size_t kOffTkMode = 64;       // uint32: 0 candidates, 1 full array
 constexpr size_t kOffTkListCount = 72;  // uint32: candidates emitted by the streaming pass
+constexpr size_t kOffErrArrive = 80;    // uint32: arrivals of the e' norm pass (zero after it)
+constexpr size_t kOffStreamErr = 88;    // double: the streaming pass's share of ||e'||^2
 // Per-call Top-k state that must start at zero, in two blocks used by
 // alternate calls on a workspace: a call's candidate stream zeroes the
 // other block (the previous call's, complete by then) for the next call.
 constexpr size_t kOffTkState = 256;
 constexpr size_t kStStreamArrive = 0;   // uint32: arrivals at the candidate stream's barrier
 constexpr size_t kStListFlags = 4;      // uint32: that pass's latched bits (overflow, timeout)
+constexpr size_t kStErrArrive = 8;      // uint32: select CTAs that published their ||e'||^2 share
 constexpr size_t kStSelect = 16;        // uint32[4]: short-list threshold published by CTA 0
 constexpr size_t kStCandCount = 32;     // uint32[6]: refine-level candidate counts
 constexpr size_t kStHist = 256;         // uint32[6][2048]: refine-level histograms
@@ -46,7 +49,12 @@ constexpr uint32_t kLwNone = 0, kLwWhole = 1, kLwSampled = 2, kLwAll = 3;
 constexpr uint32_t kLwSmemElems = 48u * 1024u;  // values one select CTA holds in shared memory
 constexpr uint32_t kLwWholeMax = 4096;          // segments at most this long: selected from e
 constexpr uint32_t kLwSampleGroups = 4096;      // groups of 4 coordinates sampled per segment
-constexpr uint32_t kLwNoBound = 0xffffffffu;    // candidate bound that admits nothing
+// Candidate bounds that admit nothing: the residual of the segment's
+// coordinates is then a, final in the streaming pass (kLwNoBound: segments
+// that send nothing), or decided by the select (kLwDeferred: short segments,
+// segments that send everything, sampled segments whose sample found no bound).
+constexpr uint32_t kLwNoBound = 0xffffffffu;
+constexpr uint32_t kLwDeferred = 0xfffffffeu;
 constexpr uint32_t kLwTileUniform = 0x80000000u;  // tile_info: the tile lies in one segment
 
 struct LwSeg {      // one segment (device and host layout, 32 bytes)
@@ -118,7 +126,8 @@ struct Workspace {
   size_t off_chunks() const {
     return align(off_counts() + sizeof(uint32_t) * kCountsPerTile * status_tiles);
   }
-  size_t off_stage() const { return align(off_chunks() + sizeof(uint64_t) * kMaxChunks); }
+  size_t off_errparts() const { return align(off_chunks() + sizeof(uint64_t) * kMaxChunks); }
+  size_t off_stage() const { return align(off_errparts() + sizeof(double) * kMaxChunks); }
   size_t total_bytes() const { return align(off_stage() + 8 * stage_cap); }
 
   uint64_t* status() const { return reinterpret_cast<uint64_t*>(base + off_status()); }
@@ -128,6 +137,8 @@ struct Workspace {
   uint32_t* offsets() const { return reinterpret_cast<uint32_t*>(base + off_offsets()); }
   uint32_t* counts() const { return reinterpret_cast<uint32_t*>(base + off_counts()); }
   uint64_t* chunks() const { return reinterpret_cast<uint64_t*>(base + off_chunks()); }
+  double* errparts() const { return reinterpret_cast<double*>(base + off_errparts()); }
+  double* stream_err() const { return reinterpret_cast<double*>(base + kOffStreamErr); }
   uint32_t* stage_idx() const { return reinterpret_cast<uint32_t*>(base + off_stage()); }
   float* stage_val() const {
     return reinterpret_cast<float*>(base + off_stage() + sizeof(uint32_t) * stage_cap);
@@ -163,6 +174,11 @@ void topk_layerwise_init_device(DeviceInfo& info);
 // their shared-memory ring on the current device and records occupancy).
 void ht_init_device(DeviceInfo& info);
 
+// ||e'||^2 of e[0, d) after a step, by one plain pass (the paths that do
+// not stream through stream_compact.cuh); written to *err_out.
+cudaError_t launch_error_norm(const float* e, uint32_t d, double* err_out, Workspace& ws,
+                              const DeviceInfo& dev);
+
 // Launch bookkeeping.
 void count_launch();
 uint64_t wait_limit_ns();
@@ -170,23 +186,25 @@ int64_t withheld_tile();
 ScanCtx next_scan_ctx(Workspace& ws, uint32_t num_tiles);
 
 // ---- launchers (return the launch's cudaError_t) ----
+// err_out (optional, device): ||e'||^2 of the step.
 cudaError_t launch_hard_threshold(const void* g, bool g_bf16, float* e, float gamma,
                                   float lambda, uint32_t d, uint32_t* idx_out, float* val_out,
-                                  uint32_t* count_out, Workspace& ws, const DeviceInfo& dev);
+                                  uint32_t* count_out, double* err_out, Workspace& ws,
+                                  const DeviceInfo& dev);
 cudaError_t launch_hard_threshold_lookback(const float* g, float* e, float gamma, float lambda,
                                            uint32_t d, uint32_t* idx_out, float* val_out,
                                            uint32_t* count_out, const ScanCtx& ctx,
                                            cudaStream_t stream);
 cudaError_t launch_topk(const void* g, bool g_bf16, float* e, float gamma, uint32_t k,
                         uint32_t d, uint32_t* idx_out, float* val_out, uint32_t* count_out,
-                        Workspace& ws, const DeviceInfo& dev);
+                        double* err_out, Workspace& ws, const DeviceInfo& dev);
 // Layer-wise Top-k: lw_prepare builds and uploads the plan of a segment
 // table (a no-op when the workspace already holds that table's plan).
 cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* seg_k,
                        uint32_t n_seg, uint64_t d, const DeviceInfo& dev);
 cudaError_t launch_topk_layerwise(const void* g, bool g_bf16, float* e, float gamma, uint32_t d,
                                   uint32_t* idx_out, float* val_out, uint32_t* count_out,
-                                  Workspace& ws, const DeviceInfo& dev);
+                                  double* err_out, Workspace& ws, const DeviceInfo& dev);
 cudaError_t launch_aggregate(uint32_t n, const uint32_t* const* idx, const float* const* val,
                              const uint32_t* counts, uint32_t d, float* dense_out,
                              Workspace& ws);

@@ -29,6 +29,14 @@
 // needed. It then scans its segments' counts in shared memory, and each warp
 // copies whole segments from staging to their final, ascending positions.
 //
+// Error norm (when sa.err_out is set): a coordinate that is neither selected
+// nor deferred (selection bits 4..7 of an op mark coordinates whose residual
+// a later kernel decides) keeps a as its residual, so a^2 is its share of
+// ||e'||^2. Each warp sums the squares of a tile segment in fp32 (fmaf per
+// lane over its 8 coordinates, then a warp tree) and adds that in fp64; the
+// CTA's share is published with its chunk total, and the last CTA adds the
+// shares in CTA order.
+//
 // Traffic beyond the step itself: 16 bytes per selected pair (staging write
 // and read) plus 4 bytes per segment. Every wait (stage arrival, stage
 // release, an earlier chunk's total) is bounded and latches kDevErrTimeout;
@@ -87,6 +95,9 @@ struct StreamArgs {
   uint64_t* chunk_sums;  // [gridDim.x] (epoch << 32) | chunk total
   uint32_t* tile_base;   // optional [num_tiles + 1]: output position of each tile's first
                          // pair, and the total (untruncated), or null
+  double* err_out;       // optional: sum of a^2 over the coordinates whose residual is final
+                         // here (not selected, not deferred), or null
+  double* err_parts;     // [gridDim.x] the CTAs' shares of it
 };
 
 // A segment's count (<= 256: 9 bits) and its warp's earlier pairs in the
@@ -118,6 +129,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   __shared__ __align__(8) uint64_t s_full[kStages];
   __shared__ __align__(8) uint64_t s_empty[kStages];
   __shared__ uint32_t s_scratch[kStreamThreads / 32];
+  __shared__ double s_err[kSWarps];
   __shared__ uint32_t s_sample_hist[Op::kPrepass ? Op::kSampleBins : 1];
   using L = StreamLayout<Op, kStages>;
   uint32_t* s_pair_idx = reinterpret_cast<uint32_t*>(smem + L::kRing);
@@ -147,6 +159,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   bool failed = false;    // a wait of this thread ran out
   bool withheld = false;  // test hook: this CTA owns the withheld tile
   uint32_t chunk_total = 0;  // compute warps: pairs selected by this warp
+  double warp_err = 0.0;     // compute warps: their share of ||e'||^2
   uint64_t policy = 0;       // producer lane
   auto fill = [&](uint32_t r) {  // producer lane
     const int s = static_cast<int>(r % kStages);
@@ -225,6 +238,17 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&s_empty[s]);  // this warp is done with the stage
+      if (sa.err_out) {
+        float sq = 0.0f;
+#pragma unroll
+        for (int v = 0; v < kSUnits; ++v)
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (!((sel[v] >> j) & 0x11u)) sq = __fmaf_rn(a[v][j], a[v][j], sq);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+        if (lane == 0) warp_err += static_cast<double>(sq);
+      }
       uint32_t off[kSUnits];
       uint32_t total = 0;
 #pragma unroll
@@ -278,10 +302,17 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   // the chunk's total (each compute warp contributes its own)
   uint32_t mine = lane == 0 && warp < kSWarps ? chunk_total : 0u;
   if (lane == 0) s_scratch[warp] = mine;
+  if (lane == 0 && warp < kSWarps) s_err[warp] = warp_err;
   __syncthreads();
   if (threadIdx.x == 0) {
     uint32_t sum = 0;
     for (int w = 0; w < kSWarps; ++w) sum += s_scratch[w];
+    if (sa.err_out) {  // the CTA's share of ||e'||^2, visible before the chunk total
+      double err = 0.0;
+      for (int w = 0; w < kSWarps; ++w) err += s_err[w];
+      sa.err_parts[c] = err;
+      __threadfence();
+    }
     st_relaxed_u64(sa.chunk_sums + c, (static_cast<uint64_t>(ctx.epoch) << 32) | sum);
   }
   // sum of the earlier chunks' totals, waiting (bounded) for missing ones
@@ -307,6 +338,16 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
       if (all_present) {
         for (int w = 0; w < kStreamThreads / 32; ++w) base += s_scratch[w];
         done = true;
+        if (sa.err_out && c == G - 1) {
+          // every earlier CTA's share was written before its chunk total
+          __threadfence();
+          __syncthreads();
+          if (threadIdx.x == 0) {
+            double err = 0.0;
+            for (uint32_t q = 0; q < G; ++q) err += __ldcg(sa.err_parts + q);
+            *sa.err_out = err;
+          }
+        }
       } else {
         const uint64_t now = global_timer_ns();
         const bool out_of_time = ++it > (1u << 26) || now - t0 > ctx.wait_limit_ns;

@@ -72,6 +72,9 @@ struct TopkArgs {
   uint64_t* chunk_sums;
   uint32_t epoch;        // tags the finalize kernel's chunk totals
   uint64_t wait_limit_ns;
+  double* err_out;       // optional ||e'||^2 of the step
+  const double* stream_err;  // the streaming pass's share (coordinates below the bound)
+  double* err_parts;     // [gridDim.x] the select CTAs' shares
 };
 
 // ------------------------------------------------------------- 1 stream
@@ -686,6 +689,8 @@ __global__ void __launch_bounds__(kSelThreads, 1)
     if (blockIdx.x == 0 && threadIdx.x == 0) {
       if (si.failed) atomicOr(args.error, kDevErrTimeout);
       *count_out = 0;
+      // nothing sent: every residual is a, all counted by the streaming pass
+      if (args.err_out) *args.err_out = si.failed ? err_invalid() : *args.stream_err;
     }
     return;
   }
@@ -706,6 +711,18 @@ __global__ void __launch_bounds__(kSelThreads, 1)
         __threadfence();
         st_release_u32(args.sel, found ? 1u : 2u);
       }
+      if (args.err_out) {
+        // the candidates not sent keep a: their squares, plus the streaming
+        // pass's share (every coordinate below the bound)
+        ErrAcc acc;
+        if (found)
+          for (uint32_t i = threadIdx.x; i < si.n; i += kSelThreads)
+            if (!selected(sel, s_mag[i], i)) acc.add(__uint_as_float(s_mag[i]));
+        acc.flush();
+        __shared__ double s_d[kSelThreads / 32];
+        const double rem = block_sum_fixed(acc.total, s_d);
+        if (threadIdx.x == 0) *args.err_out = found ? *args.stream_err + rem : err_invalid();
+      }
     }
     small_emit(args, e, si.n, k, Gs, idx_out, val_out, count_out, s_w);
     return;
@@ -713,7 +730,10 @@ __global__ void __launch_bounds__(kSelThreads, 1)
   bool ok = true;
   const uint64_t thr = radix_threshold_grid(args, e, si, k, s_hist, s_w, ok);
   if (!ok) {
-    if (blockIdx.x == 0 && threadIdx.x == 0) *count_out = 0;
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+      *count_out = 0;
+      if (args.err_out) *args.err_out = err_invalid();
+    }
     return;
   }
   // ordered compaction across the grid: chunk counts, then positions
@@ -721,6 +741,7 @@ __global__ void __launch_bounds__(kSelThreads, 1)
   const uint32_t lo = static_cast<uint32_t>(static_cast<uint64_t>(c) * si.n / G);
   const uint32_t hi = static_cast<uint32_t>(static_cast<uint64_t>(c + 1) * si.n / G);
   uint32_t mine = 0;
+  ErrAcc acc;  // squares of the source positions not sent (their residual is a)
   for (uint32_t i0 = lo + threadIdx.x; i0 < hi; i0 += 4 * kSelThreads) {
     uint64_t key[4];
 #pragma unroll
@@ -729,10 +750,24 @@ __global__ void __launch_bounds__(kSelThreads, 1)
       key[j] = i < hi ? source_key(args, e, si.mode, i) : 0ull;
     }
 #pragma unroll
-    for (int j = 0; j < 4; ++j) mine += (i0 + j * kSelThreads < hi && key[j] >= thr) ? 1u : 0u;
+    for (int j = 0; j < 4; ++j) {
+      const bool in = i0 + j * kSelThreads < hi;
+      mine += (in && key[j] >= thr) ? 1u : 0u;
+      if (args.err_out && in && key[j] < thr)
+        acc.add(__uint_as_float(static_cast<uint32_t>(key[j] >> 32)));
+    }
   }
   uint32_t total;
   block_exclusive<kSelThreads>(mine, total, s_w);
+  if (args.err_out) {
+    acc.flush();
+    __shared__ double s_d[kSelThreads / 32];
+    const double share = block_sum_fixed(acc.total, s_d);
+    if (threadIdx.x == 0) {
+      args.err_parts[c] = share;  // visible before the chunk total
+      __threadfence();
+    }
+  }
   if (threadIdx.x == 0)
     st_relaxed_u64(args.chunk_sums + c, (static_cast<uint64_t>(args.epoch) << 32) | total);
   uint32_t base = 0;
@@ -754,6 +789,18 @@ __global__ void __launch_bounds__(kSelThreads, 1)
       block_exclusive<kSelThreads>(part, sum, s_w);
       if (all_present) {
         base = sum;
+        if (args.err_out && c == G - 1) {
+          // every earlier CTA's share was written before its chunk total;
+          // with candidates, the coordinates below the bound are the
+          // streaming pass's (a full-array source covers every coordinate)
+          __threadfence();
+          __syncthreads();
+          if (threadIdx.x == 0) {
+            double err = si.mode == 0 ? *args.stream_err : 0.0;
+            for (uint32_t q = 0; q < G; ++q) err += __ldcg(args.err_parts + q);
+            *args.err_out = err;
+          }
+        }
         break;
       }
       const bool out_of_time = ++it > (1u << 26) || global_timer_ns() - t0 > args.wait_limit_ns;
@@ -788,8 +835,8 @@ int tk_stream_blocks_per_sm() {
 
 template <typename GT>
 cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_t d,
-                         uint32_t* idx_out, float* val_out, uint32_t* count_out, Workspace& ws,
-                         const DeviceInfo& dev) {
+                         uint32_t* idx_out, float* val_out, uint32_t* count_out, double* err_out,
+                         Workspace& ws, const DeviceInfo& dev) {
   const uint32_t tiles = tiles_for(d);
   cudaError_t err = cudaSuccess;
   // this call's zeroed state block, and the other one, cleared for the next call
@@ -815,6 +862,9 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
   args.error = ws.u32(kOffError);
   args.chunk_sums = ws.chunks();
   args.wait_limit_ns = wait_limit_ns();
+  args.err_out = err_out;
+  args.stream_err = ws.stream_err();
+  args.err_parts = ws.errparts();
 
   // 1 stream (sample pre-pass + candidates). The bulk copies need 16-byte
   // aligned g and e; otherwise a plain pass writes a and the selection runs in
@@ -831,7 +881,8 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
     if (slots > kMaxChunks) slots = kMaxChunks;
     const uint32_t grid = tiles < slots ? tiles : slots;
     uint32_t cap = ws.cand_cap;
-    StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks()};
+    StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks(), nullptr,
+                  err_out ? ws.stream_err() : nullptr, ws.errparts()};
     void* params[] = {&op, &d, &args.list_idx, &args.list_val, &args.list_count, &cap, &ctx, &sa};
     err = cudaLaunchCooperativeKernel(
         reinterpret_cast<const void*>(&stream_compact_kernel<TopkCandOp<GT>, kTkStages>),
@@ -847,7 +898,8 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
     count_launch();
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
   }
-  // 2 select
+  // 2 select (inputs the streaming pass could not take: the norm by a plain pass after it)
+  if (!streamable) args.err_out = nullptr;
   args.epoch = next_scan_ctx(ws, 1).epoch;
   void* params[] = {(void*)&e, (void*)&d, (void*)&k, (void*)&idx_out, (void*)&val_out,
                     (void*)&count_out, (void*)&args};
@@ -856,6 +908,7 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
   err = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(&topk_select_kernel),
                                     dim3(grid), dim3(kSelThreads), params, kSelSmem, ws.stream);
   count_launch();
+  if (err == cudaSuccess && err_out && !streamable) err = launch_error_norm(e, d, err_out, ws, dev);
   return err;
 }
 
@@ -882,12 +935,12 @@ uint32_t topk_candidate_capacity(uint64_t d) {
 
 cudaError_t launch_topk(const void* g, bool g_bf16, float* e, float gamma, uint32_t k,
                         uint32_t d, uint32_t* idx_out, float* val_out, uint32_t* count_out,
-                        Workspace& ws, const DeviceInfo& dev) {
+                        double* err_out, Workspace& ws, const DeviceInfo& dev) {
   if (g_bf16)
     return launch_typed(static_cast<const uint16_t*>(g), e, gamma, k, d, idx_out, val_out,
-                        count_out, ws, dev);
+                        count_out, err_out, ws, dev);
   return launch_typed(static_cast<const float*>(g), e, gamma, k, d, idx_out, val_out, count_out,
-                      ws, dev);
+                      err_out, ws, dev);
 }
 
 }  // namespace efs

@@ -142,7 +142,7 @@ __global__ void __launch_bounds__(kSampleThreads, 1)
   __syncthreads();
   griddep_wait();  // the previous kernel (which may read the bounds) is complete
   if (tid == 0) {
-    uint32_t bound = kLwNoBound;
+    uint32_t bound = kLwDeferred;
     // expected candidates (the sampled mass scaled to d_s) at most half the
     // list's capacity, else the segment is selected from e itself
     if (s_bin != 0xffffffffu &&
@@ -163,7 +163,7 @@ struct LwCandOp {
   float gamma;
   uint32_t d;
   const uint32_t* seg_end;    // [n_seg] exclusive segment ends
-  const uint32_t* mbound;     // [n_seg] candidate bounds (kLwNoBound: none)
+  const uint32_t* mbound;     // [n_seg] candidate bounds (kLwNoBound, kLwDeferred: none)
   const uint32_t* tile_info;  // [tiles] first segment of the tile | kLwTileUniform
   uint32_t* other_state;      // the other Top-k state block: zeroed here for the next call
   static constexpr uint32_t kGBytes = kTileElems * sizeof(GT);
@@ -185,14 +185,16 @@ struct LwCandOp {
   }
 
   // selection bits of the lane's coordinates from their segments' bounds
+  // (bit j: candidate; bit 4 + j: residual decided by the select)
   __device__ __forceinline__ void select(uint32_t t, uint64_t first, const float (&a)[kSUnits][4],
                                          uint32_t (&sel)[kSUnits]) const {
     const uint32_t info = __ldg(tile_info + t);
     if (info & kLwTileUniform) {
       const uint32_t b = __ldg(mbound + (info & ~kLwTileUniform));
+      const uint32_t defer = b == kLwDeferred ? 0xf0u : 0u;
 #pragma unroll
       for (int v = 0; v < kSUnits; ++v) {
-        sel[v] = 0;
+        sel[v] = defer;
 #pragma unroll
         for (int j = 0; j < 4; ++j) sel[v] |= (mag_bits(a[v][j]) >= b ? 1u : 0u) << j;
       }
@@ -206,7 +208,9 @@ struct LwCandOp {
           const uint64_t i = first + v * 128 + j;
           if (i < d) {
             while (__ldg(seg_end + s) <= i) ++s;
-            sel[v] |= (mag_bits(a[v][j]) >= __ldg(mbound + s) ? 1u : 0u) << j;
+            const uint32_t b = __ldg(mbound + s);
+            sel[v] |= (mag_bits(a[v][j]) >= b ? 1u : 0u) << j;
+            sel[v] |= (b == kLwDeferred ? 1u : 0u) << (4 + j);
           }
         }
       }
@@ -260,7 +264,7 @@ struct LwCandOp {
     for (int v = 0; v < kSUnits; ++v)
 #pragma unroll
       for (int j = 0; j < 4; ++j)
-        if (first + v * 128 + j >= d) sel[v] &= ~(1u << j);
+        if (first + v * 128 + j >= d) sel[v] &= ~(0x11u << j);
   }
 };
 
@@ -292,6 +296,10 @@ struct LwArgs {
   uint64_t wait_limit_ns;
   uint32_t tiles, cap, use_list;
   uint32_t total_k;
+  double* err_out;            // optional ||e'||^2 of the step
+  const double* stream_err;   // the streaming pass's share (final residuals)
+  double* err_parts;          // [gridDim.x] the select CTAs' shares
+  uint32_t* err_arrive;       // select CTAs that published their share (zero at the start)
 };
 
 // The source a segment is selected from: its candidates [c0, c1) of the
@@ -306,7 +314,7 @@ struct Source {
 };
 __device__ Source segment_source(const LwArgs& a, const LwSeg& s, uint32_t si) {
   Source src{false, 0, s.hi - s.lo};
-  if (!a.use_list || __ldcg(a.mbound + si) == kLwNoBound) return src;
+  if (!a.use_list || __ldcg(a.mbound + si) >= kLwDeferred) return src;
   const uint32_t tl = s.lo / kTileElems, th = s.hi / kTileElems;  // tl < tiles, th <= tiles
   const uint32_t p0 = __ldcg(a.tile_base + tl), p1 = __ldcg(a.tile_base + tl + 1);
   const uint32_t q0 = __ldcg(a.tile_base + th);
@@ -405,7 +413,8 @@ struct SrcGlobal {  // values in global memory; coordinates lo + i, or from a li
 };
 
 // Ordered write-out of the selected source positions of [s0, s1), in two
-// passes. Warp w owns the contiguous part [s0 + w (s1-s0)/32, ...): it counts
+// passes (the first also adds the squares of the positions not sent, with
+// magnitude bits >= err_from, to *err when it is given). Warp w owns the contiguous part [s0 + w (s1-s0)/32, ...): it counts
 // its selected positions (coalesced loads, 4 in flight per lane); the CTA's
 // counts are scanned (plus `base`, the pairs of earlier CTAs of a team, which
 // `publish` supplies once it sees the CTA's total; 0xffffffff: none, write
@@ -415,7 +424,8 @@ struct SrcGlobal {  // values in global memory; coordinates lo + i, or from a li
 template <class Src, class Publish>
 __device__ uint32_t write_out(const Src& src, uint32_t s0, uint32_t s1, const SmallSelection& sel,
                               uint32_t k, uint32_t* idx_out, float* val_out, float* e,
-                              bool& overflow, uint32_t* s_w, const Publish& publish) {
+                              bool& overflow, uint32_t* s_w, const Publish& publish,
+                              ErrAcc* err, uint32_t err_from) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   constexpr int kNumWarps = kLwThreads / 32;
   const uint32_t len = s1 - s0;
@@ -433,7 +443,12 @@ __device__ uint32_t write_out(const Src& src, uint32_t s0, uint32_t s1, const Sm
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const uint32_t i = i0 + j * 32 + lane;
-      cnt += (i < w1 && selected(sel, b[j] & 0x7fffffffu, i)) ? 1u : 0u;
+      const uint32_t mg = b[j] & 0x7fffffffu;
+      const bool take = i < w1 && selected(sel, mg, i);
+      cnt += take ? 1u : 0u;
+      // a position not sent keeps a; those at or above err_from are this
+      // kernel's share of ||e'||^2 (the rest were counted while streaming)
+      if (err && i < w1 && !take && mg >= err_from) err->add(__uint_as_float(b[j]));
     }
   }
   cnt = warp_sum(cnt);
@@ -486,10 +501,20 @@ struct NoTeam {
 
 // One CTA selects segment s on its own. Returns false when the threshold
 // was not found or the count differs from k (never for well-formed data).
+// Where the streaming pass left a segment's residuals to the select: every
+// position of a list source (candidates), and of an e source those at or above
+// the bound the stream used (all of them without one).
+__device__ __forceinline__ uint32_t err_from_for(const LwArgs& a, const LwSeg& s, uint32_t si,
+                                                 bool list) {
+  if (list || s.kind != kLwSampled) return 0u;
+  const uint32_t b = __ldcg(a.mbound + si);
+  return b >= kLwDeferred ? 0u : b;
+}
+
 __device__ bool select_single(const LwArgs& a, const LwSeg& s, uint32_t si, float* e,
                               uint32_t* idx_out, float* val_out, bool& overflow,
                               uint32_t* s_bits, uint32_t* s_hist, uint32_t* s_w, uint32_t* s_lo,
-                              uint32_t* s_hi) {
+                              uint32_t* s_hi, ErrAcc* err) {
   uint32_t* io = idx_out + s.out;
   float* vo = val_out + s.out;
   const uint32_t ds = s.hi - s.lo;
@@ -502,6 +527,7 @@ __device__ bool select_single(const LwArgs& a, const LwSeg& s, uint32_t si, floa
     return true;
   }
   const Source src = s.kind == kLwWhole ? Source{false, 0, ds} : segment_source(a, s, si);
+  const uint32_t err_from = err_from_for(a, s, si, src.list);
   const float* vals = src.list ? a.list_val + src.c0 : e + s.lo;
   const uint32_t* idxs = src.list ? a.list_idx + src.c0 : nullptr;
   SmallSelection sel;
@@ -514,13 +540,13 @@ __device__ bool select_single(const LwArgs& a, const LwSeg& s, uint32_t si, floa
     found = threshold_levels<kLwThreads>(MagsShared{s_bits}, src.n, s.k, lo, hi, s_hist, s_w, sel);
     if (found)
       got = write_out(SrcShared{s_bits, idxs, s_idx, s.lo}, 0, src.n, sel, s.k, io, vo, e,
-                      overflow, s_w, NoTeam{});
+                      overflow, s_w, NoTeam{}, err, err_from);
   } else {
     load_minmax(vals, src.n, nullptr, lo, hi, s_lo, s_hi);
     found = threshold_levels<kLwThreads>(MagsGlobal{vals}, src.n, s.k, lo, hi, s_hist, s_w, sel);
     if (found)
       got = write_out(SrcGlobal{vals, idxs, s.lo}, 0, src.n, sel, s.k, io, vo, e, overflow, s_w,
-                      NoTeam{});
+                      NoTeam{}, err, err_from);
   }
   return found && got == s.k;
 }
@@ -538,10 +564,12 @@ __device__ bool select_single(const LwArgs& a, const LwSeg& s, uint32_t si, floa
 // (latched as a timeout) or an inconsistent histogram.
 __device__ bool select_team(const LwArgs& a, const LwSeg& s, uint32_t si, uint32_t T, uint32_t r,
                             LwTeamState* st, float* e, uint32_t* idx_out, float* val_out,
-                            bool& overflow, bool& bad, uint32_t* s_hist, uint32_t* s_w) {
+                            bool& overflow, bool& bad, uint32_t* s_hist, uint32_t* s_w,
+                            ErrAcc* err) {
   __shared__ uint32_t s_found, s_last;
   const int tid = threadIdx.x;
   const Source src = segment_source(a, s, si);
+  const uint32_t err_from = err_from_for(a, s, si, src.list);
   const float* vals = src.list ? a.list_val + src.c0 : e + s.lo;
   const uint32_t* idxs = src.list ? a.list_idx + src.c0 : nullptr;
   const MagsGlobal mag{vals};
@@ -653,7 +681,7 @@ __device__ bool select_team(const LwArgs& a, const LwSeg& s, uint32_t si, uint32
     return s_base;
   };
   const SrcGlobal sg{vals, idxs, s.lo};
-  write_out(sg, s0, s1, sel, s.k, io, vo, e, overflow, s_w, publish);
+  write_out(sg, s0, s1, sel, s.k, io, vo, e, overflow, s_w, publish, err, err_from);
   if (s_base == 0xffffffffu) return false;
   // every CTA has read the level histograms (before the write-out barrier):
   // clear them for the next call
@@ -680,8 +708,13 @@ __global__ void __launch_bounds__(kLwThreads, 1)
     *a.count_out = failed ? 0u : a.total_k;
     if (failed) atomicOr(a.error, kDevErrTimeout);
   }
-  if (failed) return;  // a is incomplete: nothing is selected
+  if (failed) {  // a is incomplete: nothing is selected
+    if (blockIdx.x == 0 && tid == 0 && a.err_out) *a.err_out = err_invalid();
+    return;
+  }
   bool overflow = false, bad = false;
+  ErrAcc acc;
+  ErrAcc* err = a.err_out ? &acc : nullptr;
   const LwCta me = a.ctas[blockIdx.x];
   if (me.team == kLwNoTeam) {
     for (uint32_t w = me.a; w < me.b; ++w) {
@@ -689,16 +722,35 @@ __global__ void __launch_bounds__(kLwThreads, 1)
       const LwSeg s = a.segs[si];
       __syncthreads();  // the previous segment is done with shared memory
       if (!select_single(a, s, si, e, idx_out, val_out, overflow, s_bits, s_hist, s_w, s_lo,
-                         s_hi))
+                         s_hi, err))
         bad = true;
     }
   } else {
     const LwSeg s = a.segs[me.a];
     select_team(a, s, me.a, me.b, me.rank, a.teams + me.team, e, idx_out, val_out, overflow, bad,
-                s_hist, s_w);
+                s_hist, s_w, err);
   }
   if (__syncthreads_or(overflow) && tid == 0) atomicOr(a.error, kDevErrOverflow);
   if (__syncthreads_or(bad) && tid == 0) atomicOr(a.error, kDevErrBadInput);
+  if (a.err_out) {
+    // this CTA's share; the last CTA to arrive adds the shares in CTA order
+    // to the streaming pass's
+    __shared__ double s_d[kLwThreads / 32];
+    __shared__ uint32_t s_last_cta;
+    acc.flush();
+    const double share = block_sum_fixed(acc.total, s_d);
+    if (tid == 0) {
+      a.err_parts[blockIdx.x] = share;
+      __threadfence();
+      s_last_cta = atomicAdd(a.err_arrive, 1u) == gridDim.x - 1 ? 1u : 0u;
+      if (s_last_cta) {
+        __threadfence();
+        double t = *a.stream_err;
+        for (uint32_t q = 0; q < gridDim.x; ++q) t += __ldcg(a.err_parts + q);
+        *a.err_out = t;
+      }
+    }
+  }
 }
 
 // ------------------------------------------------------------- host side
@@ -746,7 +798,7 @@ uint64_t select_cost(const LwSeg& s) {
 
 template <typename GT>
 cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t d, uint32_t* idx_out,
-                         float* val_out, uint32_t* count_out, Workspace& ws,
+                         float* val_out, uint32_t* count_out, double* err_out, Workspace& ws,
                          const DeviceInfo& dev) {
   const LwPlan& p = *ws.lw;
   cudaError_t err = cudaSuccess;
@@ -786,7 +838,8 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t d, uint32_
     const uint32_t grid = p.tiles < slots ? p.tiles : slots;
     uint32_t cap = ws.cand_cap;
     uint32_t* list_count = ws.u32(kOffTkListCount);
-    StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks(), tile_base};
+    StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks(), tile_base,
+                  err_out ? ws.stream_err() : nullptr, ws.errparts()};
     void* params[] = {&op, &d, &list_idx, &list_val, &list_count, &cap, &ctx, &sa};
     // not cooperative: the only cross-CTA wait is on lower-numbered CTAs,
     // which are scheduled first
@@ -821,11 +874,17 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t d, uint32_
   a.cap = ws.cand_cap;
   a.use_list = streamable ? 1u : 0u;
   a.total_k = static_cast<uint32_t>(p.total_k);
+  // inputs the streaming pass could not take: the norm by a plain pass after
+  a.err_out = streamable ? err_out : nullptr;
+  a.stream_err = ws.stream_err();
+  a.err_parts = ws.errparts();
+  a.err_arrive = state + kStErrArrive / 4;
   void* params[] = {(void*)&e, (void*)&idx_out, (void*)&val_out, (void*)&a};
   // (cooperative only when there are teams: nothing else waits on another CTA)
   err = launch_pdl(reinterpret_cast<const void*>(&lw_select_kernel), p.n_select_ctas, kLwThreads,
                    kLwSelectSmem, ws.stream, params, p.n_teams > 0);
   count_launch();
+  if (err == cudaSuccess && err_out && !streamable) err = launch_error_norm(e, d, err_out, ws, dev);
   return err;
 }
 
@@ -885,6 +944,7 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
       sampled.push_back(s);
     }
     ends[s] = static_cast<uint32_t>(hi);
+    mbound[s] = x.kind == kLwNone ? kLwNoBound : kLwDeferred;  // sampled: the sampler's
     total_k += k;
     lo = hi;
   }
@@ -1050,12 +1110,12 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
 
 cudaError_t launch_topk_layerwise(const void* g, bool g_bf16, float* e, float gamma, uint32_t d,
                                   uint32_t* idx_out, float* val_out, uint32_t* count_out,
-                                  Workspace& ws, const DeviceInfo& dev) {
+                                  double* err_out, Workspace& ws, const DeviceInfo& dev) {
   if (g_bf16)
     return launch_typed(static_cast<const uint16_t*>(g), e, gamma, d, idx_out, val_out,
-                        count_out, ws, dev);
+                        count_out, err_out, ws, dev);
   return launch_typed(static_cast<const float*>(g), e, gamma, d, idx_out, val_out, count_out,
-                      ws, dev);
+                      err_out, ws, dev);
 }
 
 }  // namespace efs
