@@ -202,10 +202,11 @@ ef_status ef_topk_layerwise_bf16(const uint16_t* g, float* e, float gamma, uint3
  *
  * Precision (the paper fixes none): squares are accumulated with fmaf in fp32
  * in groups of at most 256 terms whose partial sums see at most 13 roundings,
- * and the groups are added in fp64 in a fixed order. The result is within
- * 1e-6 of the exact sum, relatively (nonnegative terms), plus the squares
- * below the fp32 range (|e'_j| < 2^-75), which contribute 0; |e'_j| >= 2^64
- * makes it +inf. It is bit-for-bit reproducible for a given device and input.
+ * and the groups are added in float-float arithmetic (about 44 bits) in a
+ * fixed order. The result is within 1e-6 of the exact sum, relatively
+ * (nonnegative terms), plus the squares below the fp32 range
+ * (|e'_j| < 2^-75), which contribute 0; a sum beyond the fp32 range
+ * (|e'_j| >= 2^64 suffices) makes it +inf. It is bit-for-bit reproducible for a given device and input.
  * The streaming kernels add it as they go; steps whose g or e are not
  * 16-byte aligned compute it with one more pass over e'. After a step that
  * failed on the device (a latched timeout) it holds a NaN.

@@ -190,16 +190,43 @@ __device__ __forceinline__ uint32_t lookback_exclusive(const ScanCtx& ctx, uint3
 // Squared error norm ||e'||^2 = sum_j e'_j^2, deterministic for a given
 // launch shape: squares are accumulated with fmaf in fp32 in fixed groups of
 // at most 8 terms (a warp tree of 32 such groups in the streaming kernels),
-// and the groups are added in fp64 in a fixed order. Every fp32 partial sum
-// carries at most 13 roundings of nonnegative terms, so the result is within
-// 13 * 2^-24 (< 1e-6) of the exact sum, relatively, plus the squares below
-// the fp32 range (|e'_j| < 2^-75) that contribute 0. |e'_j| >= 2^64 squares
-// to +inf.
+// and the groups are added in float-float arithmetic (an unevaluated pair
+// hi + lo of fp32 values, added with the error-free TwoSum of Knuth, so each
+// addition is exact up to about 2^-44 relatively) in a fixed order. Every
+// fp32 group sum carries at most 13 roundings of nonnegative terms, so the
+// result is within 13 * 2^-24 (< 1e-6) of the exact sum, relatively, plus
+// the squares below the fp32 range (|e'_j| < 2^-75), which contribute 0; a
+// sum beyond the fp32 range is +inf. Float-float instead of fp64: fp64
+// arithmetic is slow on this GPU (a 32-step fp64 chain cost microseconds).
+
 // Written as ||e'||^2 when a failed step has none.
 __device__ __forceinline__ double err_invalid() { return __longlong_as_double(0x7ff8000000000000ll); }
 
+struct FF {  // hi + lo, |lo| <= ulp(hi) / 2
+  float hi, lo;
+};
+
+// Knuth's TwoSum: s + t == a + b exactly, s = RN(a + b).
+__device__ __forceinline__ void two_sum(float a, float b, float& s, float& t) {
+  s = __fadd_rn(a, b);
+  const float bb = __fsub_rn(s, a);
+  t = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+}
+
+__device__ __forceinline__ FF ff_add(FF x, FF y) {
+  float s, t;
+  two_sum(x.hi, y.hi, s, t);
+  t = __fadd_rn(t, __fadd_rn(x.lo, y.lo));
+  const float hi = __fadd_rn(s, t);  // renormalise: |t| is small against s
+  return FF{hi, __fsub_rn(t, __fsub_rn(hi, s))};
+}
+
+__device__ __forceinline__ double ff_to_double(FF x) {
+  return static_cast<double>(x.hi) + static_cast<double>(x.lo);
+}
+
 struct ErrAcc {
-  double total = 0.0;
+  FF total{0.0f, 0.0f};
   float part = 0.0f;
   int terms = 0;
   __device__ __forceinline__ void add(float x) {
@@ -207,26 +234,45 @@ struct ErrAcc {
     if (++terms == 8) flush();
   }
   __device__ __forceinline__ void flush() {
-    total += static_cast<double>(part);
+    total = ff_add(total, FF{part, 0.0f});
     part = 0.0f;
     terms = 0;
   }
 };
 
-// Sum of one double per thread over the CTA in a fixed order (warp trees,
-// then the warps in order); the result is valid in thread 0. s_d holds
-// blockDim.x / 32 doubles.
-__device__ __forceinline__ double block_sum_fixed(double v, double* s_d) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+__device__ __forceinline__ FF warp_sum_ff(FF v) {
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  __syncthreads();  // an earlier use of s_d is complete
-  if (lane == 0) s_d[warp] = v;
+  for (int o = 16; o > 0; o >>= 1) {
+    const FF w{__shfl_xor_sync(0xffffffffu, v.hi, o), __shfl_xor_sync(0xffffffffu, v.lo, o)};
+    v = ff_add(v, w);
+  }
+  return v;
+}
+
+// Sum of one value per thread over the CTA in a fixed order (a warp tree,
+// then a tree over the warps); the result is valid in thread 0. s_ff holds
+// 32 values.
+__device__ __forceinline__ FF block_sum_ff(FF v, FF* s_ff) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nw = static_cast<int>(blockDim.x >> 5);
+  v = warp_sum_ff(v);
+  __syncthreads();  // an earlier use of s_ff is complete
+  if (lane == 0) s_ff[warp] = v;
   __syncthreads();
-  double t = 0.0;
-  if (threadIdx.x == 0)
-    for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) t += s_d[w];
-  return t;
+  FF r{0.0f, 0.0f};
+  if (warp == 0) r = warp_sum_ff(lane < nw ? s_ff[lane] : FF{0.0f, 0.0f});
+  return r;
+}
+
+// Sum of parts[0, n) by the whole CTA in a fixed order (one round of loads,
+// then the fixed trees); valid in thread 0.
+__device__ __forceinline__ FF sum_parts_ff(const FF* parts, uint32_t n, FF* s_ff) {
+  FF v{0.0f, 0.0f};
+  for (uint32_t q = threadIdx.x; q < n; q += blockDim.x) {
+    const float2 p = __ldcg(reinterpret_cast<const float2*>(parts) + q);
+    v = ff_add(v, FF{p.x, p.y});
+  }
+  return block_sum_ff(v, s_ff);
 }
 
 // Bounded grid-wide barrier for a cooperative launch (all CTAs co-resident).

@@ -7,8 +7,8 @@
 // CTA c sums the contiguous range [c d / G, (c+1) d / G): per thread, the
 // accumulator of common.cuh over coalesced positions; per CTA, a fixed-order
 // sum of the threads. Each CTA stores its share, fences, and counts itself
-// in; the last to arrive adds the G shares in CTA order, writes the result
-// and resets the counter. No CTA waits for another.
+// in; the last to arrive adds the G shares in a fixed order, writes the
+// result and resets the counter. No CTA waits for another.
 #include "internal.h"
 
 namespace efs {
@@ -17,9 +17,9 @@ namespace {
 constexpr int kErrThreads = 256;
 
 __global__ void __launch_bounds__(kErrThreads)
-    error_norm_kernel(const float* __restrict__ e, uint32_t d, double* parts, uint32_t* arrive,
+    error_norm_kernel(const float* __restrict__ e, uint32_t d, FF* parts, uint32_t* arrive,
                       double* err_out) {
-  __shared__ double s_d[kErrThreads / 32];
+  __shared__ FF s_d[32];
   __shared__ uint32_t s_last;
   const uint32_t G = gridDim.x, c = blockIdx.x;
   const uint32_t lo = static_cast<uint32_t>(static_cast<uint64_t>(c) * d / G);
@@ -36,19 +36,20 @@ __global__ void __launch_bounds__(kErrThreads)
     for (int j = 0; j < 4; ++j) acc.add(v[j]);
   }
   acc.flush();
-  const double mine = block_sum_fixed(acc.total, s_d);
+  const FF mine = block_sum_ff(acc.total, s_d);
   if (threadIdx.x == 0) {
     parts[c] = mine;
     __threadfence();
     s_last = atomicAdd(arrive, 1u) == G - 1 ? 1u : 0u;
   }
   __syncthreads();
-  if (threadIdx.x == 0 && s_last) {
+  if (s_last) {
     __threadfence();
-    double t = 0.0;
-    for (uint32_t q = 0; q < G; ++q) t += __ldcg(parts + q);
-    *err_out = t;
-    *arrive = 0;  // ready for the next pass
+    const FF t = sum_parts_ff(parts, G, s_d);
+    if (threadIdx.x == 0) {
+      *err_out = ff_to_double(t);
+      *arrive = 0;  // ready for the next pass
+    }
   }
 }
 

@@ -33,9 +33,9 @@
 // nor deferred (selection bits 4..7 of an op mark coordinates whose residual
 // a later kernel decides) keeps a as its residual, so a^2 is its share of
 // ||e'||^2. Each warp sums the squares of a tile segment in fp32 (fmaf per
-// lane over its 8 coordinates, then a warp tree) and adds that in fp64; the
-// CTA's share is published with its chunk total, and the last CTA adds the
-// shares in CTA order.
+// lane over its 8 coordinates, then a warp tree) and adds that in
+// float-float (common.cuh); the CTA's share is published with its chunk
+// total, and the last CTA adds the shares in a fixed order.
 //
 // Traffic beyond the step itself: 16 bytes per selected pair (staging write
 // and read) plus 4 bytes per segment. Every wait (stage arrival, stage
@@ -97,7 +97,7 @@ struct StreamArgs {
                          // pair, and the total (untruncated), or null
   double* err_out;       // optional: sum of a^2 over the coordinates whose residual is final
                          // here (not selected, not deferred), or null
-  double* err_parts;     // [gridDim.x] the CTAs' shares of it
+  FF* err_parts;         // [gridDim.x] the CTAs' shares of it
 };
 
 // A segment's count (<= 256: 9 bits) and its warp's earlier pairs in the
@@ -129,7 +129,8 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   __shared__ __align__(8) uint64_t s_full[kStages];
   __shared__ __align__(8) uint64_t s_empty[kStages];
   __shared__ uint32_t s_scratch[kStreamThreads / 32];
-  __shared__ double s_err[kSWarps];
+  __shared__ FF s_err[kSWarps];
+  __shared__ FF s_err_sum[32];
   __shared__ uint32_t s_sample_hist[Op::kPrepass ? Op::kSampleBins : 1];
   using L = StreamLayout<Op, kStages>;
   uint32_t* s_pair_idx = reinterpret_cast<uint32_t*>(smem + L::kRing);
@@ -159,7 +160,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   bool failed = false;    // a wait of this thread ran out
   bool withheld = false;  // test hook: this CTA owns the withheld tile
   uint32_t chunk_total = 0;  // compute warps: pairs selected by this warp
-  double warp_err = 0.0;     // compute warps: their share of ||e'||^2
+  FF warp_err{0.0f, 0.0f};   // compute warps: their share of ||e'||^2
   uint64_t policy = 0;       // producer lane
   auto fill = [&](uint32_t r) {  // producer lane
     const int s = static_cast<int>(r % kStages);
@@ -247,7 +248,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
             if (!((sel[v] >> j) & 0x11u)) sq = __fmaf_rn(a[v][j], a[v][j], sq);
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
-        if (lane == 0) warp_err += static_cast<double>(sq);
+        if (lane == 0) warp_err = ff_add(warp_err, FF{sq, 0.0f});
       }
       uint32_t off[kSUnits];
       uint32_t total = 0;
@@ -308,8 +309,8 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
     uint32_t sum = 0;
     for (int w = 0; w < kSWarps; ++w) sum += s_scratch[w];
     if (sa.err_out) {  // the CTA's share of ||e'||^2, visible before the chunk total
-      double err = 0.0;
-      for (int w = 0; w < kSWarps; ++w) err += s_err[w];
+      FF err{0.0f, 0.0f};
+      for (int w = 0; w < kSWarps; ++w) err = ff_add(err, s_err[w]);
       sa.err_parts[c] = err;
       __threadfence();
     }
@@ -342,11 +343,8 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
           // every earlier CTA's share was written before its chunk total
           __threadfence();
           __syncthreads();
-          if (threadIdx.x == 0) {
-            double err = 0.0;
-            for (uint32_t q = 0; q < G; ++q) err += __ldcg(sa.err_parts + q);
-            *sa.err_out = err;
-          }
+          const FF err = sum_parts_ff(sa.err_parts, G, s_err_sum);
+          if (threadIdx.x == 0) *sa.err_out = ff_to_double(err);
         }
       } else {
         const uint64_t now = global_timer_ns();

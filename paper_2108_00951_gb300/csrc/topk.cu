@@ -74,7 +74,7 @@ struct TopkArgs {
   uint64_t wait_limit_ns;
   double* err_out;       // optional ||e'||^2 of the step
   const double* stream_err;  // the streaming pass's share (coordinates below the bound)
-  double* err_parts;     // [gridDim.x] the select CTAs' shares
+  FF* err_parts;         // [gridDim.x] the select CTAs' shares
 };
 
 // ------------------------------------------------------------- 1 stream
@@ -719,9 +719,10 @@ __global__ void __launch_bounds__(kSelThreads, 1)
           for (uint32_t i = threadIdx.x; i < si.n; i += kSelThreads)
             if (!selected(sel, s_mag[i], i)) acc.add(__uint_as_float(s_mag[i]));
         acc.flush();
-        __shared__ double s_d[kSelThreads / 32];
-        const double rem = block_sum_fixed(acc.total, s_d);
-        if (threadIdx.x == 0) *args.err_out = found ? *args.stream_err + rem : err_invalid();
+        __shared__ FF s_d[32];
+        const FF rem = block_sum_ff(acc.total, s_d);
+        if (threadIdx.x == 0)
+          *args.err_out = found ? *args.stream_err + ff_to_double(rem) : err_invalid();
       }
     }
     small_emit(args, e, si.n, k, Gs, idx_out, val_out, count_out, s_w);
@@ -761,8 +762,8 @@ __global__ void __launch_bounds__(kSelThreads, 1)
   block_exclusive<kSelThreads>(mine, total, s_w);
   if (args.err_out) {
     acc.flush();
-    __shared__ double s_d[kSelThreads / 32];
-    const double share = block_sum_fixed(acc.total, s_d);
+    __shared__ FF s_d[32];
+    const FF share = block_sum_ff(acc.total, s_d);
     if (threadIdx.x == 0) {
       args.err_parts[c] = share;  // visible before the chunk total
       __threadfence();
@@ -795,11 +796,10 @@ __global__ void __launch_bounds__(kSelThreads, 1)
           // streaming pass's (a full-array source covers every coordinate)
           __threadfence();
           __syncthreads();
-          if (threadIdx.x == 0) {
-            double err = si.mode == 0 ? *args.stream_err : 0.0;
-            for (uint32_t q = 0; q < G; ++q) err += __ldcg(args.err_parts + q);
-            *args.err_out = err;
-          }
+          __shared__ FF s_d2[32];
+          const FF shares = sum_parts_ff(args.err_parts, G, s_d2);
+          if (threadIdx.x == 0)
+            *args.err_out = (si.mode == 0 ? *args.stream_err : 0.0) + ff_to_double(shares);
         }
         break;
       }

@@ -298,7 +298,7 @@ struct LwArgs {
   uint32_t total_k;
   double* err_out;            // optional ||e'||^2 of the step
   const double* stream_err;   // the streaming pass's share (final residuals)
-  double* err_parts;          // [gridDim.x] the select CTAs' shares
+  FF* err_parts;              // [gridDim.x] the select CTAs' shares
   uint32_t* err_arrive;       // select CTAs that published their share (zero at the start)
 };
 
@@ -735,20 +735,20 @@ __global__ void __launch_bounds__(kLwThreads, 1)
   if (a.err_out) {
     // this CTA's share; the last CTA to arrive adds the shares in CTA order
     // to the streaming pass's
-    __shared__ double s_d[kLwThreads / 32];
+    __shared__ FF s_d[32];
     __shared__ uint32_t s_last_cta;
     acc.flush();
-    const double share = block_sum_fixed(acc.total, s_d);
+    const FF share = block_sum_ff(acc.total, s_d);
     if (tid == 0) {
       a.err_parts[blockIdx.x] = share;
       __threadfence();
       s_last_cta = atomicAdd(a.err_arrive, 1u) == gridDim.x - 1 ? 1u : 0u;
-      if (s_last_cta) {
-        __threadfence();
-        double t = *a.stream_err;
-        for (uint32_t q = 0; q < gridDim.x; ++q) t += __ldcg(a.err_parts + q);
-        *a.err_out = t;
-      }
+    }
+    __syncthreads();
+    if (s_last_cta) {
+      __threadfence();
+      const FF shares = sum_parts_ff(a.err_parts, gridDim.x, s_d);
+      if (tid == 0) *a.err_out = *a.stream_err + ff_to_double(shares);
     }
   }
 }
