@@ -68,6 +68,8 @@ def parse_args(argv=None):
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="resnet18")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--error-norm", action="store_true",
+                   help="every compress call also returns ||e'||^2 (the _ex entries)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=10.0,
                    help="bound on the CPU-oracle sample of the cpu_baseline leg")
@@ -289,24 +291,30 @@ def run_ours(args):
     ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
     marks = [[ev() for _ in range(8)] for _ in range(args.steps)]
 
+    err_sq = torch.zeros(3, n, dtype=torch.float64, device=dev)
+
+    def errkw(leg, i):
+        return {"err_sq_out": err_sq[leg, i:i + 1]} if args.error_norm else {}
+
     def step(s, timed):
         g = batches[s % 2]
         m = marks[s - args.warmup] if timed else None
         if m: m[0].record(stream)
         for i in range(n):
             efs.ef_hard_threshold(g[i], e_ht[i], gamma, lam, idx_ht[i], val_ht[i],
-                                  cnt_ht[s, i:i + 1])
+                                  cnt_ht[s, i:i + 1], **errkw(0, i))
         if m: m[1].record(stream)
         efs.sparse_aggregate(idx_ht, val_ht, cnt_ht[s], d, dense_ht)
         if m: m[2].record(stream)
         for i in range(n):
-            efs.ef_topk(g[i], e_tk[i], gamma, k, idx_tk[i], val_tk[i], cnt_tk[s, i:i + 1])
+            efs.ef_topk(g[i], e_tk[i], gamma, k, idx_tk[i], val_tk[i], cnt_tk[s, i:i + 1],
+                        **errkw(1, i))
         if m: m[3].record(stream)
         efs.sparse_aggregate(idx_tk, val_tk, cnt_tk[s], d, dense_tk)
         if m: m[4].record(stream)
         for i in range(n):
             efs.ef_topk_layerwise(g[i], e_lw[i], gamma, seg_end, seg_k, idx_lw[i], val_lw[i],
-                                  cnt_lw[s, i:i + 1])
+                                  cnt_lw[s, i:i + 1], **errkw(2, i))
         if m: m[5].record(stream)
         efs.sparse_aggregate(idx_lw, val_lw, cnt_lw[s], d, dense_lw)
         if m: m[6].record(stream)
@@ -450,6 +458,11 @@ def run_ours(args):
             "algorithmic_bytes_per_launch": int(ht_bytes(d, 0) + 8 * counts_ht.mean().item()),
             "traffic": profiled_traffic("ht_kernel", w.name),
         },
+        "error_norm": ({"requested": True,
+                        "last_step_sq_norms_worker0": {
+                            "ht": float(err_sq[0, 0]), "topk": float(err_sq[1, 0]),
+                            "topk_layerwise": float(err_sq[2, 0])}}
+                       if args.error_norm else {"requested": False}),
         "gpu_launches": int(launches),
         "clocks": clocks,
         "e2e": e2e,
