@@ -17,6 +17,9 @@ passage behind every line):
 * ``sparse_aggregate(idx_list, val_list, d)`` — worker-ordered sum of the
   decompressed vectors (Algorithm 1, exchange step).
 * ``error_norm_sq(e)`` — ||e||^2 in fp64, the per-step term of the total error.
+* ``ef_scaled_round(g, e, gamma, m)``, ``int_aggregate(q_list, d, m)`` — scaled
+  integer rounding under EF (an absolute compressor, Sec. 5) and the exact
+  integer exchange of its messages.
 * ``sparse_aggregate_apply(idx_list, val_list, d, alpha, x, m, mu, lr)`` —
   that sum scaled by alpha, applied as Algorithm 1's model update, or as the
   momentum update of the Appendix's gradient-compression EF SGD.
@@ -90,6 +93,15 @@ def _load():
             lib.oracle_sparse_aggregate_apply.restype = ctypes.c_int
             lib.oracle_error_norm_sq.argtypes = [f32p, ctypes.c_uint64]
             lib.oracle_error_norm_sq.restype = ctypes.c_double
+            i32p = ctypes.POINTER(ctypes.c_int32)
+            for name, gp in (("oracle_ef_scaled_round", f32p),
+                             ("oracle_ef_scaled_round_bf16", ctypes.POINTER(ctypes.c_uint16))):
+                fn = getattr(lib, name)
+                fn.argtypes = [gp, f32p, ctypes.c_float, ctypes.c_int, ctypes.c_uint64, i32p, u32p]
+                fn.restype = ctypes.c_int
+            lib.oracle_int_aggregate.argtypes = [ctypes.c_uint32, ctypes.POINTER(i32p),
+                                                 ctypes.c_uint64, ctypes.c_int, f32p]
+            lib.oracle_int_aggregate.restype = ctypes.c_int
             _lib = lib
     return _lib
 
@@ -216,6 +228,35 @@ def sparse_aggregate_apply(idx_list, val_list, d: int, alpha: float, x, m=None, 
     if rc != 0:
         raise RuntimeError("oracle_sparse_aggregate_apply: index out of range")
     return x_new, m_new
+
+
+def ef_scaled_round(g: np.ndarray, e: np.ndarray, gamma: float, m: int):
+    """One EF step with scaled integer rounding: q = RNE(a 2^m) (int32),
+    C(a) = q 2^-m, e' = a - C(a); coordinates that do not fit are kept in e.
+    Returns (q, e_new, unsent)."""
+    lib = _load()
+    g, gctype, is_bf16 = _gradient(g)
+    e_new = np.array(e, dtype=np.float32, copy=True)
+    d = e_new.size
+    q = np.empty(max(d, 1), np.int32)
+    unsent = np.zeros(1, np.uint32)
+    fn = lib.oracle_ef_scaled_round_bf16 if is_bf16 else lib.oracle_ef_scaled_round
+    fn(_ptr(g, gctype), _ptr(e_new, ctypes.c_float), ctypes.c_float(gamma), int(m), d,
+       _ptr(q, ctypes.c_int32), _ptr(unsent, ctypes.c_uint32))
+    return q[:d].copy(), e_new, int(unsent[0])
+
+
+def int_aggregate(q_list, d: int, m: int) -> np.ndarray:
+    """Exact integer sum of n dense messages, decompressed as RN(S) 2^-m."""
+    lib = _load()
+    n = len(q_list)
+    arrs = [np.ascontiguousarray(q, dtype=np.int32) for q in q_list]
+    arrs = [a if a.size else np.zeros(1, np.int32) for a in arrs]
+    i32p = ctypes.POINTER(ctypes.c_int32)
+    ptrs = (i32p * n)(*[_ptr(a, ctypes.c_int32) for a in arrs])
+    dense = np.empty(max(d, 1), np.float32)
+    lib.oracle_int_aggregate(n, ptrs, d, int(m), _ptr(dense, ctypes.c_float))
+    return dense[:d].copy()
 
 
 def error_norm_sq(e) -> float:

@@ -30,6 +30,11 @@
  *   R7 the residual of a sent coordinate is +0.0f.
  *   R9 aggregation returns the sum (the 1/n of Algorithm 1 is the caller's),
  *      accumulated from +0.0f in ascending worker order.
+ *   R14 scaled integer rounding (Sec. 5 names it an absolute compressor):
+ *      q_j = round-half-to-even(a_j 2^m) as int32, C(a)_j = q_j 2^-m, e'_j =
+ *      a_j - C(a)_j (exact); a coordinate whose a_j 2^m has magnitude at least
+ *      2^31 (or is NaN) is not sent: q_j = 0, e'_j = a_j, and it is counted. The integer messages are summed exactly and the sum
+ *      decompressed with one rounding: RN(S_j) 2^-m.
  *   R12 model update after aggregation (the paper is silent on rounding):
  *      Delta'_j = alpha * s_j rounded once (alpha = 1/n gives the mean);
  *      without momentum x_j <- x_j - Delta'_j; with momentum
@@ -283,4 +288,55 @@ double oracle_error_norm_sq(const float* e, uint64_t d) {
   double s = 0.0;
   for (uint64_t j = 0; j < d; ++j) s += (double)e[j] * (double)e[j];
   return s;
+}
+
+/* ------------------------------------------------------------------------
+ * Scaled integer rounding (Sec. 5: any rounding with error bounded by eps
+ * is an absolute compressor with kappa^2 = d eps^2, the scaled integer
+ * rounding of in-network aggregation among them), under error feedback
+ * (Algorithm 1):
+ *   a_j = fmaf(gamma, g_j, e_j); q_j = RNE(a_j 2^m);
+ *   C(a)_j = q_j 2^-m; e'_j = a_j - C(a)_j, |e'_j| <= 2^(-m-1)  (R14)
+ * ------------------------------------------------------------------------ */
+static int scaled_round_core(const float* g_f32, const uint16_t* g_bf16, float* e, float gamma,
+                             int m, uint64_t d, int32_t* q, uint32_t* unsent) {
+  uint32_t u = 0;
+  for (uint64_t j = 0; j < d; ++j) {
+    float gj = g_f32 ? g_f32[j] : bf16_bits_to_float(g_bf16[j]);
+    float a = canonical_nan_if_nan(fmaf(gamma, gj, e[j]));    /* R2, R6 */
+    float s = ldexpf(a, m);                                    /* a 2^m (exact scaling) */
+    if (!(fabsf(s) < 2147483648.0f)) {                         /* |a 2^m| >= 2^31, or NaN */
+      q[j] = 0;                                                /* not representable: */
+      e[j] = a;                                                /* kept in e (R14) */
+      ++u;
+      continue;
+    }
+    float r = rintf(s);                                        /* round half to even */
+    q[j] = (int32_t)r;
+    float c = ldexpf((float)q[j], -m);                         /* C(a)_j */
+    e[j] = canonical_nan_if_nan(a - c);                        /* e'_j = a_j - C(a)_j */
+  }
+  *unsent = u;
+  return 0;
+}
+
+int oracle_ef_scaled_round(const float* g, float* e, float gamma, int m, uint64_t d, int32_t* q,
+                           uint32_t* unsent) {
+  return scaled_round_core(g, NULL, e, gamma, m, d, q, unsent);
+}
+
+int oracle_ef_scaled_round_bf16(const uint16_t* g, float* e, float gamma, int m, uint64_t d,
+                                int32_t* q, uint32_t* unsent) {
+  return scaled_round_core(NULL, g, e, gamma, m, d, q, unsent);
+}
+
+/* Exchange of the integer messages: S_j = sum_i q_i[j] exactly (int64, any
+ * order gives the same sum), decompressed as RN(S_j) 2^-m (R14). */
+int oracle_int_aggregate(uint32_t n, const int32_t* const* q, uint64_t d, int m, float* dense) {
+  for (uint64_t j = 0; j < d; ++j) {
+    int64_t s = 0;
+    for (uint32_t i = 0; i < n; ++i) s += q[i][j];
+    dense[j] = ldexpf((float)s, -m);
+  }
+  return 0;
 }

@@ -50,6 +50,15 @@ MUTANTS = {
     "update_wrong_sign": [("fmaf(-lr, u, x[j])", "fmaf(lr, u, x[j])")],
     "update_sgd_adds": [("x[j] = canonical_nan_if_nan(x[j] - delta);",
                          "x[j] = canonical_nan_if_nan(x[j] + delta);")],
+    "round_half_away": [("float r = rintf(s);", "float r = roundf(s);")],
+    "round_truncate": [("float r = rintf(s);", "float r = truncf(s);")],
+    "round_residual_not_subtracted": [("e[j] = canonical_nan_if_nan(a - c);",
+                                       "e[j] = canonical_nan_if_nan(a);")],
+    "round_scale_sign": [("float s = ldexpf(a, m);", "float s = ldexpf(a, -m);")],
+    "round_saturates_instead": [("      q[j] = 0;                                                /* not representable: */",
+                                 "      q[j] = a > 0 ? 2147483647 : -2147483647;")],
+    "int_aggregate_in_float": [("    int64_t s = 0;\n    for (uint32_t i = 0; i < n; ++i) s += q[i][j];",
+                                "    float s = 0;\n    for (uint32_t i = 0; i < n; ++i) s += (float)q[i][j];")],
     "error_norm_fp32_square": [("s += (double)e[j] * (double)e[j];", "s += (double)(e[j] * e[j]);")],
     "error_norm_abs": [("s += (double)e[j] * (double)e[j];", "s += fabs((double)e[j]);")],
 }
@@ -77,6 +86,10 @@ PIN_TESTS = [
     pins.test_update_rounding_follows_r12,
     pins.test_error_norm_hand_values_and_exactness,
     pins.test_error_norm_bounds_of_the_sparsifiers,
+    pins.test_scaled_round_hand_example,
+    pins.test_scaled_round_is_an_absolute_compressor,
+    pins.test_scaled_round_unsent_coordinates,
+    pins.test_int_aggregate_is_exact_and_order_free,
 ]
 
 
@@ -89,7 +102,9 @@ def _swapped_library(path):
     for name in ("oracle_ef_hard_threshold", "oracle_ef_hard_threshold_bf16",
                  "oracle_ef_topk", "oracle_ef_topk_bf16", "oracle_ef_topk_layerwise",
                  "oracle_ef_topk_layerwise_bf16", "oracle_sparse_aggregate",
-                 "oracle_sparse_aggregate_apply", "oracle_error_norm_sq"):
+                 "oracle_sparse_aggregate_apply", "oracle_error_norm_sq",
+                 "oracle_ef_scaled_round", "oracle_ef_scaled_round_bf16",
+                 "oracle_int_aggregate"):
         fn, ref = getattr(lib, name), getattr(saved, name)
         fn.argtypes, fn.restype = ref.argtypes, ref.restype
     oracle._lib = lib

@@ -567,6 +567,71 @@ def test_error_norm_bounds_of_the_sparsifiers():
 
 
 # --------------------------------------------------------------------------
+# scaled integer rounding (Sec. 5: an absolute compressor)
+# --------------------------------------------------------------------------
+def test_scaled_round_hand_example():
+    # grid 2^-2: 0.1 -> 0 (0.4), 0.125 -> 0 (0.5, to even), 0.375 -> 2 (1.5,
+    # to even), -0.625 -> -2 (-2.5, to even), 3.0 -> 12, 0.25 + tiny -> 1
+    a = _f32([0.1, 0.125, 0.375, -0.625, 3.0, 0.26])
+    q, e_new, unsent = oracle.ef_scaled_round(np.zeros(6, np.float32), a, 1.0, 2)
+    assert list(q) == [0, 0, 2, -2, 12, 1] and unsent == 0
+    assert list(e_new) == [np.float32(0.1), 0.125, -0.125, -0.125, 0.0, np.float32(0.26) - 0.25]
+
+
+def test_scaled_round_is_an_absolute_compressor():
+    # |e'_j| <= 2^(-m-1) for every coordinate, so ||e'||^2 <= d 2^(-2m-2)
+    # (kappa^2 = d eps^2, Sec. 5), and a = C(a) + e' exactly
+    rng = np.random.default_rng(31)
+    d = 4000
+    g = _f32(rng.standard_normal(d) * 10.0)
+    e = _f32(rng.standard_normal(d))
+    for m in (-3, 0, 4, 17):
+        q, e_new, unsent = oracle.ef_scaled_round(g, e, 0.1, m)
+        assert unsent == 0
+        a = [fma_f32(np.float32(0.1), gj, ej) for gj, ej in zip(g, e)]
+        eps = Fraction(2) ** (-m - 1)
+        for j in range(d):
+            c = Fraction(int(q[j])) * Fraction(2) ** (-m)
+            assert Fraction(float(a[j])) == c + Fraction(float(e_new[j]))
+            assert abs(Fraction(float(e_new[j]))) <= eps
+            # q is the nearest integer to a 2^m, ties to even
+            t = Fraction(float(a[j])) * Fraction(2) ** m
+            fl = t.numerator // t.denominator
+            want = fl + 1 if (t - fl > Fraction(1, 2) or (t - fl == Fraction(1, 2) and fl % 2)) else fl
+            assert int(q[j]) == want
+        assert oracle.error_norm_sq(e_new) <= d * float(eps) ** 2
+
+
+def test_scaled_round_unsent_coordinates():
+    # a 2^m at or beyond 2^31, infinities and NaN are not sent: q = 0, e' = a
+    a = _f32([2.0 ** 31, -(2.0 ** 31), 2.0 ** 31 - 128.0, np.inf, np.nan, 1.0])
+    q, e_new, unsent = oracle.ef_scaled_round(np.zeros(6, np.float32), a, 1.0, 0)
+    assert unsent == 4
+    assert list(q[:3]) == [0, 0, 2 ** 31 - 128] and q[3] == 0 and q[4] == 0 and q[5] == 1
+    assert e_new[0] == 2.0 ** 31 and e_new[1] == -(2.0 ** 31) and e_new[2] == 0.0
+    assert np.isinf(e_new[3]) and e_new.view(np.uint32)[4] == CANONICAL_NAN and e_new[5] == 0.0
+
+
+def test_int_aggregate_is_exact_and_order_free():
+    # the integer sum is exact whatever the order; one rounding at the end
+    big = 2 ** 30
+    q1 = np.array([big, 1, -7], np.int32)
+    q2 = np.array([big, 2, 7], np.int32)
+    q3 = np.array([-big, 4, 0], np.int32)
+    for order in ([q1, q2, q3], [q3, q2, q1], [q2, q3, q1]):
+        dense = oracle.int_aggregate(order, 3, 3)
+        assert list(dense) == [float(big) / 8, 7 / 8, 0.0]
+    # 2^25 + 1 rounds once to 2^25 (ties to even), then scales
+    dense = oracle.int_aggregate([np.array([2 ** 24 + 1], np.int32),
+                                  np.array([2 ** 24], np.int32)], 1, 0)
+    assert dense[0] == 2.0 ** 25
+    # (2^24 + 1) + 1 - 2^24 = 2 exactly; an fp32 running sum would give 0
+    dense = oracle.int_aggregate([np.array([2 ** 24 + 1], np.int32), np.array([1], np.int32),
+                                  np.array([-(2 ** 24)], np.int32)], 1, 0)
+    assert dense[0] == 2.0
+
+
+# --------------------------------------------------------------------------
 # multi-iteration EF: Lemma 9 (virtual iterate) per worker
 # --------------------------------------------------------------------------
 
