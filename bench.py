@@ -11,7 +11,10 @@ workload, through the whole hot path:
     same fraction of every tensor) on the same gradients, then
     sparse_aggregate of those messages;
   - sparse_aggregate_apply of the hard-threshold messages into a model and
-    momentum state (the momentum EF SGD update, fused with the exchange).
+    momentum state (the momentum EF SGD update, fused with the exchange);
+  - n x ef_scaled_round (scaled integer rounding, another absolute
+    compressor: dense int32 messages) on the same gradients, then
+    int_aggregate of those messages (exact integer sum).
 Gradients come from two pre-generated synthetic batches (alternating), so
 every step compresses different data; each step's working set (n workers x
 (g, e_ht, e_topk)) is far larger than the 126 MB L2.
@@ -282,6 +285,11 @@ def run_ours(args):
     dense_lw = torch.empty(d, device=dev)
     x_model = torch.zeros(d, device=dev)
     m_model = torch.zeros(d, device=dev)
+    e_rd = [torch.zeros(d, device=dev) for _ in range(n)]
+    q_rd = [torch.empty(d, dtype=torch.int32, device=dev) for _ in range(n)]
+    unsent_rd = torch.zeros(n, dtype=torch.int32, device=dev)
+    dense_rd = torch.empty(d, device=dev)
+    scale_log2 = 20  # grid 2^-20 for the rounding compressor
     total = args.warmup + args.steps
     cnt_ht = torch.zeros(total, n, dtype=torch.int32, device=dev)
     cnt_tk = torch.zeros(total, n, dtype=torch.int32, device=dev)
@@ -289,7 +297,7 @@ def run_ours(args):
     stream = torch.cuda.current_stream()
 
     ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
-    marks = [[ev() for _ in range(8)] for _ in range(args.steps)]
+    marks = [[ev() for _ in range(10)] for _ in range(args.steps)]
 
     err_sq = torch.zeros(3, n, dtype=torch.float64, device=dev)
 
@@ -321,6 +329,11 @@ def run_ours(args):
         efs.sparse_aggregate_apply(idx_ht, val_ht, cnt_ht[s], d, 1.0 / n, x_model, m_model, 0.9,
                                    gamma)
         if m: m[7].record(stream)
+        for i in range(n):
+            efs.ef_scaled_round(g[i], e_rd[i], gamma, scale_log2, q_rd[i], unsent_rd[i:i + 1])
+        if m: m[8].record(stream)
+        efs.int_aggregate(q_rd, d, scale_log2, dense_rd)
+        if m: m[9].record(stream)
 
     for s in range(args.warmup):
         step(s, False)
@@ -347,7 +360,7 @@ def run_ours(args):
 
     step_s = t0.elapsed_time(t1) / 1e3
     # per-iteration segment times (µs per call: the segment of n calls / n)
-    seg_us = [[m[a].elapsed_time(m[a + 1]) * 1e3 for m in marks] for a in range(7)]
+    seg_us = [[m[a].elapsed_time(m[a + 1]) * 1e3 for m in marks] for a in range(9)]
     ht_s = sum(m[0].elapsed_time(m[1]) for m in marks) / 1e3
     agg_ht_s = sum(m[1].elapsed_time(m[2]) for m in marks) / 1e3
     tk_s = sum(m[2].elapsed_time(m[3]) for m in marks) / 1e3
@@ -355,6 +368,8 @@ def run_ours(args):
     lw_s = sum(m[4].elapsed_time(m[5]) for m in marks) / 1e3
     agg_lw_s = sum(m[5].elapsed_time(m[6]) for m in marks) / 1e3
     upd_s = sum(m[6].elapsed_time(m[7]) for m in marks) / 1e3
+    rd_s = sum(m[7].elapsed_time(m[8]) for m in marks) / 1e3
+    iagg_s = sum(m[8].elapsed_time(m[9]) for m in marks) / 1e3
     counts_ht = cnt_ht[args.warmup:].double()
     counts_tk = cnt_tk[args.warmup:].double()
     bytes_ht = float(ht_bytes(d, 0) * n * args.steps + 8 * counts_ht.sum().item())
@@ -363,6 +378,8 @@ def run_ours(args):
     bytes_agg_ht = float(8 * counts_ht.sum().item() + 4 * d * args.steps)
     bytes_agg_tk = float(8 * counts_tk.sum().item() + 4 * d * args.steps)
     bytes_upd = float(8 * counts_ht.sum().item() + 16 * d * args.steps)
+    bytes_rd = float(16 * d * n * args.steps)
+    bytes_iagg = float((4 * n + 4) * d * args.steps)
 
     ht_s_max, bytes_ht_all = reduce_timing(dist, ht_s, bytes_ht, dev)
     step_s_max, _ = reduce_timing(dist, step_s, 0.0, dev)
@@ -435,6 +452,16 @@ def run_ours(args):
             "frac_of_peak": round(bytes_upd / upd_s / 1e9 / peak, 4),
             "bytes": "8 per hard-threshold pair + 16 per coordinate (x, m read and written)",
         },
+        "scaled_round": {
+            "scale_log2": scale_log2,
+            "ms_per_iter": round(rd_s / args.steps * 1e3, 4),
+            "gbs": round(bytes_rd / rd_s / 1e9, 2),
+            "frac_of_peak": round(bytes_rd / rd_s / 1e9 / peak, 4),
+            "int_aggregate_ms_per_iter": round(iagg_s / args.steps * 1e3, 4),
+            "int_aggregate_gbs": round(bytes_iagg / iagg_s / 1e9, 2),
+            "int_aggregate_frac_of_peak": round(bytes_iagg / iagg_s / 1e9 / peak, 4),
+            "bytes": "compress 16 per coordinate; exchange 4 n + 4 per coordinate",
+        },
         "per_call_us_p10_p50_p90": {
             "ht": percentiles([v / n for v in seg_us[0]]),
             "topk": percentiles([v / n for v in seg_us[2]]),
@@ -443,6 +470,8 @@ def run_ours(args):
             "aggregate_topk": percentiles(seg_us[3]),
             "aggregate_topk_layerwise": percentiles(seg_us[5]),
             "aggregate_apply_momentum": percentiles(seg_us[6]),
+            "scaled_round": percentiles([v / n for v in seg_us[7]]),
+            "int_aggregate": percentiles(seg_us[8]),
         },
         "frac_of_nominal_8tbs": round(value / NOMINAL_HBM_GBS, 4),
         "roofline": {

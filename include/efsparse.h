@@ -223,6 +223,44 @@ ef_status ef_topk_layerwise_ex(const void* g, ef_grad_type g_type, float* e, flo
                                uint32_t* count_out, double* err_sq_out, ef_stream_t stream);
 
 /*
+ * ef_scaled_round_ex — EF accumulate + scaled integer rounding + residual:
+ * another absolute compressor behind the same error-feedback step.
+ *
+ * Defines: Algorithm 1 with C = scaled integer rounding, which Sec. 5 names an
+ * absolute compressor (any rounding with error bounded by eps is one, with
+ * kappa^2 = d eps^2; the scaled integer rounding of in-network aggregation in
+ * particular). With a_j = fmaf(gamma, g_j, e_j):
+ *     q_j    = a_j 2^scale_log2 rounded to the nearest integer, ties to even (int32),
+ *     C(a)_j = q_j 2^-scale_log2,
+ *     e'_j   = a_j - C(a)_j   (exact: a == C(a) + e' bit for bit; |e'_j| <= 2^(-scale_log2-1)).
+ * A coordinate whose a_j 2^scale_log2 has magnitude at least 2^31 (or is NaN)
+ * is not sent: q_j = 0 and e'_j = a_j; such coordinates are counted.
+ *
+ *   g, g_type, e, gamma, d, err_sq_out   as for ef_hard_threshold_ex.
+ *   scale_log2 the scale exponent m, -100 <= m <= 100 (grid spacing 2^-m).
+ *   q_out      [out] int32[d], the dense integer message (4-byte aligned;
+ *              16-byte alignment of g, e and q_out selects vector access).
+ *   unsent_out [out] one uint32 in device memory: the coordinates not sent.
+ * One pass: 16 bytes per coordinate (14 with a bf16 gradient).
+ */
+ef_status ef_scaled_round_ex(const void* g, ef_grad_type g_type, float* e, float gamma,
+                             int32_t scale_log2, uint64_t d, int32_t* q_out,
+                             uint32_t* unsent_out, double* err_sq_out, ef_stream_t stream);
+
+/*
+ * int_aggregate — exchange of n workers' scaled-integer messages: the
+ * integer sum S_j = sum_i q[i][j] is exact (64-bit, so independent of the
+ * order), then dense_out[j] = S_j rounded once to fp32, times 2^-scale_log2.
+ *
+ *   n          1 <= n <= 256.
+ *   q          HOST array of n DEVICE pointers to int32[d] messages.
+ *   d, scale_log2   as for ef_scaled_round_ex.
+ *   dense_out  [out] fp32[d], not overlapping any message.
+ */
+ef_status int_aggregate(uint32_t n, const int32_t* const* q, uint64_t d, int32_t scale_log2,
+                        float* dense_out, ef_stream_t stream);
+
+/*
  * sparse_aggregate — decompress and sum n workers' sparse vectors.
  *
  * Defines: Algorithm 1's exchange step, Delta_bar = (1/n) sum_i Delta_{i,t},

@@ -18,12 +18,14 @@ from ._binding import (  # noqa: F401
     EfError,
     ef_check_status,
     ef_hard_threshold,
+    ef_scaled_round,
     ef_kernel_launches,
     ef_test_set_lookback_fault,
     ef_topk,
     ef_topk_layerwise,
     ef_workspace_release,
     library_path,
+    int_aggregate,
     load_library,
     sparse_aggregate,
     sparse_aggregate_apply,

@@ -65,6 +65,9 @@ def load_library(build_if_missing: bool = True):
             "ef_topk_ex": [vp, ctypes.c_int, vp, f32, u64, u64, vp, vp, vp, vp, vp],
             "ef_topk_layerwise_ex": [vp, ctypes.c_int, vp, f32, u32, vp, vp, u64, vp, vp, vp, vp,
                                      vp],
+            "ef_scaled_round_ex": [vp, ctypes.c_int, vp, f32, ctypes.c_int32, u64, vp, vp, vp,
+                                   vp],
+            "int_aggregate": [u32, ctypes.POINTER(vp), u64, ctypes.c_int32, vp, vp],
             "sparse_aggregate": [u32, ctypes.POINTER(vp), ctypes.POINTER(vp), vp, u64, vp, vp],
             "sparse_aggregate_apply": [u32, ctypes.POINTER(vp), ctypes.POINTER(vp), vp, u64, f32,
                                        vp, vp, f32, f32, vp],
@@ -239,6 +242,32 @@ def sparse_aggregate_apply(idx_list, val_list, counts, d, alpha, x, m=None, mome
                                       _dev(x, "x", torch.float32, d), m_ptr,
                                       ctypes.c_float(momentum), ctypes.c_float(lr),
                                       _stream(stream)), "sparse_aggregate_apply")
+
+
+def ef_scaled_round(g, e, gamma, scale_log2, q_out, unsent_out, stream=None, err_sq_out=None):
+    """EF accumulate + scaled integer rounding (``ef_scaled_round_ex``):
+    ``q_out`` int32 [d] = RNE(a 2^scale_log2), ``e`` becomes a - q 2^-scale_log2;
+    ``unsent_out`` int32 [>= 1] counts the coordinates that did not fit."""
+    lib = load_library()
+    bf16 = _gradient(g)
+    d = e.numel()
+    if g.numel() != d:
+        raise ValueError("g and e differ in length")
+    _check(lib.ef_scaled_round_ex(_dev(g, "g", g.dtype), int(bf16), _dev(e, "e", torch.float32),
+                                  ctypes.c_float(gamma), int(scale_log2), d,
+                                  _dev(q_out, "q_out", torch.int32, d),
+                                  _dev(unsent_out, "unsent_out", torch.int32, 1),
+                                  _err(err_sq_out), _stream(stream)), "ef_scaled_round_ex")
+
+
+def int_aggregate(q_list, d, scale_log2, dense_out, stream=None):
+    """Exact integer sum of n dense int32 messages, as RN(S) 2^-scale_log2."""
+    lib = load_library()
+    n = len(q_list)
+    arr = (ctypes.c_void_p * max(n, 1))(*[_dev(t, "q", torch.int32, d) for t in q_list])
+    _check(lib.int_aggregate(n, arr, int(d), int(scale_log2),
+                             _dev(dense_out, "dense_out", torch.float32, d), _stream(stream)),
+           "int_aggregate")
 
 
 def ef_check_status(stream=None) -> int:

@@ -409,6 +409,70 @@ ef_status sparse_aggregate_apply(uint32_t n, const uint32_t* const* idx, const f
                             ws);
 }
 
+ef_status ef_scaled_round_ex(const void* g, ef_grad_type g_type, float* e, float gamma,
+                             int32_t scale_log2, uint64_t d, int32_t* q_out,
+                             uint32_t* unsent_out, double* err_sq_out, ef_stream_t stream) {
+  using namespace efs;
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (g_type != EF_GRAD_F32 && g_type != EF_GRAD_BF16) return EF_ERR_INVALID_ARG;
+  const bool bf16 = g_type == EF_GRAD_BF16;
+  const size_t gsz = bf16 ? 2 : 4;
+  if (!std::isfinite(gamma) || scale_log2 < -100 || scale_log2 > 100) return EF_ERR_INVALID_ARG;
+  if (d > kMaxD || !unsent_out || !aligned(unsent_out, 4)) return EF_ERR_INVALID_ARG;
+  if (err_sq_out && !aligned(err_sq_out, 8)) return EF_ERR_INVALID_ARG;
+  if (d == 0) {
+    if (cudaMemsetAsync(unsent_out, 0, sizeof(uint32_t), s) != cudaSuccess) return EF_ERR_CUDA;
+    return write_err_zero(err_sq_out, s);
+  }
+  if (!g || !e || !q_out || !aligned(g, gsz) || !aligned(e, 4) || !aligned(q_out, 4))
+    return EF_ERR_INVALID_ARG;
+  const size_t nb = static_cast<size_t>(d) * 4;
+  if (overlaps(g, d * gsz, e, nb) || overlaps(q_out, nb, g, d * gsz) || overlaps(q_out, nb, e, nb) ||
+      overlaps(unsent_out, 4, g, d * gsz) || overlaps(unsent_out, 4, e, nb) ||
+      overlaps(unsent_out, 4, q_out, nb))
+    return EF_ERR_INVALID_ARG;
+  if (err_sq_out && (overlaps(err_sq_out, 8, g, d * gsz) || overlaps(err_sq_out, 8, e, nb) ||
+                     overlaps(err_sq_out, 8, q_out, nb) || overlaps(err_sq_out, 8, unsent_out, 4)))
+    return EF_ERR_INVALID_ARG;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
+  DeviceInfo info;
+  ef_status st = device_info(dev, &info);
+  if (st != EF_OK) return st;
+  Workspace* ws = nullptr;
+  st = acquire_workspace(s, 0, 0, 0, 0, &ws);
+  if (st != EF_OK) return st;
+  return finish_launch(launch_scaled_round(g, bf16, e, gamma, scale_log2,
+                                           static_cast<uint32_t>(d), q_out, unsent_out,
+                                           err_sq_out, *ws, info),
+                       ws);
+}
+
+ef_status int_aggregate(uint32_t n, const int32_t* const* q, uint64_t d, int32_t scale_log2,
+                        float* dense_out, ef_stream_t stream) {
+  using namespace efs;
+  if (n == 0 || n > kMaxWorkers || !q) return EF_ERR_INVALID_ARG;
+  if (d > kMaxD || scale_log2 < -100 || scale_log2 > 100) return EF_ERR_INVALID_ARG;
+  if (d == 0) return EF_OK;
+  if (!dense_out || !aligned(dense_out, 4)) return EF_ERR_INVALID_ARG;
+  for (uint32_t i = 0; i < n; ++i) {
+    if (!q[i] || !aligned(q[i], 4)) return EF_ERR_INVALID_ARG;
+    if (overlaps(q[i], static_cast<size_t>(d) * 4, dense_out, static_cast<size_t>(d) * 4))
+      return EF_ERR_INVALID_ARG;
+  }
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
+  DeviceInfo info;
+  ef_status st = device_info(dev, &info);
+  if (st != EF_OK) return st;
+  Workspace* ws = nullptr;
+  st = acquire_workspace(s, 0, 0, 0, 0, &ws);
+  if (st != EF_OK) return st;
+  return finish_launch(
+      launch_int_aggregate(n, q, static_cast<uint32_t>(d), scale_log2, dense_out, *ws, info), ws);
+}
+
 ef_status ef_check_status(ef_stream_t stream) {
   const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (cudaStreamSynchronize(s) != cudaSuccess) return EF_ERR_CUDA;

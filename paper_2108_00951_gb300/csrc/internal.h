@@ -174,6 +174,14 @@ void topk_layerwise_init_device(DeviceInfo& info);
 // their shared-memory ring on the current device and records occupancy).
 void ht_init_device(DeviceInfo& info);
 
+// Scaled integer rounding under error feedback, and the exact exchange of
+// its integer messages (round.cu).
+cudaError_t launch_scaled_round(const void* g, bool g_bf16, float* e, float gamma, int m,
+                                uint32_t d, int32_t* q, uint32_t* unsent, double* err_out,
+                                Workspace& ws, const DeviceInfo& dev);
+cudaError_t launch_int_aggregate(uint32_t n, const int32_t* const* q, uint32_t d, int m,
+                                 float* dense_out, Workspace& ws, const DeviceInfo& dev);
+
 // ||e'||^2 of e[0, d) after a step, by one plain pass (the paths that do
 // not stream through stream_compact.cuh); written to *err_out.
 cudaError_t launch_error_norm(const float* e, uint32_t d, double* err_out, Workspace& ws,
