@@ -127,7 +127,8 @@ struct Workspace {
     return align(off_counts() + sizeof(uint32_t) * kCountsPerTile * status_tiles);
   }
   size_t off_errparts() const { return align(off_chunks() + sizeof(uint64_t) * kMaxChunks); }
-  size_t off_stage() const { return align(off_errparts() + sizeof(FF) * kMaxChunks); }
+  size_t off_cntparts() const { return align(off_errparts() + sizeof(FF) * kMaxChunks); }
+  size_t off_stage() const { return align(off_cntparts() + sizeof(uint32_t) * kMaxChunks); }
   size_t total_bytes() const { return align(off_stage() + 8 * stage_cap); }
 
   uint64_t* status() const { return reinterpret_cast<uint64_t*>(base + off_status()); }
@@ -138,6 +139,7 @@ struct Workspace {
   uint32_t* counts() const { return reinterpret_cast<uint32_t*>(base + off_counts()); }
   uint64_t* chunks() const { return reinterpret_cast<uint64_t*>(base + off_chunks()); }
   FF* errparts() const { return reinterpret_cast<FF*>(base + off_errparts()); }
+  uint32_t* cntparts() const { return reinterpret_cast<uint32_t*>(base + off_cntparts()); }
   double* stream_err() const { return reinterpret_cast<double*>(base + kOffStreamErr); }
   uint32_t* stage_idx() const { return reinterpret_cast<uint32_t*>(base + off_stage()); }
   float* stage_val() const {

@@ -42,12 +42,16 @@ __device__ __forceinline__ bool round_one(float a, float scale, float unscale, i
   return true;
 }
 
+// Each CTA publishes its count of coordinates not sent (and its share of
+// ||e'||^2) and counts itself in; the last CTA to arrive writes the totals
+// (shares added in a fixed order) and resets the counter. No CTA waits.
 template <typename GT, bool kVec>
 __global__ void __launch_bounds__(kRoundThreads)
     scaled_round_kernel(const GT* __restrict__ g, float* __restrict__ e, float gamma, int m,
                         uint32_t d, int32_t* __restrict__ q, uint32_t* __restrict__ unsent,
-                        FF* err_parts, uint32_t* err_arrive, double* err_out) {
+                        uint32_t* cnt_parts, FF* err_parts, uint32_t* arrive, double* err_out) {
   __shared__ FF s_ff[32];
+  __shared__ uint32_t s_cnt[kRoundThreads / 32];
   __shared__ uint32_t s_last;
   const float scale = pow2f(m), unscale = pow2f(-m);
   const int lane = threadIdx.x & 31;
@@ -91,25 +95,40 @@ __global__ void __launch_bounds__(kRoundThreads)
       }
     }
   }
-  // the count of coordinates kept in e (an integer: any order gives the same)
   const uint32_t warp_total = warp_sum(not_sent);
-  if (lane == 0 && warp_total) atomicAdd(unsent, warp_total);
+  if (lane == 0) s_cnt[threadIdx.x >> 5] = warp_total;
+  FF share{0.0f, 0.0f};
   if (err_out) {
     acc.flush();
-    const FF share = block_sum_ff(acc.total, s_ff);
-    if (threadIdx.x == 0) {
-      err_parts[blockIdx.x] = share;
-      __threadfence();
-      s_last = atomicAdd(err_arrive, 1u) == gridDim.x - 1 ? 1u : 0u;
-    }
+    share = block_sum_ff(acc.total, s_ff);  // synchronises the CTA
+  } else {
     __syncthreads();
-    if (s_last) {  // the last CTA adds the shares in a fixed order
-      __threadfence();
-      const FF t = sum_parts_ff(err_parts, gridDim.x, s_ff);
-      if (threadIdx.x == 0) {
-        *err_out = ff_to_double(t);
-        *err_arrive = 0;  // ready for the next call
-      }
+  }
+  if (threadIdx.x == 0) {
+    uint32_t c = 0;
+    for (int w = 0; w < kRoundThreads / 32; ++w) c += s_cnt[w];
+    cnt_parts[blockIdx.x] = c;
+    if (err_out) err_parts[blockIdx.x] = share;
+    __threadfence();
+    s_last = atomicAdd(arrive, 1u) == gridDim.x - 1 ? 1u : 0u;
+  }
+  __syncthreads();
+  if (s_last) {
+    __threadfence();
+    uint32_t c = 0;
+    for (uint32_t b = threadIdx.x; b < gridDim.x; b += kRoundThreads) c += __ldcg(cnt_parts + b);
+    c = warp_sum(c);
+    __syncthreads();  // s_cnt is reused
+    if (lane == 0) s_cnt[threadIdx.x >> 5] = c;
+    FF t{0.0f, 0.0f};
+    if (err_out) t = sum_parts_ff(err_parts, gridDim.x, s_ff);  // synchronises the CTA
+    else __syncthreads();
+    if (threadIdx.x == 0) {
+      uint32_t total = 0;
+      for (int w = 0; w < kRoundThreads / 32; ++w) total += s_cnt[w];
+      *unsent = total;
+      if (err_out) *err_out = ff_to_double(t);
+      *arrive = 0;  // ready for the next call
     }
   }
 }
@@ -164,18 +183,18 @@ template <typename GT>
 cudaError_t launch_round_typed(const GT* g, float* e, float gamma, int m, uint32_t d, int32_t* q,
                                uint32_t* unsent, double* err_out, Workspace& ws,
                                const DeviceInfo& dev) {
-  cudaError_t err = cudaMemsetAsync(unsent, 0, sizeof(uint32_t), ws.stream);
-  if (err != cudaSuccess) return err;
   const bool vec = reinterpret_cast<uintptr_t>(g) % (4 * sizeof(GT)) == 0 &&
                    reinterpret_cast<uintptr_t>(e) % 16 == 0 &&
                    reinterpret_cast<uintptr_t>(q) % 16 == 0;
   const uint32_t grid = grid_for(d, dev);
   if (vec)
     scaled_round_kernel<GT, true><<<grid, kRoundThreads, 0, ws.stream>>>(
-        g, e, gamma, m, d, q, unsent, ws.errparts(), ws.u32(kOffErrArrive), err_out);
+        g, e, gamma, m, d, q, unsent, ws.cntparts(), ws.errparts(), ws.u32(kOffErrArrive),
+        err_out);
   else
     scaled_round_kernel<GT, false><<<grid, kRoundThreads, 0, ws.stream>>>(
-        g, e, gamma, m, d, q, unsent, ws.errparts(), ws.u32(kOffErrArrive), err_out);
+        g, e, gamma, m, d, q, unsent, ws.cntparts(), ws.errparts(), ws.u32(kOffErrArrive),
+        err_out);
   count_launch();
   return cudaGetLastError();
 }
