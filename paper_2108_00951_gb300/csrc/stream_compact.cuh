@@ -174,7 +174,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   };
   const bool producer = warp == kProducerWarp && lane == 0;
   if (producer) {
-    policy = l2_evict_first_policy();
+    policy = l2_evict_normal_policy();
     for (uint32_t r = 0; r < rounds && r < static_cast<uint32_t>(kStages); ++r) fill(r);
   }
 

@@ -42,11 +42,12 @@ def g_device(g: np.ndarray, offset=0) -> torch.Tensor:
     return to_dev(g, offset)
 
 
-def ht(g, e, gamma, lam, g_off=0, e_off=0, stream=None):
+def ht(g, e, gamma, lam, g_off=0, e_off=0, stream=None, out_off=(0, 0)):
     d = e.size
     gd, ed = g_device(g, g_off), to_dev(e, e_off)
-    idx = torch.full((max(d, 1),), -1, dtype=torch.int32, device=DEV)
-    val = torch.empty(max(d, 1), dtype=torch.float32, device=DEV)
+    # outputs `out_off` elements past an allocation boundary
+    idx = torch.full((max(d, 1) + out_off[0],), -1, dtype=torch.int32, device=DEV)[out_off[0]:]
+    val = torch.empty(max(d, 1) + out_off[1], dtype=torch.float32, device=DEV)[out_off[1]:]
     cnt = torch.full((1,), -1, dtype=torch.int32, device=DEV)
     efs.ef_hard_threshold(gd, ed, gamma, lam, idx, val, cnt, stream=stream)
     torch.cuda.synchronize()

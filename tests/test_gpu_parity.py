@@ -158,6 +158,20 @@ def test_ht_spill_mixed_density():
     _check_same((i, v, en), oracle.ef_hard_threshold(g, e, 0.1, 0.05), "mixed")
 
 
+@pytest.mark.parametrize("out_off", [(1, 0), (2, 3), (3, 1)])
+def test_ht_misaligned_outputs(out_off):
+    # the pairs are written with 16-byte stores matched to each output's own
+    # alignment; dense (several buffer pieces per CTA) and sparse chunks
+    g, e = _inputs(SPILL_D, 24)
+    g[: SPILL_D // 3] *= 1000.0
+    _check_same(gu.ht(g, e, 0.1, 0.05, out_off=out_off), oracle.ef_hard_threshold(g, e, 0.1, 0.05),
+                "outputs offset %s" % (out_off,))
+    d = 4096 + 77
+    g, e = _inputs(d, 25)
+    _check_same(gu.ht(g, e, 0.1, 1e-3, out_off=out_off), oracle.ef_hard_threshold(g, e, 0.1, 1e-3),
+                "small, outputs offset %s" % (out_off,))
+
+
 @pytest.mark.parametrize("region,k", [(SPILL_D // 50, 20_000), (SPILL_D // 5, SPILL_D // 16)])
 def test_topk_spill_concentrated_candidates(region, k):
     # all candidates in the first `region` coordinates: the few CTAs there
