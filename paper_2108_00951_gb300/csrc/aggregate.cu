@@ -78,37 +78,90 @@ __device__ __forceinline__ void apply_update(const AggOut& o, float s, float& x,
   }
 }
 
+// 4-byte asynchronous copy global -> shared (no register staging).
+__device__ __forceinline__ void cp_async_4(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(
+                   static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
+               "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.wait_all;" ::: "memory");
+}
+
 template <bool kVec, int kMode>
 __global__ void __launch_bounds__(kThreads)
     agg_reduce_kernel(AggPtrs p, uint32_t n, uint32_t d, uint32_t tiles,
                       const uint32_t* __restrict__ off, AggOut o,
                       uint32_t* __restrict__ error) {
   __shared__ __align__(16) float acc[kAggTile];
-  __shared__ uint32_t s_lo[kMaxWorkers], s_hi[kMaxWorkers];
+  __shared__ uint32_t s_lo[kMaxWorkers], s_pre[kMaxWorkers + 1];
+  __shared__ uint32_t st_idx[kAggStage];
+  __shared__ float st_val[kAggStage];
   const uint32_t t = blockIdx.x;
+  const int lane = threadIdx.x & 31;
   const uint64_t j0 = static_cast<uint64_t>(t) * kAggTile;
   for (int q = threadIdx.x; q < kAggTile / 4; q += kThreads)
     reinterpret_cast<float4*>(acc)[q] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
   for (uint32_t i = threadIdx.x; i < n; i += kThreads) {
-    s_lo[i] = off[static_cast<uint64_t>(i) * (tiles + 1) + t];
-    s_hi[i] = off[static_cast<uint64_t>(i) * (tiles + 1) + t + 1];
+    const uint32_t lo = off[static_cast<uint64_t>(i) * (tiles + 1) + t];
+    const uint32_t hi = off[static_cast<uint64_t>(i) * (tiles + 1) + t + 1];
+    s_lo[i] = lo;
+    s_pre[i + 1] = hi > lo ? hi - lo : 0u;  // this tile's pairs of worker i
+  }
+  __syncthreads();
+  if (threadIdx.x < 32) {  // s_pre: the tile's pairs of the workers before each one
+    uint32_t carry = 0;
+    for (uint32_t i0 = 0; i0 < n; i0 += 32) {
+      const uint32_t i = i0 + lane;
+      uint32_t v = i < n ? s_pre[i + 1] : 0u;
+#pragma unroll
+      for (int o2 = 1; o2 < 32; o2 <<= 1) {
+        const uint32_t x = __shfl_up_sync(0xffffffffu, v, o2);
+        if (lane >= o2) v += x;
+      }
+      if (i < n) s_pre[i + 1] = carry + v;
+      carry += __shfl_sync(0xffffffffu, v, 31);
+    }
+    if (lane == 0) s_pre[0] = 0;
   }
   __syncthreads();
   bool bad = false;
-  for (uint32_t i = 0; i < n; ++i) {
-    const uint32_t lo = s_lo[i], hi = s_hi[i];
-    if (lo >= hi) continue;  // uniform across the CTA
-    const uint32_t* __restrict__ xi = p.idx[i];
-    const float* __restrict__ vi = p.val[i];
-    for (uint32_t q = lo + threadIdx.x; q < hi; q += kThreads) {
-      const uint32_t j = __ldg(xi + q);
-      const uint64_t r = static_cast<uint64_t>(j) - j0;  // wraps when j < j0
-      if (r < kAggTile && j < d)
-        acc[r] += __ldg(vi + q);
-      else
-        bad = true;  // unsorted or out-of-range input: skipped, latched
+  const uint32_t total = s_pre[n];
+  // The tile's pairs of all workers, in worker order, a stage at a time:
+  // every copy of a stage is in flight at once (one round trip), then the
+  // stage is added worker by worker, with a barrier between workers so that
+  // each coordinate receives its contributions in worker order.
+  for (uint32_t b0 = 0; b0 < total; b0 += kAggStage) {
+    const uint32_t bn = total - b0 < kAggStage ? total - b0 : kAggStage;
+    {
+      uint32_t i = 0;
+      for (uint32_t q = threadIdx.x; q < bn; q += kThreads) {
+        const uint32_t gp = b0 + q;
+        while (s_pre[i + 1] <= gp) ++i;
+        const uint32_t src = s_lo[i] + (gp - s_pre[i]);
+        cp_async_4(st_idx + q, p.idx[i] + src);
+        cp_async_4(st_val + q, p.val[i] + src);
+      }
     }
+    cp_async_wait_all();
     __syncthreads();
+    uint32_t i = 0;
+    while (s_pre[i + 1] <= b0) ++i;  // the stage's first worker (uniform)
+    for (; i < n && s_pre[i] < b0 + bn; ++i) {
+      const uint32_t a = (s_pre[i] > b0 ? s_pre[i] : b0) - b0;
+      const uint32_t z = (s_pre[i + 1] < b0 + bn ? s_pre[i + 1] : b0 + bn) - b0;
+      if (a >= z) continue;  // uniform: no pairs of worker i here
+      for (uint32_t q = a + threadIdx.x; q < z; q += kThreads) {
+        const uint32_t j = st_idx[q];
+        const uint64_t r = static_cast<uint64_t>(j) - j0;  // wraps when j < j0
+        if (r < kAggTile && j < d)
+          acc[r] += st_val[q];
+        else
+          bad = true;  // unsorted or out-of-range input: skipped, latched
+      }
+      __syncthreads();
+    }
   }
   if (bad) atomicOr(error, kDevErrBadInput);
   if (kVec && j0 + kAggTile <= d) {
@@ -185,6 +238,20 @@ cudaError_t launch_common(uint32_t n, const uint32_t* const* idx, const float* c
   return cudaGetLastError();
 }
 }  // namespace
+
+void aggregate_init_device() {
+  const void* fns[] = {
+      reinterpret_cast<const void*>(&agg_reduce_kernel<true, kAggDense>),
+      reinterpret_cast<const void*>(&agg_reduce_kernel<false, kAggDense>),
+      reinterpret_cast<const void*>(&agg_reduce_kernel<true, kAggSgd>),
+      reinterpret_cast<const void*>(&agg_reduce_kernel<false, kAggSgd>),
+      reinterpret_cast<const void*>(&agg_reduce_kernel<true, kAggMomentum>),
+      reinterpret_cast<const void*>(&agg_reduce_kernel<false, kAggMomentum>)};
+  for (const void* f : fns)
+    cudaFuncSetAttribute(f, cudaFuncAttributePreferredSharedMemoryCarveout,
+                         cudaSharedmemCarveoutMaxShared);
+  cudaGetLastError();
+}
 
 cudaError_t launch_aggregate(uint32_t n, const uint32_t* const* idx, const float* const* val,
                              const uint32_t* counts, uint32_t d, float* dense_out,

@@ -42,6 +42,7 @@ ef_status device_info(int dev, DeviceInfo* out) {
     ht_init_device(info);
     topk_init_device(info);
     topk_layerwise_init_device(info);
+    aggregate_init_device();
     if (info.refine_blocks <= 0 || info.finalize_blocks <= 0) return EF_ERR_CUDA;
     it = g_devices.emplace(dev, info).first;
   }
@@ -374,6 +375,10 @@ ef_status sparse_aggregate(uint32_t n, const uint32_t* const* idx, const float* 
       return EF_ERR_INVALID_ARG;
   const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const uint32_t tiles = efs::agg_tiles_for(d);
+  int dev = 0;  // the per-device set-up (kernel attributes) on first use
+  efs::DeviceInfo info;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
+  if (efs::device_info(dev, &info) != EF_OK) return EF_ERR_CUDA;
   Workspace* ws = nullptr;
   const ef_status st = efs::acquire_workspace(
       s, 0, 0, static_cast<size_t>(n) * (static_cast<size_t>(tiles) + 1), 0, &ws);
@@ -399,6 +404,10 @@ ef_status sparse_aggregate_apply(uint32_t n, const uint32_t* const* idx, const f
       return EF_ERR_INVALID_ARG;
   const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const uint32_t tiles = efs::agg_tiles_for(d);
+  int dev = 0;  // the per-device set-up (kernel attributes) on first use
+  efs::DeviceInfo info;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
+  if (efs::device_info(dev, &info) != EF_OK) return EF_ERR_CUDA;
   Workspace* ws = nullptr;
   const ef_status st = efs::acquire_workspace(
       s, 0, 0, static_cast<size_t>(n) * (static_cast<size_t>(tiles) + 1), 0, &ws);

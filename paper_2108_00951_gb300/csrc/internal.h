@@ -172,6 +172,10 @@ void topk_init_device(DeviceInfo& info);
 // Per-device set-up of the layer-wise Top-k kernels.
 void topk_layerwise_init_device(DeviceInfo& info);
 
+// Per-device set-up of the aggregation kernels (prefer the largest shared
+// memory carve-out, so that 8 of their CTAs are resident per SM).
+void aggregate_init_device();
+
 // Per-device set-up of the streaming hard-threshold kernels (opts them into
 // their shared-memory ring on the current device and records occupancy).
 void ht_init_device(DeviceInfo& info);
@@ -229,6 +233,7 @@ inline uint32_t tiles_for(uint64_t d) {
   return static_cast<uint32_t>((d + kTileElems - 1) / kTileElems);
 }
 constexpr int kAggTile = 4096;             // dense elements per aggregation CTA
+constexpr int kAggStage = 1024;            // pairs an aggregation CTA stages per round trip
 constexpr uint32_t kMaxWorkers = 256;
 inline uint32_t agg_tiles_for(uint64_t d) {
   return static_cast<uint32_t>((d + kAggTile - 1) / kAggTile);
