@@ -285,6 +285,28 @@ def test_aggregate_empty_lists_and_misaligned_output():
                        oracle.sparse_aggregate(idx, val, d), "off=%d" % off)
 
 
+def test_aggregate_tile_boundary_layouts():
+    # lists with long runs of empty tiles, lists inside one tile, a list that
+    # ends in the first tile, one that starts in the last, the last coordinate,
+    # entries on tile boundaries: every per-tile offset pattern of the lists
+    d = 300 * 4096 + 123
+    rng = np.random.default_rng(31)
+    lists = [
+        np.array([0, 4095, 4096, 8191, 8192], np.uint32),
+        np.array([d - 1], np.uint32),
+        np.array([7], np.uint32),
+        np.sort(rng.choice(np.arange(150 * 4096, 151 * 4096), 900, replace=False)).astype(np.uint32),
+        np.array([5, 250 * 4096, d - 2], np.uint32),
+        np.arange(299 * 4096, d, 3, dtype=np.uint32),
+        np.zeros(0, np.uint32),
+        np.sort(rng.choice(d, 20_000, replace=False)).astype(np.uint32),
+    ]
+    vals = [rng.standard_normal(len(x)).astype(np.float32) for x in lists]
+    gu.assert_bits(gu.aggregate(lists, vals, d), oracle.sparse_aggregate(lists, vals, d),
+                   "tile layouts")
+    assert efs.ef_check_status() == efs.EF_OK
+
+
 # ------------------------------------------------------- multi-iteration EF
 @pytest.mark.parametrize("method", ["ht", "topk"])
 def test_lr_workload_all_iterations(method):
