@@ -36,6 +36,8 @@ struct AggPtrs {
 __global__ void __launch_bounds__(kThreads)
     agg_offsets_kernel(AggPtrs p, const uint32_t* __restrict__ counts, uint32_t n,
                        uint32_t tiles, uint32_t* __restrict__ off) {
+  griddep_wait();                // the lists and counts come from the kernels before
+  griddep_launch_dependents();    // the reduction may be scheduled (it waits for this grid)
   const uint64_t per = static_cast<uint64_t>(tiles) + 1;
   const uint64_t gid = static_cast<uint64_t>(blockIdx.x) * kThreads + threadIdx.x;
   if (gid >= per * n) return;
@@ -89,6 +91,11 @@ __device__ __forceinline__ void cp_async_wait_all() {
   asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
+// Bulk prefetch of [p, p + bytes) into L2 (16-byte aligned, bytes % 16 == 0).
+__device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
 template <bool kVec, int kMode>
 __global__ void __launch_bounds__(kThreads)
     agg_reduce_kernel(AggPtrs p, uint32_t n, uint32_t d, uint32_t tiles,
@@ -103,6 +110,15 @@ __global__ void __launch_bounds__(kThreads)
   const uint64_t j0 = static_cast<uint64_t>(t) * kAggTile;
   for (int q = threadIdx.x; q < kAggTile / 4; q += kThreads)
     reinterpret_cast<float4*>(acc)[q] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+  if constexpr (kMode != kAggDense) {
+    // the tile's x (and m), read by the epilogue, on their way to L2 while
+    // the pairs are gathered (a prefetch: no data moves into the CTA)
+    if (kVec && threadIdx.x == 0 && j0 + kAggTile <= d) {
+      prefetch_l2_bulk(o.out + j0, kAggTile * sizeof(float));
+      if constexpr (kMode == kAggMomentum) prefetch_l2_bulk(o.m + j0, kAggTile * sizeof(float));
+    }
+  }
+  griddep_wait();  // the offsets (and everything before them) are complete
   for (uint32_t i = threadIdx.x; i < n; i += kThreads) {
     const uint32_t lo = off[static_cast<uint64_t>(i) * (tiles + 1) + t];
     const uint32_t hi = off[static_cast<uint64_t>(i) * (tiles + 1) + t + 1];
@@ -200,14 +216,13 @@ __global__ void __launch_bounds__(kThreads)
 }
 
 template <int kMode>
-void launch_reduce(bool vec, const AggPtrs& p, uint32_t n, uint32_t d, uint32_t tiles,
-                   const uint32_t* off, const AggOut& o, Workspace& ws) {
-  if (vec)
-    agg_reduce_kernel<true, kMode><<<tiles, kThreads, 0, ws.stream>>>(p, n, d, tiles, off, o,
-                                                                      ws.u32(kOffError));
-  else
-    agg_reduce_kernel<false, kMode><<<tiles, kThreads, 0, ws.stream>>>(p, n, d, tiles, off, o,
-                                                                       ws.u32(kOffError));
+cudaError_t launch_reduce(bool vec, AggPtrs p, uint32_t n, uint32_t d, uint32_t tiles,
+                          const uint32_t* off, AggOut o, Workspace& ws) {
+  uint32_t* error = ws.u32(kOffError);
+  void* params[] = {&p, &n, &d, &tiles, &off, &o, &error};
+  const void* fn = vec ? reinterpret_cast<const void*>(&agg_reduce_kernel<true, kMode>)
+                       : reinterpret_cast<const void*>(&agg_reduce_kernel<false, kMode>);
+  return launch_pdl(fn, tiles, kThreads, 0, ws.stream, params, false);
 }
 
 cudaError_t launch_common(uint32_t n, const uint32_t* const* idx, const float* const* val,
@@ -222,20 +237,23 @@ cudaError_t launch_common(uint32_t n, const uint32_t* const* idx, const float* c
   const uint64_t entries = static_cast<uint64_t>(n) * (tiles + 1);
   const uint32_t grid1 = static_cast<uint32_t>((entries + kThreads - 1) / kThreads);
   uint32_t* off = ws.offsets();
-  agg_offsets_kernel<<<grid1, kThreads, 0, ws.stream>>>(p, counts, n, tiles, off);
+  const uint32_t* counts_arg = counts;
+  uint32_t n_arg = n, tiles_arg = tiles;
+  void* params[] = {&p, &counts_arg, &n_arg, &tiles_arg, &off};
+  cudaError_t err = launch_pdl(reinterpret_cast<const void*>(&agg_offsets_kernel), grid1,
+                               kThreads, 0, ws.stream, params, false);
   count_launch();
-  cudaError_t err = cudaGetLastError();
   if (err != cudaSuccess) return err;
   const bool vec = reinterpret_cast<uintptr_t>(o.out) % 16 == 0 &&
                    reinterpret_cast<uintptr_t>(o.m) % 16 == 0;
   if (mode == kAggDense)
-    launch_reduce<kAggDense>(vec, p, n, d, tiles, off, o, ws);
+    err = launch_reduce<kAggDense>(vec, p, n, d, tiles, off, o, ws);
   else if (mode == kAggSgd)
-    launch_reduce<kAggSgd>(vec, p, n, d, tiles, off, o, ws);
+    err = launch_reduce<kAggSgd>(vec, p, n, d, tiles, off, o, ws);
   else
-    launch_reduce<kAggMomentum>(vec, p, n, d, tiles, off, o, ws);
+    err = launch_reduce<kAggMomentum>(vec, p, n, d, tiles, off, o, ws);
   count_launch();
-  return cudaGetLastError();
+  return err;
 }
 }  // namespace
 

@@ -263,6 +263,26 @@ ef_status topk_layerwise_entry(const void* g, bool bf16, float* e, float gamma, 
 
 }  // namespace
 
+// A launch that may begin while the previous kernel on the stream finishes
+// (programmatic dependent launch; every kernel here waits for its
+// predecessor before reading what it wrote), optionally cooperative.
+cudaError_t launch_pdl(const void* fn, uint32_t grid, uint32_t block, uint32_t smem,
+                       cudaStream_t stream, void** params, bool cooperative) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(block);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeCooperative;
+  attr[1].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = cooperative ? 2 : 1;
+  return cudaLaunchKernelExC(&cfg, fn, params);
+}
+
 void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 uint64_t wait_limit_ns() { return g_wait_limit_ns.load(); }
 int64_t withheld_tile() { return g_withheld_tile.load(); }

@@ -768,26 +768,6 @@ int lw_stream_blocks_per_sm() {
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
-// A launch that may begin while the previous kernel on the stream finishes
-// (programmatic dependent launch; every kernel here waits for its
-// predecessor before reading what it wrote), optionally cooperative.
-cudaError_t launch_pdl(const void* fn, uint32_t grid, uint32_t block, uint32_t smem,
-                       cudaStream_t stream, void** params, bool cooperative) {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(block);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = stream;
-  cudaLaunchAttribute attr[2];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  attr[1].id = cudaLaunchAttributeCooperative;
-  attr[1].val.cooperative = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = cooperative ? 2 : 1;
-  return cudaLaunchKernelExC(&cfg, fn, params);
-}
-
 // Work estimate of a segment's selection by one CTA, in positions handled.
 uint64_t select_cost(const LwSeg& s) {
   const uint64_t ds = s.hi - s.lo;
