@@ -59,6 +59,7 @@ __global__ void __launch_bounds__(kRoundThreads)
   const uint64_t stride = static_cast<uint64_t>(gridDim.x) * kRoundThreads;
   ErrAcc acc;
   uint32_t not_sent = 0;
+  griddep_wait();  // g and e may come from the kernels before (programmatic launch)
   for (uint64_t gi = static_cast<uint64_t>(blockIdx.x) * kRoundThreads + threadIdx.x;
        gi < groups; gi += stride) {
     const uint64_t j0 = gi * 4;
@@ -95,6 +96,7 @@ __global__ void __launch_bounds__(kRoundThreads)
       }
     }
   }
+  griddep_launch_dependents();  // the next kernel may be scheduled (it waits for this grid)
   const uint32_t warp_total = warp_sum(not_sent);
   if (lane == 0) s_cnt[threadIdx.x >> 5] = warp_total;
   FF share{0.0f, 0.0f};
@@ -143,6 +145,8 @@ __global__ void __launch_bounds__(kRoundThreads)
   const float unscale = pow2f(-m);
   const uint64_t groups = (static_cast<uint64_t>(d) + 3) / 4;
   const uint64_t stride = static_cast<uint64_t>(gridDim.x) * kRoundThreads;
+  griddep_wait();  // the messages come from the kernels before (programmatic launch)
+  griddep_launch_dependents();
   for (uint64_t gi = static_cast<uint64_t>(blockIdx.x) * kRoundThreads + threadIdx.x;
        gi < groups; gi += stride) {
     const uint64_t j0 = gi * 4;
@@ -189,16 +193,15 @@ cudaError_t launch_round_typed(const GT* g, float* e, float gamma, int m, uint32
                    reinterpret_cast<uintptr_t>(e) % 16 == 0 &&
                    reinterpret_cast<uintptr_t>(q) % 16 == 0;
   const uint32_t grid = grid_for(d, dev);
-  if (vec)
-    scaled_round_kernel<GT, true><<<grid, kRoundThreads, 0, ws.stream>>>(
-        g, e, gamma, m, d, q, unsent, ws.cntparts(), ws.errparts(), ws.u32(kOffErrArrive),
-        err_out);
-  else
-    scaled_round_kernel<GT, false><<<grid, kRoundThreads, 0, ws.stream>>>(
-        g, e, gamma, m, d, q, unsent, ws.cntparts(), ws.errparts(), ws.u32(kOffErrArrive),
-        err_out);
+  uint32_t* cnt_parts = ws.cntparts();
+  FF* err_parts = ws.errparts();
+  uint32_t* arrive = ws.u32(kOffErrArrive);
+  void* params[] = {&g, &e, &gamma, &m, &d, &q, &unsent, &cnt_parts, &err_parts, &arrive, &err_out};
+  const void* fn = vec ? reinterpret_cast<const void*>(&scaled_round_kernel<GT, true>)
+                       : reinterpret_cast<const void*>(&scaled_round_kernel<GT, false>);
+  const cudaError_t err = launch_pdl(fn, grid, kRoundThreads, 0, ws.stream, params, false);
   count_launch();
-  return cudaGetLastError();
+  return err;
 }
 
 }  // namespace
@@ -222,12 +225,12 @@ cudaError_t launch_int_aggregate(uint32_t n, const int32_t* const* q, uint32_t d
     if (i < n && reinterpret_cast<uintptr_t>(q[i]) % 16 != 0) vec = false;
   }
   const uint32_t grid = grid_for(d, dev);
-  if (vec)
-    int_aggregate_kernel<true><<<grid, kRoundThreads, 0, ws.stream>>>(p, n, d, m, dense_out);
-  else
-    int_aggregate_kernel<false><<<grid, kRoundThreads, 0, ws.stream>>>(p, n, d, m, dense_out);
+  void* params[] = {&p, &n, &d, &m, &dense_out};
+  const void* fn = vec ? reinterpret_cast<const void*>(&int_aggregate_kernel<true>)
+                       : reinterpret_cast<const void*>(&int_aggregate_kernel<false>);
+  const cudaError_t err = launch_pdl(fn, grid, kRoundThreads, 0, ws.stream, params, false);
   count_launch();
-  return cudaGetLastError();
+  return err;
 }
 
 }  // namespace efs

@@ -684,6 +684,7 @@ __global__ void __launch_bounds__(kSelThreads, 1)
   extern __shared__ __align__(16) uint32_t s_mag[];
   __shared__ uint32_t s_hist[kHistBins];
   __shared__ uint32_t s_w[kSelThreads / 32];
+  griddep_wait();  // the streaming pass (and all before it) is complete
   const SourceInfo si = read_source(args, d, k);
   if (k == 0 || si.failed) {
     if (blockIdx.x == 0 && threadIdx.x == 0) {
@@ -884,10 +885,9 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
     StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks(), nullptr,
                   err_out ? ws.stream_err() : nullptr, ws.errparts()};
     void* params[] = {&op, &d, &args.list_idx, &args.list_val, &args.list_count, &cap, &ctx, &sa};
-    err = cudaLaunchCooperativeKernel(
-        reinterpret_cast<const void*>(&stream_compact_kernel<TopkCandOp<GT>, kTkStages>),
-        dim3(grid), dim3(kStreamThreads), params, StreamLayout<TopkCandOp<GT>, kTkStages>::kSmem,
-        ws.stream);
+    err = launch_pdl(
+        reinterpret_cast<const void*>(&stream_compact_kernel<TopkCandOp<GT>, kTkStages>), grid,
+        kStreamThreads, StreamLayout<TopkCandOp<GT>, kTkStages>::kSmem, ws.stream, params, true);
     count_launch();
     if (err != cudaSuccess) return err;
   } else {
@@ -905,8 +905,8 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
                     (void*)&count_out, (void*)&args};
   uint32_t grid = static_cast<uint32_t>(dev.refine_blocks);
   if (grid > kMaxChunks) grid = kMaxChunks;
-  err = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(&topk_select_kernel),
-                                    dim3(grid), dim3(kSelThreads), params, kSelSmem, ws.stream);
+  err = launch_pdl(reinterpret_cast<const void*>(&topk_select_kernel), grid, kSelThreads,
+                   kSelSmem, ws.stream, params, true);
   count_launch();
   if (err == cudaSuccess && err_out && !streamable) err = launch_error_norm(e, d, err_out, ws, dev);
   return err;
