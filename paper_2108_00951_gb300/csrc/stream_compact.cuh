@@ -316,6 +316,56 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
     }
     st_relaxed_u64(sa.chunk_sums + c, (static_cast<uint64_t>(ctx.epoch) << 32) | sum);
   }
+  // The chunk's segments, a window at a time (the ring is free now): their
+  // counts and their warps' earlier pairs (coalesced loads; a segment was
+  // staged on chip iff the two add up to at most the warp's share), an
+  // exclusive scan of the counts into offsets within the window, then, once
+  // the chunk's base is known, the copy. The first window is prepared before
+  // the wait for the earlier chunks' totals, which hides its loads.
+  const uint32_t lo = t_lo * kSWarps, hi = t_hi * kSWarps;
+  uint32_t* seg_off = reinterpret_cast<uint32_t*>(smem);
+  uint32_t* seg_pos = seg_off + L::kChunkSegs;  // the warp's earlier pairs
+  constexpr int kNumWarps = kStreamThreads / 32;
+  constexpr int kCopySegs = 8;
+  // per thread: its contiguous run [rb, re) of the window, the run's offset
+  // within the window, and the window's total
+  uint32_t rb = 0, re = 0, run_off = 0, window_total = 0;
+  auto prepare = [&](uint32_t w0, uint32_t n) {
+    __syncthreads();  // the previous window's copy is done with the arrays
+    for (uint32_t i = threadIdx.x; i < n; i += kStreamThreads) {
+      const uint32_t packed = __ldcg(sa.counts + w0 + i);
+      seg_off[i] = packed & 0x1ffu;
+      seg_pos[i] = packed >> 9;
+    }
+    __syncthreads();
+    const uint32_t per = (n + kStreamThreads - 1) / kStreamThreads;
+    rb = threadIdx.x * per < n ? threadIdx.x * per : n;
+    re = rb + per < n ? rb + per : n;
+    uint32_t run = 0;
+    for (uint32_t i = rb; i < re; ++i) {
+      const uint32_t cnt = seg_off[i];
+      seg_off[i] = run;
+      run += cnt;
+    }
+    uint32_t incl = run;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    if (lane == 31) s_scratch[warp] = incl;
+    __syncthreads();
+    uint32_t warp_base = 0, total = 0;
+    for (int w = 0; w < kNumWarps; ++w) {
+      const uint32_t x = s_scratch[w];
+      warp_base += w < warp ? x : 0u;
+      total += x;
+    }
+    run_off = warp_base + incl - run;
+    window_total = total;
+  };
+  prepare(lo, hi - lo < L::kChunkSegs ? hi - lo : L::kChunkSegs);
+
   // sum of the earlier chunks' totals, waiting (bounded) for missing ones
   uint32_t base = 0;
   {
@@ -357,52 +407,12 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
       }
     }
   }
-  const uint32_t lo = t_lo * kSWarps, hi = t_hi * kSWarps;
-
-  // The chunk's segments, a window at a time (the ring is free now): their
-  // counts and their warps' earlier pairs (coalesced loads; a segment was
-  // staged on chip iff the two add up to at most the warp's share), an
-  // exclusive scan of the counts into output offsets, then the copy.
-  uint32_t* seg_off = reinterpret_cast<uint32_t*>(smem);
-  uint32_t* seg_pos = seg_off + L::kChunkSegs;  // the warp's earlier pairs
-  constexpr int kNumWarps = kStreamThreads / 32;
-  constexpr int kCopySegs = 8;
   bool overflow = false;
   for (uint32_t w0 = lo; w0 < hi; w0 += L::kChunkSegs) {
     const uint32_t n = hi - w0 < L::kChunkSegs ? hi - w0 : L::kChunkSegs;
-    __syncthreads();
-    for (uint32_t i = threadIdx.x; i < n; i += kStreamThreads) {
-      const uint32_t packed = __ldcg(sa.counts + w0 + i);
-      seg_off[i] = packed & 0x1ffu;
-      seg_pos[i] = packed >> 9;
-    }
-    __syncthreads();
-    // each thread scans a contiguous run of the window in shared memory
-    const uint32_t per = (n + kStreamThreads - 1) / kStreamThreads;
-    const uint32_t b = threadIdx.x * per < n ? threadIdx.x * per : n;
-    const uint32_t e = b + per < n ? b + per : n;
-    uint32_t run = 0;
-    for (uint32_t i = b; i < e; ++i) {
-      const uint32_t cnt = seg_off[i];
-      seg_off[i] = run;
-      run += cnt;
-    }
-    uint32_t incl = run;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const uint32_t v = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += v;
-    }
-    if (lane == 31) s_scratch[warp] = incl;
-    __syncthreads();
-    uint32_t warp_base = 0, window_total = 0;
-    for (int w = 0; w < kNumWarps; ++w) {
-      const uint32_t x = s_scratch[w];
-      warp_base += w < warp ? x : 0u;
-      window_total += x;
-    }
-    const uint32_t thread_base = base + warp_base + incl - run;
-    for (uint32_t i = b; i < e; ++i) {
+    if (w0 != lo) prepare(w0, n);
+    const uint32_t thread_base = base + run_off;
+    for (uint32_t i = rb; i < re; ++i) {
       seg_off[i] += thread_base;
       // windows start at whole tiles, so a tile's first segment has i % kSWarps == 0
       if (sa.tile_base && i % kSWarps == 0) sa.tile_base[(w0 + i) / kSWarps] = seg_off[i];
