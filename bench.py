@@ -278,6 +278,9 @@ def run_ours(args):
     e_tk = [torch.zeros(d, device=dev) for _ in range(n)]
     e_lw = [torch.zeros(d, device=dev) for _ in range(n)]
     idx_ht, val_ht = outputs(d)
+    # the hard-threshold messages' tile indexes, written by the compress calls
+    # and read by the aggregations of those messages
+    tiles_ht = [torch.empty(efs.tiles_for(d), dtype=torch.int32, device=dev) for _ in range(n)]
     idx_tk, val_tk = outputs(k)
     idx_lw, val_lw = outputs(k_lw)
     dense_ht = torch.empty(d, device=dev)
@@ -310,9 +313,9 @@ def run_ours(args):
         if m: m[0].record(stream)
         for i in range(n):
             efs.ef_hard_threshold(g[i], e_ht[i], gamma, lam, idx_ht[i], val_ht[i],
-                                  cnt_ht[s, i:i + 1], **errkw(0, i))
+                                  cnt_ht[s, i:i + 1], tiles_out=tiles_ht[i], **errkw(0, i))
         if m: m[1].record(stream)
-        efs.sparse_aggregate(idx_ht, val_ht, cnt_ht[s], d, dense_ht)
+        efs.sparse_aggregate(idx_ht, val_ht, cnt_ht[s], d, dense_ht, tiles=tiles_ht)
         if m: m[2].record(stream)
         for i in range(n):
             efs.ef_topk(g[i], e_tk[i], gamma, k, idx_tk[i], val_tk[i], cnt_tk[s, i:i + 1],
@@ -327,7 +330,7 @@ def run_ours(args):
         efs.sparse_aggregate(idx_lw, val_lw, cnt_lw[s], d, dense_lw)
         if m: m[6].record(stream)
         efs.sparse_aggregate_apply(idx_ht, val_ht, cnt_ht[s], d, 1.0 / n, x_model, m_model, 0.9,
-                                   gamma)
+                                   gamma, tiles=tiles_ht)
         if m: m[7].record(stream)
         for i in range(n):
             efs.ef_scaled_round(g[i], e_rd[i], gamma, scale_log2, q_rd[i], unsent_rd[i:i + 1])
@@ -434,6 +437,7 @@ def run_ours(args):
         "topk_gbs": round(bytes_tk / tk_s / 1e9, 2),
         "topk_frac_of_peak": round(bytes_tk / tk_s / 1e9 / peak, 4),
         "aggregate_ms_per_iter": round(agg_ht_s / args.steps * 1e3, 4),
+        "aggregate_tile_index": "hard-threshold messages: from the compress calls; Top-k: searched",
         "aggregate_gbs": round(bytes_agg_ht / agg_ht_s / 1e9, 2),
         "aggregate_frac_of_peak": round(bytes_agg_ht / agg_ht_s / 1e9 / peak, 4),
         "aggregate_topk_ms_per_iter": round(agg_tk_s / args.steps * 1e3, 4),
@@ -451,6 +455,7 @@ def run_ours(args):
             "gbs": round(bytes_upd / upd_s / 1e9, 2),
             "frac_of_peak": round(bytes_upd / upd_s / 1e9 / peak, 4),
             "bytes": "8 per hard-threshold pair + 16 per coordinate (x, m read and written)",
+            "tile_index": "the messages' tile indexes written by the compress calls",
         },
         "scaled_round": {
             "scale_log2": scale_log2,
@@ -513,6 +518,7 @@ def run_e2e(args, efs, torch, dev, dist, grads, d, n, gamma, lam, stream):
     e = [torch.zeros(d, device=dev) for _ in range(n)]
     idx = [torch.empty(d, dtype=torch.int32, device=dev) for _ in range(n)]
     val = [torch.empty(d, dtype=torch.float32, device=dev) for _ in range(n)]
+    tiles = [torch.empty(efs.tiles_for(d), dtype=torch.int32, device=dev) for _ in range(n)]
     cnt = torch.zeros(args.steps + args.warmup, n, dtype=torch.int32, device=dev)
     dense = [torch.empty(d, device=dev) for _ in range(2)]
     up, down = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
@@ -536,10 +542,10 @@ def run_e2e(args, efs, torch, dev, dist, grads, d, n, gamma, lam, stream):
         for i in range(n):
             stream.wait_event(uploaded[b][i])
             efs.ef_hard_threshold(dev_g[b][i], e[i], gamma, lam, idx[i], val[i],
-                                  cnt[s, i:i + 1], stream=stream)
+                                  cnt[s, i:i + 1], stream=stream, tiles_out=tiles[i])
             consumed[b][i].record(stream)
         stream.wait_event(fetched[b])
-        efs.sparse_aggregate(idx, val, cnt[s], d, dense[b], stream=stream)
+        efs.sparse_aggregate(idx, val, cnt[s], d, dense[b], stream=stream, tiles=tiles)
         reduced[b].record(stream)
         with torch.cuda.stream(down):
             down.wait_event(reduced[b])

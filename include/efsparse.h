@@ -320,6 +320,49 @@ ef_status sparse_aggregate_apply(uint32_t n, const uint32_t* const* idx,
                                  float momentum, float lr, ef_stream_t stream);
 
 /*
+ * Tile index of a sparse message (an implementation device; the paper's
+ * messages are the (index, value) lists alone). The coordinates [0, d) are cut
+ * into T = ceil(d / EF_TILE) tiles of EF_TILE coordinates; a message's tile
+ * index is uint32[T + 1] with
+ *     tiles[t] = the number of its pairs with index < EF_TILE * t, t < T,
+ *     tiles[T] = its count.
+ * The aggregation works tile by tile and otherwise finds these positions by a
+ * binary search of every list at every tile boundary (one more kernel, whose
+ * chains of dependent loads make it latency-bound); the hard-threshold kernel
+ * knows them as it places the pairs and writes them for T + 1 words. A worker
+ * can send the tile index with its message (4 (T + 1) bytes against 8 bytes per
+ * pair).
+ *
+ * ef_hard_threshold_tiled — ef_hard_threshold_ex (identical outputs) that also
+ * writes the message's tile index.
+ *   tiles_out  [out] uint32[ceil(d / EF_TILE) + 1], 4-byte aligned, device,
+ *              not overlapping any other argument; required (non-NULL).
+ *
+ * sparse_aggregate_tiled, sparse_aggregate_apply_tiled — sparse_aggregate and
+ * sparse_aggregate_apply (identical outputs for well-formed input) given the
+ * lists' tile indexes.
+ *   tiles      HOST array of n DEVICE pointers; tiles[i] is list i's tile index
+ *              (uint32[ceil(d / EF_TILE) + 1], 4-byte aligned).
+ * A tile index that does not match its list never causes an out-of-bounds
+ * access: every position is clamped to [0, counts[i]], and a pair read for a
+ * tile it does not belong to is skipped and latches EF_ERR_BAD_INPUT.
+ */
+#define EF_TILE 4096
+ef_status ef_hard_threshold_tiled(const void* g, ef_grad_type g_type, float* e, float gamma,
+                                  float lambda, uint64_t d, uint32_t* idx_out, float* val_out,
+                                  uint32_t* count_out, uint32_t* tiles_out, double* err_sq_out,
+                                  ef_stream_t stream);
+ef_status sparse_aggregate_tiled(uint32_t n, const uint32_t* const* idx,
+                                 const float* const* val, const uint32_t* const* tiles,
+                                 const uint32_t* counts, uint64_t d, float* dense_out,
+                                 ef_stream_t stream);
+ef_status sparse_aggregate_apply_tiled(uint32_t n, const uint32_t* const* idx,
+                                       const float* const* val, const uint32_t* const* tiles,
+                                       const uint32_t* counts, uint64_t d, float alpha,
+                                       float* x, float* m, float momentum, float lr,
+                                       ef_stream_t stream);
+
+/*
  * ef_hard_threshold_noalloc — ef_hard_threshold for callers that cannot
  * allocate device memory. (An implementation convenience; the paper has no
  * counterpart.)

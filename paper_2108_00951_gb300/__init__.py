@@ -15,6 +15,7 @@ from ._binding import (  # noqa: F401
     EF_ERR_NO_MEMORY,
     EF_ERR_TIMEOUT,
     EF_OK,
+    TILE,
     EfError,
     ef_check_status,
     ef_hard_threshold,
@@ -30,4 +31,5 @@ from ._binding import (  # noqa: F401
     sparse_aggregate,
     sparse_aggregate_apply,
     status_string,
+    tiles_for,
 )

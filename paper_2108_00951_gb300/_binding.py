@@ -71,6 +71,13 @@ def load_library(build_if_missing: bool = True):
             "sparse_aggregate": [u32, ctypes.POINTER(vp), ctypes.POINTER(vp), vp, u64, vp, vp],
             "sparse_aggregate_apply": [u32, ctypes.POINTER(vp), ctypes.POINTER(vp), vp, u64, f32,
                                        vp, vp, f32, f32, vp],
+            "ef_hard_threshold_tiled": [vp, ctypes.c_int, vp, f32, f32, u64, vp, vp, vp, vp, vp,
+                                        vp],
+            "sparse_aggregate_tiled": [u32, ctypes.POINTER(vp), ctypes.POINTER(vp),
+                                       ctypes.POINTER(vp), vp, u64, vp, vp],
+            "sparse_aggregate_apply_tiled": [u32, ctypes.POINTER(vp), ctypes.POINTER(vp),
+                                             ctypes.POINTER(vp), vp, u64, f32, vp, vp, f32, f32,
+                                             vp],
             "ef_check_status": [vp],
             "ef_workspace_release": [],
         }
@@ -129,15 +136,25 @@ def _err(err_sq_out):
     return _dev(err_sq_out, "err_sq_out", torch.float64, 1)
 
 
+TILE = 4096  # coordinates per tile of a message's tile index
+
+
+def tiles_for(d: int) -> int:
+    """Length of a message's tile index for dimension d: ceil(d / TILE) + 1."""
+    return (int(d) + TILE - 1) // TILE + 1
+
+
 def ef_hard_threshold(g, e, gamma, lam, idx_out, val_out, count_out, stream=None,
-                      err_sq_out=None):
+                      err_sq_out=None, tiles_out=None):
     """EF accumulate + hard-threshold + compaction (``ef_hard_threshold[_bf16]``;
-    ``ef_hard_threshold_ex`` when ``err_sq_out`` is given).
+    ``ef_hard_threshold_ex`` when ``err_sq_out`` is given,
+    ``ef_hard_threshold_tiled`` when ``tiles_out`` is given).
 
     ``g`` float32 or bfloat16 [d]; ``e`` float32 [d], updated in place;
     ``idx_out`` int32 [>= d] (uint32 bit patterns), ``val_out`` float32 [>= d],
     ``count_out`` int32 [>= 1]; ``err_sq_out`` optional float64 [>= 1]:
-    ||e'||^2 of the step.
+    ||e'||^2 of the step; ``tiles_out`` optional int32 [>= tiles_for(d)]: the
+    message's tile index (pairs below each multiple of TILE, then the count).
     """
     lib = load_library()
     bf16 = _gradient(g)
@@ -148,6 +165,12 @@ def ef_hard_threshold(g, e, gamma, lam, idx_out, val_out, count_out, stream=None
             ctypes.c_float(lam), d, _dev(idx_out, "idx_out", torch.int32, d),
             _dev(val_out, "val_out", torch.float32, d),
             _dev(count_out, "count_out", torch.int32, 1))
+    if tiles_out is not None:
+        _check(lib.ef_hard_threshold_tiled(
+            head[0], int(bf16), *head[1:], _dev(tiles_out, "tiles_out", torch.int32, tiles_for(d)),
+            ctypes.c_void_p(0) if err_sq_out is None else _err(err_sq_out), _stream(stream)),
+            "ef_hard_threshold_tiled")
+        return
     if err_sq_out is not None:
         _check(lib.ef_hard_threshold_ex(head[0], int(bf16), *head[1:], _err(err_sq_out),
                                         _stream(stream)), "ef_hard_threshold_ex")
@@ -207,11 +230,19 @@ def ef_topk_layerwise(g, e, gamma, seg_end, seg_k, idx_out, val_out, count_out, 
     _check(fn(*head, _stream(stream)), "ef_topk_layerwise")
 
 
-def sparse_aggregate(idx_list, val_list, counts, d, dense_out, stream=None):
+def _tile_array(tiles, n, d):
+    if len(tiles) != n:
+        raise ValueError("one tile index per list")
+    return (ctypes.c_void_p * max(n, 1))(*[_dev(t, "tiles", torch.int32, tiles_for(d))
+                                           for t in tiles])
+
+
+def sparse_aggregate(idx_list, val_list, counts, d, dense_out, stream=None, tiles=None):
     """Worker-ordered sum of n sparse vectors into ``dense_out`` (float32 [d]).
 
     ``idx_list``/``val_list``: n int32 / float32 CUDA tensors; ``counts``: int32
-    CUDA tensor of n pair counts.
+    CUDA tensor of n pair counts; ``tiles`` optional: the n lists' tile indexes
+    (``sparse_aggregate_tiled``).
     """
     lib = load_library()
     n = len(idx_list)
@@ -219,17 +250,23 @@ def sparse_aggregate(idx_list, val_list, counts, d, dense_out, stream=None):
         raise ValueError("idx_list and val_list differ in length")
     idx_arr = (ctypes.c_void_p * max(n, 1))(*[_dev(t, "idx", torch.int32) for t in idx_list])
     val_arr = (ctypes.c_void_p * max(n, 1))(*[_dev(t, "val", torch.float32) for t in val_list])
-    _check(lib.sparse_aggregate(n, idx_arr, val_arr, _dev(counts, "counts", torch.int32, n),
-                                int(d), _dev(dense_out, "dense_out", torch.float32, d),
-                                _stream(stream)), "sparse_aggregate")
+    cnt = _dev(counts, "counts", torch.int32, n)
+    out = _dev(dense_out, "dense_out", torch.float32, d)
+    if tiles is not None:
+        _check(lib.sparse_aggregate_tiled(n, idx_arr, val_arr, _tile_array(tiles, n, d), cnt,
+                                          int(d), out, _stream(stream)), "sparse_aggregate_tiled")
+        return
+    _check(lib.sparse_aggregate(n, idx_arr, val_arr, cnt, int(d), out, _stream(stream)),
+           "sparse_aggregate")
 
 
 def sparse_aggregate_apply(idx_list, val_list, counts, d, alpha, x, m=None, momentum=0.0, lr=0.0,
-                           stream=None):
+                           stream=None, tiles=None):
     """Worker-ordered sum of n sparse vectors, scaled by ``alpha``, applied to
     the model ``x`` (float32 [d], in place): ``x -= Delta'`` without ``m``;
     with ``m`` (float32 [d], in place) ``m = fmaf(momentum, m, Delta')`` and
-    ``x = fmaf(-lr, Delta' + m, x)``."""
+    ``x = fmaf(-lr, Delta' + m, x)``. ``tiles`` optional: the lists' tile
+    indexes (``sparse_aggregate_apply_tiled``)."""
     lib = load_library()
     n = len(idx_list)
     if n != len(val_list):
@@ -237,11 +274,14 @@ def sparse_aggregate_apply(idx_list, val_list, counts, d, alpha, x, m=None, mome
     idx_arr = (ctypes.c_void_p * max(n, 1))(*[_dev(t, "idx", torch.int32) for t in idx_list])
     val_arr = (ctypes.c_void_p * max(n, 1))(*[_dev(t, "val", torch.float32) for t in val_list])
     m_ptr = ctypes.c_void_p(0) if m is None else _dev(m, "m", torch.float32, d)
-    _check(lib.sparse_aggregate_apply(n, idx_arr, val_arr, _dev(counts, "counts", torch.int32, n),
-                                      int(d), ctypes.c_float(alpha),
-                                      _dev(x, "x", torch.float32, d), m_ptr,
-                                      ctypes.c_float(momentum), ctypes.c_float(lr),
-                                      _stream(stream)), "sparse_aggregate_apply")
+    tail = (_dev(counts, "counts", torch.int32, n), int(d), ctypes.c_float(alpha),
+            _dev(x, "x", torch.float32, d), m_ptr, ctypes.c_float(momentum), ctypes.c_float(lr),
+            _stream(stream))
+    if tiles is not None:
+        _check(lib.sparse_aggregate_apply_tiled(n, idx_arr, val_arr, _tile_array(tiles, n, d),
+                                                *tail), "sparse_aggregate_apply_tiled")
+        return
+    _check(lib.sparse_aggregate_apply(n, idx_arr, val_arr, *tail), "sparse_aggregate_apply")
 
 
 def ef_scaled_round(g, e, gamma, scale_log2, q_out, unsent_out, stream=None, err_sq_out=None):

@@ -29,6 +29,7 @@ namespace {
 struct AggPtrs {
   const uint32_t* idx[kMaxWorkers];
   const float* val[kMaxWorkers];
+  const uint32_t* tiles[kMaxWorkers];  // the lists' tile indexes, when the caller has them
 };
 
 // off[i * (tiles + 1) + t] = number of entries of list i below t * kAggTile;
@@ -99,8 +100,8 @@ __device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes) 
 template <bool kVec, int kMode>
 __global__ void __launch_bounds__(kThreads)
     agg_reduce_kernel(AggPtrs p, uint32_t n, uint32_t d, uint32_t tiles,
-                      const uint32_t* __restrict__ off, AggOut o,
-                      uint32_t* __restrict__ error) {
+                      const uint32_t* __restrict__ off, const uint32_t* __restrict__ counts,
+                      AggOut o, uint32_t* __restrict__ error) {
   __shared__ __align__(16) float acc[kAggTile];
   __shared__ uint32_t s_lo[kMaxWorkers], s_pre[kMaxWorkers + 1];
   __shared__ uint32_t st_idx[kAggStage];
@@ -120,8 +121,15 @@ __global__ void __launch_bounds__(kThreads)
   }
   griddep_wait();  // the offsets (and everything before them) are complete
   for (uint32_t i = threadIdx.x; i < n; i += kThreads) {
-    const uint32_t lo = off[static_cast<uint64_t>(i) * (tiles + 1) + t];
-    const uint32_t hi = off[static_cast<uint64_t>(i) * (tiles + 1) + t + 1];
+    // the list's range in this tile: from the offsets kernel, or from the
+    // caller's tile index (clamped to the list, so never out of bounds)
+    const uint32_t* r = off ? off + static_cast<uint64_t>(i) * (tiles + 1) : p.tiles[i];
+    uint32_t lo = r[t], hi = r[t + 1];
+    if (!off) {
+      const uint32_t cnt = counts[i];
+      lo = min(lo, cnt);
+      hi = min(hi, cnt);
+    }
     s_lo[i] = lo;
     s_pre[i + 1] = hi > lo ? hi - lo : 0u;  // this tile's pairs of worker i
   }
@@ -217,41 +225,46 @@ __global__ void __launch_bounds__(kThreads)
 
 template <int kMode>
 cudaError_t launch_reduce(bool vec, AggPtrs p, uint32_t n, uint32_t d, uint32_t tiles,
-                          const uint32_t* off, AggOut o, Workspace& ws) {
+                          const uint32_t* off, const uint32_t* counts, AggOut o, Workspace& ws) {
   uint32_t* error = ws.u32(kOffError);
-  void* params[] = {&p, &n, &d, &tiles, &off, &o, &error};
+  void* params[] = {&p, &n, &d, &tiles, &off, &counts, &o, &error};
   const void* fn = vec ? reinterpret_cast<const void*>(&agg_reduce_kernel<true, kMode>)
                        : reinterpret_cast<const void*>(&agg_reduce_kernel<false, kMode>);
   return launch_pdl(fn, tiles, kThreads, 0, ws.stream, params, false);
 }
 
 cudaError_t launch_common(uint32_t n, const uint32_t* const* idx, const float* const* val,
-                          const uint32_t* counts, uint32_t d, const AggOut& o, int mode,
-                          Workspace& ws) {
+                          const uint32_t* const* tile_index, const uint32_t* counts, uint32_t d,
+                          const AggOut& o, int mode, Workspace& ws) {
   AggPtrs p;
   for (uint32_t i = 0; i < kMaxWorkers; ++i) {
     p.idx[i] = i < n ? idx[i] : nullptr;
     p.val[i] = i < n ? val[i] : nullptr;
+    p.tiles[i] = i < n && tile_index ? tile_index[i] : nullptr;
   }
   const uint32_t tiles = agg_tiles_for(d);
-  const uint64_t entries = static_cast<uint64_t>(n) * (tiles + 1);
-  const uint32_t grid1 = static_cast<uint32_t>((entries + kThreads - 1) / kThreads);
-  uint32_t* off = ws.offsets();
-  const uint32_t* counts_arg = counts;
-  uint32_t n_arg = n, tiles_arg = tiles;
-  void* params[] = {&p, &counts_arg, &n_arg, &tiles_arg, &off};
-  cudaError_t err = launch_pdl(reinterpret_cast<const void*>(&agg_offsets_kernel), grid1,
-                               kThreads, 0, ws.stream, params, false);
-  count_launch();
-  if (err != cudaSuccess) return err;
+  cudaError_t err = cudaSuccess;
+  uint32_t* off = nullptr;
+  if (!tile_index) {  // locate each list's tile boundaries first
+    const uint64_t entries = static_cast<uint64_t>(n) * (tiles + 1);
+    const uint32_t grid1 = static_cast<uint32_t>((entries + kThreads - 1) / kThreads);
+    off = ws.offsets();
+    const uint32_t* counts_arg = counts;
+    uint32_t n_arg = n, tiles_arg = tiles;
+    void* params[] = {&p, &counts_arg, &n_arg, &tiles_arg, &off};
+    err = launch_pdl(reinterpret_cast<const void*>(&agg_offsets_kernel), grid1, kThreads, 0,
+                     ws.stream, params, false);
+    count_launch();
+    if (err != cudaSuccess) return err;
+  }
   const bool vec = reinterpret_cast<uintptr_t>(o.out) % 16 == 0 &&
                    reinterpret_cast<uintptr_t>(o.m) % 16 == 0;
   if (mode == kAggDense)
-    err = launch_reduce<kAggDense>(vec, p, n, d, tiles, off, o, ws);
+    err = launch_reduce<kAggDense>(vec, p, n, d, tiles, off, counts, o, ws);
   else if (mode == kAggSgd)
-    err = launch_reduce<kAggSgd>(vec, p, n, d, tiles, off, o, ws);
+    err = launch_reduce<kAggSgd>(vec, p, n, d, tiles, off, counts, o, ws);
   else
-    err = launch_reduce<kAggMomentum>(vec, p, n, d, tiles, off, o, ws);
+    err = launch_reduce<kAggMomentum>(vec, p, n, d, tiles, off, counts, o, ws);
   count_launch();
   return err;
 }
@@ -272,18 +285,35 @@ void aggregate_init_device() {
 }
 
 cudaError_t launch_aggregate(uint32_t n, const uint32_t* const* idx, const float* const* val,
-                             const uint32_t* counts, uint32_t d, float* dense_out,
-                             Workspace& ws) {
-  return launch_common(n, idx, val, counts, d, AggOut{dense_out, nullptr, 1.0f, 0.0f, 0.0f},
-                       kAggDense, ws);
+                             const uint32_t* const* tiles, const uint32_t* counts, uint32_t d,
+                             float* dense_out, Workspace& ws) {
+  return launch_common(n, idx, val, tiles, counts, d,
+                       AggOut{dense_out, nullptr, 1.0f, 0.0f, 0.0f}, kAggDense, ws);
 }
 
 cudaError_t launch_aggregate_apply(uint32_t n, const uint32_t* const* idx,
-                                   const float* const* val, const uint32_t* counts, uint32_t d,
-                                   float alpha, float* x, float* m, float mu, float lr,
-                                   Workspace& ws) {
-  return launch_common(n, idx, val, counts, d, AggOut{x, m, alpha, mu, lr},
+                                   const float* const* val, const uint32_t* const* tiles,
+                                   const uint32_t* counts, uint32_t d, float alpha, float* x,
+                                   float* m, float mu, float lr, Workspace& ws) {
+  return launch_common(n, idx, val, tiles, counts, d, AggOut{x, m, alpha, mu, lr},
                        m ? kAggMomentum : kAggSgd, ws);
+}
+
+cudaError_t launch_list_tiles(const uint32_t* idx, const uint32_t* count, uint32_t d,
+                              uint32_t* tiles_out, Workspace& ws) {
+  AggPtrs p;
+  for (uint32_t i = 0; i < kMaxWorkers; ++i) {
+    p.idx[i] = i == 0 ? idx : nullptr;
+    p.val[i] = nullptr;
+    p.tiles[i] = nullptr;
+  }
+  uint32_t n = 1, tiles = agg_tiles_for(d);
+  const uint32_t grid = (tiles + 1 + kThreads - 1) / kThreads;
+  void* params[] = {&p, &count, &n, &tiles, &tiles_out};
+  const cudaError_t err = launch_pdl(reinterpret_cast<const void*>(&agg_offsets_kernel), grid,
+                                     kThreads, 0, ws.stream, params, false);
+  count_launch();
+  return err;
 }
 
 }  // namespace efs

@@ -121,14 +121,17 @@ ef_status write_err_zero(double* err_out, cudaStream_t stream) {
 
 ef_status hard_threshold_entry(const void* g, bool bf16, float* e, float gamma, float lambda,
                                uint64_t d, uint32_t* idx_out, float* val_out,
-                               uint32_t* count_out, double* err_out, cudaStream_t stream) {
+                               uint32_t* count_out, double* err_out, uint32_t* tiles_out,
+                               cudaStream_t stream) {
   const size_t gsz = bf16 ? 2 : 4;
   if (!count_out || !aligned(count_out, 4)) return EF_ERR_INVALID_ARG;
   if (!std::isfinite(gamma) || !(lambda >= 0.0f)) return EF_ERR_INVALID_ARG;
   if (d > kMaxD) return EF_ERR_INVALID_ARG;
   if (err_out && !aligned(err_out, 8)) return EF_ERR_INVALID_ARG;
+  if (tiles_out && !aligned(tiles_out, 4)) return EF_ERR_INVALID_ARG;
   if (d == 0) {
-    const ef_status z = write_zero_count(count_out, stream);
+    ef_status z = write_zero_count(count_out, stream);
+    if (z == EF_OK && tiles_out) z = write_zero_count(tiles_out, stream);  // one entry: 0
     return z != EF_OK ? z : write_err_zero(err_out, stream);
   }
   if (!g || !e || !idx_out || !val_out) return EF_ERR_INVALID_ARG;
@@ -157,8 +160,15 @@ ef_status hard_threshold_entry(const void* g, bool bf16, float* e, float gamma, 
                   overlaps(err_out, 8, idx_out, nb) || overlaps(err_out, 8, val_out, nb) ||
                   overlaps(err_out, 8, count_out, 4)))
     return EF_ERR_INVALID_ARG;
+  const size_t tb = (static_cast<size_t>(tiles_for(d)) + 1) * 4;
+  if (tiles_out && (overlaps(tiles_out, tb, e, nb) || overlaps(tiles_out, tb, g, d * gsz) ||
+                    overlaps(tiles_out, tb, idx_out, nb) || overlaps(tiles_out, tb, val_out, nb) ||
+                    overlaps(tiles_out, tb, count_out, 4) ||
+                    (err_out && overlaps(tiles_out, tb, err_out, 8))))
+    return EF_ERR_INVALID_ARG;
   return finish_launch(launch_hard_threshold(g, bf16, e, gamma, lambda, static_cast<uint32_t>(d),
-                                             idx_out, val_out, count_out, err_out, *ws, info),
+                                             idx_out, val_out, count_out, err_out, tiles_out, *ws,
+                                             info),
                        ws);
 }
 
@@ -304,6 +314,48 @@ ScanCtx next_scan_ctx(Workspace& ws, uint32_t num_tiles) {
   return c;
 }
 
+// The aggregate entries: the plain sum (dense_out set) or the fused update
+// (x set); tiles optional.
+ef_status aggregate_entry(uint32_t n, const uint32_t* const* idx, const float* const* val,
+                          const uint32_t* const* tiles, const uint32_t* counts, uint64_t d,
+                          float* dense_out, float alpha, float* x, float* m, float momentum,
+                          float lr, cudaStream_t s) {
+  if (n == 0 || n > kMaxWorkers || !idx || !val || !counts) return EF_ERR_INVALID_ARG;
+  if (d > kMaxD) return EF_ERR_INVALID_ARG;
+  const bool apply = x != nullptr;
+  if (apply && (!std::isfinite(alpha) || !std::isfinite(momentum) || !std::isfinite(lr)))
+    return EF_ERR_INVALID_ARG;
+  if (d == 0) return EF_OK;
+  const size_t nb = static_cast<size_t>(d) * 4;
+  if (!aligned(counts, 4)) return EF_ERR_INVALID_ARG;
+  if (apply) {
+    if (!aligned(x, 4) || (m && !aligned(m, 4))) return EF_ERR_INVALID_ARG;
+    if (m && overlaps(x, nb, m, nb)) return EF_ERR_INVALID_ARG;
+  } else if (!dense_out || !aligned(dense_out, 4)) {
+    return EF_ERR_INVALID_ARG;
+  }
+  for (uint32_t i = 0; i < n; ++i) {
+    if (!idx[i] || !val[i] || !aligned(idx[i], 4) || !aligned(val[i], 4))
+      return EF_ERR_INVALID_ARG;
+    if (tiles && (!tiles[i] || !aligned(tiles[i], 4))) return EF_ERR_INVALID_ARG;
+  }
+  const uint32_t nt = agg_tiles_for(d);
+  int dev = 0;  // the per-device set-up (kernel attributes) on first use
+  DeviceInfo info;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
+  if (device_info(dev, &info) != EF_OK) return EF_ERR_CUDA;
+  Workspace* ws = nullptr;
+  const size_t offsets = tiles ? 0 : static_cast<size_t>(n) * (static_cast<size_t>(nt) + 1);
+  const ef_status st = acquire_workspace(s, 0, 0, offsets, 0, &ws);
+  if (st != EF_OK) return st;
+  const uint32_t d32 = static_cast<uint32_t>(d);
+  if (apply)
+    return finish_launch(
+        launch_aggregate_apply(n, idx, val, tiles, counts, d32, alpha, x, m, momentum, lr, *ws),
+        ws);
+  return finish_launch(launch_aggregate(n, idx, val, tiles, counts, d32, dense_out, *ws), ws);
+}
+
 }  // namespace efs
 
 using efs::Workspace;
@@ -314,14 +366,14 @@ ef_status ef_hard_threshold(const float* g, float* e, float gamma, float lambda,
                             uint32_t* idx_out, float* val_out, uint32_t* count_out,
                             ef_stream_t stream) {
   return efs::hard_threshold_entry(g, false, e, gamma, lambda, d, idx_out, val_out, count_out,
-                                   nullptr, reinterpret_cast<cudaStream_t>(stream));
+                                   nullptr, nullptr, reinterpret_cast<cudaStream_t>(stream));
 }
 
 ef_status ef_hard_threshold_bf16(const uint16_t* g, float* e, float gamma, float lambda,
                                  uint64_t d, uint32_t* idx_out, float* val_out,
                                  uint32_t* count_out, ef_stream_t stream) {
   return efs::hard_threshold_entry(g, true, e, gamma, lambda, d, idx_out, val_out, count_out,
-                                   nullptr, reinterpret_cast<cudaStream_t>(stream));
+                                   nullptr, nullptr, reinterpret_cast<cudaStream_t>(stream));
 }
 
 ef_status ef_topk(const float* g, float* e, float gamma, uint64_t k, uint64_t d,
@@ -360,7 +412,18 @@ ef_status ef_hard_threshold_ex(const void* g, ef_grad_type g_type, float* e, flo
                                uint32_t* count_out, double* err_sq_out, ef_stream_t stream) {
   if (g_type != EF_GRAD_F32 && g_type != EF_GRAD_BF16) return EF_ERR_INVALID_ARG;
   return efs::hard_threshold_entry(g, g_type == EF_GRAD_BF16, e, gamma, lambda, d, idx_out,
-                                   val_out, count_out, err_sq_out,
+                                   val_out, count_out, err_sq_out, nullptr,
+                                   reinterpret_cast<cudaStream_t>(stream));
+}
+
+ef_status ef_hard_threshold_tiled(const void* g, ef_grad_type g_type, float* e, float gamma,
+                                  float lambda, uint64_t d, uint32_t* idx_out, float* val_out,
+                                  uint32_t* count_out, uint32_t* tiles_out, double* err_sq_out,
+                                  ef_stream_t stream) {
+  if (g_type != EF_GRAD_F32 && g_type != EF_GRAD_BF16) return EF_ERR_INVALID_ARG;
+  if (!tiles_out) return EF_ERR_INVALID_ARG;
+  return efs::hard_threshold_entry(g, g_type == EF_GRAD_BF16, e, gamma, lambda, d, idx_out,
+                                   val_out, count_out, err_sq_out, tiles_out,
                                    reinterpret_cast<cudaStream_t>(stream));
 }
 
@@ -385,57 +448,33 @@ ef_status ef_topk_layerwise_ex(const void* g, ef_grad_type g_type, float* e, flo
 ef_status sparse_aggregate(uint32_t n, const uint32_t* const* idx, const float* const* val,
                            const uint32_t* counts, uint64_t d, float* dense_out,
                            ef_stream_t stream) {
-  if (n == 0 || n > efs::kMaxWorkers || !idx || !val || !counts) return EF_ERR_INVALID_ARG;
-  if (d > efs::kMaxD) return EF_ERR_INVALID_ARG;
-  if (d == 0) return EF_OK;
-  if (!dense_out || !efs::aligned(dense_out, 4) || !efs::aligned(counts, 4))
-    return EF_ERR_INVALID_ARG;
-  for (uint32_t i = 0; i < n; ++i)
-    if (!idx[i] || !val[i] || !efs::aligned(idx[i], 4) || !efs::aligned(val[i], 4))
-      return EF_ERR_INVALID_ARG;
-  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  const uint32_t tiles = efs::agg_tiles_for(d);
-  int dev = 0;  // the per-device set-up (kernel attributes) on first use
-  efs::DeviceInfo info;
-  if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
-  if (efs::device_info(dev, &info) != EF_OK) return EF_ERR_CUDA;
-  Workspace* ws = nullptr;
-  const ef_status st = efs::acquire_workspace(
-      s, 0, 0, static_cast<size_t>(n) * (static_cast<size_t>(tiles) + 1), 0, &ws);
-  if (st != EF_OK) return st;
-  return efs::finish_launch(
-      efs::launch_aggregate(n, idx, val, counts, static_cast<uint32_t>(d), dense_out, *ws), ws);
+  return efs::aggregate_entry(n, idx, val, nullptr, counts, d, dense_out, 0.0f, nullptr,
+                              nullptr, 0.0f, 0.0f, reinterpret_cast<cudaStream_t>(stream));
+}
+
+ef_status sparse_aggregate_tiled(uint32_t n, const uint32_t* const* idx, const float* const* val,
+                                 const uint32_t* const* tiles, const uint32_t* counts, uint64_t d,
+                                 float* dense_out, ef_stream_t stream) {
+  if (!tiles) return EF_ERR_INVALID_ARG;
+  return efs::aggregate_entry(n, idx, val, tiles, counts, d, dense_out, 0.0f, nullptr, nullptr,
+                              0.0f, 0.0f, reinterpret_cast<cudaStream_t>(stream));
 }
 
 ef_status sparse_aggregate_apply(uint32_t n, const uint32_t* const* idx, const float* const* val,
                                  const uint32_t* counts, uint64_t d, float alpha, float* x,
                                  float* m, float momentum, float lr, ef_stream_t stream) {
-  if (n == 0 || n > efs::kMaxWorkers || !idx || !val || !counts) return EF_ERR_INVALID_ARG;
-  if (d > efs::kMaxD) return EF_ERR_INVALID_ARG;
-  if (!std::isfinite(alpha) || !std::isfinite(momentum) || !std::isfinite(lr))
-    return EF_ERR_INVALID_ARG;
-  if (d == 0) return EF_OK;
-  if (!x || !efs::aligned(x, 4) || !efs::aligned(counts, 4) || (m && !efs::aligned(m, 4)))
-    return EF_ERR_INVALID_ARG;
-  if (m && efs::overlaps(x, static_cast<size_t>(d) * 4, m, static_cast<size_t>(d) * 4))
-    return EF_ERR_INVALID_ARG;
-  for (uint32_t i = 0; i < n; ++i)
-    if (!idx[i] || !val[i] || !efs::aligned(idx[i], 4) || !efs::aligned(val[i], 4))
-      return EF_ERR_INVALID_ARG;
-  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  const uint32_t tiles = efs::agg_tiles_for(d);
-  int dev = 0;  // the per-device set-up (kernel attributes) on first use
-  efs::DeviceInfo info;
-  if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
-  if (efs::device_info(dev, &info) != EF_OK) return EF_ERR_CUDA;
-  Workspace* ws = nullptr;
-  const ef_status st = efs::acquire_workspace(
-      s, 0, 0, static_cast<size_t>(n) * (static_cast<size_t>(tiles) + 1), 0, &ws);
-  if (st != EF_OK) return st;
-  return efs::finish_launch(efs::launch_aggregate_apply(n, idx, val, counts,
-                                                        static_cast<uint32_t>(d), alpha, x, m,
-                                                        momentum, lr, *ws),
-                            ws);
+  if (!x) return EF_ERR_INVALID_ARG;
+  return efs::aggregate_entry(n, idx, val, nullptr, counts, d, nullptr, alpha, x, m, momentum,
+                              lr, reinterpret_cast<cudaStream_t>(stream));
+}
+
+ef_status sparse_aggregate_apply_tiled(uint32_t n, const uint32_t* const* idx,
+                                       const float* const* val, const uint32_t* const* tiles,
+                                       const uint32_t* counts, uint64_t d, float alpha, float* x,
+                                       float* m, float momentum, float lr, ef_stream_t stream) {
+  if (!tiles || !x) return EF_ERR_INVALID_ARG;
+  return efs::aggregate_entry(n, idx, val, tiles, counts, d, nullptr, alpha, x, m, momentum, lr,
+                              reinterpret_cast<cudaStream_t>(stream));
 }
 
 ef_status ef_scaled_round_ex(const void* g, ef_grad_type g_type, float* e, float gamma,

@@ -159,7 +159,7 @@ using HtStreamKernel = StreamLayout<HtOp<GT>, kHtStages>;
 template <typename GT>
 cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint32_t d,
                          uint32_t* idx_out, float* val_out, uint32_t* count_out, double* err_out,
-                         Workspace& ws, const DeviceInfo& dev) {
+                         uint32_t* tiles_out, Workspace& ws, const DeviceInfo& dev) {
   const uint32_t tiles = tiles_for(d);
   const ScanCtx ctx = next_scan_ctx(ws, tiles);
   const uintptr_t ga = reinterpret_cast<uintptr_t>(g), ea = reinterpret_cast<uintptr_t>(e);
@@ -172,7 +172,8 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
     const uint32_t grid = tiles < slots ? tiles : slots;
     uint32_t cap = d;
     ScanCtx c = ctx;
-    StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks(), nullptr, err_out,
+    // the placement writes each tile's first output position (the tile index)
+    StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks(), tiles_out, err_out,
                   ws.errparts()};
     void* params[] = {&op, &d, &idx_out, &val_out, &count_out, &cap, &c, &sa};
     // A plain launch suffices: the only cross-CTA wait is on lower-numbered
@@ -204,6 +205,7 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
   count_launch();
   cudaError_t err = cudaGetLastError();
   if (err == cudaSuccess && err_out) err = launch_error_norm(e, d, err_out, ws, dev);
+  if (err == cudaSuccess && tiles_out) err = launch_list_tiles(idx_out, count_out, d, tiles_out, ws);
   return err;
 }
 
@@ -248,13 +250,13 @@ cudaError_t launch_hard_threshold_lookback(const float* g, float* e, float gamma
 
 cudaError_t launch_hard_threshold(const void* g, bool g_bf16, float* e, float gamma,
                                   float lambda, uint32_t d, uint32_t* idx_out, float* val_out,
-                                  uint32_t* count_out, double* err_out, Workspace& ws,
-                                  const DeviceInfo& dev) {
+                                  uint32_t* count_out, double* err_out, uint32_t* tiles_out,
+                                  Workspace& ws, const DeviceInfo& dev) {
   if (g_bf16)
     return launch_typed(static_cast<const uint16_t*>(g), e, gamma, lambda, d, idx_out, val_out,
-                        count_out, err_out, ws, dev);
+                        count_out, err_out, tiles_out, ws, dev);
   return launch_typed(static_cast<const float*>(g), e, gamma, lambda, d, idx_out, val_out,
-                      count_out, err_out, ws, dev);
+                      count_out, err_out, tiles_out, ws, dev);
 }
 
 }  // namespace efs

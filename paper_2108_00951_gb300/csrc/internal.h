@@ -206,10 +206,16 @@ ScanCtx next_scan_ctx(Workspace& ws, uint32_t num_tiles);
 
 // ---- launchers (return the launch's cudaError_t) ----
 // err_out (optional, device): ||e'||^2 of the step.
+// tiles_out (optional, device, uint32[tiles_for(d) + 1]): the message's tile
+// index, tiles_out[t] = pairs with index < t * kTileElems, the last = count.
 cudaError_t launch_hard_threshold(const void* g, bool g_bf16, float* e, float gamma,
                                   float lambda, uint32_t d, uint32_t* idx_out, float* val_out,
-                                  uint32_t* count_out, double* err_out, Workspace& ws,
-                                  const DeviceInfo& dev);
+                                  uint32_t* count_out, double* err_out, uint32_t* tiles_out,
+                                  Workspace& ws, const DeviceInfo& dev);
+// The tile index of one ascending list (binary searches), for the paths whose
+// kernel does not produce it.
+cudaError_t launch_list_tiles(const uint32_t* idx, const uint32_t* count, uint32_t d,
+                              uint32_t* tiles_out, Workspace& ws);
 cudaError_t launch_hard_threshold_lookback(const float* g, float* e, float gamma, float lambda,
                                            uint32_t d, uint32_t* idx_out, float* val_out,
                                            uint32_t* count_out, const ScanCtx& ctx,
@@ -224,13 +230,15 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
 cudaError_t launch_topk_layerwise(const void* g, bool g_bf16, float* e, float gamma, uint32_t d,
                                   uint32_t* idx_out, float* val_out, uint32_t* count_out,
                                   double* err_out, Workspace& ws, const DeviceInfo& dev);
+// tiles (optional): HOST array of n DEVICE pointers to the lists' tile
+// indexes; without it the kernel before the reduction finds them.
 cudaError_t launch_aggregate(uint32_t n, const uint32_t* const* idx, const float* const* val,
-                             const uint32_t* counts, uint32_t d, float* dense_out,
-                             Workspace& ws);
+                             const uint32_t* const* tiles, const uint32_t* counts, uint32_t d,
+                             float* dense_out, Workspace& ws);
 cudaError_t launch_aggregate_apply(uint32_t n, const uint32_t* const* idx,
-                                   const float* const* val, const uint32_t* counts, uint32_t d,
-                                   float alpha, float* x, float* m, float mu, float lr,
-                                   Workspace& ws);
+                                   const float* const* val, const uint32_t* const* tiles,
+                                   const uint32_t* counts, uint32_t d, float alpha, float* x,
+                                   float* m, float mu, float lr, Workspace& ws);
 
 
 // Workspace sizing helpers.
@@ -239,6 +247,7 @@ inline uint32_t tiles_for(uint64_t d) {
 }
 constexpr int kAggTile = 4096;             // dense elements per aggregation CTA
 constexpr int kAggStage = 1024;            // pairs an aggregation CTA stages per round trip
+static_assert(kAggTile == kTileElems, "a message's tile index serves the aggregation");
 constexpr uint32_t kMaxWorkers = 256;
 inline uint32_t agg_tiles_for(uint64_t d) {
   return static_cast<uint32_t>((d + kAggTile - 1) / kAggTile);
