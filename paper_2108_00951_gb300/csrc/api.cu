@@ -147,15 +147,6 @@ ef_status hard_threshold_entry(const void* g, bool bf16, float* e, float gamma, 
       if (overlaps(outs[o], out_n[o], outs[p], out_n[p])) return EF_ERR_INVALID_ARG;
   }
   if (overlaps(g, d * gsz, e, nb)) return EF_ERR_INVALID_ARG;
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
-  DeviceInfo info;
-  ef_status st = device_info(dev, &info);
-  if (st != EF_OK) return st;
-  Workspace* ws = nullptr;
-  st = acquire_workspace(stream, tiles_for(d), 0, 0,
-                         static_cast<size_t>(tiles_for(d)) * kTileElems, &ws);
-  if (st != EF_OK) return st;
   if (err_out && (overlaps(err_out, 8, e, nb) || overlaps(err_out, 8, g, d * gsz) ||
                   overlaps(err_out, 8, idx_out, nb) || overlaps(err_out, 8, val_out, nb) ||
                   overlaps(err_out, 8, count_out, 4)))
@@ -166,6 +157,15 @@ ef_status hard_threshold_entry(const void* g, bool bf16, float* e, float gamma, 
                     overlaps(tiles_out, tb, count_out, 4) ||
                     (err_out && overlaps(tiles_out, tb, err_out, 8))))
     return EF_ERR_INVALID_ARG;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EF_ERR_CUDA;
+  DeviceInfo info;
+  ef_status st = device_info(dev, &info);
+  if (st != EF_OK) return st;
+  Workspace* ws = nullptr;
+  st = acquire_workspace(stream, tiles_for(d), 0, 0,
+                         static_cast<size_t>(tiles_for(d)) * kTileElems, &ws);
+  if (st != EF_OK) return st;
   return finish_launch(launch_hard_threshold(g, bf16, e, gamma, lambda, static_cast<uint32_t>(d),
                                              idx_out, val_out, count_out, err_out, tiles_out, *ws,
                                              info),

@@ -133,6 +133,53 @@ def test_aggregate_apply_rejects():
         assert call(**kwargs) == efs.EF_ERR_INVALID_ARG, kwargs
 
 
+TILES = 0x60000000
+
+
+def _ht_tiled(tiles=TILES, d=1000, err=0, **kw):
+    lib = efs.load_library()
+    a = dict(g=G, e=E, idx=IDX, val=VAL, cnt=CNT)
+    a.update(kw)
+    return lib.ef_hard_threshold_tiled(vp(a["g"]), 0, vp(a["e"]), ctypes.c_float(0.1),
+                                       ctypes.c_float(1e-3), d, vp(a["idx"]), vp(a["val"]),
+                                       vp(a["cnt"]), vp(tiles), vp(err), vp(0))
+
+
+@pytest.mark.parametrize("kwargs", [
+    dict(tiles=0), dict(tiles=TILES + 2),
+    dict(tiles=IDX + 3996),   # the index's 2 words overlap the last index entry
+    dict(tiles=CNT - 4),      # its second word is the count
+    dict(tiles=E + 100), dict(tiles=G),
+    dict(err=TILES + 4),      # the error norm inside the index
+    dict(cnt=0), dict(g=G + 1),
+])
+def test_hard_threshold_tiled_rejects(kwargs):
+    assert _ht_tiled(**kwargs) == efs.EF_ERR_INVALID_ARG
+
+
+def test_aggregate_tiled_rejects():
+    lib = efs.load_library()
+    arr = (vp * 1)(vp(IDX))
+    varr = (vp * 1)(vp(VAL))
+    tarr = (vp * 1)(vp(TILES))
+    f = ctypes.c_float
+    assert lib.sparse_aggregate_tiled(1, arr, varr, None, vp(CNT), 100, vp(G),
+                                      vp(0)) == efs.EF_ERR_INVALID_ARG
+    for t in (0, TILES + 2):
+        bad = (vp * 1)(vp(t))
+        assert lib.sparse_aggregate_tiled(1, arr, varr, bad, vp(CNT), 100, vp(G),
+                                          vp(0)) == efs.EF_ERR_INVALID_ARG
+        assert lib.sparse_aggregate_apply_tiled(1, arr, varr, bad, vp(CNT), 100, f(0.5), vp(G),
+                                                vp(E), f(0.9), f(0.1),
+                                                vp(0)) == efs.EF_ERR_INVALID_ARG
+    assert lib.sparse_aggregate_tiled(0, arr, varr, tarr, vp(CNT), 100, vp(G),
+                                      vp(0)) == efs.EF_ERR_INVALID_ARG
+    assert lib.sparse_aggregate_apply_tiled(1, arr, varr, None, vp(CNT), 100, f(0.5), vp(G), vp(E),
+                                            f(0.9), f(0.1), vp(0)) == efs.EF_ERR_INVALID_ARG
+    assert lib.sparse_aggregate_apply_tiled(1, arr, varr, tarr, vp(CNT), 100, f(0.5), vp(0), vp(E),
+                                            f(0.9), f(0.1), vp(0)) == efs.EF_ERR_INVALID_ARG
+
+
 def test_binding_fails_loudly_on_cpu_tensors():
     torch = pytest.importorskip("torch")
     x = torch.zeros(8)
