@@ -55,6 +55,8 @@
 //        for the partial last tile.
 //   (tile_smem and tile_global also receive `aux`, the pre-pass result or 0)
 //   void prologue()                     every thread, once, at the start
+//   static constexpr uint32_t kPrefetchTiles;  tiles of the chunk pulled toward
+//   void prefetch(uint32_t tile)               L2 before the wait for the previous kernel
 // Optional pre-pass (kPrepass): before streaming, the compute threads sample
 // their CTA's chunk of tiles [t_lo, t_hi) with
 //   void sample(uint32_t t_lo, uint32_t t_hi, int tid, uint32_t* s_hist)
@@ -151,8 +153,15 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
     mbar_init_fence();
   }
   __syncthreads();
-  // a dependent launch may start early: everything the previous kernels on
-  // the stream wrote is read only after this
+  // A dependent launch starts while the previous kernel's last CTAs place
+  // their pairs, a phase that leaves DRAM mostly idle: pull the chunk's first
+  // tiles toward L2 meanwhile. A prefetch is not a read of the data: L2 is the
+  // point of coherence, so the previous kernel's writes still land before the
+  // bulk copies below read these lines.
+  if (threadIdx.x == 0)
+    for (uint32_t r = 0; r < rounds && r < Op::kPrefetchTiles; ++r)
+      if (t_lo + r < full_tiles) op.prefetch(t_lo + r);
+  // everything the previous kernels on the stream wrote is read only after this
   griddep_wait();
   op.prologue();
 

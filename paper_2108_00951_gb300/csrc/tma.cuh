@@ -71,6 +71,12 @@ __device__ __forceinline__ void tma_load_1d(void* dst, const void* src, uint32_t
       : "memory");
 }
 
+// Bulk prefetch of [src, src + bytes) into L2 (16-byte aligned, bytes a
+// multiple of 16): no data moves into the CTA and nothing waits for it.
+__device__ __forceinline__ void prefetch_l2_1d(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 // L2 policies: data read once per call, and data the next pass re-reads.
 __device__ __forceinline__ uint64_t l2_evict_first_policy() {
   uint64_t p;

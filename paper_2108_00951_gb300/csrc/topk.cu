@@ -102,6 +102,13 @@ struct TopkCandOp {
   static constexpr int kSampleBins = efs::kSampleBins;
   static constexpr int kSampleShift = 31 - kSampleBits;  // key bits below the sampled ones
 
+  // no L2 prefetch before the wait: measured 3 %% slower (the previous call's
+  // select, still running, re-reads its candidate list from L2)
+  static constexpr uint32_t kPrefetchTiles = 0;
+  __device__ __forceinline__ void prefetch(uint32_t t) const {
+    prefetch_l2_1d(g + static_cast<size_t>(t) * kTileElems, kGBytes);
+    prefetch_l2_1d(e + static_cast<size_t>(t) * kTileElems, kTileElems * sizeof(float));
+  }
   __device__ __forceinline__ void fill(unsigned char* stage, uint32_t t, uint64_t* bar,
                                        uint64_t policy) const {
     tma_load_1d(stage, g + static_cast<size_t>(t) * kTileElems, kGBytes, bar, policy);

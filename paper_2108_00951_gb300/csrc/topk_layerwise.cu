@@ -177,6 +177,13 @@ struct LwCandOp {
   __device__ bool barrier(uint64_t, uint32_t*) const { return true; }
   __device__ uint64_t choose() const { return 0; }
 
+  // the chunk's first tiles of g and e toward L2 before the wait for the
+  // previous kernel (its tail leaves DRAM mostly idle)
+  static constexpr uint32_t kPrefetchTiles = 8;
+  __device__ __forceinline__ void prefetch(uint32_t t) const {
+    prefetch_l2_1d(g + static_cast<size_t>(t) * kTileElems, kGBytes);
+    prefetch_l2_1d(e + static_cast<size_t>(t) * kTileElems, kTileElems * sizeof(float));
+  }
   __device__ __forceinline__ void fill(unsigned char* stage, uint32_t t, uint64_t* bar,
                                        uint64_t policy) const {
     tma_load_1d(stage, g + static_cast<size_t>(t) * kTileElems, kGBytes, bar, policy);
