@@ -1,5 +1,5 @@
 // stream_compact.cuh — ordered stream compaction at memory speed: one
-// cooperative launch of persistent CTAs, TMA-fed tiles, warp-independent
+// launch of persistent CTAs (one per SM), TMA-fed tiles, warp-independent
 // streaming of contiguous chunks, then pair placement.
 //
 // Why not a decoupled look-back, one tile per CTA: each CTA holds its tile
@@ -22,12 +22,16 @@
 // segment's count, and releases the stage. No CTA-wide barrier.
 //
 // Phase 2 (placement). Segments are ordered (tile, warp), which is coordinate
-// order. Each CTA publishes its chunk's total (tagged with the launch's epoch)
-// and sums the totals of all earlier chunks in one batched load, waiting
-// (bounded) for any not yet published; all CTAs finish phase 1 at about the
-// same time, so this is about one L2 round trip and no grid-wide barrier is
-// needed. It then scans its segments' counts in shared memory, and each warp
+// order. Each CTA publishes its chunk's total (tagged with the launch's epoch),
+// loads and scans its own segments' counts in shared memory, and then sums
+// the totals of all earlier chunks in one batched load, waiting (bounded) for
+// any not yet published; no grid-wide barrier is needed. Each warp then
 // copies whole segments from staging to their final, ascending positions.
+//
+// Before its wait for the previous kernel on the stream (programmatic
+// launch: the CTA becomes resident while that kernel's last CTAs place their
+// pairs) a CTA pulls the first Op::kPrefetchTiles tiles of its chunk toward
+// L2 with bulk prefetches.
 //
 // Error norm (when sa.err_out is set): a coordinate that is neither selected
 // nor deferred (selection bits 4..7 of an op mark coordinates whose residual
