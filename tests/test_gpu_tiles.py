@@ -73,6 +73,31 @@ def test_hard_threshold_writes_the_tile_index(d, bf16):
     assert efs.ef_check_status() == efs.EF_OK
 
 
+@pytest.mark.parametrize("offs", [(0, 0), (1, 0)])
+def test_tile_index_with_the_error_norm(offs):
+    # both optional outputs of ef_hard_threshold_tiled at once, on the
+    # streaming and on the misaligned path; the norm within the relative
+    # 1e-6 of the error-norm tests, the other outputs bit-exact
+    d = 3 * 2**20 + 4099
+    g, e = _inputs(d, 3)
+    ri, rv, re_ = oracle.ef_hard_threshold(g, e, 0.1, 1.5e-3)
+    gd, ed = gu.g_device(g, offs[0]), gu.to_dev(e, offs[1])
+    idx = torch.empty(d, dtype=torch.int32, device=DEV)
+    val = torch.empty(d, dtype=torch.float32, device=DEV)
+    cnt = torch.empty(1, dtype=torch.int32, device=DEV)
+    tiles = torch.empty(efs.tiles_for(d), dtype=torch.int32, device=DEV)
+    err = torch.full((1,), float("nan"), dtype=torch.float64, device=DEV)
+    efs.ef_hard_threshold(gd, ed, 0.1, 1.5e-3, idx, val, cnt, err_sq_out=err, tiles_out=tiles)
+    c = int(cnt.item())
+    gu.assert_bits(idx[:c].cpu().numpy().view(np.uint32), ri, "idx")
+    gu.assert_bits(val[:c].cpu().numpy(), rv, "val")
+    gu.assert_bits(ed.cpu().numpy(), re_, "e'")
+    gu.assert_bits(tiles.cpu().numpy().view(np.uint32), _tile_index(ri, d), "tile index")
+    want = oracle.error_norm_sq(re_)
+    assert abs(float(err.item()) - want) <= 1e-6 * want
+    assert efs.ef_check_status() == efs.EF_OK
+
+
 @pytest.mark.parametrize("offs", [(1, 0), (0, 3)])
 def test_tile_index_on_the_misaligned_path(offs):
     d = 5 * 4096 + 999
