@@ -43,10 +43,11 @@
  *     and the paper's data volume counts non-zeros, Sec. 6 "average density").
  *   - The residual of a sent coordinate is +0.0f; of an unsent one it is a[j].
  *     Hence a == C(a) + e' holds exactly for every finite a.
- *   - NaN: never satisfies |a| >= lambda (not sent by hard-threshold); in the
- *     Top-k order, magnitudes compare by IEEE-754 totalOrder of |a|, so NaN
- *     ranks above +inf. Every NaN the library writes (accumulator, residual,
- *     sent value, aggregate sum) is the canonical quiet NaN 0x7fffffff.
+ *   - NaN (the paper is silent on it): never satisfies |a| >= lambda (not
+ *     sent by hard-threshold); in the Top-k order every NaN is one magnitude,
+ *     above +inf, so NaNs tie and the lowest indices win. A NaN carries no
+ *     value and its encoding is not part of the result (CUDA arithmetic writes
+ *     the quiet NaN 0x7fffffff for every NaN it produces).
  *   - Top-k ties go to the lowest index; exactly k pairs are emitted.
  *
  * Workspace: the library keeps one grow-only device workspace per (device,

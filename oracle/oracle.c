@@ -22,11 +22,11 @@
  *   R4 a coordinate equal to +-0 is never sent (it adds nothing to C(a) and
  *      ||C(a)||_0 does not count it).
  *   R5 Top-k ties go to the lowest index; exactly k pairs are sent.
- *   R6 magnitude order = IEEE-754 totalOrder of |a| (NaN above +inf); the
- *      hard-threshold test |a| >= lambda is false for NaN. The paper is
- *      silent on NaN; a NaN carries no value, so every NaN the step produces
- *      (accumulator or aggregate sum) is written as the one canonical quiet
- *      NaN, encoding 0x7fffffff.
+ *   R6 NaN (the paper is silent on it): a NaN carries no value, so every
+ *      NaN is the same magnitude, above +inf (equal magnitudes tie by index
+ *      as in R5); the hard-threshold test |a| >= lambda is false for NaN.
+ *      NaN results keep whatever encoding the host arithmetic gives them;
+ *      results are compared with any NaN equal to any other NaN.
  *   R7 the residual of a sent coordinate is +0.0f.
  *   R9 aggregation returns the sum (the 1/n of Algorithm 1 is the caller's),
  *      accumulated from +0.0f in ascending worker order.
@@ -45,15 +45,6 @@
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
-
-/* R6: the canonical encoding of a NaN result. */
-static float canonical_nan_if_nan(float x) {
-  if (!isnan(x)) return x;
-  uint32_t w = 0x7fffffffu;
-  float f;
-  memcpy(&f, &w, sizeof f);
-  return f;
-}
 
 /* Widen a bfloat16 bit pattern to the fp32 value it denotes: the 16 stored
  * bits are the high half of the fp32 encoding, the low half is zero. */
@@ -77,7 +68,7 @@ static int hard_threshold_core(const float* g_f32, const uint16_t* g_bf16,
   uint64_t c = 0;
   for (uint64_t j = 0; j < d; ++j) {
     float gj = g_f32 ? g_f32[j] : bf16_bits_to_float(g_bf16[j]);
-    float a = canonical_nan_if_nan(fmaf(gamma, gj, e[j])); /* R2, R6 */
+    float a = fmaf(gamma, gj, e[j]);                       /* R2 */
     int in_support = (fabsf(a) >= lambda) && (a != 0.0f); /* R3, R4, R6 */
     if (in_support) {
       idx[c] = (uint32_t)j;
@@ -109,19 +100,14 @@ int oracle_ef_hard_threshold_bf16(const uint16_t* g, float* e, float gamma,
  * largest-magnitude entries minimises ||p - C(p)||^2 under ||C(p)||_0 <= k).
  * ------------------------------------------------------------------------ */
 
-/* Magnitude order of R6: compare |x| and |y| under IEEE-754 totalOrder.
- * For non-NaN values this is the ordinary order of fabsf; every NaN ranks
- * above +inf, and two NaNs rank by their payloads. Returns -1, 0 or +1. */
+/* Magnitude order of R6: the ordinary order of fabsf for numbers; every NaN
+ * ranks above +inf, and two NaNs are equal. Returns -1, 0 or +1. */
 static int magnitude_cmp(float x, float y) {
   float ax = fabsf(x), ay = fabsf(y);
   int nx = isnan(ax), ny = isnan(ay);
   if (nx || ny) {
-    if (!ny) return 1;
-    if (!nx) return -1;
-    uint32_t px, py;
-    memcpy(&px, &ax, sizeof px);
-    memcpy(&py, &ay, sizeof py);
-    return (px > py) - (px < py);
+    if (nx && ny) return 0;
+    return nx ? 1 : -1;
   }
   return (ax > ay) - (ax < ay);
 }
@@ -152,7 +138,7 @@ static int topk_core(const float* g_f32, const uint16_t* g_bf16, float* e,
   /* corrected update p = e + gamma g (Algorithm 1), one fma each (R2) */
   for (uint64_t j = 0; j < d; ++j) {
     float gj = g_f32 ? g_f32[j] : bf16_bits_to_float(g_bf16[j]);
-    a[j] = canonical_nan_if_nan(fmaf(gamma, gj, e[j]));    /* R6 */
+    a[j] = fmaf(gamma, gj, e[j]);
     order[j] = (uint32_t)j;
   }
   /* S = the first k coordinates in decreasing magnitude, ties by index */
@@ -240,7 +226,7 @@ int oracle_sparse_aggregate(uint32_t n, const uint32_t* const* idx,
     for (uint32_t p = 0; p < counts[i]; ++p) {
       uint32_t j = idx[i][p];
       if ((uint64_t)j >= d) return 1;
-      dense[j] = canonical_nan_if_nan(dense[j] + val[i][p]); /* R6 */
+      dense[j] = dense[j] + val[i][p];
     }
   }
   return 0;
@@ -264,13 +250,13 @@ int oracle_sparse_aggregate_apply(uint32_t n, const uint32_t* const* idx,
   int rc = oracle_sparse_aggregate(n, idx, val, counts, d, s);
   if (rc == 0) {
     for (uint64_t j = 0; j < d; ++j) {
-      float delta = canonical_nan_if_nan(alpha * s[j]);          /* Delta'_j */
+      float delta = alpha * s[j];                    /* Delta'_j */
       if (m) {
-        m[j] = canonical_nan_if_nan(fmaf(mu, m[j], delta));      /* m <- mu m + Delta' */
-        float u = canonical_nan_if_nan(delta + m[j]);            /* Delta' + m */
-        x[j] = canonical_nan_if_nan(fmaf(-lr, u, x[j]));         /* x <- x - lr (Delta' + m) */
+        m[j] = fmaf(mu, m[j], delta);                /* m <- mu m + Delta' */
+        float u = delta + m[j];                      /* Delta' + m */
+        x[j] = fmaf(-lr, u, x[j]);                   /* x <- x - lr (Delta' + m) */
       } else {
-        x[j] = canonical_nan_if_nan(x[j] - delta);               /* x <- x - Delta_bar */
+        x[j] = x[j] - delta;                         /* x <- x - Delta_bar */
       }
     }
   }
@@ -303,7 +289,7 @@ static int scaled_round_core(const float* g_f32, const uint16_t* g_bf16, float* 
   uint32_t u = 0;
   for (uint64_t j = 0; j < d; ++j) {
     float gj = g_f32 ? g_f32[j] : bf16_bits_to_float(g_bf16[j]);
-    float a = canonical_nan_if_nan(fmaf(gamma, gj, e[j]));    /* R2, R6 */
+    float a = fmaf(gamma, gj, e[j]);                           /* R2 */
     float s = ldexpf(a, m);                                    /* a 2^m (exact scaling) */
     if (!(fabsf(s) < 2147483648.0f)) {                         /* |a 2^m| >= 2^31, or NaN */
       q[j] = 0;                                                /* not representable: */
@@ -314,7 +300,7 @@ static int scaled_round_core(const float* g_f32, const uint16_t* g_bf16, float* 
     float r = rintf(s);                                        /* round half to even */
     q[j] = (int32_t)r;
     float c = ldexpf((float)q[j], -m);                         /* C(a)_j */
-    e[j] = canonical_nan_if_nan(a - c);                        /* e'_j = a_j - C(a)_j */
+    e[j] = a - c;                                              /* e'_j = a_j - C(a)_j */
   }
   *unsent = u;
   return 0;

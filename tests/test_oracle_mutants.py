@@ -30,30 +30,41 @@ MUTANTS = {
     "topk_highest_index_ties": [("  return (ia > ib) - (ia < ib);", "  return (ia < ib) - (ia > ib);")],
     "topk_residual_kept": [("    e[j] = 0.0f;                                      /* R7 */",
                             "    e[j] = a[j];")],
-    "nan_payload_kept": [("  if (!isnan(x)) return x;", "  return x;")],
+    "nan_ranked_by_payload": [("    if (nx && ny) return 0;",
+                               "    if (nx && ny) { uint32_t px, py; memcpy(&px, &ax, 4);"
+                               " memcpy(&py, &ay, 4); return (px > py) - (px < py); }")],
     "aggregate_reverse_order": [("for (uint32_t i = 0; i < n; ++i) {",
                                  "for (uint32_t i = n; i-- > 0;) {")],
-    "nan_ranks_lowest": [("    if (!ny) return 1;\n    if (!nx) return -1;",
-                          "    if (!ny) return -1;\n    if (!nx) return 1;")],
+    "nan_ranks_lowest": [("    return nx ? 1 : -1;", "    return nx ? -1 : 1;")],
     "layerwise_local_indices": [("idx[sent + p] += (uint32_t)lo;", "idx[sent + p] += 0u;")],
     "layerwise_first_k_everywhere": [("                       seg_k[s], hi - lo,",
                                       "                       seg_k[0] < hi - lo ? seg_k[0] : hi - lo, hi - lo,")],
     "layerwise_error_not_sliced": [("e + lo, gamma,", "e, gamma,")],
     "update_uses_old_momentum": [
-        ("        m[j] = canonical_nan_if_nan(fmaf(mu, m[j], delta));      /* m <- mu m + Delta' */\n"
-         "        float u = canonical_nan_if_nan(delta + m[j]);            /* Delta' + m */",
-         "        float u = canonical_nan_if_nan(delta + m[j]);            /* Delta' + m */\n"
-         "        m[j] = canonical_nan_if_nan(fmaf(mu, m[j], delta));      /* m <- mu m + Delta' */")],
-    "update_alpha_dropped": [("float delta = canonical_nan_if_nan(alpha * s[j]);",
-                              "float delta = canonical_nan_if_nan(s[j]);")],
+        ("        m[j] = fmaf(mu, m[j], delta);                /* m <- mu m + Delta' */\n"
+         "        float u = delta + m[j];                      /* Delta' + m */",
+         "        float u = delta + m[j];                      /* Delta' + m */\n"
+         "        m[j] = fmaf(mu, m[j], delta);                /* m <- mu m + Delta' */")],
+    "update_alpha_dropped": [("float delta = alpha * s[j];", "float delta = s[j];")],
     "update_momentum_two_step": [("fmaf(mu, m[j], delta)", "(mu * m[j] + delta)")],
     "update_wrong_sign": [("fmaf(-lr, u, x[j])", "fmaf(lr, u, x[j])")],
-    "update_sgd_adds": [("x[j] = canonical_nan_if_nan(x[j] - delta);",
-                         "x[j] = canonical_nan_if_nan(x[j] + delta);")],
+    "update_sgd_adds": [("x[j] = x[j] - delta;", "x[j] = x[j] + delta;")],
     "round_half_away": [("float r = rintf(s);", "float r = roundf(s);")],
     "round_truncate": [("float r = rintf(s);", "float r = truncf(s);")],
-    "round_residual_not_subtracted": [("e[j] = canonical_nan_if_nan(a - c);",
-                                       "e[j] = canonical_nan_if_nan(a);")],
+    "round_residual_not_subtracted": [("e[j] = a - c;", "e[j] = a;")],
+    # the bf16 widening inside the scaled-rounding step only (the line is
+    # followed there by the scaling, not by the threshold or the sort)
+    "round_bf16_integer_value": [
+        ("bf16_bits_to_float(g_bf16[j]);\n    float a = fmaf(gamma, gj, e[j]);"
+         "                           /* R2 */\n    float s = ldexpf(a, m);",
+         "(float)g_bf16[j];\n    float a = fmaf(gamma, gj, e[j]);"
+         "                           /* R2 */\n    float s = ldexpf(a, m);")],
+    "round_bf16_sign_dropped": [
+        ("bf16_bits_to_float(g_bf16[j]);\n    float a = fmaf(gamma, gj, e[j]);"
+         "                           /* R2 */\n    float s = ldexpf(a, m);",
+         "bf16_bits_to_float(g_bf16[j] & 0x7fff);\n    float a = fmaf(gamma, gj, e[j]);"
+         "                           /* R2 */\n    float s = ldexpf(a, m);")],
+    "bf16_widening_shift": [("((uint32_t)bits) << 16", "((uint32_t)bits) << 15")],
     "round_scale_sign": [("float s = ldexpf(a, m);", "float s = ldexpf(a, -m);")],
     "round_saturates_instead": [("      q[j] = 0;                                                /* not representable: */",
                                  "      q[j] = a > 0 ? 2147483647 : -2147483647;")],
@@ -89,6 +100,9 @@ PIN_TESTS = [
     pins.test_scaled_round_hand_example,
     pins.test_scaled_round_is_an_absolute_compressor,
     pins.test_scaled_round_unsent_coordinates,
+    pins.test_scaled_round_bf16_hand_example,
+    pins.test_scaled_round_bf16_is_the_widened_fp32,
+    pins.test_ht_bf16_widening,
     pins.test_int_aggregate_is_exact_and_order_free,
 ]
 

@@ -111,9 +111,6 @@ def test_ht_lambda_above_max_sends_nothing():
     assert _same_bits(e_new, a)
 
 
-CANONICAL_NAN = 0x7FFFFFFF
-
-
 def test_ht_nan_and_inf():
     # NaN never passes |a| >= lambda; +-inf does; 0 * inf is NaN (invalid)
     e = _f32([np.nan, np.inf, -np.inf, 1.0, 5.0])
@@ -122,11 +119,13 @@ def test_ht_nan_and_inf():
     assert idx.tolist() == [1, 2, 3, 4]
     assert val.tolist() == [np.inf, -np.inf, 1.0, np.inf]
     assert e_new[1:].tolist() == [0.0, 0.0, 0.0, 0.0]
-    # every NaN result carries the one canonical encoding (reading R6)
-    e = _f32([np.nan, 2.0])
-    e[0] = np.uint32(0x7FC00001).view(np.float32)        # a NaN with a payload
-    _, _, e_new = oracle.ef_hard_threshold(_f32([0.0, np.inf]), e, 0.0, 0.5)
-    assert e_new.view(np.uint32).tolist() == [CANONICAL_NAN, CANONICAL_NAN]
+    # a NaN accumulator (a NaN error, or 0 * inf) is never sent and stays in
+    # the residual as a NaN, whatever its encoding (reading R6)
+    e = _f32([np.nan, 2.0, -1.0])
+    e[0] = np.uint32(0xFFC00001).view(np.float32)        # a negative NaN with a payload
+    idx, _, e_new = oracle.ef_hard_threshold(_f32([0.0, np.inf, 0.0]), e, 0.0, 0.5)
+    assert idx.tolist() == [2]
+    assert np.isnan(e_new[0]) and np.isnan(e_new[1]) and e_new[2] == 0.0
 
 
 @pytest.mark.parametrize("d", [1, 7, 64, 3001])
@@ -265,6 +264,15 @@ def test_topk_nan_inf_order():
     assert idx.tolist() == [1, 2, 3]    # +inf and -inf tie: lower index first
     idx, _, _ = oracle.ef_topk(g, e, 1.0, 4)
     assert idx.tolist() == [1, 2, 3, 4]
+    # every NaN is one magnitude (a NaN carries no value): NaNs with different
+    # payloads and signs tie, so the lowest indices win, never the payloads
+    nans = np.array([0x7FC00001, 0x7FFFFFFF, 0xFFC00000, 0x7FC00002], np.uint32).view(np.float32)
+    e = _f32([1.0, nans[0], np.inf, nans[1], nans[2], nans[3]])
+    idx, val, e_new = oracle.ef_topk(np.zeros(6, np.float32), e, 1.0, 2)
+    assert idx.tolist() == [1, 3] and np.all(np.isnan(val))
+    assert e_new[1] == 0.0 and e_new[3] == 0.0 and np.isnan(e_new[4]) and np.isnan(e_new[5])
+    idx, _, _ = oracle.ef_topk(np.zeros(6, np.float32), e, 1.0, 5)
+    assert idx.tolist() == [1, 2, 3, 4, 5]
 
 
 # --------------------------------------------------------------------------
@@ -431,11 +439,11 @@ def test_aggregate_sums_in_worker_order():
     assert dense[5] == 1.0
 
 
-def test_aggregate_nan_is_canonical():
+def test_aggregate_nan_propagates():
     nan = np.uint32(0x7FC00001).view(np.float32)
-    dense = oracle.sparse_aggregate([np.array([1], np.uint32), np.array([1], np.uint32)],
-                                    [_f32([nan]), _f32([1.0])], 3)
-    assert dense.view(np.uint32)[1] == CANONICAL_NAN
+    dense = oracle.sparse_aggregate([np.array([1], np.uint32), np.array([1, 2], np.uint32)],
+                                    [_f32([nan]), _f32([1.0, np.inf])], 3)
+    assert dense[0] == 0.0 and np.isnan(dense[1]) and dense[2] == np.inf
 
 
 def test_aggregate_rejects_out_of_range():
@@ -609,7 +617,41 @@ def test_scaled_round_unsent_coordinates():
     assert unsent == 4
     assert list(q[:3]) == [0, 0, 2 ** 31 - 128] and q[3] == 0 and q[4] == 0 and q[5] == 1
     assert e_new[0] == 2.0 ** 31 and e_new[1] == -(2.0 ** 31) and e_new[2] == 0.0
-    assert np.isinf(e_new[3]) and e_new.view(np.uint32)[4] == CANONICAL_NAN and e_new[5] == 0.0
+    assert np.isinf(e_new[3]) and np.isnan(e_new[4]) and e_new[5] == 0.0
+
+
+def test_scaled_round_bf16_hand_example():
+    # bf16 bit patterns widened by hand: 0x3F80 = 1.0, 0xBFC0 = -1.5,
+    # 0x4049 = 3.140625, 0x0001 = 2^-133 (a subnormal), 0x7F80 = +inf,
+    # 0xC780 = -65536; grid 2^-2 (m = 2), gamma = 1, e = 0
+    bits = np.array([0x3F80, 0xBFC0, 0x4049, 0x0001, 0x7F80, 0xC780], np.uint16)
+    q, e_new, unsent = oracle.ef_scaled_round(bits, np.zeros(6, np.float32), 1.0, 2)
+    assert list(q) == [4, -6, 13, 0, 0, -262144] and unsent == 1
+    assert e_new[0] == 0.0 and e_new[1] == 0.0 and e_new[2] == 3.140625 - 3.25
+    assert e_new[3] == np.float32(2.0 ** -133) and e_new[4] == np.inf and e_new[5] == 0.0
+
+
+def test_scaled_round_bf16_is_the_widened_fp32():
+    # on bf16 bit patterns the step equals the fp32 step on the values they
+    # denote, bit for bit: q, e' and the unsent count; the widening here is
+    # torch's own bf16 -> fp32 conversion
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(77)
+    x = torch.from_numpy(_f32(rng.standard_normal(6000) *
+                              np.exp2(rng.integers(-130, 40, 6000))))
+    gb = x.to(torch.bfloat16)
+    bits = gb.view(torch.int16).numpy().view(np.uint16).copy()
+    bits[:4] = [0x7F80, 0xFF80, 0x7FC0, 0x8000]           # +inf, -inf, NaN, -0
+    widened = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).to(torch.float32).numpy()
+    e = _f32(rng.standard_normal(6000) * 1e-3)
+    for m in (0, 7, 20, 40):
+        q16, e16, u16 = oracle.ef_scaled_round(bits, e, 0.1, m)
+        q32, e32, u32 = oracle.ef_scaled_round(widened, e, 0.1, m)
+        assert u16 == u32 and u16 >= 3
+        assert np.array_equal(q16, q32)
+        assert np.array_equal(np.isnan(e16), np.isnan(e32))
+        ok = ~np.isnan(e16)
+        assert _same_bits(e16[ok], e32[ok])
 
 
 def test_int_aggregate_is_exact_and_order_free():
