@@ -15,9 +15,19 @@ workload, through the whole hot path:
   - n x ef_scaled_round (scaled integer rounding, another absolute
     compressor: dense int32 messages) on the same gradients, then
     int_aggregate of those messages (exact integer sum).
+  - n x ef_hard_threshold_bf16 on the same gradients rounded to bfloat16
+    (the bf16-gradient variant, widened exactly in the kernel).
 Gradients come from two pre-generated synthetic batches (alternating), so
 every step compresses different data; each step's working set (n workers x
 (g, e_ht, e_topk)) is far larger than the 126 MB L2.
+
+The default workload is the VGG-16-shaped vector (d = 138,357,544, 8
+workers), the largest one that fits one GPU. After the timed steps, further
+legs time the rest of the d >= 25 M regime on the same GPU: hard-threshold
+and Top-k on the LSTM-shaped vector and on the ResNet-50-shaped vector at
+each of its thresholds and Top-k fractions; a cold-L2 variant of the
+headline call (L2 flushed before every call); and the latency of the
+logistic-regression-sized case (d = 100,000, which fits in L2).
 
 Headline (`value`): hard-threshold compress throughput in GB/s of
 algorithmic traffic, 12 B/coordinate (read g, read e, write e) + 8 B per sent
@@ -28,7 +38,9 @@ HBM roofline. `e2e` repeats the hard-threshold iteration through the public
 API with the n gradients copied host->device from pinned memory and the
 dense aggregate copied back, every step.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload resnet18]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload vgg16]
+  python bench.py --harness ht --workload vgg16 --steps 3 --warmup 3
+      # one worker's calls only (a few GB on the device), for ncu captures
   python bench.py --impl reference ...   # the CPU oracle as the reference arm
 
 For N > 1 (one process per GPU under torch.distributed.run) every rank runs
@@ -69,7 +81,15 @@ def parse_args(argv=None):
     p.add_argument("--steps", type=int, default=200)
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    p.add_argument("--workload", default="resnet18")
+    p.add_argument("--workload", default="vgg16")
+    p.add_argument("--harness", choices=["ht", "ht_bf16", "topk", "topk_layerwise", "aggregate"],
+                   default=None,
+                   help="run only one kind of call, for one worker (aggregate: the n workers' "
+                        "hard-threshold messages), and print a short summary")
+    p.add_argument("--lam-index", type=int, default=0,
+                   help="which of the workload's fixed lambdas (or Top-k fractions) to use")
+    p.add_argument("--no-extra-legs", action="store_true",
+                   help="skip the d >= 25 M regime, cold-L2 and latency legs")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--error-norm", action="store_true",
                    help="every compress call also returns ||e'||^2 (the _ex entries)")
@@ -260,15 +280,16 @@ def run_ours(args):
 
     w = workloads.BY_NAME[args.workload]
     d, n, gamma = w.d, w.n, w.gamma
-    k = w.topk_values()[0]
-    frac = w.topk_fracs[0] if w.topk_fracs else k / d
+    ks = w.topk_values()
+    k = ks[min(args.lam_index, len(ks) - 1)]
+    frac = k / d if not w.topk_fracs else w.topk_fracs[min(args.lam_index, len(w.topk_fracs) - 1)]
     seg_end = workloads.segment_ends(w)
     seg_k = workloads.layerwise_k(w, frac)
     k_lw = sum(seg_k)
     wr = replica_workload(w, rank)
     batches = [[workloads.gradient(wr, i, b, device=dev) for i in range(n)] for b in range(2)]
     lam = (workloads.density_lambda(wr, batches[0][0], w.density) if w.density is not None
-           else w.lambdas[0])
+           else w.lambdas[args.lam_index])
 
     def outputs(cap):
         return ([torch.empty(cap, dtype=torch.int32, device=dev) for _ in range(n)],
@@ -289,6 +310,10 @@ def run_ours(args):
     x_model = torch.zeros(d, device=dev)
     m_model = torch.zeros(d, device=dev)
     e_rd = [torch.zeros(d, device=dev) for _ in range(n)]
+    # the bf16-gradient variant: the same gradients rounded to bfloat16
+    batches_bf = [[g.to(torch.bfloat16) for g in b] for b in batches]
+    e_bf = [torch.zeros(d, device=dev) for _ in range(n)]
+    idx_bf, val_bf = outputs(d)
     q_rd = [torch.empty(d, dtype=torch.int32, device=dev) for _ in range(n)]
     unsent_rd = torch.zeros(n, dtype=torch.int32, device=dev)
     dense_rd = torch.empty(d, device=dev)
@@ -297,10 +322,11 @@ def run_ours(args):
     cnt_ht = torch.zeros(total, n, dtype=torch.int32, device=dev)
     cnt_tk = torch.zeros(total, n, dtype=torch.int32, device=dev)
     cnt_lw = torch.zeros(total, n, dtype=torch.int32, device=dev)
+    cnt_bf = torch.zeros(total, n, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream()
 
     ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
-    marks = [[ev() for _ in range(10)] for _ in range(args.steps)]
+    marks = [[ev() for _ in range(11)] for _ in range(args.steps)]
 
     err_sq = torch.zeros(3, n, dtype=torch.float64, device=dev)
 
@@ -337,6 +363,11 @@ def run_ours(args):
         if m: m[8].record(stream)
         efs.int_aggregate(q_rd, d, scale_log2, dense_rd)
         if m: m[9].record(stream)
+        gb = batches_bf[s % 2]
+        for i in range(n):
+            efs.ef_hard_threshold(gb[i], e_bf[i], gamma, lam, idx_bf[i], val_bf[i],
+                                  cnt_bf[s, i:i + 1])
+        if m: m[10].record(stream)
 
     for s in range(args.warmup):
         step(s, False)
@@ -363,7 +394,7 @@ def run_ours(args):
 
     step_s = t0.elapsed_time(t1) / 1e3
     # per-iteration segment times (µs per call: the segment of n calls / n)
-    seg_us = [[m[a].elapsed_time(m[a + 1]) * 1e3 for m in marks] for a in range(9)]
+    seg_us = [[m[a].elapsed_time(m[a + 1]) * 1e3 for m in marks] for a in range(10)]
     ht_s = sum(m[0].elapsed_time(m[1]) for m in marks) / 1e3
     agg_ht_s = sum(m[1].elapsed_time(m[2]) for m in marks) / 1e3
     tk_s = sum(m[2].elapsed_time(m[3]) for m in marks) / 1e3
@@ -373,6 +404,9 @@ def run_ours(args):
     upd_s = sum(m[6].elapsed_time(m[7]) for m in marks) / 1e3
     rd_s = sum(m[7].elapsed_time(m[8]) for m in marks) / 1e3
     iagg_s = sum(m[8].elapsed_time(m[9]) for m in marks) / 1e3
+    bf_s = sum(m[9].elapsed_time(m[10]) for m in marks) / 1e3
+    counts_bf = cnt_bf[args.warmup:].double()
+    bytes_bf = float(ht_bytes(d, 0, 2) * n * args.steps + 8 * counts_bf.sum().item())
     counts_ht = cnt_ht[args.warmup:].double()
     counts_tk = cnt_tk[args.warmup:].double()
     bytes_ht = float(ht_bytes(d, 0) * n * args.steps + 8 * counts_ht.sum().item())
@@ -394,13 +428,24 @@ def run_ours(args):
     avg_launch = ht_s / (n * args.steps)
     achieved = (ht_bytes(d, 0) + 8 * counts_ht.mean().item()) / avg_launch / 1e9
 
+    # free the main legs' buffers before the extra legs allocate theirs
+    del batches, batches_bf, e_ht, e_tk, e_lw, e_rd, e_bf, idx_ht, val_ht, idx_tk, val_tk
+    del idx_lw, val_lw, idx_bf, val_bf, q_rd, dense_tk, dense_lw, dense_rd, x_model, m_model
+    torch.cuda.empty_cache()
+    extra = None
+    if not args.no_extra_legs:
+        extra = extra_legs(args, efs, torch, dev, dist, rank, w, peak)
+
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(args, efs, torch, dev, dist, batches[0], d, n, gamma, lam, stream)
+        grads0 = [workloads.gradient(wr, i, 0, device=dev) for i in range(n)]
+        e2e = run_e2e(args, efs, torch, dev, dist, grads0, d, n, gamma, lam, stream)
+        del grads0
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(args, [b.cpu().numpy() for b in batches[0][:2]], d, gamma, lam, k)
+        cpu = cpu_baseline(args, [workloads.gradient(wr, i, 0, device=dev).cpu().numpy()
+                                  for i in range(2)], d, gamma, lam, k)
 
     if rank != 0:
         return None
@@ -467,6 +512,13 @@ def run_ours(args):
             "int_aggregate_frac_of_peak": round(bytes_iagg / iagg_s / 1e9 / peak, 4),
             "bytes": "compress 16 per coordinate; exchange 4 n + 4 per coordinate",
         },
+        "ht_bf16": {
+            "ms_per_iter": round(bf_s / args.steps * 1e3, 4),
+            "gbs": round(bytes_bf / bf_s / 1e9, 2),
+            "frac_of_peak": round(bytes_bf / bf_s / 1e9 / peak, 4),
+            "density": round(counts_bf.mean().item() / d, 6),
+            "bytes": "10 per coordinate (bf16 g, fp32 e read and written) + 8 per sent pair",
+        },
         "per_call_us_p10_p50_p90": {
             "ht": percentiles([v / n for v in seg_us[0]]),
             "topk": percentiles([v / n for v in seg_us[2]]),
@@ -477,6 +529,7 @@ def run_ours(args):
             "aggregate_apply_momentum": percentiles(seg_us[6]),
             "scaled_round": percentiles([v / n for v in seg_us[7]]),
             "int_aggregate": percentiles(seg_us[8]),
+            "ht_bf16": percentiles([v / n for v in seg_us[9]]),
         },
         "frac_of_nominal_8tbs": round(value / NOMINAL_HBM_GBS, 4),
         "roofline": {
@@ -497,11 +550,202 @@ def run_ours(args):
                             "ht": float(err_sq[0, 0]), "topk": float(err_sq[1, 0]),
                             "topk_layerwise": float(err_sq[2, 0])}}
                        if args.error_norm else {"requested": False}),
+        "extra_legs": extra,
         "gpu_launches": int(launches),
         "clocks": clocks,
         "e2e": e2e,
         "cpu_baseline": cpu,
     }
+
+
+def compress_leg(efs, torch, dev, dist, w, method, param, steps, warmup, peak, flush=None):
+    """Time an EF loop of workload w's n workers through one compress method
+    ("ht": param = lambda; "topk": param = k): `warmup` untimed iterations,
+    then `steps` timed ones (CUDA events around each iteration's n calls on
+    the launching stream). With `flush` (a device buffer larger than L2) the
+    buffer is rewritten before every call and each call is timed alone: the
+    cold-L2 variant."""
+    n, d = w.n, w.d
+    batches = [[workloads_gradient(w, i, b, dev) for i in range(n)] for b in range(2)]
+    e = [torch.zeros(d, device=dev) for _ in range(n)]
+    cap = d if method == "ht" else param
+    idx = [torch.empty(cap, dtype=torch.int32, device=dev) for _ in range(n)]
+    val = [torch.empty(cap, dtype=torch.float32, device=dev) for _ in range(n)]
+    cnt = torch.zeros(warmup + steps, n, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+    ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    per = n if flush is not None else 1
+    marks = [[(ev(), ev()) for _ in range(per)] for _ in range(steps)]
+
+    def call(s, i):
+        g = batches[s % 2][i]
+        if method == "ht":
+            efs.ef_hard_threshold(g, e[i], w.gamma, param, idx[i], val[i], cnt[s, i:i + 1])
+        else:
+            efs.ef_topk(g, e[i], w.gamma, param, idx[i], val[i], cnt[s, i:i + 1])
+
+    for s in range(warmup + steps):
+        m = marks[s - warmup] if s >= warmup else None
+        if flush is None:
+            if m: m[0][0].record(stream)
+            for i in range(n):
+                call(s, i)
+            if m: m[0][1].record(stream)
+        else:
+            for i in range(n):
+                flush.add_(1.0)
+                if m: m[i][0].record(stream)
+                call(s, i)
+                if m: m[i][1].record(stream)
+    torch.cuda.synchronize()
+    if efs.ef_check_status() != efs.EF_OK:
+        raise RuntimeError("device error in the %s leg of %s" % (method, w.name))
+    secs = sum(a.elapsed_time(b) for m in marks for a, b in m) / 1e3
+    calls_us = ([a.elapsed_time(b) * 1e3 / n for m in marks for a, b in m] if flush is None else
+                [a.elapsed_time(b) * 1e3 for m in marks for a, b in m])
+    counts = cnt[warmup:].double()
+    byts = float(12 * d * n * steps + 8 * counts.sum().item())
+    secs_max, byts_all = reduce_timing(dist, secs, byts, dev)
+    gbs = byts_all / secs_max / 1e9 if dist is None else byts / secs / 1e9
+    return {"workload": w.name, "d": d, "n": n,
+            ("lambda" if method == "ht" else "k"): param,
+            "density": round(counts.mean().item() / d, 6),
+            "us_per_call_p10_p50_p90": percentiles(calls_us),
+            "gbs": round(gbs, 2), "frac_of_peak": round(gbs / peak, 4),
+            "iterations": steps, "warmup": warmup}
+
+
+def workloads_gradient(w, i, t, dev):
+    from paper_2108_00951_gb300 import workloads
+    return workloads.gradient(w, i, t, device=dev)
+
+
+def extra_legs(args, efs, torch, dev, dist, rank, w_main, peak):
+    """The rest of the d >= 25 M regime (LSTM-shaped at its threshold and
+    Top-k fraction, ResNet-50-shaped at each threshold and Top-k fraction),
+    the cold-L2 variant of the headline call, and the latency of the
+    L2-resident logistic-regression-sized case."""
+    from paper_2108_00951_gb300 import workloads
+    steps, warmup = max(3, min(args.steps, 20)), max(3, args.warmup)
+    out = {"regime_d_ge_25M": [], "bytes": "12 per coordinate + 8 per sent pair"}
+    for name in ("lstm", "resnet50"):
+        if name == w_main.name:
+            continue
+        w = replica_workload(workloads.BY_NAME[name], rank)
+        if w.density is not None:
+            lams = [workloads.density_lambda(w, workloads_gradient(w, 0, 0, dev), w.density)]
+        else:
+            lams = list(w.lambdas)
+        for lam in lams:
+            out["regime_d_ge_25M"].append(
+                {"method": "hard_threshold",
+                 **compress_leg(efs, torch, dev, dist, w, "ht", lam, steps, warmup, peak)})
+            torch.cuda.empty_cache()
+        for k in w.topk_values():
+            out["regime_d_ge_25M"].append(
+                {"method": "topk",
+                 **compress_leg(efs, torch, dev, dist, w, "topk", k, steps, warmup, peak)})
+            torch.cuda.empty_cache()
+    # cold L2: a 512 MB buffer (4x the L2) rewritten before every call
+    flush = torch.zeros(128 << 20, device=dev)
+    w = replica_workload(w_main, rank)
+    lam = (workloads.density_lambda(w, workloads_gradient(w, 0, 0, dev), w.density)
+           if w.density is not None else w.lambdas[args.lam_index])
+    out["cold_l2_ht"] = compress_leg(efs, torch, dev, dist, w, "ht", lam, 3, warmup, peak,
+                                     flush=flush)
+    del flush
+    torch.cuda.empty_cache()
+    # latency of the L2-resident case (d = 100,000, 4 workers)
+    w = replica_workload(workloads.BY_NAME["lr"], rank)
+    lat = {}
+    for method, param in (("ht", w.lambdas[0]), ("topk", w.topk_k[0])):
+        r = compress_leg(efs, torch, dev, dist, w, method, param, 50, warmup, peak)
+        lat[method + "_us_per_call_p10_p50_p90"] = r["us_per_call_p10_p50_p90"]
+    out["latency_lr"] = {"d": w.d, "n": w.n, **lat,
+                         "note": "the working set fits in L2: reported as latency"}
+    return out
+
+
+def run_harness(args):
+    """One kind of call on one worker of the workload (a few GB on the
+    device), for profiler captures: `--warmup` then `--steps` calls on
+    alternating gradients; the aggregate harness compresses the n workers'
+    gradients once (hard-threshold) and aggregates their messages."""
+    import torch
+    import paper_2108_00951_gb300 as efs
+    from paper_2108_00951_gb300 import workloads
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    efs.load_library()
+    w = workloads.BY_NAME[args.workload]
+    d = w.d
+    lam = (workloads.density_lambda(w, workloads_gradient(w, 0, 0, dev), w.density)
+           if w.density is not None else w.lambdas[args.lam_index])
+    ks = w.topk_values()
+    k = ks[min(args.lam_index, len(ks) - 1)]
+    e = torch.zeros(d, device=dev)
+    cnt = torch.zeros(1, dtype=torch.int32, device=dev)
+    ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    t0, t1 = ev(), ev()
+    if args.harness == "aggregate":
+        idx_s = torch.empty(d, dtype=torch.int32, device=dev)
+        val_s = torch.empty(d, dtype=torch.float32, device=dev)
+        idx, val, tiles, counts = [], [], [], []
+        for i in range(w.n):
+            e.zero_()
+            tl = torch.empty(efs.tiles_for(d), dtype=torch.int32, device=dev)
+            efs.ef_hard_threshold(workloads_gradient(w, i, 0, dev), e, w.gamma, lam, idx_s, val_s,
+                                  cnt, tiles_out=tl)
+            c = int(cnt.item())
+            idx.append(idx_s[:max(c, 1)].clone())
+            val.append(val_s[:max(c, 1)].clone())
+            tiles.append(tl)
+            counts.append(c)
+        del idx_s, val_s
+        cnt_n = torch.tensor(counts, dtype=torch.int32, device=dev)
+        dense = torch.empty(d, device=dev)
+        for s in range(args.warmup + args.steps):
+            if s == args.warmup:
+                t0.record()
+            efs.sparse_aggregate(idx, val, cnt_n, d, dense, tiles=tiles)
+        t1.record()
+        torch.cuda.synchronize()
+        per = t0.elapsed_time(t1) * 1e3 / max(args.steps, 1)
+        byts = 8 * sum(counts) + 4 * d
+    else:
+        dtype = torch.bfloat16 if args.harness == "ht_bf16" else torch.float32
+        grads = [workloads.gradient(w, 0, t, device=dev, dtype=dtype) for t in range(2)]
+        cap = k if args.harness == "topk" else d
+        if args.harness == "topk_layerwise":
+            frac = w.topk_fracs[min(args.lam_index, len(w.topk_fracs) - 1)] if w.topk_fracs \
+                else k / d
+            seg_end, seg_k = workloads.segment_ends(w), workloads.layerwise_k(w, frac)
+            cap = sum(seg_k)
+        idx = torch.empty(cap, dtype=torch.int32, device=dev)
+        val = torch.empty(cap, dtype=torch.float32, device=dev)
+        for s in range(args.warmup + args.steps):
+            if s == args.warmup:
+                t0.record()
+            g = grads[s % 2]
+            if args.harness in ("ht", "ht_bf16"):
+                efs.ef_hard_threshold(g, e, w.gamma, lam, idx, val, cnt)
+            elif args.harness == "topk":
+                efs.ef_topk(g, e, w.gamma, k, idx, val, cnt)
+            else:
+                efs.ef_topk_layerwise(g, e, w.gamma, seg_end, seg_k, idx, val, cnt)
+        t1.record()
+        torch.cuda.synchronize()
+        per = t0.elapsed_time(t1) * 1e3 / max(args.steps, 1)
+        gb = 2 if args.harness == "ht_bf16" else 4
+        byts = (gb + 8) * d + 8 * int(cnt.item())
+    if efs.ef_check_status() != efs.EF_OK:
+        raise RuntimeError("device error in the harness")
+    return {"harness": args.harness, "workload": w.name, "d": d, "steps": args.steps,
+            "warmup": args.warmup, "us_per_call": round(per, 2),
+            "last_call_algorithmic_bytes": int(byts),
+            "note": "one worker's calls back to back: a harness for profiler captures, "
+                    "not a bench value"}
 
 
 def run_e2e(args, efs, torch, dev, dist, grads, d, n, gamma, lam, stream):
@@ -576,6 +820,26 @@ def run_e2e(args, efs, torch, dev, dist, grads, d, n, gamma, lam, stream):
 
 
 # ------------------------------------------------------------ CPU oracle legs
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith(("model name", "cpu model")):
+                    return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    import platform
+    return platform.processor() or platform.machine()
+
+
 def cpu_baseline(args, grads, d, gamma, lam, k):
     """The oracle as it stands, single-threaded on this host: hard-threshold
     calls on the first workers' full-size gradients for about
@@ -594,7 +858,7 @@ def cpu_baseline(args, grads, d, gamma, lam, k):
     return {"value": round(byts / el / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
             "sample": "%d single-threaded oracle hard-threshold calls at full d=%d (%.1f s)"
                       % (calls, d, el),
-            "host_cores_available": os.cpu_count()}
+            "host_cores_available": os.cpu_count(), "cpu_model": cpu_model()}
 
 
 def run_reference(args):
@@ -640,7 +904,8 @@ def run_reference(args):
                                % (w.name, w.d), "global_batch": 1, "seq_len": None,
                    "parallelism": "single CPU thread"},
         "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
-                         "sample": "%d full-size oracle hard-threshold calls" % args.steps},
+                         "sample": "%d full-size oracle hard-threshold calls" % args.steps,
+                         "cpu_model": cpu_model()},
         "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -650,6 +915,8 @@ def main(argv=None):
     args = parse_args(argv)
     if args.impl == "reference":
         out = run_reference(args)
+    elif args.harness:
+        out = run_harness(args)
     else:
         out = run_ours(args)
     if out is not None:
