@@ -52,9 +52,25 @@
  *
  * Workspace: the library keeps one grow-only device workspace per (device,
  * stream) pair (scan tile status, histograms, candidate buffers, offsets).
- * Growing it synchronises `stream` once. Calls on DIFFERENT streams never
- * share a workspace and may run concurrently; calls on the same stream are
- * ordered by the stream. ef_workspace_release() frees all workspaces.
+ * Growing it synchronises `stream` once. Its size follows the largest d seen
+ * on that stream: about 8 bytes per coordinate of pair staging (the size of
+ * the outputs: 1.1 GB at d = 138 M) plus, once Top-k has run, 3 x 8 bytes per
+ * candidate slot (min(d, max(2^20, d/16)) slots), plus 8 bytes per 4096
+ * coordinates and about 260 KB of fixed state. Memory is therefore bounded by
+ * (number of streams used) x that size; ef_workspace_release() frees all
+ * workspaces of the current device (for example after a phase that used
+ * extra streams), and ef_hard_threshold_noalloc needs none. Calls on
+ * DIFFERENT streams never share a workspace and may run concurrently; calls
+ * on the same stream are ordered by the stream.
+ *
+ * Concurrency: a compress call's CTAs wait (bounded) for lower-numbered CTAs
+ * of the same launch, which the device dispatches first and which fit the
+ * device together when it is otherwise idle. If kernels on other streams or
+ * other processes (MPS) hold SMs long enough that such a CTA cannot start
+ * within the bound (2 s), the call fails with EF_ERR_TIMEOUT (reported by
+ * ef_check_status); it never hangs and never returns a wrong result. The
+ * one-tile-per-CTA path (misaligned g or e, ef_hard_threshold_noalloc) takes
+ * its tiles in the order CTAs start and needs no co-residency.
  */
 #ifndef EFSPARSE_H
 #define EFSPARSE_H
@@ -385,13 +401,19 @@ ef_status sparse_aggregate_apply_tiled(uint32_t n, const uint32_t* const* idx,
  *              the call it holds the device-side error bits of this call
  *              (0 = success; nonzero = a bounded wait ran out or an output
  *              position overflowed). ef_check_status() does not see them.
+ *              It must not overlap g, e, idx_out, val_out or count_out
+ *              (EF_ERR_INVALID_ARG otherwise, nothing launched).
  *
  * The scratch (512 KiB + 256 bytes) is held on every device that loads the
  * library until the process exits. The first call on a device looks up the
  * scratch's device address; make that first call before any stream capture.
  * All calls on one device share the scratch: calls that overlap on the GPU
  * (on different streams, or from host threads without ordering between them)
- * race and must not be made.
+ * race and must not be made. The scratch keeps the last call's contents;
+ * each call clears what must start at zero. The test hook
+ * ef_test_set_lookback_fault applies to this entry too. Testing aid: the
+ * environment variable EF_NOALLOC_FIRST_EPOCH, read at a device's first call,
+ * starts the per-call tag count there (it wraps at 2^30 - 1).
  */
 ef_status ef_hard_threshold_noalloc(const float* g, float* e, float gamma, float lambda,
                                     uint64_t d, uint32_t* idx_out, float* val_out,

@@ -311,6 +311,7 @@ ScanCtx next_scan_ctx(Workspace& ws, uint32_t num_tiles) {
   c.num_tiles = num_tiles;
   c.withheld_tile = withheld_tile();
   c.wait_limit_ns = wait_limit_ns();
+  c.tile_claim = ws.u32(kOffTileClaim);
   return c;
 }
 

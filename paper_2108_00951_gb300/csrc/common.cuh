@@ -7,10 +7,13 @@
 // "Single-pass Parallel Prefix Scan with Decoupled Look-back", NVIDIA
 // NVR-2016-002): every tile publishes its own count as soon as it is known,
 // then reads its predecessors' published counts until it meets an inclusive
-// prefix. A tile's id is its CTA's linear index; CTAs of a one-dimensional
-// grid are dispatched in increasing index order, so every predecessor a tile
-// waits for has started before it. Every wait is bounded in iterations and
-// wall time and latches an error instead of hanging.
+// prefix. In the one-tile-per-CTA kernel a CTA takes its tile id from a
+// global counter when it starts (not from its block index), so every tile it
+// waits for belongs to a CTA that is already running: the scan makes progress
+// whatever order or concurrency the hardware schedules CTAs in. The streaming
+// kernels wait only on lower-numbered CTAs of a cooperative launch, which are
+// all resident. Every wait is bounded in iterations and wall time and latches
+// an error instead of hanging.
 //
 // Throughput of the scan: a tile can only finish once it sees an inclusive
 // prefix, so the set of resolved tiles grows by at most one look-back window
@@ -47,6 +50,10 @@ struct ScanCtx {
   uint32_t num_tiles;
   int64_t withheld_tile;   // test hook: this tile never publishes (-1: none)
   uint64_t wait_limit_ns;  // bound on any single wait
+  // Tile dispenser of the one-tile-per-CTA kernel: [0] tiles handed out,
+  // [1] CTAs finished. Zero between launches: the last CTA to finish resets
+  // both.
+  uint32_t* tile_claim;
 };
 
 // --------------------------------------------------------- memory helpers

@@ -25,7 +25,24 @@ __global__ void __launch_bounds__(kThreads)
     ht_kernel(const GT* __restrict__ g, float* __restrict__ e, float gamma, float lambda,
               uint32_t d, uint32_t* __restrict__ idx_out, float* __restrict__ val_out,
               uint32_t* __restrict__ count_out, ScanCtx ctx) {
-  const uint32_t tile = blockIdx.x;
+  // The tile comes from the dispenser, in the order CTAs start, so every
+  // lower tile this CTA's look-back waits for is held by a running CTA.
+  __shared__ uint32_t s_tile;
+  if (threadIdx.x == 0) s_tile = atomicAdd(ctx.tile_claim, 1u);
+  __syncthreads();
+  const uint32_t tile = s_tile;
+  if (tile >= ctx.num_tiles) {
+    // the dispenser did not start at zero (an earlier launch was cut short):
+    // touch nothing, report it, and still count this CTA as finished
+    if (threadIdx.x == 0) {
+      atomicOr(ctx.error, kDevErrTimeout);
+      if (atomicAdd(ctx.tile_claim + 1, 1u) == gridDim.x - 1) {
+        ctx.tile_claim[0] = 0;
+        ctx.tile_claim[1] = 0;
+      }
+    }
+    return;
+  }
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const uint64_t first = element_index(tile, warp, 0, lane, 0);
 
@@ -72,6 +89,15 @@ __global__ void __launch_bounds__(kThreads)
     }
   }
   compact_tile(ctx, tile, sel, a, idx_out, val_out, count_out, d);
+  if (threadIdx.x == 0) {
+    // every CTA took its tile before it counts itself finished; the last one
+    // leaves the dispenser at zero for the next launch
+    __threadfence();
+    if (atomicAdd(ctx.tile_claim + 1, 1u) == gridDim.x - 1) {
+      ctx.tile_claim[0] = 0;
+      ctx.tile_claim[1] = 0;
+    }
+  }
 }
 
 // The hard-threshold step as a streaming-compaction op: a stage holds a
@@ -183,21 +209,18 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
     StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks(), tiles_out, err_out,
                   ws.errparts()};
     void* params[] = {&op, &d, &idx_out, &val_out, &count_out, &cap, &c, &sa};
-    // A plain launch suffices: the only cross-CTA wait is on lower-numbered
-    // CTAs, which are scheduled first. It may start while the previous kernel
-    // on the stream finishes (the kernel waits for it before its first read).
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(grid);
-    cfg.blockDim = dim3(kStreamThreads);
-    cfg.dynamicSmemBytes = HtStreamKernel<GT>::kSmem;
-    cfg.stream = ws.stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    const cudaError_t err = cudaLaunchKernelExC(
-        &cfg, reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages>), params);
+    // CTAs wait on the chunk totals of lower-numbered CTAs. The grid fits the
+    // device at once (one CTA per SM) and CTAs are dispatched in index order,
+    // so those CTAs are running; the launch is not cooperative because a
+    // cooperative grid cannot start until the previous kernel's CTAs have
+    // all left (5 us per call on the ResNet-18-sized vector). If other work
+    // holds SMs long enough that a lower-numbered CTA cannot start, the
+    // bounded wait ends the call with EF_ERR_TIMEOUT (never a hang or a wrong
+    // result). Programmatic: it may start while the previous kernel on the
+    // stream finishes (the kernel waits for it before its first read).
+    const cudaError_t err = launch_pdl(
+        reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages>), grid,
+        kStreamThreads, HtStreamKernel<GT>::kSmem, ws.stream, params, false);
     count_launch();
     return err;
   }

@@ -2,13 +2,16 @@
 library calls the benchmark times.
 
 Hard-threshold: every output of two workers over two EF iterations is
-compared bit for bit with the oracle, and so is their aggregate. Top-k: the
-ResNet-18-sized case is compared with the oracle over two iterations; the
-larger ones are checked at iteration 0 against properties that fix the Top-k
-result uniquely at any size: exactly k ascending indices, values equal to the
-oracle's a at those indices, residual equal to a with those coordinates
-zeroed, and every selected composite key (|a| bits, then lower index)
-greater than every unselected one.
+compared bit for bit with the oracle, and so is their aggregate; the
+ResNet-50-sized vector at each of its three thresholds. The aggregate of all
+16 ResNet-50 workers' messages is compared with the oracle's over two
+iterations. Top-k: the ResNet-18- and ResNet-50-sized cases (the latter at
+both Top-k fractions, 0.1 % and 1 %) are compared with the oracle over two
+iterations; the larger ones are checked at iteration 0 against properties
+that fix the Top-k result uniquely at any size: exactly k ascending indices,
+values equal to the oracle's a at those indices, residual equal to a with
+those coordinates zeroed, and every selected composite key (|a| bits, then
+lower index) greater than every unselected one.
 """
 import numpy as np
 import pytest
@@ -35,18 +38,19 @@ def _host(g):
     return _bf16_bits(g) if g.dtype == torch.bfloat16 else g.cpu().numpy()
 
 
-def _lambda(w):
+def _lambda(w, which=0):
     if w.density is not None:
         return workloads.density_lambda(w, workloads.gradient(w, 0, 0, device=DEV), w.density)
-    return w.lambdas[0]
+    return w.lambdas[which]
 
 
-@pytest.mark.parametrize("name,dtype", [("resnet18", torch.float32), ("lstm", torch.float32),
-                                        ("resnet50", torch.float32), ("vgg16", torch.float32),
-                                        ("vgg16", torch.bfloat16)])
-def test_full_size_hard_threshold(name, dtype):
+@pytest.mark.parametrize("name,dtype,which", [
+    ("resnet18", torch.float32, 0), ("lstm", torch.float32, 0), ("resnet50", torch.float32, 0),
+    ("resnet50", torch.float32, 1), ("resnet50", torch.float32, 2), ("vgg16", torch.float32, 0),
+    ("vgg16", torch.bfloat16, 0)])
+def test_full_size_hard_threshold(name, dtype, which):
     w = workloads.BY_NAME[name]
-    lam = _lambda(w)
+    lam = _lambda(w, which)
     workers = (0, w.n - 1)
     e_gpu = {i: torch.zeros(w.d, device=DEV) for i in workers}
     e_ref = {i: np.zeros(w.d, np.float32) for i in workers}
@@ -90,16 +94,53 @@ def _check_topk_properties(a, k, gi, gv, ge):
         assert key[sel].min() > key[~sel].max()
 
 
-@pytest.mark.parametrize("name", ["resnet18", "lstm", "resnet50", "vgg16"])
-def test_full_size_topk(name):
+def test_full_size_aggregate_all_workers():
+    # all 16 ResNet-50-sized workers at the densest threshold (1e-4), two EF
+    # iterations: every worker's message against the oracle, then the
+    # aggregate of the 16 messages (with and without their tile indexes)
+    w = workloads.BY_NAME["resnet50"]
+    lam = w.lambdas[0]
+    e_gpu = [torch.zeros(w.d, device=DEV) for _ in range(w.n)]
+    e_ref = [np.zeros(w.d, np.float32) for _ in range(w.n)]
+    idx = [torch.empty(w.d, dtype=torch.int32, device=DEV) for _ in range(w.n)]
+    val = [torch.empty(w.d, dtype=torch.float32, device=DEV) for _ in range(w.n)]
+    tiles = [torch.empty(efs.tiles_for(w.d), dtype=torch.int32, device=DEV) for _ in range(w.n)]
+    cnt = torch.empty(w.n, dtype=torch.int32, device=DEV)
+    for t in range(2):
+        refs = []
+        for i in range(w.n):
+            g = workloads.gradient(w, i, t, device=DEV)
+            efs.ef_hard_threshold(g, e_gpu[i], w.gamma, lam, idx[i], val[i], cnt[i:i + 1],
+                                  tiles_out=tiles[i])
+            ri, rv, e_ref[i] = oracle.ef_hard_threshold(g.cpu().numpy(), e_ref[i], w.gamma, lam)
+            c = int(cnt[i].item())
+            assert c == ri.size, (t, i, c, ri.size)
+            gu.assert_bits(idx[i][:c].cpu().numpy().view(np.uint32), ri, "idx")
+            gu.assert_bits(val[i][:c].cpu().numpy(), rv, "val")
+            gu.assert_bits(e_gpu[i].cpu().numpy(), e_ref[i], "e'")
+            refs.append((ri, rv))
+        want = oracle.sparse_aggregate([r[0] for r in refs], [r[1] for r in refs], w.d)
+        dense = torch.empty(w.d, device=DEV)
+        efs.sparse_aggregate(idx, val, cnt, w.d, dense)
+        gu.assert_bits(dense.cpu().numpy(), want, "aggregate")
+        dense.fill_(float("nan"))
+        efs.sparse_aggregate(idx, val, cnt, w.d, dense, tiles=tiles)
+        gu.assert_bits(dense.cpu().numpy(), want, "aggregate with tile indexes")
+    assert efs.ef_check_status() == efs.EF_OK
+
+
+@pytest.mark.parametrize("name,which", [("resnet18", 0), ("lstm", 0), ("resnet50", 0),
+                                        ("resnet50", 1), ("vgg16", 0)])
+def test_full_size_topk(name, which):
     w = workloads.BY_NAME[name]
-    k = w.topk_values()[0]
+    k = w.topk_values()[which]
     idx = torch.empty(k, dtype=torch.int32, device=DEV)
     val = torch.empty(k, dtype=torch.float32, device=DEV)
     cnt = torch.empty(1, dtype=torch.int32, device=DEV)
     e_gpu = torch.zeros(w.d, device=DEV)
     e_ref = np.zeros(w.d, np.float32)
-    iterations = 2 if name == "resnet18" else 1
+    compare_oracle = name in ("resnet18", "resnet50")
+    iterations = 2 if compare_oracle else 1
     for t in range(iterations):
         g = workloads.gradient(w, 0, t, device=DEV)
         g_host = g.cpu().numpy()
@@ -114,7 +155,7 @@ def test_full_size_topk(name):
         _, _, a = oracle.ef_hard_threshold(g_host, e_before, w.gamma, float("inf"))
         assert np.all(np.isfinite(a))
         _check_topk_properties(a, k, gi, gv, ge)
-        if name == "resnet18":
+        if compare_oracle:
             ri, rv, e_ref = oracle.ef_topk(g_host, e_before, w.gamma, k)
             gu.assert_bits(gi, ri, "idx")
             gu.assert_bits(gv, rv, "val")

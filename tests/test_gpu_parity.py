@@ -110,15 +110,17 @@ def test_ht_zero_length():
     assert int(cnt.item()) == 0
 
 
-def test_ht_concurrent_streams():
+@pytest.mark.parametrize("off", [0, 1])
+def test_ht_concurrent_streams(off):
     # calls on different streams use different workspaces and may overlap
+    # (off = 1: misaligned bases, the look-back kernel and its tile dispenser)
     d = 300_000
     g1, e1 = _inputs(d, 4)
     g2, e2 = _inputs(d, 5)
     s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
     outs = []
     for (g, e), s in (((g1, e1), s1), ((g2, e2), s2)):
-        gd, ed = gu.to_dev(g), gu.to_dev(e)
+        gd, ed = gu.to_dev(g, off), gu.to_dev(e, off)
         idx = torch.empty(d, dtype=torch.int32, device=gu.DEV)
         val = torch.empty(d, dtype=torch.float32, device=gu.DEV)
         cnt = torch.empty(1, dtype=torch.int32, device=gu.DEV)
@@ -133,6 +135,17 @@ def test_ht_concurrent_streams():
         c = int(cnt.item())
         _check_same((idx[:c].cpu().numpy().view(np.uint32), val[:c].cpu().numpy(),
                      ed.cpu().numpy()), oracle.ef_hard_threshold(g, e, 0.1, 1e-3), "stream")
+
+
+def test_ht_lookback_dispenser_back_to_back():
+    # the look-back kernel (misaligned bases) takes its tile ids from a
+    # per-stream dispenser that the last CTA to finish leaves at zero: launches
+    # of different tile counts in a row on one stream, each equal to the oracle
+    for r, d in enumerate([5 * 4096 + 3, 1, 4096, 700_001, 3 * 4096 + 17, 2 * 4096]):
+        g, e = _inputs(d, 30 + r)
+        _check_same(gu.ht(g, e, 0.1, 1.5e-3, g_off=1, e_off=1),
+                    oracle.ef_hard_threshold(g, e, 0.1, 1.5e-3), "back to back d=%d" % d)
+    assert efs.ef_check_status() == efs.EF_OK
 
 
 # ---------------------------------------------------------------------- Top-k

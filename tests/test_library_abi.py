@@ -186,3 +186,26 @@ def test_binding_fails_loudly_on_cpu_tensors():
     i = torch.zeros(8, dtype=torch.int32)
     with pytest.raises(TypeError):
         efs.ef_hard_threshold(x, x.clone(), 0.1, 1e-3, i, x.clone(), i[:1])
+
+
+ST = 0x60000000
+
+
+def _noalloc(g=G, e=E, gamma=0.1, lam=1e-3, d=1000, idx=IDX, val=VAL, cnt=CNT, status=ST):
+    lib = efs.load_library()
+    fn = lib.ef_hard_threshold_noalloc
+    fn.argtypes = [vp, vp, ctypes.c_float, ctypes.c_float, ctypes.c_uint64, vp, vp, vp, vp, vp]
+    fn.restype = ctypes.c_int
+    return fn(vp(g), vp(e), gamma, lam, d, vp(idx), vp(val), vp(cnt), vp(status), vp(0))
+
+
+@pytest.mark.parametrize("kwargs", [
+    dict(d=(1 << 28) + 1), dict(cnt=0), dict(g=0), dict(e=0), dict(idx=0), dict(val=0),
+    dict(lam=-1.0), dict(gamma=float("nan")), dict(e=E + 2), dict(status=ST + 2),
+    dict(idx=E + 64), dict(cnt=VAL + 8),
+    # the status word may not overlap any other buffer
+    dict(status=G), dict(status=E + 400), dict(status=IDX + 3996), dict(status=VAL),
+    dict(status=CNT), dict(d=0, status=CNT),
+])
+def test_noalloc_rejects(kwargs):
+    assert _noalloc(**kwargs) == efs.EF_ERR_INVALID_ARG
