@@ -93,9 +93,13 @@ ef_status acquire_workspace(cudaStream_t stream, uint32_t tiles, uint32_t cand_c
     // everything tagged with an epoch restarts from zero with the epochs
     const size_t clear = kHeaderBytes + sizeof(uint64_t) * ws->status_tiles;
     if (cudaMemsetAsync(ws->base, 0, clear, stream) != cudaSuccess ||
-        cudaMemsetAsync(ws->chunks(), 0, sizeof(uint64_t) * kMaxChunks, stream) != cudaSuccess)
+        cudaMemsetAsync(ws->chunks(), 0, sizeof(uint64_t) * kMaxChunks, stream) != cudaSuccess ||
+        cudaMemsetAsync(ws->ht_chunks(0), 0, 2 * sizeof(uint64_t) * kMaxChunks, stream) !=
+            cudaSuccess)
       return EF_ERR_CUDA;
     ws->epoch = 0;
+    ws->ht_part_ready = false;  // no boundaries written for the next call
+    ws->ht_last_tiles = 0;
     ws->dirty = false;
     if (ws->lw) ws->lw->valid = false;  // re-upload the tables, re-zero their counters
   }

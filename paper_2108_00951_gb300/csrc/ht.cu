@@ -206,8 +206,21 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
     uint32_t cap = d;
     ScanCtx c = ctx;
     // the placement writes each tile's first output position (the tile index)
-    StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks(), tiles_out, err_out,
-                  ws.errparts()};
+    StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.ht_chunks(ws.ht_seq), tiles_out,
+                  err_out, ws.errparts()};
+    // Balanced chunks: the previous call of this size wrote this call's chunk
+    // boundaries; this call writes the next call's from the previous call's
+    // chunk totals (dense regions get fewer tiles). Any boundaries partition
+    // the tiles, so the result never depends on them.
+    const uint32_t seq = ws.ht_seq;
+    const bool same = seq > 0 && ws.ht_last_tiles == tiles && ws.ht_last_grid == grid;
+    // (a call that returns ||e'||^2 uses equal chunks: the norm's summation
+    // order follows the chunks, and it is reproducible for an input)
+    sa.part_in = same && ws.ht_part_ready && !err_out ? ws.ht_part(seq) : nullptr;
+    sa.prev_sums = same ? ws.ht_chunks(seq + 1) : nullptr;   // the other parity: seq - 1
+    sa.prev_part = same && ws.ht_prev_balanced ? ws.ht_part(seq + 2) : nullptr;  // seq - 1
+    sa.prev_epoch = ws.ht_last_epoch;
+    sa.part_out = ws.ht_part(seq + 1);
     void* params[] = {&op, &d, &idx_out, &val_out, &count_out, &cap, &c, &sa};
     // CTAs wait on the chunk totals of lower-numbered CTAs. The grid fits the
     // device at once (one CTA per SM) and CTAs are dispatched in index order,
@@ -222,6 +235,12 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
         reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages>), grid,
         kStreamThreads, HtStreamKernel<GT>::kSmem, ws.stream, params, false);
     count_launch();
+    ws.ht_prev_balanced = sa.part_in != nullptr;
+    ws.ht_part_ready = err == cudaSuccess;
+    ws.ht_last_tiles = tiles;
+    ws.ht_last_grid = grid;
+    ws.ht_last_epoch = c.epoch;
+    ++ws.ht_seq;
     return err;
   }
   const bool vec = (ga % (4 * sizeof(GT)) == 0) && (ea % 16 == 0);

@@ -114,6 +114,14 @@ struct Workspace {
   size_t stage_cap = 0;        // capacity of the pair staging buffers (pairs)
   uint32_t epoch = 0;          // last epoch handed to a compaction launch
   uint32_t topk_calls = 0;     // Top-k calls so far: their parity picks the state block
+  // Balanced chunks of the streaming hard-threshold kernel: each call computes
+  // the next call's chunk boundaries from the previous call's chunk totals.
+  uint32_t ht_seq = 0;          // streaming hard-threshold calls so far
+  uint32_t ht_last_tiles = 0;   // the previous such call's tiles, grid and epoch
+  uint32_t ht_last_grid = 0;
+  uint32_t ht_last_epoch = 0;
+  bool ht_part_ready = false;   // the previous call wrote the boundaries for this one
+  bool ht_prev_balanced = false;  // the previous call used written boundaries
   bool dirty = false;          // header must be re-cleared (failed launch or device timeout)
   LwPlan* lw = nullptr;        // layer-wise Top-k tables (created on first use)
 
@@ -130,7 +138,19 @@ struct Workspace {
   size_t off_errparts() const { return align(off_chunks() + sizeof(uint64_t) * kMaxChunks); }
   size_t off_cntparts() const { return align(off_errparts() + sizeof(FF) * kMaxChunks); }
   size_t off_stage() const { return align(off_cntparts() + sizeof(uint32_t) * kMaxChunks); }
-  size_t total_bytes() const { return align(off_stage() + 8 * stage_cap); }
+  // hard-threshold balancing: chunk totals of the last two calls (by call
+  // parity), then three boundary arrays (by call number mod 3)
+  size_t off_ht() const { return align(off_stage() + 8 * stage_cap); }
+  size_t total_bytes() const {
+    return align(off_ht() + 2 * sizeof(uint64_t) * kMaxChunks + 3 * sizeof(uint32_t) * (kMaxChunks + 1));
+  }
+  uint64_t* ht_chunks(uint32_t parity) const {
+    return reinterpret_cast<uint64_t*>(base + off_ht()) + (parity & 1u) * kMaxChunks;
+  }
+  uint32_t* ht_part(uint32_t which) const {
+    return reinterpret_cast<uint32_t*>(base + off_ht() + 2 * sizeof(uint64_t) * kMaxChunks) +
+           (which % 3u) * (kMaxChunks + 1);
+  }
 
   uint64_t* status() const { return reinterpret_cast<uint64_t*>(base + off_status()); }
   uint64_t* cand(int i) const {
@@ -156,7 +176,7 @@ struct Workspace {
 // Per-device facts queried once.
 struct DeviceInfo {
   int sm_count = 0;
-  int refine_blocks = 0;          // co-resident CTAs for the cooperative Top-k refine
+  int refine_blocks = 0;          // co-resident CTAs of the Top-k select (one wave)
   int finalize_blocks = 0;        // co-resident CTAs for the Top-k finalize
   int ht_stream_per_sm_f32 = 0;   // streaming hard-threshold CTAs per SM (0: unavailable)
   int ht_stream_per_sm_bf16 = 0;

@@ -104,7 +104,83 @@ struct StreamArgs {
   double* err_out;       // optional: sum of a^2 over the coordinates whose residual is final
                          // here (not selected, not deferred), or null
   FF* err_parts;         // [gridDim.x] the CTAs' shares of it
+  // Chunk boundaries (all optional; null: equal chunks of tiles):
+  const uint32_t* part_in;    // [gridDim.x + 1] this launch's boundaries (tiles)
+  const uint64_t* prev_sums;  // the previous launch's chunk totals, (epoch << 32) | total
+  const uint32_t* prev_part;  // the previous launch's boundaries (null: equal chunks)
+  uint32_t prev_epoch;        // the previous launch's epoch
+  uint32_t* part_out;         // [gridDim.x + 1] boundaries computed for the next launch
 };
+
+// Weight of a chunk when the next launch's chunks are balanced: a coordinate
+// counts 2, a selected pair 3 (a staged pair costs about one and a half
+// coordinates of streaming time: the measured per-SM rates of sparse and
+// dense chunks).
+constexpr uint64_t kBalCoord = 2, kBalPair = 3;
+
+// The next launch's left boundary of chunk c, from the previous launch's
+// chunk totals and boundaries, by lanes 1..31 of one warp (lane 0 is busy
+// elsewhere). The chunks' weights are summed, the target c/G of the total
+// is located in one chunk, and the boundary is interpolated inside it
+// (uniform density within a chunk). Monotone in c for any inputs, so the
+// boundaries always partition the tiles. Equal chunks when the previous
+// totals are missing or from another launch.
+__device__ __forceinline__ static uint32_t next_chunk_boundary(const StreamArgs& sa, uint32_t c, uint32_t G, uint32_t T,
+                                        int lane) {
+  constexpr uint32_t kMask = 0xfffffffeu;
+  const uint32_t eq = static_cast<uint32_t>(static_cast<uint64_t>(c) * T / G);
+  if (!sa.prev_sums || c == 0) return c == 0 ? 0u : eq;
+  const uint32_t L = lane - 1;  // 0..30
+  const uint32_t qa = static_cast<uint32_t>(static_cast<uint64_t>(L) * G / 31);
+  const uint32_t qb = static_cast<uint32_t>(static_cast<uint64_t>(L + 1) * G / 31);
+  auto bounds = [&](uint32_t q, uint32_t& lo, uint32_t& hi) {
+    if (sa.prev_part) {
+      lo = min(__ldcg(sa.prev_part + q), T);
+      hi = min(max(__ldcg(sa.prev_part + q + 1), lo), T);
+    } else {
+      lo = static_cast<uint32_t>(static_cast<uint64_t>(q) * T / G);
+      hi = static_cast<uint32_t>(static_cast<uint64_t>(q + 1) * T / G);
+    }
+  };
+  uint64_t mine = 0;
+  bool ok = true;
+  for (uint32_t q = qa; q < qb; ++q) {
+    const uint64_t w = __ldcg(sa.prev_sums + q);
+    uint32_t lo, hi;
+    bounds(q, lo, hi);
+    if (static_cast<uint32_t>(w >> 32) != sa.prev_epoch) ok = false;
+    mine += kBalCoord * kTileElems * (hi - lo) + kBalPair * static_cast<uint32_t>(w);
+  }
+  if (__any_sync(kMask, !ok)) return eq;
+  uint64_t incl = mine;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint64_t v = __shfl_up_sync(kMask, incl, o);
+    if (static_cast<int>(L) >= o) incl += v;
+  }
+  const uint64_t total = __shfl_sync(kMask, incl, 31);
+  const uint64_t target = total / G * c + total % G * c / G;  // floor(total * c / G)
+  const uint64_t excl = incl - mine;
+  uint32_t b = 0;
+  bool here = target >= excl && target < incl;
+  if (here) {
+    uint64_t acc = excl;
+    for (uint32_t q = qa; q < qb; ++q) {
+      const uint64_t w = __ldcg(sa.prev_sums + q);
+      uint32_t lo, hi;
+      bounds(q, lo, hi);
+      const uint64_t wq = kBalCoord * kTileElems * (hi - lo) + kBalPair * static_cast<uint32_t>(w);
+      if (acc + wq > target) {
+        b = lo + static_cast<uint32_t>((target - acc) * (hi - lo) / wq);
+        break;
+      }
+      acc += wq;
+    }
+  }
+  const uint32_t who = __ballot_sync(kMask, here);
+  if (!who) return eq;
+  return min(__shfl_sync(kMask, b, __ffs(who) - 1), T);
+}
 
 // A segment's count (<= 256: 9 bits) and its warp's earlier pairs in the
 // chunk, saturated to 23 bits, in one word.
@@ -143,8 +219,14 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   float* s_pair_val = reinterpret_cast<float*>(smem + L::kRing + kSWarps * L::kWarpPairs * 4);
 
   const uint32_t T = ctx.num_tiles, G = gridDim.x, c = blockIdx.x;
-  const uint32_t t_lo = static_cast<uint32_t>(static_cast<uint64_t>(c) * T / G);
-  const uint32_t t_hi = static_cast<uint32_t>(static_cast<uint64_t>(c + 1) * T / G);
+  // the chunk: written boundaries (by the previous launch, before it let this
+  // one start), else equal chunks
+  uint32_t t_lo = static_cast<uint32_t>(static_cast<uint64_t>(c) * T / G);
+  uint32_t t_hi = static_cast<uint32_t>(static_cast<uint64_t>(c + 1) * T / G);
+  if (sa.part_in) {
+    t_lo = min(__ldcg(sa.part_in + c), T);
+    t_hi = min(max(__ldcg(sa.part_in + c + 1), t_lo), T);
+  }
   const uint32_t rounds = t_hi - t_lo;
   const uint32_t full_tiles = d / kTileElems;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -215,7 +297,18 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   }
 
   if (warp == kProducerWarp) {
-    if (lane == 0) {
+    if (lane != 0) {
+      // lanes 1..31: the next launch's boundary of this chunk, while lane 0
+      // keeps the ring filled; visible before this launch lets the next start
+      if (sa.part_out) {
+        const uint32_t b = next_chunk_boundary(sa, c, G, T, lane);
+        if (lane == 1) {
+          sa.part_out[c] = b;
+          if (c == G - 1) sa.part_out[G] = T;
+          __threadfence();
+        }
+      }
+    } else {
       uint32_t r = rounds < static_cast<uint32_t>(kStages) ? rounds : kStages;
       for (; r < rounds; ++r) {
         const int s = static_cast<int>(r % kStages);

@@ -147,3 +147,24 @@ def test_error_norm_full_size_resnet18():
     _check("ht", g, e, w.gamma, lam, "resnet18 ht")
     _check("topk", g, e, w.gamma, w.topk_values()[0], "resnet18 topk")
     _check("lw", g, e, w.gamma, (ends, ks), "resnet18 layer-wise")
+
+
+@pytest.mark.parametrize("kind", ["ht", "topk"])
+def test_error_norm_reproducible_over_calls(kind):
+    # calls that return the norm use equal chunks and the sampled Top-k bound
+    # (the norm's summation order follows them), so identical inputs give the
+    # same bits however many calls of the size ran before on the stream
+    d = 4 * 2**20 + 3
+    g, e = _inputs(d, 9)
+    g[: d // 5] *= 20.0   # a dense region: balanced chunks would differ from equal ones
+    arg = 1.5e-3 if kind == "ht" else 20_000
+    bits = set()
+    for _ in range(4):
+        bits.add(np.float64(_run(kind, g, e, 0.1, arg)[3]).view(np.uint64).item())
+        # calls without the norm in between (they may balance and use the bound)
+        if kind == "ht":
+            gu.ht(g, e, 0.1, arg)
+        else:
+            gu.topk(g, e, 0.1, arg)
+    assert len(bits) == 1
+    assert efs.ef_check_status() == efs.EF_OK

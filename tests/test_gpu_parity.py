@@ -148,6 +148,37 @@ def test_ht_lookback_dispenser_back_to_back():
     assert efs.ef_check_status() == efs.EF_OK
 
 
+def test_ht_balanced_chunks_over_calls():
+    # each streaming call computes the next call's chunk boundaries from the
+    # previous call's chunk totals; a dense quarter moves them. Calls of one
+    # size in a row (the boundaries in use), a call of another size and a bf16
+    # call between them (the boundaries dropped and rebuilt): every call equal
+    # to the oracle
+    d1, d2 = 5 * 2**20 + 77, 3 * 2**20 + 4099
+    rng = np.random.default_rng(17)
+    e_gpu = {d1: gu.to_dev(np.zeros(d1, np.float32)), d2: gu.to_dev(np.zeros(d2, np.float32))}
+    e_ref = {d1: np.zeros(d1, np.float32), d2: np.zeros(d2, np.float32)}
+    for r, (d, bf16) in enumerate([(d1, False)] * 4 + [(d2, False), (d1, False), (d1, True),
+                                                         (d1, False), (d1, False)]):
+        g = (rng.standard_normal(d) * 1e-2).astype(np.float32)
+        g[: d // 4] *= 30.0 if r % 2 else 1.0          # the dense region comes and goes
+        g[d // 2: d // 2 + d // 8] *= 10.0
+        if bf16:
+            g = (g.view(np.uint32) >> 16).astype(np.uint16)
+        gd = gu.g_device(g)
+        idx = torch.full((d,), -1, dtype=torch.int32, device=gu.DEV)
+        val = torch.empty(d, dtype=torch.float32, device=gu.DEV)
+        cnt = torch.zeros(1, dtype=torch.int32, device=gu.DEV)
+        efs.ef_hard_threshold(gd, e_gpu[d], 0.1, 2e-3, idx, val, cnt)
+        ri, rv, e_ref[d] = oracle.ef_hard_threshold(g, e_ref[d], 0.1, 2e-3)
+        c = int(cnt.item())
+        assert c == ri.size, (r, c, ri.size)
+        gu.assert_bits(idx[:c].cpu().numpy().view(np.uint32), ri, "idx call %d" % r)
+        gu.assert_bits(val[:c].cpu().numpy(), rv, "val call %d" % r)
+        gu.assert_bits(e_gpu[d].cpu().numpy(), e_ref[d], "e' call %d" % r)
+    assert efs.ef_check_status() == efs.EF_OK
+
+
 # ---------------------------------------------------------------------- Top-k
 # ------------------------------------------- on-chip staging and its spill
 # The streaming compaction keeps each compute warp's first pairs of its CTA's
@@ -256,6 +287,30 @@ def test_topk_nan_inf():
         _check_same(gu.topk(g, e, 0.1, k), oracle.ef_topk(g, e, 0.1, k), "nan k=%d" % k)
 
 
+def test_topk_calls_in_a_row_with_jumping_scales():
+    # calls of one (k, d) on one stream whose scales jump by 100x between
+    # calls, and a call with another k between them (the per-call state and
+    # the sampled bound start afresh each time): every call equal to the oracle
+    d, k = 3 * 2**20 + 517, 3000
+    rng = np.random.default_rng(23)
+    e_gpu = gu.to_dev(np.zeros(d, np.float32))
+    e_ref = np.zeros(d, np.float32)
+    for r, (scale, kk) in enumerate([(1.0, k), (1.0, k), (100.0, k), (1.0, k), (0.01, k),
+                                     (0.01, k), (1.0, k + 1), (1.0, k), (1.0, k)]):
+        g = (rng.standard_normal(d) * 1e-2 * scale).astype(np.float32)
+        gd = gu.to_dev(g)
+        idx = torch.full((kk,), -1, dtype=torch.int32, device=gu.DEV)
+        val = torch.empty(kk, dtype=torch.float32, device=gu.DEV)
+        cnt = torch.zeros(1, dtype=torch.int32, device=gu.DEV)
+        efs.ef_topk(gd, e_gpu, 0.1, kk, idx, val, cnt)
+        ri, rv, e_ref = oracle.ef_topk(g, e_ref, 0.1, kk)
+        assert int(cnt.item()) == kk
+        gu.assert_bits(idx.cpu().numpy().view(np.uint32), ri, "idx call %d" % r)
+        gu.assert_bits(val.cpu().numpy(), rv, "val call %d" % r)
+        gu.assert_bits(e_gpu.cpu().numpy(), e_ref, "e' call %d" % r)
+    assert efs.ef_check_status() == efs.EF_OK
+
+
 # ---------------------------------------------------------------- aggregation
 def _sparse_lists(n, d, density, seed, integer=False):
     rng = _rng("agg", n, d, seed)
@@ -317,6 +372,51 @@ def test_aggregate_tile_boundary_layouts():
     vals = [rng.standard_normal(len(x)).astype(np.float32) for x in lists]
     gu.assert_bits(gu.aggregate(lists, vals, d), oracle.sparse_aggregate(lists, vals, d),
                    "tile layouts")
+    assert efs.ef_check_status() == efs.EF_OK
+
+
+@pytest.mark.parametrize("n", [33, 100])
+def test_aggregate_many_workers(n):
+    # more workers than one stage takes (32 runs): the runs of a tile are
+    # staged in several groups, in worker order
+    d = 3 * 4096 + 7
+    for density in (0.01, 0.4):
+        idx, val = _sparse_lists(n, d, density, 5)
+        gu.assert_bits(gu.aggregate(idx, val, d), oracle.sparse_aggregate(idx, val, d),
+                       "n=%d rho=%g" % (n, density))
+
+
+@pytest.mark.parametrize("offs", [(1, 0), (0, 3), (2, 2)])
+def test_aggregate_misaligned_lists(offs):
+    # lists that are not 16-byte aligned take the 4-byte staging path; one
+    # such list is enough
+    d = 5 * 4096 + 11
+    idx, val = _sparse_lists(6, d, 0.2, 6)
+    idx_t = [gu.to_dev(i.view(np.int32), offs[0] if w == 3 else 0) for w, i in enumerate(idx)]
+    val_t = [gu.to_dev(v, offs[1] if w == 3 else 0) for w, v in enumerate(val)]
+    counts = torch.tensor([len(i) for i in idx], dtype=torch.int32, device=gu.DEV)
+    dense = torch.full((d,), float("nan"), device=gu.DEV)
+    efs.sparse_aggregate(idx_t, val_t, counts, d, dense)
+    torch.cuda.synchronize()
+    gu.assert_bits(dense.cpu().numpy(), oracle.sparse_aggregate(idx, val, d), "offs %s" % (offs,))
+    assert efs.ef_check_status() == efs.EF_OK
+
+
+def test_aggregate_runs_across_stages():
+    # runs longer than a stage (1024 staged elements), runs that start and
+    # end at every residue modulo 4, and a tile whose pairs are all in one
+    # warp's coordinates
+    d = 8 * 4096
+    rng = np.random.default_rng(41)
+    lists = []
+    for w in range(7):
+        start = 4096 + w            # every start residue
+        lists.append(np.arange(start, 3 * 4096 - w, 1 + (w % 3), dtype=np.uint32))
+    lists.append(np.arange(5 * 4096 + 600, 5 * 4096 + 1000, dtype=np.uint32))
+    lists.append(np.sort(rng.choice(d, 9000, replace=False)).astype(np.uint32))
+    vals = [rng.standard_normal(len(x)).astype(np.float32) for x in lists]
+    gu.assert_bits(gu.aggregate(lists, vals, d), oracle.sparse_aggregate(lists, vals, d),
+                   "long runs")
     assert efs.ef_check_status() == efs.EF_OK
 
 
