@@ -63,12 +63,13 @@
  * DIFFERENT streams never share a workspace and may run concurrently; calls
  * on the same stream are ordered by the stream.
  *
- * Concurrency: a compress call's CTAs wait (bounded) for lower-numbered CTAs
- * of the same launch, which the device dispatches first and which fit the
- * device together when it is otherwise idle. If kernels on other streams or
- * other processes (MPS) hold SMs long enough that such a CTA cannot start
- * within the bound (2 s), the call fails with EF_ERR_TIMEOUT (reported by
- * ef_check_status); it never hangs and never returns a wrong result. The
+ * Concurrency: the streaming kernels' CTAs wait (bounded) only for
+ * lower-numbered CTAs of the same launch, which the device dispatches first;
+ * kernels that wait on every CTA of their grid (the Top-k kernels, the
+ * layer-wise select with teams) are cooperative launches. If kernels on other
+ * streams or other processes (MPS) hold SMs long enough that a CTA cannot
+ * start within the bound (2 s), the call fails with EF_ERR_TIMEOUT (reported
+ * by ef_check_status); it never hangs and never returns a wrong result. The
  * one-tile-per-CTA path (misaligned g or e, ef_hard_threshold_noalloc) takes
  * its tiles in the order CTAs start and needs no co-residency.
  */

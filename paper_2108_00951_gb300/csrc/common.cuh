@@ -11,11 +11,10 @@
 // global counter when it starts (not from its block index), so every tile it
 // waits for belongs to a CTA that is already running: the scan makes progress
 // whatever order or concurrency the hardware schedules CTAs in. The streaming
-// kernels' grids are one CTA per SM: they fit the device at once and their
-// CTAs are dispatched in index order, so the lower-numbered CTAs they wait
-// for are running (with other work holding SMs, a bounded wait can run out:
-// a latched timeout, never a hang). Every wait is bounded in iterations and wall time and latches
-// an error instead of hanging.
+// kernels' CTAs wait only for lower-numbered CTAs of their grid, which are
+// dispatched first; kernels with grid-wide barriers are cooperative launches.
+// Every wait is bounded in iterations and wall time and latches an error
+// instead of hanging.
 //
 // Throughput of the scan: a tile can only finish once it sees an inclusive
 // prefix, so the set of resolved tiles grows by at most one look-back window
@@ -284,7 +283,7 @@ __device__ __forceinline__ FF sum_parts_ff(const FF* parts, uint32_t n, FF* s_ff
   return block_sum_ff(v, s_ff);
 }
 
-// Bounded grid-wide barrier for a grid whose CTAs are all resident at once.
+// Bounded grid-wide barrier for a cooperative launch (all CTAs co-resident).
 // Returns false, latching kDevErrTimeout, if the wait ran out.
 // Programmatic dependent launch: wait until the grids this one depends on
 // have completed and their memory is visible (a no-op when the launch did

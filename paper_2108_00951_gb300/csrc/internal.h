@@ -176,7 +176,7 @@ struct Workspace {
 // Per-device facts queried once.
 struct DeviceInfo {
   int sm_count = 0;
-  int refine_blocks = 0;          // co-resident CTAs of the Top-k select (one wave)
+  int refine_blocks = 0;          // co-resident CTAs for the cooperative Top-k select
   int finalize_blocks = 0;        // co-resident CTAs for the Top-k finalize
   int ht_stream_per_sm_f32 = 0;   // streaming hard-threshold CTAs per SM (0: unavailable)
   int ht_stream_per_sm_bf16 = 0;

@@ -113,10 +113,10 @@ struct StreamArgs {
 };
 
 // Weight of a chunk when the next launch's chunks are balanced: a coordinate
-// counts 2, a selected pair 3 (a staged pair costs about one and a half
-// coordinates of streaming time: the measured per-SM rates of sparse and
-// dense chunks).
-constexpr uint64_t kBalCoord = 2, kBalPair = 3;
+// counts 2, a selected pair 5 (a staged pair costs about two and a half
+// coordinates of a CTA's time, staging and placement together; 3 and 8 were
+// measured slower on dense vectors).
+constexpr uint64_t kBalCoord = 2, kBalPair = 5;
 
 // The next launch's left boundary of chunk c, from the previous launch's
 // chunk totals and boundaries, by lanes 1..31 of one warp (lane 0 is busy

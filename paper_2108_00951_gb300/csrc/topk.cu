@@ -892,15 +892,14 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
     StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks(), nullptr,
                   err_out ? ws.stream_err() : nullptr, ws.errparts()};
     void* params[] = {&op, &d, &args.list_idx, &args.list_val, &args.list_count, &cap, &ctx, &sa};
-    // Not a cooperative launch, although the pre-pass has a grid barrier: the
-    // grid (one CTA per SM) fits the device at once, so once the previous
-    // kernel's CTAs leave every CTA becomes resident; a cooperative grid
-    // could not start before they all have left (3-5 us per call). If other
-    // work holds SMs beyond the bounded wait, the call ends with
-    // EF_ERR_TIMEOUT instead of hanging.
+    // A cooperative launch: the pre-pass ends in a grid barrier, which needs
+    // every CTA resident at once even when calls on other streams compete
+    // for the SMs (a plain launch was 3-5 us per call faster, but two such
+    // grids dispatched in part side by side could each wait on CTAs that
+    // cannot start).
     err = launch_pdl(
         reinterpret_cast<const void*>(&stream_compact_kernel<TopkCandOp<GT>, kTkStages>), grid,
-        kStreamThreads, StreamLayout<TopkCandOp<GT>, kTkStages>::kSmem, ws.stream, params, false);
+        kStreamThreads, StreamLayout<TopkCandOp<GT>, kTkStages>::kSmem, ws.stream, params, true);
     count_launch();
     if (err != cudaSuccess) return err;
   } else {
@@ -918,9 +917,9 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
                     (void*)&count_out, (void*)&args};
   uint32_t grid = static_cast<uint32_t>(dev.refine_blocks);
   if (grid > kMaxChunks) grid = kMaxChunks;
-  // (one resident wave: not cooperative, for the reason given for the stream)
+  // (cooperative, for the reason given for the stream: grid barriers)
   err = launch_pdl(reinterpret_cast<const void*>(&topk_select_kernel), grid, kSelThreads,
-                   kSelSmem, ws.stream, params, false);
+                   kSelSmem, ws.stream, params, true);
   count_launch();
   if (err == cudaSuccess && err_out && !streamable) err = launch_error_norm(e, d, err_out, ws, dev);
   return err;

@@ -842,10 +842,8 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t d, uint32_
     count_launch();
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
   }
-  // 3 select: the teams' CTAs wait for one another; the grid is one resident
-  // wave (the plan keeps it within the co-resident budget), so it is a plain
-  // programmatic launch like the streaming kernels (a cooperative one could
-  // not start before the previous kernel's CTAs have all left)
+  // 3 select: a cooperative launch when there are teams, so that every
+  // team's CTAs are resident
   LwArgs a;
   a.segs = segs;
   a.mbound = mbound;
@@ -869,8 +867,9 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t d, uint32_
   a.err_parts = ws.errparts();
   a.err_arrive = state + kStErrArrive / 4;
   void* params[] = {(void*)&e, (void*)&idx_out, (void*)&val_out, (void*)&a};
+  // (cooperative only when there are teams: nothing else waits on another CTA)
   err = launch_pdl(reinterpret_cast<const void*>(&lw_select_kernel), p.n_select_ctas, kLwThreads,
-                   kLwSelectSmem, ws.stream, params, false);
+                   kLwSelectSmem, ws.stream, params, p.n_teams > 0);
   count_launch();
   if (err == cudaSuccess && err_out && !streamable) err = launch_error_norm(e, d, err_out, ws, dev);
   return err;
@@ -951,7 +950,7 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
   // memory, or whose own length would make a selection from e slow for one
   // CTA, gets a team of co-resident CTAs; the others go, longest first, onto
   // the least loaded of the remaining CTAs. At most sm_count x (select CTAs
-  // per SM) CTAs in all, so that the whole grid is resident at once.
+  // per SM) CTAs in all, so that the cooperative launch is resident.
   const uint32_t budget =
       static_cast<uint32_t>(std::max(1, dev.sm_count * std::max(1, dev.lw_select_per_sm)));
   std::vector<uint32_t> team_seg, team_size, singles;

@@ -137,6 +137,41 @@ def test_ht_concurrent_streams(off):
                      ed.cpu().numpy()), oracle.ef_hard_threshold(g, e, 0.1, 1e-3), "stream")
 
 
+@pytest.mark.parametrize("kind", ["topk", "topk_layerwise"])
+def test_topk_concurrent_streams(kind):
+    # Top-k calls on different streams (their own workspaces) may overlap on
+    # the device; their grid-wide barriers need every CTA resident, which the
+    # cooperative launches guarantee whatever the other stream runs
+    d, k = 2 * 2**20 + 333, 4000
+    seg_end = [d // 3, d // 2, d]
+    seg_k = [1500, 1000, 1500]
+    ins = [_inputs(d, 40), _inputs(d, 41), _inputs(d, 42)]
+    streams = [torch.cuda.Stream() for _ in ins]
+    outs = []
+    for (g, e), s in zip(ins, streams):
+        gd, ed = gu.to_dev(g), gu.to_dev(e)
+        idx = torch.empty(k, dtype=torch.int32, device=gu.DEV)
+        val = torch.empty(k, dtype=torch.float32, device=gu.DEV)
+        cnt = torch.empty(1, dtype=torch.int32, device=gu.DEV)
+        outs.append((gd, ed, idx, val, cnt))
+    torch.cuda.synchronize()
+    for rep in range(3):
+        for (g, e), s, (gd, ed, idx, val, cnt) in zip(ins, streams, outs):
+            with torch.cuda.stream(s):
+                ed.copy_(torch.from_numpy(e).to(gu.DEV, non_blocking=True))
+                if kind == "topk":
+                    efs.ef_topk(gd, ed, 0.1, k, idx, val, cnt)
+                else:
+                    efs.ef_topk_layerwise(gd, ed, 0.1, seg_end, seg_k, idx, val, cnt)
+    torch.cuda.synchronize()
+    for (g, e), (gd, ed, idx, val, cnt) in zip(ins, outs):
+        want = (oracle.ef_topk(g, e, 0.1, k) if kind == "topk"
+                else oracle.ef_topk_layerwise(g, e, 0.1, seg_end, seg_k))
+        _check_same((idx.cpu().numpy().view(np.uint32), val.cpu().numpy(), ed.cpu().numpy()),
+                    want, kind + " concurrent")
+    assert efs.ef_check_status() == efs.EF_OK
+
+
 def test_ht_lookback_dispenser_back_to_back():
     # the look-back kernel (misaligned bases) takes its tile ids from a
     # per-stream dispenser that the last CTA to finish leaves at zero: launches
