@@ -33,33 +33,79 @@ struct AggPtrs {
 };
 
 // off[i * (tiles + 1) + t] = number of entries of list i below t * kAggTile;
-// off[i * (tiles + 1) + tiles] = counts[i].
+// off[i * (tiles + 1) + tiles] = counts[i]. Grid: blockIdx.y = list, x over
+// the tiles + 1 entries. Two ways to the same numbers, chosen per list:
+//  - a list with at least (tiles + 1) / 16 and at most 8 (tiles + 1) entries
+//    is scattered: entry p (p = 0..count, count standing for the end) owns the
+//    tiles t with list[p - 1] < t * kAggTile <= list[p] and writes p there —
+//    two loads per entry and no dependent chain; a run of more than 8 tiles
+//    is written by the whole warp;
+//  - other lists: one binary search per tile (14-23 dependent loads, but
+//    independent of the list's length).
+// Either way every entry lies in [0, count]; a list that is not strictly
+// ascending is latched as bad input (scatter) and may leave entries the
+// reduction clamps to the list.
 __global__ void __launch_bounds__(kThreads)
     agg_offsets_kernel(AggPtrs p, const uint32_t* __restrict__ counts, uint32_t n,
-                       uint32_t tiles, uint32_t* __restrict__ off) {
+                       uint32_t tiles, uint32_t* __restrict__ off, uint32_t* __restrict__ error) {
   griddep_wait();                // the lists and counts come from the kernels before
   griddep_launch_dependents();    // the reduction may be scheduled (it waits for this grid)
-  const uint64_t per = static_cast<uint64_t>(tiles) + 1;
-  const uint64_t gid = static_cast<uint64_t>(blockIdx.x) * kThreads + threadIdx.x;
-  if (gid >= per * n) return;
-  const uint32_t i = static_cast<uint32_t>(gid / per);
-  const uint32_t t = static_cast<uint32_t>(gid % per);
+  const uint32_t per = tiles + 1;
+  const uint32_t i = blockIdx.y;
+  const uint32_t tx = blockIdx.x * kThreads + threadIdx.x;
+  const uint32_t stride = gridDim.x * kThreads;  // >= per
+  const int lane = threadIdx.x & 31;
   const uint32_t cnt = counts[i];
-  uint32_t result = cnt;
-  if (t < tiles) {
-    const uint64_t target = static_cast<uint64_t>(t) * kAggTile;
-    const uint32_t* x = p.idx[i];
-    uint32_t lo = 0, hi = cnt;
-    while (lo < hi) {
-      const uint32_t mid = lo + (hi - lo) / 2;
-      if (static_cast<uint64_t>(__ldg(x + mid)) < target)
-        lo = mid + 1;
-      else
-        hi = mid;
+  const uint32_t* x = p.idx[i];
+  uint32_t* o = off + static_cast<uint64_t>(i) * per;
+  const bool scatter = cnt >= per / 16 && static_cast<uint64_t>(cnt) <= 8ull * per;
+  if (!scatter) {
+    if (tx >= per) return;
+    uint32_t result = cnt;
+    if (tx < tiles) {
+      const uint64_t target = static_cast<uint64_t>(tx) * kAggTile;
+      uint32_t lo = 0, hi = cnt;
+      while (lo < hi) {
+        const uint32_t mid = lo + (hi - lo) / 2;
+        if (static_cast<uint64_t>(__ldg(x + mid)) < target)
+          lo = mid + 1;
+        else
+          hi = mid;
+      }
+      result = lo;
     }
-    result = lo;
+    o[tx] = result;
+    return;
   }
-  off[gid] = result;
+  bool bad = false;
+#pragma unroll 1
+  for (uint32_t q = 0; q < 9; ++q) {  // positions tx + q * stride <= cnt (cnt <= 8 per)
+    const uint32_t pos = tx + q * stride;
+    const bool has = pos <= cnt;
+    uint32_t t_lo = 1, t_hi = 0;  // empty
+    if (has) {
+      const uint32_t cur = pos < cnt ? __ldg(x + pos) : 0u;
+      const uint32_t prev = pos > 0 ? __ldg(x + pos - 1) : 0u;
+      if (pos > 0 && pos < cnt && prev >= cur) bad = true;  // not strictly ascending
+      t_lo = pos == 0 ? 0u : min(prev / kAggTile + 1u, per);
+      t_hi = pos == cnt ? tiles : min(cur / kAggTile, tiles - 1u);
+      if (pos < cnt && t_hi < t_lo) t_lo = t_hi + 1;  // nothing (malformed, or a shared tile)
+    }
+    const bool mine = has && t_lo <= t_hi && t_hi - t_lo < 8;
+    if (mine)
+      for (uint32_t t = t_lo; t <= t_hi; ++t) o[t] = pos;
+    // longer runs: the whole warp writes them, one run after another
+    uint32_t m = __ballot_sync(0xffffffffu, has && t_lo <= t_hi && !mine);
+    while (m) {
+      const int l = __ffs(m) - 1;
+      m &= m - 1;
+      const uint32_t a = __shfl_sync(0xffffffffu, t_lo, l);
+      const uint32_t b = __shfl_sync(0xffffffffu, t_hi, l);
+      const uint32_t v = __shfl_sync(0xffffffffu, pos, l);
+      for (uint32_t t = a + lane; t <= b; t += 32) o[t] = v;
+    }
+  }
+  if (bad) atomicOr(error, kDevErrBadInput);
 }
 
 // What the reduction does with a finished tile.
@@ -122,14 +168,10 @@ __global__ void __launch_bounds__(kThreads)
   griddep_wait();  // the offsets (and everything before them) are complete
   for (uint32_t i = threadIdx.x; i < n; i += kThreads) {
     // the list's range in this tile: from the offsets kernel, or from the
-    // caller's tile index (clamped to the list, so never out of bounds)
+    // caller's tile index, clamped to the list (never out of bounds)
     const uint32_t* r = off ? off + static_cast<uint64_t>(i) * (tiles + 1) : p.tiles[i];
-    uint32_t lo = r[t], hi = r[t + 1];
-    if (!off) {
-      const uint32_t cnt = counts[i];
-      lo = min(lo, cnt);
-      hi = min(hi, cnt);
-    }
+    const uint32_t cnt = counts[i];
+    uint32_t lo = min(r[t], cnt), hi = min(r[t + 1], cnt);
     s_lo[i] = lo;
     s_pre[i + 1] = hi > lo ? hi - lo : 0u;  // this tile's pairs of worker i
   }
@@ -246,12 +288,12 @@ cudaError_t launch_common(uint32_t n, const uint32_t* const* idx, const float* c
   cudaError_t err = cudaSuccess;
   uint32_t* off = nullptr;
   if (!tile_index) {  // locate each list's tile boundaries first
-    const uint64_t entries = static_cast<uint64_t>(n) * (tiles + 1);
-    const uint32_t grid1 = static_cast<uint32_t>((entries + kThreads - 1) / kThreads);
+    const dim3 grid1((tiles + 1 + kThreads - 1) / kThreads, n);
     off = ws.offsets();
     const uint32_t* counts_arg = counts;
     uint32_t n_arg = n, tiles_arg = tiles;
-    void* params[] = {&p, &counts_arg, &n_arg, &tiles_arg, &off};
+    uint32_t* error = ws.u32(kOffError);
+    void* params[] = {&p, &counts_arg, &n_arg, &tiles_arg, &off, &error};
     err = launch_pdl(reinterpret_cast<const void*>(&agg_offsets_kernel), grid1, kThreads, 0,
                      ws.stream, params, false);
     count_launch();
@@ -308,8 +350,9 @@ cudaError_t launch_list_tiles(const uint32_t* idx, const uint32_t* count, uint32
     p.tiles[i] = nullptr;
   }
   uint32_t n = 1, tiles = agg_tiles_for(d);
-  const uint32_t grid = (tiles + 1 + kThreads - 1) / kThreads;
-  void* params[] = {&p, &count, &n, &tiles, &tiles_out};
+  const dim3 grid((tiles + 1 + kThreads - 1) / kThreads, 1);
+  uint32_t* error = ws.u32(kOffError);
+  void* params[] = {&p, &count, &n, &tiles, &tiles_out, &error};
   const cudaError_t err = launch_pdl(reinterpret_cast<const void*>(&agg_offsets_kernel), grid,
                                      kThreads, 0, ws.stream, params, false);
   count_launch();

@@ -280,10 +280,10 @@ ef_status topk_layerwise_entry(const void* g, bool bf16, float* e, float gamma, 
 // A launch that may begin while the previous kernel on the stream finishes
 // (programmatic dependent launch; every kernel here waits for its
 // predecessor before reading what it wrote), optionally cooperative.
-cudaError_t launch_pdl(const void* fn, uint32_t grid, uint32_t block, uint32_t smem,
+cudaError_t launch_pdl(const void* fn, dim3 grid, uint32_t block, uint32_t smem,
                        cudaStream_t stream, void** params, bool cooperative) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid);
+  cfg.gridDim = grid;
   cfg.blockDim = dim3(block);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;

@@ -218,7 +218,7 @@ cudaError_t launch_error_norm(const float* e, uint32_t d, double* err_out, Works
 // A launch that may begin while the previous kernel on the stream finishes
 // (programmatic dependent launch: the kernel waits for its predecessor with
 // griddepcontrol.wait before reading what it wrote), optionally cooperative.
-cudaError_t launch_pdl(const void* fn, uint32_t grid, uint32_t block, uint32_t smem,
+cudaError_t launch_pdl(const void* fn, dim3 grid, uint32_t block, uint32_t smem,
                        cudaStream_t stream, void** params, bool cooperative);
 void count_launch();
 uint64_t wait_limit_ns();
