@@ -65,7 +65,7 @@
  *
  * Concurrency: the streaming kernels' CTAs wait (bounded) only for
  * lower-numbered CTAs of the same launch, which the device dispatches first;
- * kernels that wait on every CTA of their grid (the Top-k kernels, the
+ * kernels that wait on every CTA of their grid (the Top-k select, the
  * layer-wise select with teams) are cooperative launches. If kernels on other
  * streams or other processes (MPS) hold SMs long enough that a CTA cannot
  * start within the bound (2 s), the call fails with EF_ERR_TIMEOUT (reported

@@ -48,7 +48,6 @@
 //
 // An Op supplies the per-segment work:
 //   static constexpr uint32_t kStageBytes;            bytes of one stage
-//   static constexpr bool kPrepass;                   see below
 //   void fill(unsigned char* stage, uint32_t tile, uint64_t* bar, uint64_t pol)
 //        issue the bulk copies of a full tile (after expect_tx)
 //   void tile_smem(const unsigned char* stage, uint32_t tile, int warp, int lane,
@@ -57,20 +56,12 @@
 //        compute values and selection bits (and side effects) of the calling
 //        warp's segment, from the stage of a full tile, or from global memory
 //        for the partial last tile.
-//   (tile_smem and tile_global also receive `aux`, the pre-pass result or 0)
+//   (tile_smem and tile_global also receive `aux`, from
+//   uint64_t initial_aux()  (all threads, after the wait for the previous
+//   kernel; uniform))
 //   void prologue()                     every thread, once, at the start
 //   static constexpr uint32_t kPrefetchTiles;  tiles of the chunk pulled toward
 //   void prefetch(uint32_t tile)               L2 before the wait for the previous kernel
-// Optional pre-pass (kPrepass): before streaming, the compute threads sample
-// their CTA's chunk of tiles [t_lo, t_hi) with
-//   void sample(uint32_t t_lo, uint32_t t_hi, int tid, uint32_t* s_hist)
-//                                       (accumulate a kSampleBins histogram)
-// the CTA merges its histogram with
-//   void merge(const uint32_t* s_hist)  (all threads)
-// and after a grid barrier every CTA computes the same value with
-//   uint64_t choose()                   (all threads; uniform result)
-// which becomes `aux`. The producer warp issues its first fills before the
-// pre-pass, so the ring is loading while the CTAs sample and synchronise.
 // Element layout: unit v of lane l of warp w covers the 4 coordinates from
 // tile * kTileElems + w * 256 + v * 128 + l * 4 (see stream_element_index).
 #pragma once
@@ -213,7 +204,6 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   __shared__ uint32_t s_scratch[kStreamThreads / 32];
   __shared__ FF s_err[kSWarps];
   __shared__ FF s_err_sum[32];
-  __shared__ uint32_t s_sample_hist[Op::kPrepass ? Op::kSampleBins : 1];
   using L = StreamLayout<Op, kStages>;
   uint32_t* s_pair_idx = reinterpret_cast<uint32_t*>(smem + L::kRing);
   float* s_pair_val = reinterpret_cast<float*>(smem + L::kRing + kSWarps * L::kWarpPairs * 4);
@@ -273,28 +263,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
     for (uint32_t r = 0; r < rounds && r < static_cast<uint32_t>(kStages); ++r) fill(r);
   }
 
-  uint64_t aux = 0;
-  if constexpr (Op::kPrepass) {
-    for (int b = threadIdx.x; b < Op::kSampleBins; b += kStreamThreads) s_sample_hist[b] = 0;
-    __syncthreads();
-    if (warp < kSWarps && rounds > 0) op.sample(t_lo, t_hi, threadIdx.x, s_sample_hist);
-    if (__syncthreads_or(failed)) {
-      if (threadIdx.x == 0) atomicOr(ctx.error, kDevErrTimeout);
-      if (producer)  // no copy may land after the CTA exits
-        for (uint32_t q = 0; q < rounds && q < static_cast<uint32_t>(kStages); ++q)
-          mbar_wait(&s_full[q], 0, ctx.wait_limit_ns);
-      return;
-    }
-    op.merge(s_sample_hist);
-    const bool passed = op.barrier(ctx.wait_limit_ns, ctx.error);
-    if (!passed) {
-      if (producer)
-        for (uint32_t q = 0; q < rounds && q < static_cast<uint32_t>(kStages); ++q)
-          mbar_wait(&s_full[q], 0, ctx.wait_limit_ns);
-      return;
-    }
-    aux = op.choose();
-  }
+  const uint64_t aux = op.initial_aux();  // uniform
 
   if (warp == kProducerWarp) {
     if (lane != 0) {

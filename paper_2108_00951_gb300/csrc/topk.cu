@@ -11,18 +11,18 @@
 // { j : K_j >= K_(k) } for the k-th largest key K_(k).
 //
 // Kernels of one call:
-//  1 stream   the streaming compaction of stream_compact.cuh with a sampling
-//             pre-pass: every CTA histograms the top 13 key bits of 2048
-//             coordinates spread over its chunk, the histograms are merged,
-//             and after a grid barrier every CTA derives the same lower bound
-//             B with about 1.5 times the needed mass above it (or, when the
-//             candidates would not fit, the full-array mode). Then
-//             a = fmaf(γ,g,e) is written over e (12 B per coordinate, the
+//  1 sample   every CTA histograms the top 13 key bits of 2048 coordinates
+//             spread over its share of the tiles, the histograms are merged,
+//             and the last CTA to arrive derives the lower bound B with about
+//             1.5 times the needed mass above it (or, when the candidates
+//             would not fit, the full-array mode).
+//  2 stream   the streaming compaction of stream_compact.cuh: a =
+//             fmaf(γ,g,e) is written over e (12 B per coordinate, the
 //             algorithmic bytes) and the coordinates with K_j >= B are
 //             emitted as an ordered (index, value) candidate list. This
 //             kernel also zeroes the other of the two per-call state blocks
 //             for the next call.
-//  2 select   the exact threshold K_(k) over the candidates — or over all of
+//  3 select   the exact threshold K_(k) over the candidates — or over all of
 //             a when the candidates are short of k, overflowed, or were not
 //             gathered — then the ordered compaction of K_j >= K_(k), zeroing
 //             e at the selected coordinates. Up to 48 K candidates CTA 0
@@ -78,12 +78,14 @@ struct TopkArgs {
 };
 
 // ------------------------------------------------------------- 1 stream
-// The streaming pass as a stream_compact op. Pre-pass: every CTA histograms
-// the top 13 key bits of 2048 coordinates spread evenly over its chunk, the
-// histograms are merged, and after a grid barrier every CTA derives the same
-// lower bound B with about 1.5 times the needed mass above it — or, when the candidates would not fit, chooses the
-// full-array mode and gathers none. Streaming: a = fmaf(γ,g,e) is written over
-// e and the coordinates with K_j >= B are selected (ordered candidates).
+// The streaming pass as a stream_compact op, with the sampling of its bound
+// (run by topk_sample_kernel): every sample CTA histograms the top 13 key
+// bits of 2048 coordinates spread evenly over its share of the tiles, the
+// histograms are merged, and the last CTA derives the lower bound B with about
+// 1.5 times the needed mass above it — or, when the candidates would not fit,
+// chooses the full-array mode (nothing gathered). Streaming: a = fmaf(γ,g,e)
+// is written over e and the coordinates with K_j >= B are selected (ordered
+// candidates).
 template <typename GT>
 struct TopkCandOp {
   const GT* g;
@@ -91,14 +93,13 @@ struct TopkCandOp {
   float gamma;
   uint32_t d, k, cand_cap;
   uint32_t* hist;      // global sample histogram [kSampleBins]
-  uint32_t* stream_arrive;  // arrivals at the pre-pass barrier (zero at the call's start)
+  uint32_t* stream_arrive;  // arrivals of the sample kernel's CTAs (zero at the call's start)
   uint32_t* mode;      // published for the select kernel
   uint64_t* lower_bound;
   uint32_t* other_state;    // the other state block: zeroed here for the next call
   static constexpr uint32_t kGBytes = kTileElems * sizeof(GT);
   static constexpr uint32_t kStageBytes = kGBytes + kTileElems * sizeof(float);
   static constexpr uint32_t kWarpStagePairs = 512;  // on-chip staged pairs per compute warp
-  static constexpr bool kPrepass = true;
   static constexpr int kSampleBins = efs::kSampleBins;
   static constexpr int kSampleShift = 31 - kSampleBits;  // key bits below the sampled ones
 
@@ -175,36 +176,30 @@ struct TopkCandOp {
   // every CTA, first thing, whatever happens later in the launch
   __device__ void prologue() const { clear_state(other_state); }
 
-  // One-shot grid barrier: the arrival counter starts at zero in every call
-  // (the per-call reset of the control block), so a CTA arrives once, after a
-  // fence that publishes its merged histogram, and waits (bounded) until all
-  // have arrived.
-  __device__ bool barrier(uint64_t limit_ns, uint32_t* error) const {
-    __shared__ int s_ok;
+  // The sample kernel's CTAs arrive once each, after a fence that publishes
+  // their merged histogram (the arrival counter starts at zero in every call:
+  // the per-call reset of the control block); the last to arrive sees every
+  // sample. Nothing waits, so the grid needs no co-residency.
+  __device__ bool arrive_last() const {
+    __shared__ int s_last;
     __syncthreads();
     if (threadIdx.x == 0) {
       __threadfence();
-      atomicAdd(stream_arrive, 1u);
-      int ok = 1;
-      const uint64_t t0 = global_timer_ns();
-      for (uint32_t it = 0; ld_acquire_u32(stream_arrive) < gridDim.x; ++it) {
-        if (it > (1u << 26) || global_timer_ns() - t0 > limit_ns) {
-          atomicOr(error, kDevErrTimeout);
-          ok = 0;
-          break;
-        }
-      }
-      s_ok = ok;
+      s_last = atomicAdd(stream_arrive, 1u) == gridDim.x - 1 ? 1 : 0;
+      if (s_last) __threadfence();  // the other CTAs' merges before its reads
     }
     __syncthreads();
-    return s_ok != 0;
+    return s_last != 0;
   }
 
-  // Every CTA computes the same bound: each compute thread loads 16
-  // consecutive bins of the merged histogram (vector loads, all in flight
-  // together), a block suffix scan gives the sampled mass above each
-  // thread's bins, and the thread holding the target-th largest sample finds
-  // its bin; CTA 0 publishes the bound with the mode.
+  // the bound the sample kernel published (complete: the kernel before this)
+  __device__ uint64_t initial_aux() const { return __ldcg(lower_bound); }
+
+  // The bound, by the last sample CTA (every thread of it): each compute
+  // thread loads 16 consecutive bins of the merged histogram (vector loads,
+  // all in flight together), a block suffix scan gives the sampled mass above
+  // each thread's bins, and the thread holding the target-th largest sample
+  // finds its bin; the bound is published with the mode.
   __device__ uint64_t choose() const {
     constexpr int kPer = kSampleBins / kComputeThreads;
     static_assert(kPer % 4 == 0 && kPer * kComputeThreads == kSampleBins, "sample bins");
@@ -276,10 +271,8 @@ struct TopkCandOp {
         bound = kSelectNone;  // and none gathered while streaming
       }
       s_bound = bound;
-      if (blockIdx.x == 0) {
-        *mode = m;
-        *lower_bound = bound;
-      }
+      *mode = m;
+      *lower_bound = bound;
     }
     __syncthreads();
     return s_bound;
@@ -323,6 +316,32 @@ struct TopkCandOp {
 };
 
 constexpr int kTkStages = 4;
+
+// The candidate bound of the streaming pass, in a kernel of its own before
+// it: every CTA histograms the top 13 key bits of 2048 coordinates spread
+// over its share of the tiles — loaded before the wait for the previous
+// kernel, since a stale value only moves the bound, never the result (the
+// select checks the candidates and falls back to the whole array) — merges
+// its histogram into the call's global one, and the last CTA to arrive
+// derives the bound and publishes it with the mode. No CTA waits for
+// another, so the launch needs no co-residency; the streaming pass then has
+// no grid barrier and is a plain programmatic launch.
+template <typename GT>
+__global__ void __launch_bounds__(kStreamThreads)
+    topk_sample_kernel(TopkCandOp<GT> op, uint32_t num_tiles) {
+  __shared__ uint32_t s_hist[TopkCandOp<GT>::kSampleBins];
+  const uint32_t T = num_tiles, G = gridDim.x, c = blockIdx.x;
+  const uint32_t t_lo = static_cast<uint32_t>(static_cast<uint64_t>(c) * T / G);
+  const uint32_t t_hi = static_cast<uint32_t>(static_cast<uint64_t>(c + 1) * T / G);
+  for (int b = threadIdx.x; b < TopkCandOp<GT>::kSampleBins; b += blockDim.x) s_hist[b] = 0;
+  __syncthreads();
+  if (threadIdx.x < kComputeThreads && t_hi > t_lo) op.sample(t_lo, t_hi, threadIdx.x, s_hist);
+  __syncthreads();
+  griddep_wait();  // the call's state block and the published words are free now
+  griddep_launch_dependents();
+  op.merge(s_hist);
+  if (op.arrive_last()) op.choose();
+}
 
 // Inputs the bulk copies cannot take (not 16-byte aligned): a = fmaf(γ,g,e)
 // written over e with plain loads, and the selection switched to the
@@ -874,7 +893,7 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
   args.stream_err = ws.stream_err();
   args.err_parts = ws.errparts();
 
-  // 1 stream (sample pre-pass + candidates). The bulk copies need 16-byte
+  // 1 sample + 2 stream (candidates). The bulk copies need 16-byte
   // aligned g and e; otherwise a plain pass writes a and the selection runs in
   // the full-array mode.
   ScanCtx ctx = next_scan_ctx(ws, tiles);
@@ -892,14 +911,17 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
     StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks(), nullptr,
                   err_out ? ws.stream_err() : nullptr, ws.errparts()};
     void* params[] = {&op, &d, &args.list_idx, &args.list_val, &args.list_count, &cap, &ctx, &sa};
-    // A cooperative launch: the pre-pass ends in a grid barrier, which needs
-    // every CTA resident at once even when calls on other streams compete
-    // for the SMs (a plain launch was 3-5 us per call faster, but two such
-    // grids dispatched in part side by side could each wait on CTAs that
-    // cannot start).
+    // the bound first (a small kernel without waits), then the streaming
+    // pass, whose CTAs only wait for lower-numbered ones: plain launches
+    uint32_t tiles_arg = tiles;
+    void* sp[] = {&op, &tiles_arg};
+    err = launch_pdl(reinterpret_cast<const void*>(&topk_sample_kernel<GT>), grid, kStreamThreads,
+                     0, ws.stream, sp, false);
+    count_launch();
+    if (err != cudaSuccess) return err;
     err = launch_pdl(
         reinterpret_cast<const void*>(&stream_compact_kernel<TopkCandOp<GT>, kTkStages>), grid,
-        kStreamThreads, StreamLayout<TopkCandOp<GT>, kTkStages>::kSmem, ws.stream, params, true);
+        kStreamThreads, StreamLayout<TopkCandOp<GT>, kTkStages>::kSmem, ws.stream, params, false);
     count_launch();
     if (err != cudaSuccess) return err;
   } else {
@@ -910,7 +932,7 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
     count_launch();
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
   }
-  // 2 select (inputs the streaming pass could not take: the norm by a plain pass after it)
+  // 3 select (inputs the streaming pass could not take: the norm by a plain pass after it)
   if (!streamable) args.err_out = nullptr;
   args.epoch = next_scan_ctx(ws, 1).epoch;
   void* params[] = {(void*)&e, (void*)&d, (void*)&k, (void*)&idx_out, (void*)&val_out,

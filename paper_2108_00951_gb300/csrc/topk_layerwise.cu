@@ -169,13 +169,8 @@ struct LwCandOp {
   static constexpr uint32_t kGBytes = kTileElems * sizeof(GT);
   static constexpr uint32_t kStageBytes = kGBytes + kTileElems * sizeof(float);
   static constexpr uint32_t kWarpStagePairs = 512;  // on-chip staged pairs per compute warp
-  static constexpr bool kPrepass = false;
-  static constexpr int kSampleBins = 1;
-  __device__ void sample(uint32_t, uint32_t, int, uint32_t*) const {}
-  __device__ void merge(const uint32_t*) const {}
   __device__ void prologue() const { clear_state(other_state); }
-  __device__ bool barrier(uint64_t, uint32_t*) const { return true; }
-  __device__ uint64_t choose() const { return 0; }
+  __device__ uint64_t initial_aux() const { return 0; }
 
   // the chunk's first tiles of g and e toward L2 before the wait for the
   // previous kernel (its tail leaves DRAM mostly idle)
