@@ -166,6 +166,7 @@ __global__ void __launch_bounds__(kThreads)
     }
   }
   griddep_wait();  // the offsets (and everything before them) are complete
+  griddep_launch_dependents();  // the next kernel waits for this grid before its reads
   for (uint32_t i = threadIdx.x; i < n; i += kThreads) {
     // the list's range in this tile: from the offsets kernel, or from the
     // caller's tile index, clamped to the list (never out of bounds)

@@ -722,6 +722,10 @@ __global__ void __launch_bounds__(kSelThreads, 1)
     return;
   }
   if (si.mode == 0 && si.n <= kSmallCand) {
+    // a few CTAs do the work: let the next kernel be scheduled on the rest of
+    // the device (every kernel of this library waits for this grid before it
+    // reads what this one writes; the whole grid's barriers are not used here)
+    griddep_launch_dependents();
     const uint32_t Gs = min(gridDim.x, (si.n + kSliceElems - 1) / kSliceElems);
     if (blockIdx.x >= Gs) return;
     if (blockIdx.x == 0) {
