@@ -179,10 +179,13 @@ struct HtOp {
   }
 };
 
-constexpr int kHtStages = 4;
+// ring stages: 4 of 32 KB (fp32 g); bf16 g makes a stage 24 KB, and a fifth
+// stage keeps about as many bytes in flight within the same shared memory
+template <typename GT>
+constexpr int kHtStages = sizeof(GT) == 2 ? 5 : 4;
 
 template <typename GT>
-using HtStreamKernel = StreamLayout<HtOp<GT>, kHtStages>;
+using HtStreamKernel = StreamLayout<HtOp<GT>, kHtStages<GT>>;
 
 template <typename GT>
 cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint32_t d,
@@ -227,7 +230,7 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
     // result). Programmatic: it may start while the previous kernel on the
     // stream finishes (the kernel waits for it before its first read).
     const cudaError_t err = launch_pdl(
-        reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages>), grid,
+        reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages<GT>>), grid,
         kStreamThreads, HtStreamKernel<GT>::kSmem, ws.stream, params, false);
     count_launch();
     ws.ht_prev_balanced = sa.part_in != nullptr;
@@ -255,7 +258,7 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
 
 template <typename GT>
 int stream_blocks_per_sm() {
-  const void* fn = reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages>);
+  const void* fn = reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages<GT>>);
   int n = 0;
   if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            HtStreamKernel<GT>::kSmem) != cudaSuccess ||
