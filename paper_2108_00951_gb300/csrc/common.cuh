@@ -129,11 +129,13 @@ __device__ __forceinline__ void publish(const ScanCtx& ctx, uint32_t tile, uint3
 
 // Decoupled look-back, executed by one full warp: returns the number of
 // selected elements in all tiles before `tile`. The window holds the 128
-// nearest unresolved predecessors: lane l inspects tiles base-4l .. base-4l-3
-// (nearest first). It slides back 128 tiles at a time until it contains an
-// inclusive prefix; only the positions up to the nearest prefix must be ready.
-// On a wait that runs out, `timed_out` is set (uniformly) and a partial sum is
-// returned; the caller must not use it for addressing.
+// nearest unresolved predecessors: load j of lane l inspects tile
+// base - 32j - l, so each load instruction of the warp reads 32 consecutive
+// status words (coalesced) and the distance order is (j, lane). It slides
+// back 128 tiles at a time until it contains an inclusive prefix; only the
+// positions up to the nearest prefix must be ready. On a wait that runs out,
+// `timed_out` is set (uniformly) and a partial sum is returned; the caller
+// must not use it for addressing.
 constexpr int kLookbackPerLane = 4;
 constexpr int kLookbackWindow = 32 * kLookbackPerLane;
 
@@ -149,7 +151,7 @@ __device__ __forceinline__ uint32_t lookback_exclusive(const ScanCtx& ctx, uint3
     uint64_t word[kLookbackPerLane];
 #pragma unroll
     for (int j = 0; j < kLookbackPerLane; ++j) {  // all loads in flight together
-      const int64_t t = base - (lane * kLookbackPerLane + j);
+      const int64_t t = base - (32 * j + lane);
       word[j] = t >= 0 ? ld_relaxed_u64(ctx.status + t)
                        : pack_status(ctx.epoch, kFlagPrefix, 0);  // before tile 0: prefix 0
     }
@@ -160,18 +162,21 @@ __device__ __forceinline__ uint32_t lookback_exclusive(const ScanCtx& ctx, uint3
       flag[j] = current ? (static_cast<uint32_t>(word[j] >> 32) & 3u) : kFlagNone;
       value[j] = current ? static_cast<uint32_t>(word[j]) : 0u;
     }
-    int jp = kLookbackPerLane;  // nearest prefix position within this lane
+    // the nearest prefix: the first load with one, its lowest lane
+    int jp = kLookbackPerLane, lp = 32;
 #pragma unroll
-    for (int j = kLookbackPerLane - 1; j >= 0; --j)
-      if (flag[j] == kFlagPrefix) jp = j;
-    const uint32_t prefix_lanes = __ballot_sync(0xffffffffu, jp < kLookbackPerLane);
-    const int lp = prefix_lanes ? __ffs(prefix_lanes) - 1 : 32;  // lane of the nearest prefix
-    const int upto = lane < lp ? kLookbackPerLane - 1 : (lane == lp ? jp : -1);
+    for (int j = kLookbackPerLane - 1; j >= 0; --j) {
+      const uint32_t b = __ballot_sync(0xffffffffu, flag[j] == kFlagPrefix);
+      if (b) {
+        jp = j;
+        lp = __ffs(b) - 1;
+      }
+    }
     bool ready = true;
     uint32_t sum = 0, ready_sum = 0;
 #pragma unroll
     for (int j = 0; j < kLookbackPerLane; ++j) {
-      if (j <= upto) {
+      if (j < jp || (j == jp && lane <= lp)) {  // up to and including the nearest prefix
         ready = ready && flag[j] != kFlagNone;
         sum += value[j];
         if (flag[j] != kFlagNone) ready_sum += value[j];
@@ -185,11 +190,11 @@ __device__ __forceinline__ uint32_t lookback_exclusive(const ScanCtx& ctx, uint3
         timed_out = true;
         return excl + warp_sum(ready_sum);
       }
-      __nanosleep(32);
+      __nanosleep(64);
       continue;
     }
     excl += warp_sum(sum);
-    if (prefix_lanes) return excl;
+    if (jp < kLookbackPerLane) return excl;
     base -= kLookbackWindow;
   }
 }

@@ -11,7 +11,7 @@
 #include "compact.cuh"
 #include "gradient.cuh"
 #include "internal.h"
-#include "stream_compact.cuh"
+#include "stream_lookback.cuh"
 
 namespace efs {
 namespace {
@@ -136,6 +136,9 @@ struct HtOp {
     const float* es = reinterpret_cast<const float*>(stage + kGBytes);
     const int local = warp * kSWarpElems + lane * 4;
     float* eg = e + stream_element_index(t, warp, 0, lane, 0);
+    // with lambda > 0, |a| >= lambda already excludes a == 0 (and NaN): one
+    // comparison a coordinate; lambda == 0 keeps the a != 0 test
+    const bool pos = lambda > 0.0f;
 #pragma unroll
     for (int v = 0; v < kSUnits; ++v) {
       GradVec<GT> gv;
@@ -148,11 +151,13 @@ struct HtOp {
       a[v][1] = __fmaf_rn(gamma, gv[1], ev.y);
       a[v][2] = __fmaf_rn(gamma, gv[2], ev.z);
       a[v][3] = __fmaf_rn(gamma, gv[3], ev.w);
-      sel[v] = in_support(a[v][0], lambda) | (in_support(a[v][1], lambda) << 1) |
-               (in_support(a[v][2], lambda) << 2) | (in_support(a[v][3], lambda) << 3);
-      st_stream_f4(eg + v * 128,
-                   make_float4((sel[v] & 1u) ? 0.0f : a[v][0], (sel[v] & 2u) ? 0.0f : a[v][1],
-                               (sel[v] & 4u) ? 0.0f : a[v][2], (sel[v] & 8u) ? 0.0f : a[v][3]));
+      bool s[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        s[j] = pos ? fabsf(a[v][j]) >= lambda : in_support(a[v][j], lambda) != 0u;
+      sel[v] = (s[0] ? 1u : 0u) | (s[1] ? 2u : 0u) | (s[2] ? 4u : 0u) | (s[3] ? 8u : 0u);
+      st_stream_f4(eg + v * 128, make_float4(s[0] ? 0.0f : a[v][0], s[1] ? 0.0f : a[v][1],
+                                             s[2] ? 0.0f : a[v][2], s[3] ? 0.0f : a[v][3]));
     }
   }
 
@@ -185,7 +190,7 @@ template <typename GT>
 constexpr int kHtStages = sizeof(GT) == 2 ? 5 : 4;
 
 template <typename GT>
-using HtStreamKernel = StreamLayout<HtOp<GT>, kHtStages<GT>>;
+using HtStreamKernel = LbLayout<HtOp<GT>, kHtStages<GT>>;
 
 template <typename GT>
 cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint32_t d,
@@ -196,49 +201,25 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
   const uintptr_t ga = reinterpret_cast<uintptr_t>(g), ea = reinterpret_cast<uintptr_t>(e);
   const int per_sm = sizeof(GT) == 4 ? dev.ht_stream_per_sm_f32 : dev.ht_stream_per_sm_bf16;
   if (ga % 16 == 0 && ea % 16 == 0 && per_sm > 0) {
-    // TMA-fed streaming compaction: one CTA per SM
+    // TMA-fed streaming compaction over dynamically claimed groups of tiles:
+    // one CTA per SM. A group waits only for groups claimed before it, held
+    // by running CTAs, so the launch needs no co-residency. Programmatic: it
+    // may start while the previous kernel on the stream finishes (the kernel
+    // waits for it before its first read).
     HtOp<GT> op{g, e, gamma, lambda, d};
-    uint32_t slots = static_cast<uint32_t>(per_sm * dev.sm_count);
-    if (slots > kMaxChunks) slots = kMaxChunks;
-    const uint32_t grid = tiles < slots ? tiles : slots;
+    const uint32_t groups = (tiles + kLbGroupTiles - 1) / kLbGroupTiles;
+    const uint32_t slots = static_cast<uint32_t>(per_sm * dev.sm_count);
+    const uint32_t grid = groups < slots ? groups : slots;
     uint32_t cap = d;
     ScanCtx c = ctx;
-    // the placement writes each tile's first output position (the tile index)
-    StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.ht_chunks(ws.ht_seq), tiles_out,
-                  err_out, ws.errparts()};
-    // Balanced chunks: the previous call of this size wrote this call's chunk
-    // boundaries; this call writes the next call's from the previous call's
-    // chunk totals (dense regions get fewer tiles). Any boundaries partition
-    // the tiles, so the result never depends on them.
-    const uint32_t seq = ws.ht_seq;
-    const bool same = seq > 0 && ws.ht_last_tiles == tiles && ws.ht_last_grid == grid;
-    // (a call that returns ||e'||^2 uses equal chunks: the norm's summation
-    // order follows the chunks, and it is reproducible for an input)
-    sa.part_in = same && ws.ht_part_ready && !err_out ? ws.ht_part(seq) : nullptr;
-    sa.prev_sums = same ? ws.ht_chunks(seq + 1) : nullptr;   // the other parity: seq - 1
-    sa.prev_part = same && ws.ht_prev_balanced ? ws.ht_part(seq + 2) : nullptr;  // seq - 1
-    sa.prev_epoch = ws.ht_last_epoch;
-    sa.part_out = ws.ht_part(seq + 1);
-    void* params[] = {&op, &d, &idx_out, &val_out, &count_out, &cap, &c, &sa};
-    // CTAs wait on the chunk totals of lower-numbered CTAs. The grid fits the
-    // device at once (one CTA per SM) and CTAs are dispatched in index order,
-    // so those CTAs are running; the launch is not cooperative because a
-    // cooperative grid cannot start until the previous kernel's CTAs have
-    // all left (5 us per call on the ResNet-18-sized vector). If other work
-    // holds SMs long enough that a lower-numbered CTA cannot start, the
-    // bounded wait ends the call with EF_ERR_TIMEOUT (never a hang or a wrong
-    // result). Programmatic: it may start while the previous kernel on the
-    // stream finishes (the kernel waits for it before its first read).
+    // the groups' shares of ||e'||^2 use the per-tile count area (16 words a tile)
+    LbArgs la{tiles_out, err_out, reinterpret_cast<FF*>(ws.counts()), ws.stage_idx(),
+              ws.stage_val()};
+    void* params[] = {&op, &d, &idx_out, &val_out, &count_out, &cap, &c, &la};
     const cudaError_t err = launch_pdl(
-        reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages<GT>>), grid,
-        kStreamThreads, HtStreamKernel<GT>::kSmem, ws.stream, params, false);
+        reinterpret_cast<const void*>(&lookback_stream_kernel<HtOp<GT>, kHtStages<GT>>), grid,
+        kLbThreads, HtStreamKernel<GT>::kSmem, ws.stream, params, false);
     count_launch();
-    ws.ht_prev_balanced = sa.part_in != nullptr;
-    ws.ht_part_ready = err == cudaSuccess;
-    ws.ht_last_tiles = tiles;
-    ws.ht_last_grid = grid;
-    ws.ht_last_epoch = c.epoch;
-    ++ws.ht_seq;
     return err;
   }
   const bool vec = (ga % (4 * sizeof(GT)) == 0) && (ea % 16 == 0);
@@ -258,11 +239,11 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
 
 template <typename GT>
 int stream_blocks_per_sm() {
-  const void* fn = reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages<GT>>);
+  const void* fn = reinterpret_cast<const void*>(&lookback_stream_kernel<HtOp<GT>, kHtStages<GT>>);
   int n = 0;
   if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            HtStreamKernel<GT>::kSmem) != cudaSuccess ||
-      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, kStreamThreads,
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, kLbThreads,
                                                     HtStreamKernel<GT>::kSmem) != cudaSuccess)
     n = 0;
   cudaGetLastError();

@@ -15,7 +15,8 @@ namespace efs {
 constexpr size_t kOffBarGen = 0;        // uint32: grid-barrier generation (never reset)
 constexpr size_t kOffError = 8;         // uint32: latched device error bits
 constexpr size_t kOffBarArrive = 16;    // uint32: grid-barrier arrivals (zero after each barrier)
-constexpr size_t kOffTileClaim = 24;    // uint32[2]: look-back tile dispenser (zero between calls)
+constexpr size_t kOffTileClaim = 24;    // uint32[3]: work dispenser: handed out, CTAs finished,
+                                        // groups resolved (zero between calls)
 constexpr size_t kOffTkLowerBound = 56; // uint64: sampled lower bound of the candidates' keys
 constexpr size_t kOffTkMode = 64;       // uint32: 0 candidates, 1 full array
 constexpr size_t kOffTkListCount = 72;  // uint32: candidates emitted by the streaming pass

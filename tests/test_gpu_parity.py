@@ -126,8 +126,8 @@ def test_ht_concurrent_streams(off):
         cnt = torch.empty(1, dtype=torch.int32, device=gu.DEV)
         torch.cuda.synchronize()
         for _ in range(3):
-            ed.copy_(torch.from_numpy(e))
-            with torch.cuda.stream(s):
+            with torch.cuda.stream(s):  # the reset of e is ordered before the call
+                ed.copy_(torch.from_numpy(e))
                 efs.ef_hard_threshold(gd, ed, 0.1, 1e-3, idx, val, cnt)
         outs.append((idx, val, cnt, ed))
     torch.cuda.synchronize()
