@@ -190,7 +190,89 @@ template <typename GT>
 constexpr int kHtStages = sizeof(GT) == 2 ? 5 : 4;
 
 template <typename GT>
-using HtStreamKernel = LbLayout<HtOp<GT>, kHtStages<GT>>;
+using HtGroupKernel = LbLayout<HtOp<GT>, kHtStages<GT>>;
+template <typename GT>
+using HtChunkKernel = StreamLayout<HtOp<GT>, kHtStages<GT>>;
+
+// From this many tiles on (16.8 M coordinates) the group look-back kernel is
+// used; below, the static-chunk kernel, whose call has less fixed cost (no
+// look-back chain to drain at the end of a short call).
+constexpr uint32_t kGroupKernelMinTiles = 4096;
+
+// Streaming hard-threshold over dynamically claimed groups of tiles: one CTA
+// per SM. A group waits only for groups claimed before it, held by running
+// CTAs, so the launch needs no co-residency. Programmatic: it may start while
+// the previous kernel on the stream finishes (the kernel waits for it before
+// its first read).
+template <typename GT>
+cudaError_t launch_groups(const GT* g, float* e, float gamma, float lambda, uint32_t d,
+                          uint32_t* idx_out, float* val_out, uint32_t* count_out, double* err_out,
+                          uint32_t* tiles_out, Workspace& ws, const DeviceInfo& dev,
+                          const ScanCtx& ctx, int per_sm) {
+  const uint32_t tiles = tiles_for(d);
+  HtOp<GT> op{g, e, gamma, lambda, d};
+  const uint32_t groups = (tiles + kLbGroupTiles - 1) / kLbGroupTiles;
+  const uint32_t slots = static_cast<uint32_t>(per_sm * dev.sm_count);
+  const uint32_t grid = groups < slots ? groups : slots;
+  uint32_t cap = d;
+  ScanCtx c = ctx;
+  // the groups' shares of ||e'||^2 use the per-tile count area (16 words a tile)
+  LbArgs la{tiles_out, err_out, reinterpret_cast<FF*>(ws.counts()), ws.stage_idx(),
+            ws.stage_val()};
+  void* params[] = {&op, &d, &idx_out, &val_out, &count_out, &cap, &c, &la};
+  const cudaError_t err = launch_pdl(
+      reinterpret_cast<const void*>(&lookback_stream_kernel<HtOp<GT>, kHtStages<GT>>), grid,
+      kLbThreads, HtGroupKernel<GT>::kSmem, ws.stream, params, false);
+  count_launch();
+  ws.ht_part_ready = false;  // the chunk kernel's boundaries are not written by this kernel
+  return err;
+}
+
+// Streaming hard-threshold over static chunks (stream_compact.cuh): one CTA
+// per SM, CTA c waiting only on the chunk totals of lower-numbered CTAs. The
+// grid fits the device at once and CTAs are dispatched in index order, so
+// those CTAs are running; if other work holds SMs long enough that one cannot
+// start, the bounded wait ends the call with EF_ERR_TIMEOUT (never a hang or a
+// wrong result). Balanced chunks: the previous call of this size wrote this
+// call's chunk boundaries from its chunk totals (dense regions get fewer
+// tiles); any boundaries partition the tiles, so the result never depends on
+// them.
+template <typename GT>
+cudaError_t launch_chunks(const GT* g, float* e, float gamma, float lambda, uint32_t d,
+                          uint32_t* idx_out, float* val_out, uint32_t* count_out, double* err_out,
+                          uint32_t* tiles_out, Workspace& ws, const DeviceInfo& dev,
+                          const ScanCtx& ctx, int per_sm) {
+  const uint32_t tiles = tiles_for(d);
+  HtOp<GT> op{g, e, gamma, lambda, d};
+  uint32_t slots = static_cast<uint32_t>(per_sm * dev.sm_count);
+  if (slots > kMaxChunks) slots = kMaxChunks;
+  const uint32_t grid = tiles < slots ? tiles : slots;
+  uint32_t cap = d;
+  ScanCtx c = ctx;
+  StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.ht_chunks(ws.ht_seq), tiles_out,
+                err_out, ws.errparts()};
+  const uint32_t seq = ws.ht_seq;
+  const bool same = seq > 0 && ws.ht_last_tiles == tiles && ws.ht_last_grid == grid;
+  // (a call that returns ||e'||^2 uses equal chunks: the norm's summation
+  // order follows the chunks, and it is reproducible for an input)
+  sa.part_in = same && ws.ht_part_ready && !err_out ? ws.ht_part(seq) : nullptr;
+  sa.prev_sums = same ? ws.ht_chunks(seq + 1) : nullptr;   // the other parity: seq - 1
+  sa.prev_part = same && ws.ht_prev_balanced ? ws.ht_part(seq + 2) : nullptr;  // seq - 1
+  sa.prev_epoch = ws.ht_last_epoch;
+  sa.part_out = ws.ht_part(seq + 1);
+  void* params[] = {&op, &d, &idx_out, &val_out, &count_out, &cap, &c, &sa};
+  const cudaError_t err = launch_pdl(
+      reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages<GT>>), grid,
+      kStreamThreads, HtChunkKernel<GT>::kSmem, ws.stream, params, false);
+  count_launch();
+  ws.ht_prev_balanced = sa.part_in != nullptr;
+  ws.ht_part_ready = err == cudaSuccess;
+  ws.ht_last_tiles = tiles;
+  ws.ht_last_grid = grid;
+  ws.ht_last_epoch = c.epoch;
+  ++ws.ht_seq;
+  return err;
+}
 
 template <typename GT>
 cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint32_t d,
@@ -199,28 +281,17 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
   const uint32_t tiles = tiles_for(d);
   const ScanCtx ctx = next_scan_ctx(ws, tiles);
   const uintptr_t ga = reinterpret_cast<uintptr_t>(g), ea = reinterpret_cast<uintptr_t>(e);
-  const int per_sm = sizeof(GT) == 4 ? dev.ht_stream_per_sm_f32 : dev.ht_stream_per_sm_bf16;
-  if (ga % 16 == 0 && ea % 16 == 0 && per_sm > 0) {
-    // TMA-fed streaming compaction over dynamically claimed groups of tiles:
-    // one CTA per SM. A group waits only for groups claimed before it, held
-    // by running CTAs, so the launch needs no co-residency. Programmatic: it
-    // may start while the previous kernel on the stream finishes (the kernel
-    // waits for it before its first read).
-    HtOp<GT> op{g, e, gamma, lambda, d};
-    const uint32_t groups = (tiles + kLbGroupTiles - 1) / kLbGroupTiles;
-    const uint32_t slots = static_cast<uint32_t>(per_sm * dev.sm_count);
-    const uint32_t grid = groups < slots ? groups : slots;
-    uint32_t cap = d;
-    ScanCtx c = ctx;
-    // the groups' shares of ||e'||^2 use the per-tile count area (16 words a tile)
-    LbArgs la{tiles_out, err_out, reinterpret_cast<FF*>(ws.counts()), ws.stage_idx(),
-              ws.stage_val()};
-    void* params[] = {&op, &d, &idx_out, &val_out, &count_out, &cap, &c, &la};
-    const cudaError_t err = launch_pdl(
-        reinterpret_cast<const void*>(&lookback_stream_kernel<HtOp<GT>, kHtStages<GT>>), grid,
-        kLbThreads, HtStreamKernel<GT>::kSmem, ws.stream, params, false);
-    count_launch();
-    return err;
+  if (ga % 16 == 0 && ea % 16 == 0) {
+    const int per_group = sizeof(GT) == 4 ? dev.ht_group_per_sm_f32 : dev.ht_group_per_sm_bf16;
+    const int per_chunk = sizeof(GT) == 4 ? dev.ht_stream_per_sm_f32 : dev.ht_stream_per_sm_bf16;
+    const int mode = ht_stream_mode();  // 0 by size, 1 chunks, 2 groups (testing aid)
+    const bool groups = mode == 2 || (mode == 0 && tiles >= kGroupKernelMinTiles);
+    if (groups && per_group > 0)
+      return launch_groups(g, e, gamma, lambda, d, idx_out, val_out, count_out, err_out,
+                           tiles_out, ws, dev, ctx, per_group);
+    if (per_chunk > 0)
+      return launch_chunks(g, e, gamma, lambda, d, idx_out, val_out, count_out, err_out,
+                           tiles_out, ws, dev, ctx, per_chunk);
   }
   const bool vec = (ga % (4 * sizeof(GT)) == 0) && (ea % 16 == 0);
   if (vec) {
@@ -237,24 +308,36 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
   return err;
 }
 
-template <typename GT>
-int stream_blocks_per_sm() {
-  const void* fn = reinterpret_cast<const void*>(&lookback_stream_kernel<HtOp<GT>, kHtStages<GT>>);
+template <typename GT, typename Layout>
+int blocks_per_sm(const void* fn, int threads) {
   int n = 0;
-  if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           HtStreamKernel<GT>::kSmem) != cudaSuccess ||
-      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, kLbThreads,
-                                                    HtStreamKernel<GT>::kSmem) != cudaSuccess)
+  if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, Layout::kSmem) !=
+          cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, threads, Layout::kSmem) != cudaSuccess)
     n = 0;
   cudaGetLastError();
   return n;
 }
 
+template <typename GT>
+int group_blocks_per_sm() {
+  return blocks_per_sm<GT, HtGroupKernel<GT>>(
+      reinterpret_cast<const void*>(&lookback_stream_kernel<HtOp<GT>, kHtStages<GT>>), kLbThreads);
+}
+template <typename GT>
+int chunk_blocks_per_sm() {
+  return blocks_per_sm<GT, HtChunkKernel<GT>>(
+      reinterpret_cast<const void*>(&stream_compact_kernel<HtOp<GT>, kHtStages<GT>>),
+      kStreamThreads);
+}
+
 }  // namespace
 
 void ht_init_device(DeviceInfo& info) {
-  info.ht_stream_per_sm_f32 = stream_blocks_per_sm<float>();
-  info.ht_stream_per_sm_bf16 = stream_blocks_per_sm<uint16_t>();
+  info.ht_stream_per_sm_f32 = chunk_blocks_per_sm<float>();
+  info.ht_stream_per_sm_bf16 = chunk_blocks_per_sm<uint16_t>();
+  info.ht_group_per_sm_f32 = group_blocks_per_sm<float>();
+  info.ht_group_per_sm_bf16 = group_blocks_per_sm<uint16_t>();
 }
 
 // Launch the look-back kernel over caller-provided scratch (the tile-status

@@ -181,6 +181,8 @@ struct DeviceInfo {
   int finalize_blocks = 0;        // co-resident CTAs for the Top-k finalize
   int ht_stream_per_sm_f32 = 0;   // streaming hard-threshold CTAs per SM (0: unavailable)
   int ht_stream_per_sm_bf16 = 0;
+  int ht_group_per_sm_f32 = 0;    // hard-threshold claimed-group CTAs per SM (0: unavailable)
+  int ht_group_per_sm_bf16 = 0;
   int tk_stream_per_sm_f32 = 0;   // streaming Top-k candidate pass CTAs per SM
   int tk_stream_per_sm_bf16 = 0;
   int lw_stream_per_sm_f32 = 0;   // streaming layer-wise candidate pass CTAs per SM
@@ -224,6 +226,7 @@ cudaError_t launch_pdl(const void* fn, dim3 grid, uint32_t block, uint32_t smem,
 void count_launch();
 uint64_t wait_limit_ns();
 int64_t withheld_tile();
+int ht_stream_mode();  // ef_test_set_ht_stream: 0 by size, 1 static chunks, 2 claimed groups
 ScanCtx next_scan_ctx(Workspace& ws, uint32_t num_tiles);
 
 // ---- launchers (return the launch's cudaError_t) ----

@@ -14,3 +14,16 @@ if HERE not in sys.path:
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (GB300, sm_103a)")
     config.addinivalue_line("markers", "slow: full-size parity cases")
+
+
+@pytest.fixture(params=["chunks", "groups"])
+def ht_kernel(request):
+    """Runs a hard-threshold test with each streaming kernel: the static-chunk
+    kernel and the claimed-group look-back kernel (by default the library
+    picks by size; small test inputs would reach only the first)."""
+    import paper_2108_00951_gb300 as efs
+    efs.ef_test_set_ht_stream({"chunks": 1, "groups": 2}[request.param])
+    try:
+        yield request.param
+    finally:
+        efs.ef_test_set_ht_stream(0)

@@ -46,6 +46,7 @@ def _check_same(gpu, ref, what):
 
 
 # ------------------------------------------------------------ hard-threshold
+@pytest.mark.usefixtures("ht_kernel")
 @pytest.mark.parametrize("bf16", [False, True])
 @pytest.mark.parametrize("d", RAGGED)
 def test_ht_random(d, bf16):
@@ -64,6 +65,7 @@ def test_ht_misaligned_bases(offs, bf16):
                 oracle.ef_hard_threshold(g, e, 0.1, 1.5e-3), "offsets %s" % (offs,))
 
 
+@pytest.mark.usefixtures("ht_kernel")
 def test_ht_adversarial_values():
     d = 3 * 4096 + 5
     rng = _rng("adv")
@@ -79,6 +81,7 @@ def test_ht_adversarial_values():
                     "adversarial lam=%g" % lam_)
 
 
+@pytest.mark.usefixtures("ht_kernel")
 def test_ht_fma_sensitive_values():
     # e = -round(gamma*g): a is the product's rounding error, which only a
     # single-rounding fma preserves
@@ -91,6 +94,7 @@ def test_ht_fma_sensitive_values():
                 "fma")
 
 
+@pytest.mark.usefixtures("ht_kernel")
 def test_ht_all_and_nothing_sent():
     d = 5 * 4096 + 1
     g, e = _inputs(d, 3)
@@ -110,6 +114,7 @@ def test_ht_zero_length():
     assert int(cnt.item()) == 0
 
 
+@pytest.mark.usefixtures("ht_kernel")
 @pytest.mark.parametrize("off", [0, 1])
 def test_ht_concurrent_streams(off):
     # calls on different streams use different workspaces and may overlap
@@ -223,12 +228,14 @@ def test_ht_balanced_chunks_over_calls():
 SPILL_D = 3 * 2**20 + 4099
 
 
+@pytest.mark.usefixtures("ht_kernel")
 @pytest.mark.parametrize("bf16", [False, True])
 def test_ht_spill_everything_sent(bf16):
     g, e = _inputs(SPILL_D, 21, bf16=bf16)
     _check_same(gu.ht(g, e, 0.1, 0.0), oracle.ef_hard_threshold(g, e, 0.1, 0.0), "all sent")
 
 
+@pytest.mark.usefixtures("ht_kernel")
 def test_ht_spill_mixed_density():
     g, e = _inputs(SPILL_D, 22)
     g[: SPILL_D // 4] *= 1000.0  # a dense quarter (~96 % sent), the rest sends nothing
@@ -237,6 +244,7 @@ def test_ht_spill_mixed_density():
     _check_same((i, v, en), oracle.ef_hard_threshold(g, e, 0.1, 0.05), "mixed")
 
 
+@pytest.mark.usefixtures("ht_kernel")
 @pytest.mark.parametrize("out_off", [(1, 0), (2, 3), (3, 1)])
 def test_ht_misaligned_outputs(out_off):
     # the pairs are written with 16-byte stores matched to each output's own
