@@ -69,6 +69,7 @@ NOMINAL_HBM_GBS = 8000.0
 METRIC = "EF hard-threshold compress GB/s & elem/s vs HBM peak; Top-k and aggregate ms/iter"
 HT_KERNEL_SOURCES = ["paper_2108_00951_gb300/csrc/ht.cu",
                      "paper_2108_00951_gb300/csrc/stream_compact.cuh",
+                     "paper_2108_00951_gb300/csrc/stream_lookback.cuh",
                      "paper_2108_00951_gb300/csrc/tma.cuh",
                      "paper_2108_00951_gb300/csrc/compact.cuh",
                      "paper_2108_00951_gb300/csrc/common.cuh",
@@ -534,8 +535,10 @@ def run_ours(args):
         "frac_of_nominal_8tbs": round(value / NOMINAL_HBM_GBS, 4),
         "roofline": {
             "bound": "hbm",
-            "kernel": "stream_compact_kernel<HtOp> (fused EF accumulate + hard-threshold + "
-                      "compaction + residual)",
+            "kernel": (("lookback_stream_kernel<HtOp> (claimed tile groups, decoupled look-back)"
+                        if (d + 4095) // 4096 >= 4096 else
+                        "stream_compact_kernel<HtOp> (static chunks)") +
+                       ": fused EF accumulate + hard-threshold + compaction + residual"),
             "achieved": round(achieved, 2),
             "peak": peak,
             "peak_kind": peak_kind,
