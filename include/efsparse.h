@@ -453,14 +453,15 @@ uint64_t ef_kernel_launches(void);
 void ef_test_set_lookback_fault(int64_t withheld_tile, uint32_t spin_limit_us);
 
 /*
- * ef_test_set_ht_stream — test hook choosing the hard-threshold streaming
- * kernel for 16-byte aligned g and e: 0 (the default) by size (claimed
- * groups of tiles with look-back from 4096 tiles, 16,777,216 coordinates, on;
- * static chunks below), 1 static chunks, 2 claimed groups. Any other value
- * means 0. The results are the same whichever kernel runs; the hook lets tests
- * run both on small inputs. Process-wide; never needed in production.
+ * ef_test_set_stream_kernel — test hook choosing the streaming kernel of the
+ * hard-threshold step and of the Top-k and layer-wise Top-k candidate passes
+ * (16-byte aligned g and e): 0 (the default) by size (claimed groups of tiles
+ * with look-back from 4096 tiles, 16,777,216 coordinates, on; static chunks
+ * below), 1 static chunks, 2 claimed groups. Any other value means 0. The
+ * results are the same whichever kernel runs; the hook lets tests run both on
+ * small inputs. Process-wide; never needed in production.
  */
-void ef_test_set_ht_stream(int mode);
+void ef_test_set_stream_kernel(int mode);
 
 #ifdef __cplusplus
 }

@@ -22,7 +22,7 @@ from ._binding import (  # noqa: F401
     ef_scaled_round,
     ef_kernel_launches,
     ef_test_set_lookback_fault,
-    ef_test_set_ht_stream,
+    ef_test_set_stream_kernel,
     ef_topk,
     ef_topk_layerwise,
     ef_workspace_release,

@@ -91,8 +91,8 @@ def load_library(build_if_missing: bool = True):
         lib.ef_kernel_launches.restype = ctypes.c_uint64
         lib.ef_test_set_lookback_fault.argtypes = [ctypes.c_int64, ctypes.c_uint32]
         lib.ef_test_set_lookback_fault.restype = None
-        lib.ef_test_set_ht_stream.argtypes = [ctypes.c_int]
-        lib.ef_test_set_ht_stream.restype = None
+        lib.ef_test_set_stream_kernel.argtypes = [ctypes.c_int]
+        lib.ef_test_set_stream_kernel.restype = None
         _lib = lib
         return lib
 
@@ -329,5 +329,5 @@ def ef_test_set_lookback_fault(withheld_tile: int, spin_limit_us: int = 0):
     load_library().ef_test_set_lookback_fault(int(withheld_tile), int(spin_limit_us))
 
 
-def ef_test_set_ht_stream(mode: int):
-    load_library().ef_test_set_ht_stream(int(mode))
+def ef_test_set_stream_kernel(mode: int):
+    load_library().ef_test_set_stream_kernel(int(mode))

@@ -21,7 +21,7 @@ std::map<int, DeviceInfo> g_devices;
 std::atomic<uint64_t> g_launches{0};
 std::atomic<int64_t> g_withheld_tile{-1};
 std::atomic<uint64_t> g_wait_limit_ns{2000000000ull};  // 2 s per wait
-std::atomic<int> g_ht_stream_mode{0};  // 0: by size, 1: static chunks, 2: claimed groups
+std::atomic<int> g_stream_kernel_mode{0};  // 0: by size, 1: static chunks, 2: claimed groups
 
 constexpr uint64_t kMaxD = 0xffffffffull;
 
@@ -301,7 +301,7 @@ cudaError_t launch_pdl(const void* fn, dim3 grid, uint32_t block, uint32_t smem,
 void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 uint64_t wait_limit_ns() { return g_wait_limit_ns.load(); }
 int64_t withheld_tile() { return g_withheld_tile.load(); }
-int ht_stream_mode() { return g_ht_stream_mode.load(); }
+int stream_kernel_mode() { return g_stream_kernel_mode.load(); }
 
 ScanCtx next_scan_ctx(Workspace& ws, uint32_t num_tiles) {
   if (ws.epoch >= (1u << 30) - 1) {  // epoch wrap: old words must not match again
@@ -620,8 +620,8 @@ void ef_test_set_lookback_fault(int64_t withheld_tile, uint32_t spin_limit_us) {
                                                : static_cast<uint64_t>(spin_limit_us) * 1000ull);
 }
 
-void ef_test_set_ht_stream(int mode) {
-  efs::g_ht_stream_mode.store(mode == 1 || mode == 2 ? mode : 0);
+void ef_test_set_stream_kernel(int mode) {
+  efs::g_stream_kernel_mode.store(mode == 1 || mode == 2 ? mode : 0);
 }
 
 }  // extern "C"

@@ -194,11 +194,6 @@ using HtGroupKernel = LbLayout<HtOp<GT>, kHtStages<GT>>;
 template <typename GT>
 using HtChunkKernel = StreamLayout<HtOp<GT>, kHtStages<GT>>;
 
-// From this many tiles on (16.8 M coordinates) the group look-back kernel is
-// used; below, the static-chunk kernel, whose call has less fixed cost (no
-// look-back chain to drain at the end of a short call).
-constexpr uint32_t kGroupKernelMinTiles = 4096;
-
 // Streaming hard-threshold over dynamically claimed groups of tiles: one CTA
 // per SM. A group waits only for groups claimed before it, held by running
 // CTAs, so the launch needs no co-residency. Programmatic: it may start while
@@ -284,9 +279,7 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
   if (ga % 16 == 0 && ea % 16 == 0) {
     const int per_group = sizeof(GT) == 4 ? dev.ht_group_per_sm_f32 : dev.ht_group_per_sm_bf16;
     const int per_chunk = sizeof(GT) == 4 ? dev.ht_stream_per_sm_f32 : dev.ht_stream_per_sm_bf16;
-    const int mode = ht_stream_mode();  // 0 by size, 1 chunks, 2 groups (testing aid)
-    const bool groups = mode == 2 || (mode == 0 && tiles >= kGroupKernelMinTiles);
-    if (groups && per_group > 0)
+    if (use_group_kernel(tiles) && per_group > 0)
       return launch_groups(g, e, gamma, lambda, d, idx_out, val_out, count_out, err_out,
                            tiles_out, ws, dev, ctx, per_group);
     if (per_chunk > 0)

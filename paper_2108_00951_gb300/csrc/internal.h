@@ -185,8 +185,12 @@ struct DeviceInfo {
   int ht_group_per_sm_bf16 = 0;
   int tk_stream_per_sm_f32 = 0;   // streaming Top-k candidate pass CTAs per SM
   int tk_stream_per_sm_bf16 = 0;
+  int tk_group_per_sm_f32 = 0;    // Top-k candidate pass, claimed-group kernel CTAs per SM
+  int tk_group_per_sm_bf16 = 0;
   int lw_stream_per_sm_f32 = 0;   // streaming layer-wise candidate pass CTAs per SM
   int lw_stream_per_sm_bf16 = 0;
+  int lw_group_per_sm_f32 = 0;    // layer-wise candidate pass, claimed-group kernel CTAs per SM
+  int lw_group_per_sm_bf16 = 0;
   int lw_select_per_sm = 0;       // co-resident layer-wise select CTAs per SM
 };
 
@@ -226,7 +230,18 @@ cudaError_t launch_pdl(const void* fn, dim3 grid, uint32_t block, uint32_t smem,
 void count_launch();
 uint64_t wait_limit_ns();
 int64_t withheld_tile();
-int ht_stream_mode();  // ef_test_set_ht_stream: 0 by size, 1 static chunks, 2 claimed groups
+int stream_kernel_mode();  // ef_test_set_stream_kernel: 0 by size, 1 static chunks, 2 claimed groups
+
+// The streaming passes (hard-threshold, Top-k and layer-wise candidates) use
+// the claimed-group look-back kernel from this many tiles on (16.8 M
+// coordinates), the static-chunk kernel below, whose call has less fixed cost
+// (no look-back chain to drain at the end of a short call); the test hook
+// ef_test_set_stream_kernel can force either.
+constexpr uint32_t kGroupKernelMinTiles = 4096;
+inline bool use_group_kernel(uint32_t tiles) {
+  const int mode = stream_kernel_mode();
+  return mode == 2 || (mode == 0 && tiles >= kGroupKernelMinTiles);
+}
 ScanCtx next_scan_ctx(Workspace& ws, uint32_t num_tiles);
 
 // ---- launchers (return the launch's cudaError_t) ----

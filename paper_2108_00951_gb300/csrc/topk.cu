@@ -36,7 +36,7 @@
 #include "gradient.cuh"
 #include "internal.h"
 #include "select.cuh"
-#include "stream_compact.cuh"
+#include "stream_lookback.cuh"
 
 namespace efs {
 namespace {
@@ -853,6 +853,19 @@ __global__ void __launch_bounds__(kSelThreads, 1)
 }
 
 template <typename GT>
+int tk_group_blocks_per_sm() {
+  const void* fn =
+      reinterpret_cast<const void*>(&lookback_stream_kernel<TopkCandOp<GT>, kTkStages>);
+  const uint32_t smem = LbLayout<TopkCandOp<GT>, kTkStages>::kSmem;
+  int n = 0;
+  if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, kLbThreads, smem) != cudaSuccess)
+    n = 0;
+  cudaGetLastError();
+  return n;
+}
+
+template <typename GT>
 int tk_stream_blocks_per_sm() {
   const void* fn = reinterpret_cast<const void*>(&stream_compact_kernel<TopkCandOp<GT>, kTkStages>);
   const uint32_t smem = StreamLayout<TopkCandOp<GT>, kTkStages>::kSmem;
@@ -903,6 +916,8 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
   ScanCtx ctx = next_scan_ctx(ws, tiles);
   ctx.error = args.list_flags;
   const int per_sm = sizeof(GT) == 4 ? dev.tk_stream_per_sm_f32 : dev.tk_stream_per_sm_bf16;
+  const int per_sm_groups =
+      sizeof(GT) == 4 ? dev.tk_group_per_sm_f32 : dev.tk_group_per_sm_bf16;
   const bool streamable = reinterpret_cast<uintptr_t>(e) % 16 == 0 &&
                           reinterpret_cast<uintptr_t>(g) % 16 == 0 && per_sm > 0;
   if (streamable) {
@@ -923,9 +938,24 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
                      0, ws.stream, sp, false);
     count_launch();
     if (err != cudaSuccess) return err;
-    err = launch_pdl(
-        reinterpret_cast<const void*>(&stream_compact_kernel<TopkCandOp<GT>, kTkStages>), grid,
-        kStreamThreads, StreamLayout<TopkCandOp<GT>, kTkStages>::kSmem, ws.stream, params, false);
+    if (use_group_kernel(tiles) && per_sm_groups > 0) {
+      // claimed groups of tiles with look-back (stream_lookback.cuh): no
+      // wait depends on which CTAs are resident
+      const uint32_t groups = (tiles + kLbGroupTiles - 1) / kLbGroupTiles;
+      const uint32_t gslots = static_cast<uint32_t>(per_sm_groups * dev.sm_count);
+      const uint32_t ggrid = groups < gslots ? groups : gslots;
+      LbArgs la{nullptr, err_out ? ws.stream_err() : nullptr, reinterpret_cast<FF*>(ws.counts()),
+                ws.stage_idx(), ws.stage_val()};
+      void* gp[] = {&op, &d, &args.list_idx, &args.list_val, &args.list_count, &cap, &ctx, &la};
+      err = launch_pdl(
+          reinterpret_cast<const void*>(&lookback_stream_kernel<TopkCandOp<GT>, kTkStages>),
+          ggrid, kLbThreads, LbLayout<TopkCandOp<GT>, kTkStages>::kSmem, ws.stream, gp, false);
+    } else {
+      err = launch_pdl(
+          reinterpret_cast<const void*>(&stream_compact_kernel<TopkCandOp<GT>, kTkStages>), grid,
+          kStreamThreads, StreamLayout<TopkCandOp<GT>, kTkStages>::kSmem, ws.stream, params,
+          false);
+    }
     count_launch();
     if (err != cudaSuccess) return err;
   } else {
@@ -961,6 +991,8 @@ void topk_init_device(DeviceInfo& info) {
   info.finalize_blocks = info.refine_blocks;
   info.tk_stream_per_sm_f32 = tk_stream_blocks_per_sm<float>();
   info.tk_stream_per_sm_bf16 = tk_stream_blocks_per_sm<uint16_t>();
+  info.tk_group_per_sm_f32 = tk_group_blocks_per_sm<float>();
+  info.tk_group_per_sm_bf16 = tk_group_blocks_per_sm<uint16_t>();
   cudaGetLastError();
 }
 

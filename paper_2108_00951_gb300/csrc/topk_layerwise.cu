@@ -38,7 +38,7 @@
 #include "gradient.cuh"
 #include "internal.h"
 #include "select.cuh"
-#include "stream_compact.cuh"
+#include "stream_lookback.cuh"
 
 namespace efs {
 namespace {
@@ -757,6 +757,18 @@ __global__ void __launch_bounds__(kLwThreads, 1)
 
 // ------------------------------------------------------------- host side
 template <typename GT>
+int lw_group_blocks_per_sm() {
+  const void* fn = reinterpret_cast<const void*>(&lookback_stream_kernel<LwCandOp<GT>, kLwStages>);
+  const uint32_t smem = LbLayout<LwCandOp<GT>, kLwStages>::kSmem;
+  int n = 0;
+  if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, kLbThreads, smem) != cudaSuccess)
+    n = 0;
+  cudaGetLastError();
+  return n;
+}
+
+template <typename GT>
 int lw_stream_blocks_per_sm() {
   const void* fn = reinterpret_cast<const void*>(&stream_compact_kernel<LwCandOp<GT>, kLwStages>);
   const uint32_t smem = StreamLayout<LwCandOp<GT>, kLwStages>::kSmem;
@@ -820,14 +832,30 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t d, uint32_
     const uint32_t grid = p.tiles < slots ? p.tiles : slots;
     uint32_t cap = ws.cand_cap;
     uint32_t* list_count = ws.u32(kOffTkListCount);
-    StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks(), tile_base,
-                  err_out ? ws.stream_err() : nullptr, ws.errparts()};
-    void* params[] = {&op, &d, &list_idx, &list_val, &list_count, &cap, &ctx, &sa};
-    // not cooperative: the only cross-CTA wait is on lower-numbered CTAs,
-    // which are scheduled first
-    err = launch_pdl(
-        reinterpret_cast<const void*>(&stream_compact_kernel<LwCandOp<GT>, kLwStages>), grid,
-        kStreamThreads, StreamLayout<LwCandOp<GT>, kLwStages>::kSmem, ws.stream, params, false);
+    const int per_sm_groups =
+        sizeof(GT) == 4 ? dev.lw_group_per_sm_f32 : dev.lw_group_per_sm_bf16;
+    if (use_group_kernel(p.tiles) && per_sm_groups > 0) {
+      // claimed groups of tiles with look-back (stream_lookback.cuh): no
+      // wait depends on which CTAs are resident
+      const uint32_t groups = (p.tiles + kLbGroupTiles - 1) / kLbGroupTiles;
+      const uint32_t gslots = static_cast<uint32_t>(per_sm_groups * dev.sm_count);
+      const uint32_t ggrid = groups < gslots ? groups : gslots;
+      LbArgs la{tile_base, err_out ? ws.stream_err() : nullptr, reinterpret_cast<FF*>(ws.counts()),
+                ws.stage_idx(), ws.stage_val()};
+      void* gp[] = {&op, &d, &list_idx, &list_val, &list_count, &cap, &ctx, &la};
+      err = launch_pdl(
+          reinterpret_cast<const void*>(&lookback_stream_kernel<LwCandOp<GT>, kLwStages>), ggrid,
+          kLbThreads, LbLayout<LwCandOp<GT>, kLwStages>::kSmem, ws.stream, gp, false);
+    } else {
+      StreamArgs sa{ws.stage_idx(), ws.stage_val(), ws.counts(), ws.chunks(), tile_base,
+                    err_out ? ws.stream_err() : nullptr, ws.errparts()};
+      void* params[] = {&op, &d, &list_idx, &list_val, &list_count, &cap, &ctx, &sa};
+      // not cooperative: the only cross-CTA wait is on lower-numbered CTAs,
+      // which are scheduled first
+      err = launch_pdl(
+          reinterpret_cast<const void*>(&stream_compact_kernel<LwCandOp<GT>, kLwStages>), grid,
+          kStreamThreads, StreamLayout<LwCandOp<GT>, kLwStages>::kSmem, ws.stream, params, false);
+    }
     count_launch();
     if (err != cudaSuccess) return err;
   } else {
@@ -882,6 +910,8 @@ void topk_layerwise_init_device(DeviceInfo& info) {
   info.lw_select_per_sm = n;
   info.lw_stream_per_sm_f32 = lw_stream_blocks_per_sm<float>();
   info.lw_stream_per_sm_bf16 = lw_stream_blocks_per_sm<uint16_t>();
+  info.lw_group_per_sm_f32 = lw_group_blocks_per_sm<float>();
+  info.lw_group_per_sm_bf16 = lw_group_blocks_per_sm<uint16_t>();
   cudaGetLastError();
 }
 

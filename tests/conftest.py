@@ -17,13 +17,14 @@ def pytest_configure(config):
 
 
 @pytest.fixture(params=["chunks", "groups"])
-def ht_kernel(request):
-    """Runs a hard-threshold test with each streaming kernel: the static-chunk
+def stream_kernel(request):
+    """Runs a streaming-pass test (hard-threshold, Top-k or layer-wise Top-k)
+    with each streaming kernel: the static-chunk
     kernel and the claimed-group look-back kernel (by default the library
     picks by size; small test inputs would reach only the first)."""
     import paper_2108_00951_gb300 as efs
-    efs.ef_test_set_ht_stream({"chunks": 1, "groups": 2}[request.param])
+    efs.ef_test_set_stream_kernel({"chunks": 1, "groups": 2}[request.param])
     try:
         yield request.param
     finally:
-        efs.ef_test_set_ht_stream(0)
+        efs.ef_test_set_stream_kernel(0)

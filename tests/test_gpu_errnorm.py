@@ -88,7 +88,7 @@ def _check(kind, g, e, gamma, arg, what, off=0):
     return gerr, want
 
 
-@pytest.mark.usefixtures("ht_kernel")
+@pytest.mark.usefixtures("stream_kernel")
 @pytest.mark.parametrize("d", [1, 4097, 3 * 4096 + 17, 300_001])
 @pytest.mark.parametrize("off", [0, 1])
 def test_ht_error_norm(d, off):
@@ -97,7 +97,7 @@ def test_ht_error_norm(d, off):
         _check("ht", g, e, 0.1, lam, "ht d=%d off=%d lam=%g" % (d, off, lam), off=off)
 
 
-@pytest.mark.usefixtures("ht_kernel")
+@pytest.mark.usefixtures("stream_kernel")
 def test_ht_error_norm_bf16():
     d = 100_003
     g, e = _inputs(d, 2)
@@ -109,6 +109,7 @@ def test_ht_error_norm_bf16():
                                  (1_000_000, 60_000),  # list beyond shared memory
                                  (300_000, 150_000),   # full-array mode
                                  (50_000, 0), (50_000, 50_000), (7, 3)])
+@pytest.mark.usefixtures("stream_kernel")
 def test_topk_error_norm(d, k):
     g, e = _inputs(d, 3)
     _check("topk", g, e, 0.1, k, "topk d=%d k=%d" % (d, k))
@@ -123,6 +124,7 @@ KINDS_SIZES = [0, 5, 64, 4097, 49152, 49153, 100_003, 3 * 4096 + 17, 1, 200_000,
 KINDS_K = [0, 5, 3, 40, 491, 1, 1000, 0, 1, 2000, 6, 65_535]
 
 
+@pytest.mark.usefixtures("stream_kernel")
 @pytest.mark.parametrize("case", ["kinds", "team", "from_e", "cut_off", "misaligned"])
 def test_layerwise_error_norm(case):
     if case in ("kinds", "misaligned"):
@@ -151,6 +153,7 @@ def test_error_norm_full_size_resnet18():
     _check("lw", g, e, w.gamma, (ends, ks), "resnet18 layer-wise")
 
 
+@pytest.mark.usefixtures("stream_kernel")
 @pytest.mark.parametrize("kind", ["ht", "topk"])
 def test_error_norm_reproducible_over_calls(kind):
     # calls that return the norm use equal chunks and the sampled Top-k bound

@@ -30,6 +30,7 @@ def _healthy_call_matches_oracle(g, e):
     assert efs.ef_check_status() == efs.EF_OK
 
 
+@pytest.mark.usefixtures("stream_kernel")
 @pytest.mark.parametrize("method", ["ht", "topk"])
 def test_lookback_wait_runs_out_and_recovers(method):
     d = 40 * 4096 + 9

@@ -67,6 +67,7 @@ KINDS_SIZES = [0, 5, 64, 4097, 49152, 49153, 100_003, 3 * 4096 + 17, 1, 200_000,
 KINDS_K = [0, 5, 3, 40, 491, 1, 1000, 0, 1, 2000, 6, 65_535, 4095, 66, 1]
 
 
+@pytest.mark.usefixtures("stream_kernel")
 @pytest.mark.parametrize("bf16", [False, True])
 def test_layerwise_every_kind(bf16):
     g, e = _inputs(sum(KINDS_SIZES), 1, bf16=bf16)
@@ -79,6 +80,7 @@ def test_layerwise_misaligned_bases(offs):
     _check(g, e, 0.1, KINDS_SIZES, KINDS_K, "offsets %s" % (offs,), g_off=offs[0], e_off=offs[1])
 
 
+@pytest.mark.usefixtures("stream_kernel")
 def test_layerwise_single_segment_is_entire_vector_topk():
     d, k = 300_001, 3000
     g, e = _inputs(d, 3)
@@ -88,6 +90,7 @@ def test_layerwise_single_segment_is_entire_vector_topk():
     gu.assert_bits(ref[2], te, "e' vs entire")
 
 
+@pytest.mark.usefixtures("stream_kernel")
 def test_layerwise_candidates_beyond_shared_memory():
     # one sampled segment whose candidate list exceeds a CTA's shared memory
     sizes, ks = [400_000, 70_000], [60_000, 700]
@@ -95,6 +98,7 @@ def test_layerwise_candidates_beyond_shared_memory():
     _check(g, e, 0.1, sizes, ks, "long candidate list")
 
 
+@pytest.mark.usefixtures("stream_kernel")
 def test_layerwise_long_list_from_ties_one_cta():
     # a modest k whose cut falls inside a block of 100,000 equal magnitudes:
     # the candidates far exceed shared memory but the segment is not given a
@@ -109,6 +113,7 @@ def test_layerwise_long_list_from_ties_one_cta():
     _check(g, e, 1.0, [n, 5000], [15_000, 5], "tie block")
 
 
+@pytest.mark.usefixtures("stream_kernel")
 def test_layerwise_bound_admits_too_many():
     # half of a large segment: the candidates would not fit, so the segment
     # is selected from e itself
@@ -117,6 +122,7 @@ def test_layerwise_bound_admits_too_many():
     _check(g, e, 0.1, sizes, ks, "selection from e")
 
 
+@pytest.mark.usefixtures("stream_kernel")
 def test_layerwise_candidate_list_cut_off():
     # the segments' candidates together overflow the list's capacity: the
     # segments whose candidates were cut off are selected from e
@@ -126,6 +132,7 @@ def test_layerwise_candidate_list_cut_off():
     _check(g, e, 0.1, sizes, ks, "cut-off list")
 
 
+@pytest.mark.usefixtures("stream_kernel")
 def test_layerwise_ties_zeros_nan_inf():
     rng = _rng("ties")
     sizes = [60_000, 30_000, 120_000, 9, 50_000]
@@ -145,6 +152,7 @@ def test_layerwise_ties_zeros_nan_inf():
     _check(g, e, 1.0, sizes, ks, "ties")
 
 
+@pytest.mark.usefixtures("stream_kernel")
 def test_layerwise_iterations_table_change_and_interleaving():
     sizes_a = [70_000, 1_000, 200_003, 4_096, 55_555]
     sizes_b = [100_000, 230_654]  # same d, another table

@@ -46,7 +46,7 @@ def _check_same(gpu, ref, what):
 
 
 # ------------------------------------------------------------ hard-threshold
-@pytest.mark.usefixtures("ht_kernel")
+@pytest.mark.usefixtures("stream_kernel")
 @pytest.mark.parametrize("bf16", [False, True])
 @pytest.mark.parametrize("d", RAGGED)
 def test_ht_random(d, bf16):
@@ -65,7 +65,7 @@ def test_ht_misaligned_bases(offs, bf16):
                 oracle.ef_hard_threshold(g, e, 0.1, 1.5e-3), "offsets %s" % (offs,))
 
 
-@pytest.mark.usefixtures("ht_kernel")
+@pytest.mark.usefixtures("stream_kernel")
 def test_ht_adversarial_values():
     d = 3 * 4096 + 5
     rng = _rng("adv")
@@ -81,7 +81,7 @@ def test_ht_adversarial_values():
                     "adversarial lam=%g" % lam_)
 
 
-@pytest.mark.usefixtures("ht_kernel")
+@pytest.mark.usefixtures("stream_kernel")
 def test_ht_fma_sensitive_values():
     # e = -round(gamma*g): a is the product's rounding error, which only a
     # single-rounding fma preserves
@@ -94,7 +94,7 @@ def test_ht_fma_sensitive_values():
                 "fma")
 
 
-@pytest.mark.usefixtures("ht_kernel")
+@pytest.mark.usefixtures("stream_kernel")
 def test_ht_all_and_nothing_sent():
     d = 5 * 4096 + 1
     g, e = _inputs(d, 3)
@@ -114,7 +114,7 @@ def test_ht_zero_length():
     assert int(cnt.item()) == 0
 
 
-@pytest.mark.usefixtures("ht_kernel")
+@pytest.mark.usefixtures("stream_kernel")
 @pytest.mark.parametrize("off", [0, 1])
 def test_ht_concurrent_streams(off):
     # calls on different streams use different workspaces and may overlap
@@ -142,6 +142,7 @@ def test_ht_concurrent_streams(off):
                      ed.cpu().numpy()), oracle.ef_hard_threshold(g, e, 0.1, 1e-3), "stream")
 
 
+@pytest.mark.usefixtures("stream_kernel")
 @pytest.mark.parametrize("kind", ["topk", "topk_layerwise"])
 def test_topk_concurrent_streams(kind):
     # Top-k calls on different streams (their own workspaces) may overlap on
@@ -228,14 +229,14 @@ def test_ht_balanced_chunks_over_calls():
 SPILL_D = 3 * 2**20 + 4099
 
 
-@pytest.mark.usefixtures("ht_kernel")
+@pytest.mark.usefixtures("stream_kernel")
 @pytest.mark.parametrize("bf16", [False, True])
 def test_ht_spill_everything_sent(bf16):
     g, e = _inputs(SPILL_D, 21, bf16=bf16)
     _check_same(gu.ht(g, e, 0.1, 0.0), oracle.ef_hard_threshold(g, e, 0.1, 0.0), "all sent")
 
 
-@pytest.mark.usefixtures("ht_kernel")
+@pytest.mark.usefixtures("stream_kernel")
 def test_ht_spill_mixed_density():
     g, e = _inputs(SPILL_D, 22)
     g[: SPILL_D // 4] *= 1000.0  # a dense quarter (~96 % sent), the rest sends nothing
@@ -244,7 +245,7 @@ def test_ht_spill_mixed_density():
     _check_same((i, v, en), oracle.ef_hard_threshold(g, e, 0.1, 0.05), "mixed")
 
 
-@pytest.mark.usefixtures("ht_kernel")
+@pytest.mark.usefixtures("stream_kernel")
 @pytest.mark.parametrize("out_off", [(1, 0), (2, 3), (3, 1)])
 def test_ht_misaligned_outputs(out_off):
     # the pairs are written with 16-byte stores matched to each output's own
@@ -259,6 +260,7 @@ def test_ht_misaligned_outputs(out_off):
                 "small, outputs offset %s" % (out_off,))
 
 
+@pytest.mark.usefixtures("stream_kernel")
 @pytest.mark.parametrize("region,k", [(SPILL_D // 50, 20_000), (SPILL_D // 5, SPILL_D // 16)])
 def test_topk_spill_concentrated_candidates(region, k):
     # all candidates in the first `region` coordinates: the few CTAs there
@@ -269,6 +271,7 @@ def test_topk_spill_concentrated_candidates(region, k):
                 "region=%d k=%d" % (region, k))
 
 
+@pytest.mark.usefixtures("stream_kernel")
 @pytest.mark.parametrize("d", RAGGED)
 def test_topk_random(d):
     g, e = _inputs(d, 11)
@@ -284,6 +287,7 @@ def test_topk_bf16_and_misaligned():
                     oracle.ef_topk(g, e, 0.1, 500), "offs %s" % (offs,))
 
 
+@pytest.mark.usefixtures("stream_kernel")
 def test_topk_heavy_ties():
     d = 200_003
     rng = _rng("ties")
@@ -294,6 +298,7 @@ def test_topk_heavy_ties():
         _check_same(gu.topk(g, e, 1.0, k), oracle.ef_topk(g, e, 1.0, k), "ties k=%d" % k)
 
 
+@pytest.mark.usefixtures("stream_kernel")
 def test_topk_mostly_zero_like_lstm_embedding():
     # ~62% exact zeros; k beyond the non-zeros forces the choice into the zero bucket
     d = 400_000
@@ -306,6 +311,7 @@ def test_topk_mostly_zero_like_lstm_embedding():
         _check_same(gu.topk(g, e, 0.1, k), oracle.ef_topk(g, e, 0.1, k), "zeros k=%d" % k)
 
 
+@pytest.mark.usefixtures("stream_kernel")
 def test_topk_all_equal_magnitude_large():
     # all keys tie in the magnitude bits: the index digits decide, through
     # full-array refine passes (the bucket exceeds the candidate buffer)
@@ -322,6 +328,7 @@ def test_topk_all_equal_magnitude_large():
         gu.assert_bits(ge, want, "e'")
 
 
+@pytest.mark.usefixtures("stream_kernel")
 def test_topk_nan_inf():
     d = 9000
     g, e = _inputs(d, 13)
@@ -330,6 +337,7 @@ def test_topk_nan_inf():
         _check_same(gu.topk(g, e, 0.1, k), oracle.ef_topk(g, e, 0.1, k), "nan k=%d" % k)
 
 
+@pytest.mark.usefixtures("stream_kernel")
 def test_topk_calls_in_a_row_with_jumping_scales():
     # calls of one (k, d) on one stream whose scales jump by 100x between
     # calls, and a call with another k between them (the per-call state and
