@@ -487,15 +487,11 @@ __global__ void __launch_bounds__(kLbThreads, 1)
     uint32_t appended = 0;  // pairs appended so far (the placer counts the freed ones)
     FF warp_err{0.0f, 0.0f};  // lane 0: share of ||e'||^2 in the current group
 
-    for (uint32_t r = 0;; ++r) {
-      const int s = static_cast<int>(r % kStages);
-      const bool arrived = lb_mbar_wait(&s_full[s], (r / kStages) & 1u, &s_failed, ctx);
-      if (!__all_sync(0xffffffffu, arrived)) break;
-      const uint32_t t = s_stage_tile[s];
-      const uint32_t info = s_stage_info[s];
-      if (t == kLbStageEnd) break;
-      float a[kSUnits][4];
-      uint32_t sel[kSUnits];
+    // A group's tiles arrive in consecutive ring uses; each tile is computed
+    // and its stage released at once, and the group's bookkeeping (positions,
+    // buffer, counts, arrival) is done once for both tiles.
+    auto compute_tile = [&](int s, uint32_t t, float (&a)[kSUnits][4],
+                            uint32_t (&sel)[kSUnits]) {
       if (t < full_tiles) {
         op.tile_smem(smem + s * Op::kStageBytes, t, warp, lane, a, sel, aux);
       } else {
@@ -514,80 +510,114 @@ __global__ void __launch_bounds__(kLbThreads, 1)
         for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
         if (lane == 0) warp_err = ff_add(warp_err, FF{sq, 0.0f});
       }
-      // positions in coordinate order (unit 0's lanes, then unit 1's): one
-      // warp scan of both units' per-lane counts packed in 16-bit halves
-      static_assert(kSUnits == 2, "two units packed in one scan");
-      const uint32_t cnt2 = __popc(sel[0] & 0xfu) | (__popc(sel[1] & 0xfu) << 16);
-      uint32_t incl2 = cnt2;
+    };
+    static_assert(kSUnits == 2 && kLbGroupTiles == 2, "four units of a group packed in one scan");
+    for (uint32_t r = 0;;) {
+      int s = static_cast<int>(r % kStages);
+      bool arrived = lb_mbar_wait(&s_full[s], (r / kStages) & 1u, &s_failed, ctx);
+      if (!__all_sync(0xffffffffu, arrived)) break;
+      const uint32_t t0 = s_stage_tile[s];
+      const uint32_t slot = s_stage_info[s] & 0xffu;
+      if (t0 == kLbStageEnd) break;
+      LbEntry& en = ent[slot];
+      const uint32_t nt = en.ntiles;
+      float a[kLbGroupTiles][kSUnits][4];
+      uint32_t sel[kLbGroupTiles][kSUnits] = {{0u, 0u}, {0u, 0u}};
+      compute_tile(s, t0, a[0], sel[0]);
+      ++r;
+      if (nt == 2) {
+        s = static_cast<int>(r % kStages);
+        arrived = lb_mbar_wait(&s_full[s], (r / kStages) & 1u, &s_failed, ctx);
+        if (!__all_sync(0xffffffffu, arrived)) break;
+        compute_tile(s, t0 + 1, a[1], sel[1]);
+        ++r;
+      }
+      // positions in coordinate order: one warp scan of the four units'
+      // per-lane counts (at most 4 each, 128 a warp) packed in bytes
+      const uint32_t cnt4 = __popc(sel[0][0] & 0xfu) | (__popc(sel[0][1] & 0xfu) << 8) |
+                            (__popc(sel[1][0] & 0xfu) << 16) | (__popc(sel[1][1] & 0xfu) << 24);
+      uint32_t incl4 = cnt4;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t x = __shfl_up_sync(0xffffffffu, incl2, o);
-        if (lane >= o) incl2 += x;
+        const uint32_t x = __shfl_up_sync(0xffffffffu, incl4, o);
+        if (lane >= o) incl4 += x;
       }
-      const uint32_t all2 = __shfl_sync(0xffffffffu, incl2, 31);
-      const uint32_t excl2 = incl2 - cnt2;
-      const uint32_t total0 = all2 & 0xffffu;
-      uint32_t off[kSUnits];
-      off[0] = excl2 & 0xffffu;
-      off[1] = total0 + (excl2 >> 16);
-      const uint32_t total = total0 + (all2 >> 16);
-      // the segment's pairs go to the warp's buffer when it has room (the
-      // placer frees it group by group), else to the segment's global slot
+      const uint32_t all4 = __shfl_sync(0xffffffffu, incl4, 31);
+      const uint32_t excl4 = incl4 - cnt4;
+      const uint32_t u0 = all4 & 0xffu, u1 = (all4 >> 8) & 0xffu;
+      const uint32_t u2 = (all4 >> 16) & 0xffu, u3 = all4 >> 24;
+      const uint32_t seg_total[kLbGroupTiles] = {u0 + u1, u2 + u3};
+      // each unit's first position within its tile's segment
+      const uint32_t off[kLbGroupTiles][kSUnits] = {
+          {excl4 & 0xffu, u0 + ((excl4 >> 8) & 0xffu)},
+          {(excl4 >> 16) & 0xffu, u2 + (excl4 >> 24)}};
+      // each segment's pairs go to the warp's buffer when it has room (the
+      // placer frees it group by group), else to the segment's global slot;
+      // bit q of to_slot: segment q goes to its slot
       uint32_t to_slot = 0;
-      if (total && lane == 0) {
-        to_slot = appended + total - vld(s_freed[warp]) > L::kFifo ? 1u : 0u;
-        if (!to_slot) __threadfence_block();  // the buffer writes after the placer's reads
+      if ((seg_total[0] | seg_total[1]) && lane == 0) {
+        const uint32_t held = appended - vld(s_freed[warp]);
+        if (held + seg_total[0] > L::kFifo) to_slot |= 1u;
+        const uint32_t held1 = held + ((to_slot & 1u) ? 0u : seg_total[0]);
+        if (held1 + seg_total[1] > L::kFifo) to_slot |= 2u;
+        if (to_slot != 3u) __threadfence_block();  // the buffer writes after the placer's reads
       }
       to_slot = __shfl_sync(0xffffffffu, to_slot, 0);
       __syncwarp();
+      const uint32_t buf_total = ((to_slot & 1u) ? 0u : seg_total[0]) +
+                                 ((to_slot & 2u) ? 0u : seg_total[1]);
       // each lane writes its selected pairs in coordinate order, one set
       // selection bit at a time (at a few percent density most lanes have
       // none, and the warp takes as many rounds as its fullest lane)
-      const uint32_t first_elem = static_cast<uint32_t>(stream_element_index(t, warp, 0, lane, 0));
-      if (to_slot) {
-        const size_t sb = (static_cast<size_t>(t) * kSWarps + warp) * kSWarpElems;
 #pragma unroll
-        for (int v = 0; v < kSUnits; ++v) {
-          uint32_t p = off[v];
-          for (uint32_t bits = sel[v] & 0xfu; bits; bits &= bits - 1, ++p) {
-            const int j = __ffs(bits) - 1;
-            la.slot_idx[sb + p] = first_elem + v * 128 + j;
-            la.slot_val[sb + p] = lb_pick(a[v], j);
+      for (int q = 0; q < 2; ++q) {
+        const uint32_t t = t0 + q;
+        const uint32_t first_elem =
+            static_cast<uint32_t>(stream_element_index(t, warp, 0, lane, 0));
+        if ((to_slot >> q) & 1u) {
+          const size_t sb = (static_cast<size_t>(t) * kSWarps + warp) * kSWarpElems;
+#pragma unroll
+          for (int v = 0; v < kSUnits; ++v) {
+            uint32_t p = off[q][v];
+            for (uint32_t bits = sel[q][v] & 0xfu; bits; bits &= bits - 1, ++p) {
+              const int j = __ffs(bits) - 1;
+              la.slot_idx[sb + p] = first_elem + v * 128 + j;
+              la.slot_val[sb + p] = lb_pick(a[q][v], j);
+            }
+          }
+        } else {
+#pragma unroll
+          for (int v = 0; v < kSUnits; ++v) {
+            uint32_t p = tail + ((q && !(to_slot & 1u)) ? seg_total[0] : 0u) + off[q][v];
+            if (p >= L::kFifo) p -= L::kFifo;
+            for (uint32_t bits = sel[q][v] & 0xfu; bits; bits &= bits - 1) {
+              const int j = __ffs(bits) - 1;
+              my_idx[p] = first_elem + v * 128 + j;
+              my_val[p] = lb_pick(a[q][v], j);
+              if (++p == L::kFifo) p = 0;
+            }
           }
         }
-      } else {
-#pragma unroll
-        for (int v = 0; v < kSUnits; ++v) {
-          uint32_t p = tail + off[v];
-          if (p >= L::kFifo) p -= L::kFifo;
-          for (uint32_t bits = sel[v] & 0xfu; bits; bits &= bits - 1) {
-            const int j = __ffs(bits) - 1;
-            my_idx[p] = first_elem + v * 128 + j;
-            my_val[p] = lb_pick(a[v], j);
-            if (++p == L::kFifo) p = 0;
-          }
-        }
-        tail += total;
-        if (tail >= L::kFifo) tail -= L::kFifo;
-        appended += total;
       }
-      const uint32_t slot = info & 0xffu, q = info >> 8;
-      LbEntry& en = ent[slot];
-      const uint32_t nt = en.ntiles;
+      tail += buf_total;
+      if (tail >= L::kFifo) tail -= L::kFifo;
+      appended += buf_total;
       uint32_t before = 0;
       if (lane == 0) {
-        en.cnt[q * kSWarps + warp] = total;
-        if (to_slot) atomicOr(&en.spilled, 1u << (q * kSWarps + warp));
-        if (la.err_out && q + 1 == nt) {
+        en.cnt[warp] = seg_total[0];
+        if (nt == 2) en.cnt[kSWarps + warp] = seg_total[1];
+        if (to_slot)
+          atomicOr(&en.spilled, ((to_slot & 1u) << warp) | ((to_slot >> 1) << (kSWarps + warp)));
+        if (la.err_out) {
           en.err[warp] = warp_err;
           warp_err = FF{0.0f, 0.0f};
         }
-        __threadfence_block();  // the pairs and the count before the arrival
-        before = atomicAdd(&en.arrivals, 1u);
+        __threadfence_block();  // the pairs and the counts before the arrival
+        before = atomicAdd(&en.arrivals, nt);
       }
       before = __shfl_sync(0xffffffffu, before, 0);
-      if (before + 1 == nt * kSWarps) {
-        // this warp counted the group's last segment: its aggregate
+      if (before + nt == nt * kSWarps) {
+        // this warp counted the group's last segments: its aggregate
         if (lane == 0) __threadfence_block();
         __syncwarp();
         const uint32_t nseg = nt * kSWarps;
