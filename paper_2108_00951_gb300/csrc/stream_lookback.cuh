@@ -14,41 +14,49 @@
 //
 // Roles (warps of a CTA):
 //  - 16 compute warps. Warp w owns the 256-coordinate segment [w*256,
-//    (w+1)*256) of every tile (the element layout of stream_compact.cuh). For
-//    each stage it computes the op's values and selection bits, releases the
-//    stage, compacts its selected pairs with ballots into its own circular
-//    pair buffer in shared memory, and records the segment's count in the
-//    group's entry. The warp that completes a group (the last of its
-//    ntiles * 16 segments) publishes the group's aggregate. Whenever the
-//    oldest group it holds pairs of has its offsets, the warp copies those
-//    pairs to the output (its own segments only), freeing buffer space; it
-//    waits for that only when its buffer has no room for the next segment.
-//  - a producer warp (lane 0): claims a group when an entry is free, then
-//    issues the bulk copies (cp.async.bulk, completing on the stage's "full"
-//    mbarrier) of its tiles as ring stages are released; after the last
-//    group, an end marker.
+//    (w+1)*256) of every tile (the element layout of stream_compact.cuh). A
+//    group's two tiles arrive in consecutive ring stages; the warp computes
+//    each tile's values and selection bits and releases its stage at once,
+//    then, once for the group: the positions of its selected pairs (one warp
+//    scan of the four units' counts), the pairs appended to its own circular
+//    buffer in shared memory — or, for a segment that finds no room, to the
+//    segment's slot in global memory —, the counts recorded in the group's
+//    entry. The warp that completes a group publishes its aggregate.
+//  - a producer warp: lane 1 claims groups, up to kLbClaimAhead ahead; lane 0
+//    takes a claimed group when an entry is free and issues the bulk copies
+//    (cp.async.bulk, completing on the stage's "full" mbarrier) of its tiles
+//    as ring stages are released; after the last group, an end marker.
 //  - a look-back warp: for each group of the CTA in claim order, the
 //    decoupled look-back over the published group totals (Merrill & Garland,
-//    the same routine as the one-tile-per-CTA kernel), the inclusive total
+//    the routine of the one-tile-per-CTA kernel), the inclusive total
 //    published, then the output position of each of the group's segments in
 //    (tile, warp) order, which is coordinate order.
+//  - kLbPlaceWarps placer warps: for each group, once its positions are
+//    there, they copy its segments (placer p: segments p, p + kLbPlaceWarps,
+//    ...; a warp's lanes on consecutive pairs, so loads and stores are
+//    coalesced) from the buffers or slots to the output, then hand the
+//    buffers' space back and free the entry.
 //
 // Deadlock freedom. Take the lowest group m that is claimed but whose
 // aggregate is not published. Groups below m have published aggregates, so
-// the look-back of any group <= m completes. The warps of the CTA holding m
-// are never blocked on buffer space by anything but their own oldest group,
-// which is <= m: if that is m itself, the buffer holds only m's earlier
-// segments, and a buffer of at least kLbGroupTiles * 256 pairs always has
-// room for the next one. So m is completed and the argument repeats. Every
-// wait is nevertheless bounded in time; one that runs out latches
-// kDevErrTimeout, and the CTA stops (after its bulk copies have landed).
+// the look-back (and then the placement) of every group below m completes,
+// which frees every entry and buffer space they hold. The CTA holding m waits
+// for nothing else: a compute warp never waits for buffer space (a segment
+// without room goes to its slot), the producer waits only for entries of
+// older groups of its own CTA and for its ring, and the ring's stages are
+// released by the compute warps as soon as they have read them. So m is
+// completed and the argument repeats; no wait depends on which CTAs are
+// resident. Every wait is nevertheless bounded in time; one that runs out
+// latches kDevErrTimeout, and the CTA stops (after its bulk copies have
+// landed).
 //
-// Traffic: the op's own bytes plus 8 bytes per selected pair, written once;
-// 8 bytes of look-back status per group. The error norm (when la.err_out is
-// set) follows stream_compact.cuh's rule per coordinate; each group's share
-// (its warps' float-float shares in warp order) is stored per group, and the
-// last CTA to finish adds the groups' shares in group order, so the value
-// does not depend on which CTA took which group.
+// Traffic: the op's own bytes plus 8 bytes per selected pair, written once,
+// plus 16 bytes per pair that goes through a slot; 8 bytes of look-back
+// status per group. The error norm (when la.err_out is set) follows
+// stream_compact.cuh's rule per coordinate; each group's share (its warps'
+// float-float shares in warp order) is stored per group, and the last CTA to
+// finish adds the groups' shares in group order, so the value does not
+// depend on which CTA took which group.
 #pragma once
 
 #include "stream_compact.cuh"
@@ -66,7 +74,7 @@ constexpr uint32_t kLbGroupSegs = kLbGroupTiles * kSWarps;
 constexpr uint32_t kLbClaimAhead = 2;          // groups claimed before the producer needs them
 constexpr uint32_t kLbEntries = 8;             // groups of a CTA in flight or pending
 constexpr uint32_t kLbStageEnd = 0xffffffffu;
-constexpr uint32_t kLbSuspendNs = 1000;        // a waiting warp checks its other duties this often
+constexpr uint32_t kLbSuspendNs = 1000;        // a suspended wait re-checks its flag and limit this often
 constexpr uint32_t kLbSegsPerLane = kLbGroupSegs / 32;  // segments per lane in the offset scan
 static_assert(kLbGroupSegs % 32 == 0 && kLbSegsPerLane <= 2, "segments per look-back lane");
 
@@ -95,7 +103,9 @@ struct LbLayout {
   static constexpr uint32_t kEntryBytes = kLbEntries * sizeof(LbEntry);
   static constexpr uint32_t kBudget = 227u * 1024u - 2048u;
   static constexpr uint32_t kFifo = ((kBudget - kRing - kEntryBytes) / (kSWarps * 8u)) / 32u * 32u;
-  static_assert(kFifo >= kLbGroupTiles * kSWarpElems, "a group's segments fit a warp's buffer");
+  // (a segment that finds no room goes to its global slot, so nothing waits
+  // for buffer space; a buffer smaller than a segment would only spill more)
+  static_assert(kFifo >= kSWarpElems, "a whole segment fits a warp's buffer");
   static constexpr uint32_t kOffEntries = kRing + kSWarps * kFifo * 8u;
   static constexpr uint32_t kSmem = kOffEntries + kEntryBytes;  // dynamic shared memory
 };
