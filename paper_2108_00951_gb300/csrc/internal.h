@@ -50,7 +50,9 @@ constexpr uint32_t kCountsPerTile = 16; // per-segment counts of the streaming c
 constexpr uint32_t kLwNone = 0, kLwWhole = 1, kLwSampled = 2, kLwAll = 3;
 constexpr uint32_t kLwSmemElems = 48u * 1024u;  // values one select CTA holds in shared memory
 constexpr uint32_t kLwWholeMax = 4096;          // segments at most this long: selected from e
-constexpr uint32_t kLwSampleGroups = 4096;      // groups of 4 coordinates sampled per segment
+constexpr uint32_t kLwSampleGroups = 4096;      // groups of 4 coordinates sampled per CTA
+constexpr uint32_t kLwMaxParts = 16;            // sampling CTAs of one long segment, at most
+constexpr uint32_t kLwPartHistWords = kSampleBins + 32;  // merged histogram + arrival word
 // Candidate bounds that admit nothing: the residual of the segment's
 // coordinates is then a, final in the streaming pass (kLwNoBound: segments
 // that send nothing), or decided by the select (kLwDeferred: short segments,
@@ -101,7 +103,8 @@ struct LwPlan {
   // byte offsets in dev: uploaded tables, then zero-initialised counters
   // and histograms (each user resets its own), then per-call outputs
   size_t off_segs = 0, off_seg_end = 0, off_mbound = 0, off_tile_info = 0, off_samples = 0,
-         off_ctas = 0, off_work_seg = 0, off_teams = 0, off_tile_base = 0, total = 0;
+         off_ctas = 0, off_work_seg = 0, off_teams = 0, off_part_hist = 0, off_tile_base = 0,
+         total = 0;
 };
 
 struct Workspace {

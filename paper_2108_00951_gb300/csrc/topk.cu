@@ -16,7 +16,8 @@
 //             and the last CTA to arrive derives the lower bound B with about
 //             1.5 times the needed mass above it (or, when the candidates
 //             would not fit, the full-array mode).
-//  2 stream   the streaming compaction of stream_compact.cuh: a =
+//  2 stream   the streaming compaction (stream_compact.cuh, or from 4096
+//             tiles on stream_lookback.cuh): a =
 //             fmaf(γ,g,e) is written over e (12 B per coordinate, the
 //             algorithmic bytes) and the coordinates with K_j >= B are
 //             emitted as an ordered (index, value) candidate list. This

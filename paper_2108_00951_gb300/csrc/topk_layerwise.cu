@@ -15,7 +15,8 @@
 //             in shared memory and picks the candidate bound: the bin holding
 //             k_s samples when every group was read, else about 1.5 times the
 //             needed mass above it.
-//  2 stream   the streaming compaction of stream_compact.cuh: a = fmaf(γ,g,e)
+//  2 stream   the streaming compaction (stream_compact.cuh, or from 4096
+//             tiles on stream_lookback.cuh): a = fmaf(γ,g,e)
 //             is written over e (12 B per coordinate, the algorithmic bytes)
 //             and the coordinates at or above their segment's bound are
 //             emitted as one ordered candidate list, with the list position
@@ -69,17 +70,30 @@ constexpr int kSampleThreads = 1024;
 template <typename GT>
 __global__ void __launch_bounds__(kSampleThreads, 1)
     lw_sample_kernel(const GT* __restrict__ g, const float* __restrict__ e, float gamma,
-                     const LwSeg* __restrict__ segs, const uint32_t* __restrict__ sampled,
-                     uint32_t* mbound, uint32_t cand_cap) {
+                     const LwSeg* __restrict__ segs, const uint2* __restrict__ sampled,
+                     uint32_t* mbound, uint32_t cand_cap, uint32_t* part_hist) {
   __shared__ uint32_t s_hist[kSampleBins];
   __shared__ uint32_t s_w[kSampleThreads / 32];
-  __shared__ uint32_t s_bin, s_mass;
+  __shared__ uint32_t s_bin, s_mass, s_last;
   const int tid = threadIdx.x;
   griddep_launch_dependents();  // the stream pass may be scheduled (it waits for this grid)
-  const uint32_t si = sampled[blockIdx.x];
-  const LwSeg s = segs[si];
+  // this CTA's part of the segment: part `part` of `parts` equal runs of its
+  // aligned groups (one part: the host's sampling plan), with merge slot `slot`
+  const uint2 rec = sampled[blockIdx.x];
+  const uint32_t si = rec.x, part = rec.y & 0xffu, parts = (rec.y >> 8) & 0xffu,
+                 slot = rec.y >> 16;
+  LwSeg s = segs[si];
   for (int b = tid; b < kSampleBins; b += kSampleThreads) s_hist[b] = 0;
-  const uint64_t a0 = (static_cast<uint64_t>(s.lo) + 3u) & ~static_cast<uint64_t>(3);
+  uint64_t a0 = (static_cast<uint64_t>(s.lo) + 3u) & ~static_cast<uint64_t>(3);
+  if (parts > 1) {
+    const uint64_t avail = (static_cast<uint64_t>(s.hi) - a0) / 4;  // whole groups inside
+    const uint64_t g0 = part * avail / parts, g1 = (part + 1) * avail / parts;
+    const uint64_t n = g1 - g0;
+    s.groups = static_cast<uint32_t>(n < kLwSampleGroups ? n : kLwSampleGroups);
+    s.step = s.groups > 1 ? ((n - 1) << 32) / (s.groups - 1) : 0;
+    s.exact = 0;
+    a0 += 4 * g0;
+  }
   constexpr int kG = static_cast<int>(kLwSampleGroups / kSampleThreads);
   GradVec<GT> gv[kG];
   float4 ev[kG];
@@ -109,6 +123,29 @@ __global__ void __launch_bounds__(kSampleThreads, 1)
       if (in[q]) atomicAdd(&s_hist[mag_bits(x[j]) >> kLwSampleShift], 1u);
   }
   __syncthreads();
+  if (parts > 1) {
+    // add the part's histogram to the segment's merged one (after the wait:
+    // the previous call's last part left it at zero); the last part to
+    // arrive takes the merged histogram, leaves it at zero, and goes on
+    griddep_wait();
+    uint32_t* gh = part_hist + static_cast<size_t>(slot) * kLwPartHistWords;
+    for (int b = tid; b < kSampleBins; b += kSampleThreads)
+      if (s_hist[b]) atomicAdd(&gh[b], s_hist[b]);
+    __syncthreads();
+    if (tid == 0) {
+      __threadfence();
+      s_last = atomicAdd(&gh[kSampleBins], 1u) == parts - 1 ? 1u : 0u;
+      if (s_last) __threadfence();  // the other parts' adds before the reads
+    }
+    __syncthreads();
+    if (!s_last) return;
+    for (int b = tid; b < kSampleBins; b += kSampleThreads) {
+      s_hist[b] = __ldcg(&gh[b]);
+      gh[b] = 0;
+    }
+    if (tid == 0) gh[kSampleBins] = 0;
+    __syncthreads();
+  }
   // kPer consecutive bins per thread
   constexpr int kPer = kSampleBins / kSampleThreads;
   uint32_t c[kPer];
@@ -812,10 +849,11 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t d, uint32_
   if (streamable) {
     // 1 sample
     if (p.n_sampled > 0) {
-      const uint32_t* sampled = reinterpret_cast<const uint32_t*>(p.dev + p.off_samples);
+      const uint2* sampled = reinterpret_cast<const uint2*>(p.dev + p.off_samples);
       uint32_t cap = ws.cand_cap;
+      uint32_t* part_hist = reinterpret_cast<uint32_t*>(p.dev + p.off_part_hist);
       void* sp[] = {(void*)&g, (void*)&e, (void*)&gamma, (void*)&segs, (void*)&sampled,
-                    (void*)&mbound, (void*)&cap};
+                    (void*)&mbound, (void*)&cap, (void*)&part_hist};
       err = launch_pdl(reinterpret_cast<const void*>(&lw_sample_kernel<GT>), p.n_sampled,
                        kSampleThreads, 0, ws.stream, sp, false);
       count_launch();
@@ -928,8 +966,10 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
   // segments, sampling CTAs
   std::vector<LwSeg> segs(n_seg);
   std::vector<uint32_t> ends(n_seg), mbound(n_seg, kLwNoBound);
-  std::vector<uint32_t> sampled;  // the sampled segments, one sampling CTA each
-  uint32_t n_sampled = 0;
+  // the sampling CTAs: (segment, part | parts << 8 | merge slot << 16)
+  std::vector<uint2> sampled;
+  std::vector<uint32_t> parts_of(n_seg, 1);
+  uint32_t n_sampled = 0, n_part_hist = 0;
   uint64_t lo = 0, total_k = 0;
   for (uint32_t s = 0; s < n_seg; ++s) {
     const uint64_t hi = seg_end[s], ds = hi - lo, k = seg_k[s];
@@ -952,8 +992,26 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
       x.groups = static_cast<uint32_t>(std::min<uint64_t>(avail, kLwSampleGroups));
       x.exact = x.groups == avail ? 1u : 0u;
       x.step = ((avail - 1) << 32) / (x.groups - 1);  // a segment of > 4096 holds > 1000 groups
-      ++n_sampled;
-      sampled.push_back(s);
+      // A long segment with a small k_s would admit far more candidates
+      // than one CTA holds: the bound keeps 32 samples' slack, i.e.
+      // 32 d_s / (4 groups) coordinates. Up to kLwMaxParts CTAs then sample
+      // equal runs of it (kLwSampleGroups groups each) into one merged
+      // histogram, shrinking that slack.
+      uint32_t parts = 1;
+      if (!x.exact) {
+        const uint64_t need = 3ull * k / 2, fit = kLwSmemElems * 3ull / 4;
+        const uint64_t slack = 32ull * ds / (4ull * x.groups);
+        if (need + slack > fit && need < fit / 2) {
+          const uint64_t want = (slack + (fit - need) - 1) / (fit - need);
+          parts = static_cast<uint32_t>(std::min<uint64_t>(
+              std::min<uint64_t>(want, kLwMaxParts), avail / kLwSampleGroups));
+          if (parts < 1) parts = 1;
+        }
+      }
+      parts_of[s] = parts;
+      const uint32_t slot = parts > 1 ? n_part_hist++ : 0u;
+      for (uint32_t j = 0; j < parts; ++j) sampled.push_back(make_uint2(s, j | (parts << 8) | (slot << 16)));
+      n_sampled += parts;
     }
     ends[s] = static_cast<uint32_t>(hi);
     mbound[s] = x.kind == kLwNone ? kLwNoBound : kLwDeferred;  // sampled: the sampler's
@@ -986,9 +1044,13 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
     if (x.kind == kLwSampled) {
       // candidates the bound aims at: 1.5 k_s, plus 32 samples' worth
       const uint64_t ds = x.hi - x.lo;
-      const uint64_t est = x.exact ? x.k + 2048 : 3ull * x.k / 2 + 32ull * ds / (4ull * x.groups);
+      const uint64_t sampled_groups = static_cast<uint64_t>(x.groups) * parts_of[s];
+      const uint64_t est =
+          x.exact ? x.k + 2048 : 3ull * x.k / 2 + 32ull * ds / (4ull * sampled_groups);
       uint64_t want = est > kLwSmemElems * 3ull / 4 ? (est + 24575) / 24576 : 1;
-      want = std::max<uint64_t>(want, (ds + (1u << 24) - 1) >> 24);
+      // a segment one CTA would select slowly from e if its bound missed
+      // gets a team, unless its merged sample makes a miss implausible
+      if (parts_of[s] == 1) want = std::max<uint64_t>(want, (ds + (1u << 24) - 1) >> 24);
       t = static_cast<uint32_t>(std::min<uint64_t>(want, kLwMaxTeam));
     }
     if (t > 1) {
@@ -1063,11 +1125,12 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
   p.off_seg_end = take(sizeof(uint32_t) * n_seg);
   p.off_mbound = take(sizeof(uint32_t) * n_seg);
   p.off_tile_info = take(sizeof(uint32_t) * tiles);
-  p.off_samples = take(sizeof(uint32_t) * sampled.size());
+  p.off_samples = take(sizeof(uint2) * sampled.size());
   p.off_ctas = take(sizeof(LwCta) * ctas.size());
   p.off_work_seg = take(sizeof(uint32_t) * work_seg.size());
   const size_t upload = off;
   p.off_teams = take(sizeof(LwTeamState) * n_teams);
+  p.off_part_hist = take(sizeof(uint32_t) * kLwPartHistWords * n_part_hist);
   const size_t zero_end = off;
   p.off_tile_base = take(sizeof(uint32_t) * (tiles + 1));
   p.total = off;
@@ -1080,7 +1143,7 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
   put(p.off_seg_end, ends.data(), sizeof(uint32_t) * n_seg);
   put(p.off_mbound, mbound.data(), sizeof(uint32_t) * n_seg);
   put(p.off_tile_info, tile_info.data(), sizeof(uint32_t) * tiles);
-  put(p.off_samples, sampled.data(), sizeof(uint32_t) * sampled.size());
+  put(p.off_samples, sampled.data(), sizeof(uint2) * sampled.size());
   put(p.off_ctas, ctas.data(), sizeof(LwCta) * ctas.size());
   put(p.off_work_seg, work_seg.data(), sizeof(uint32_t) * work_seg.size());
 
