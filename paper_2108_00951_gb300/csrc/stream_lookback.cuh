@@ -66,8 +66,10 @@ namespace efs {
 constexpr int kLbProducerWarp = kSWarps;       // 16
 constexpr int kLbScanWarp = kSWarps + 1;       // 17
 constexpr int kLbPlaceWarp = kSWarps + 2;      // 18: the first placer warp
-constexpr int kLbPlaceWarps = 8;
-constexpr int kLbThreads = 32 * (kSWarps + 2 + kLbPlaceWarps);  // 832
+constexpr int kLbPlaceWarps = 12;  // with 8, placement bounds calls that send ~a quarter of a
+                                   // vector; 12 cost nothing on sparser ones
+constexpr int kLbThreads = 32 * (kSWarps + 2 + kLbPlaceWarps);  // 960
+static_assert(kLbThreads <= 1024, "one CTA of at most 1024 threads");
 constexpr uint32_t kLbGroupTiles = 2;          // tiles per claimed group (the placement
                                                // assumes 2: 32 segments, one per lane)
 constexpr uint32_t kLbGroupSegs = kLbGroupTiles * kSWarps;
