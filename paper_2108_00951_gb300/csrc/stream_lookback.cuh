@@ -80,7 +80,7 @@ constexpr uint32_t kLbSuspendNs = 1000;        // a suspended wait re-checks its
 constexpr uint32_t kLbSegsPerLane = kLbGroupSegs / 32;  // segments per lane in the offset scan
 static_assert(kLbGroupSegs % 32 == 0 && kLbSegsPerLane <= 2, "segments per look-back lane");
 
-// One group of a CTA, from its claim until every warp placed its pairs.
+// One group of a CTA, from the producer taking it until its pairs are placed.
 struct LbEntry {
   uint32_t cnt[kLbGroupSegs];  // pairs of segment (q, w) at q * 16 + w
   uint32_t off[kLbGroupSegs];  // output position of each segment's first pair
@@ -91,7 +91,7 @@ struct LbEntry {
   uint32_t ntiles;             // tiles of the group (the last group may have fewer)
   uint32_t arrivals;           // segments counted so far (complete: ntiles * 16)
   uint32_t total;              // the group's aggregate (once complete)
-  uint32_t placed;             // kSWarps: the entry is free
+  uint32_t placed;             // kSWarps: the entry is free (set by the placers)
   uint32_t spilled;            // bit l: segment l's pairs are in its global slot
   uint32_t pad;
 };
@@ -191,9 +191,9 @@ __global__ void __launch_bounds__(kLbThreads, 1)
   __shared__ __align__(8) uint64_t s_full[kStages];
   __shared__ __align__(8) uint64_t s_empty[kStages];
   __shared__ uint32_t s_stage_tile[kStages];  // tile of the stage's current use, or the end
-  __shared__ uint32_t s_stage_info[kStages];  // its entry slot | (tile within group << 8)
-  __shared__ uint32_t s_claimed;              // groups this CTA claimed so far
-  __shared__ uint32_t s_claim_done;           // the producer claims no more
+  __shared__ uint32_t s_stage_info[kStages];  // its group's entry slot | (tile in the group << 8)
+  __shared__ uint32_t s_claimed;              // groups the producer took so far
+  __shared__ uint32_t s_claim_done;           // the producer takes no more
   __shared__ uint32_t s_failed;               // a wait of this CTA ran out
   __shared__ uint32_t s_resolved;             // groups the look-back warp resolved
   __shared__ uint32_t s_freed[kSWarps];       // pairs of each compute warp placed so far
