@@ -56,7 +56,9 @@
  * on that stream: about 8 bytes per coordinate of pair staging (the size of
  * the outputs: 1.1 GB at d = 138 M) plus, once Top-k has run, 3 x 8 bytes per
  * candidate slot (min(d, max(2^20, d/16)) slots), plus 8 bytes per 4096
- * coordinates and about 260 KB of fixed state. Memory is therefore bounded by
+ * coordinates and about 260 KB of fixed state, and one 4-byte word of mapped
+ * pinned host memory (the density hint of the hard-threshold step's kernel
+ * choice, written by the device). Memory is therefore bounded by
  * (number of streams used) x that size; ef_workspace_release() frees all
  * workspaces of the current device (for example after a phase that used
  * extra streams), and ef_hard_threshold_noalloc needs none. Calls on
@@ -457,9 +459,13 @@ void ef_test_set_lookback_fault(int64_t withheld_tile, uint32_t spin_limit_us);
  * hard-threshold step and of the Top-k and layer-wise Top-k candidate passes
  * (16-byte aligned g and e): 0 (the default) by size (claimed groups of tiles
  * with look-back from 4096 tiles, 16,777,216 coordinates, on; static chunks
- * below), 1 static chunks, 2 claimed groups. Any other value means 0. The
- * results are the same whichever kernel runs; the hook lets tests run both on
- * small inputs. Process-wide; never needed in production.
+ * below; for the hard-threshold step, a shallower ring with larger pair
+ * buffers once an earlier call on the same stream sent at least 1/12 of its
+ * coordinates), 1 static chunks, 2 claimed groups, 3 claimed groups with the
+ * shallower ring (hard-threshold; the candidate passes treat 3 as 2). Any
+ * other value means 0. The results are the same whichever kernel runs; the
+ * hook lets tests run each on small inputs. Process-wide; never needed in
+ * production.
  */
 void ef_test_set_stream_kernel(int mode);
 

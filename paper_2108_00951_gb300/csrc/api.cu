@@ -21,7 +21,7 @@ std::map<int, DeviceInfo> g_devices;
 std::atomic<uint64_t> g_launches{0};
 std::atomic<int64_t> g_withheld_tile{-1};
 std::atomic<uint64_t> g_wait_limit_ns{2000000000ull};  // 2 s per wait
-std::atomic<int> g_stream_kernel_mode{0};  // 0: by size, 1: static chunks, 2: claimed groups
+std::atomic<int> g_stream_kernel_mode{0};  // 0: by size, 1: chunks, 2: groups, 3: shallow ring
 
 constexpr uint64_t kMaxD = 0xffffffffull;
 
@@ -64,6 +64,19 @@ ef_status acquire_workspace(cudaStream_t stream, uint32_t tiles, uint32_t cand_c
     ws = new Workspace;
     ws->device = dev;
     ws->stream = stream;
+    // the density hint (no hint when mapped host memory is unavailable)
+    void* h = nullptr;
+    if (cudaHostAlloc(&h, sizeof(uint32_t), cudaHostAllocMapped) == cudaSuccess) {
+      void* dp = nullptr;
+      *static_cast<volatile uint32_t*>(h) = 0u;
+      if (cudaHostGetDevicePointer(&dp, h, 0) == cudaSuccess) {
+        ws->density_host = static_cast<uint32_t*>(h);
+        ws->density_dev = static_cast<uint32_t*>(dp);
+      } else {
+        cudaFreeHost(h);
+      }
+    }
+    cudaGetLastError();
   }
   if (!ws->base || tiles > ws->status_tiles || cand_cap > ws->cand_cap ||
       offsets > ws->offsets_cap || stage > ws->stage_cap) {
@@ -599,6 +612,7 @@ ef_status ef_workspace_release(void) {
   for (auto it = efs::g_workspaces.begin(); it != efs::g_workspaces.end();) {
     if (it->first.first == dev) {
       if (it->second->base) cudaFree(it->second->base);
+      if (it->second->density_host) cudaFreeHost(it->second->density_host);
       if (it->second->lw) {
         if (it->second->lw->dev) cudaFree(it->second->lw->dev);
         delete it->second->lw;
@@ -621,7 +635,7 @@ void ef_test_set_lookback_fault(int64_t withheld_tile, uint32_t spin_limit_us) {
 }
 
 void ef_test_set_stream_kernel(int mode) {
-  efs::g_stream_kernel_mode.store(mode == 1 || mode == 2 ? mode : 0);
+  efs::g_stream_kernel_mode.store(mode >= 1 && mode <= 3 ? mode : 0);
 }
 
 }  // extern "C"

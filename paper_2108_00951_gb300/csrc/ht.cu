@@ -189,8 +189,8 @@ struct HtOp {
 template <typename GT>
 constexpr int kHtStages = sizeof(GT) == 2 ? 5 : 4;
 
-template <typename GT>
-using HtGroupKernel = LbLayout<HtOp<GT>, kHtStages<GT>>;
+template <typename GT, int kStages = kHtStages<GT>>
+using HtGroupKernel = LbLayout<HtOp<GT>, kStages>;
 template <typename GT>
 using HtChunkKernel = StreamLayout<HtOp<GT>, kHtStages<GT>>;
 
@@ -198,8 +198,9 @@ using HtChunkKernel = StreamLayout<HtOp<GT>, kHtStages<GT>>;
 // per SM. A group waits only for groups claimed before it, held by running
 // CTAs, so the launch needs no co-residency. Programmatic: it may start while
 // the previous kernel on the stream finishes (the kernel waits for it before
-// its first read).
-template <typename GT>
+// its first read). kStages: the ring depth (one stage fewer for dense calls,
+// whose pair buffers then take the freed shared memory).
+template <typename GT, int kStages>
 cudaError_t launch_groups(const GT* g, float* e, float gamma, float lambda, uint32_t d,
                           uint32_t* idx_out, float* val_out, uint32_t* count_out, double* err_out,
                           uint32_t* tiles_out, Workspace& ws, const DeviceInfo& dev,
@@ -213,11 +214,11 @@ cudaError_t launch_groups(const GT* g, float* e, float gamma, float lambda, uint
   ScanCtx c = ctx;
   // the groups' shares of ||e'||^2 use the per-tile count area (16 words a tile)
   LbArgs la{tiles_out, err_out, reinterpret_cast<FF*>(ws.counts()), ws.stage_idx(),
-            ws.stage_val()};
+            ws.stage_val(), ws.density_dev};
   void* params[] = {&op, &d, &idx_out, &val_out, &count_out, &cap, &c, &la};
   const cudaError_t err = launch_pdl(
-      reinterpret_cast<const void*>(&lookback_stream_kernel<HtOp<GT>, kHtStages<GT>>), grid,
-      kLbThreads, HtGroupKernel<GT>::kSmem, ws.stream, params, false);
+      reinterpret_cast<const void*>(&lookback_stream_kernel<HtOp<GT>, kStages>), grid,
+      kLbThreads, HtGroupKernel<GT, kStages>::kSmem, ws.stream, params, false);
   count_launch();
   ws.ht_part_ready = false;  // the chunk kernel's boundaries are not written by this kernel
   return err;
@@ -278,10 +279,22 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, float lambda, uint3
   const uintptr_t ga = reinterpret_cast<uintptr_t>(g), ea = reinterpret_cast<uintptr_t>(e);
   if (ga % 16 == 0 && ea % 16 == 0) {
     const int per_group = sizeof(GT) == 4 ? dev.ht_group_per_sm_f32 : dev.ht_group_per_sm_bf16;
+    const int per_dense = sizeof(GT) == 4 ? dev.ht_dense_per_sm_f32 : dev.ht_dense_per_sm_bf16;
     const int per_chunk = sizeof(GT) == 4 ? dev.ht_stream_per_sm_f32 : dev.ht_stream_per_sm_bf16;
-    if (use_group_kernel(tiles) && per_group > 0)
-      return launch_groups(g, e, gamma, lambda, d, idx_out, val_out, count_out, err_out,
-                           tiles_out, ws, dev, ctx, per_group);
+    if (use_group_kernel(tiles)) {
+      const int mode = stream_kernel_mode();
+      const bool dense =
+          mode == 3 || (mode == 0 && ws.density_host &&
+                        *static_cast<volatile uint32_t*>(ws.density_host) >= kDenseRingHint);
+      if (dense && per_dense > 0)
+        return launch_groups<GT, kHtStages<GT> - 1>(g, e, gamma, lambda, d, idx_out, val_out,
+                                                    count_out, err_out, tiles_out, ws, dev, ctx,
+                                                    per_dense);
+      if (per_group > 0)
+        return launch_groups<GT, kHtStages<GT>>(g, e, gamma, lambda, d, idx_out, val_out,
+                                                count_out, err_out, tiles_out, ws, dev, ctx,
+                                                per_group);
+    }
     if (per_chunk > 0)
       return launch_chunks(g, e, gamma, lambda, d, idx_out, val_out, count_out, err_out,
                            tiles_out, ws, dev, ctx, per_chunk);
@@ -312,10 +325,10 @@ int blocks_per_sm(const void* fn, int threads) {
   return n;
 }
 
-template <typename GT>
+template <typename GT, int kStages>
 int group_blocks_per_sm() {
-  return blocks_per_sm<GT, HtGroupKernel<GT>>(
-      reinterpret_cast<const void*>(&lookback_stream_kernel<HtOp<GT>, kHtStages<GT>>), kLbThreads);
+  return blocks_per_sm<GT, HtGroupKernel<GT, kStages>>(
+      reinterpret_cast<const void*>(&lookback_stream_kernel<HtOp<GT>, kStages>), kLbThreads);
 }
 template <typename GT>
 int chunk_blocks_per_sm() {
@@ -329,8 +342,10 @@ int chunk_blocks_per_sm() {
 void ht_init_device(DeviceInfo& info) {
   info.ht_stream_per_sm_f32 = chunk_blocks_per_sm<float>();
   info.ht_stream_per_sm_bf16 = chunk_blocks_per_sm<uint16_t>();
-  info.ht_group_per_sm_f32 = group_blocks_per_sm<float>();
-  info.ht_group_per_sm_bf16 = group_blocks_per_sm<uint16_t>();
+  info.ht_group_per_sm_f32 = group_blocks_per_sm<float, kHtStages<float>>();
+  info.ht_group_per_sm_bf16 = group_blocks_per_sm<uint16_t, kHtStages<uint16_t>>();
+  info.ht_dense_per_sm_f32 = group_blocks_per_sm<float, kHtStages<float> - 1>();
+  info.ht_dense_per_sm_bf16 = group_blocks_per_sm<uint16_t, kHtStages<uint16_t> - 1>();
 }
 
 // Launch the look-back kernel over caller-provided scratch (the tile-status

@@ -126,6 +126,11 @@ struct Workspace {
   uint32_t ht_last_epoch = 0;
   bool ht_part_ready = false;   // the previous call wrote the boundaries for this one
   bool ht_prev_balanced = false;  // the previous call used written boundaries
+  // Host-mapped word the claimed-group hard-threshold kernel writes (the
+  // call's pairs * 65536 / d): read without synchronising, it may be a few
+  // calls old, and only picks the next calls' ring depth (never a result).
+  uint32_t* density_host = nullptr;
+  uint32_t* density_dev = nullptr;
   bool dirty = false;          // header must be re-cleared (failed launch or device timeout)
   LwPlan* lw = nullptr;        // layer-wise Top-k tables (created on first use)
 
@@ -186,6 +191,8 @@ struct DeviceInfo {
   int ht_stream_per_sm_bf16 = 0;
   int ht_group_per_sm_f32 = 0;    // hard-threshold claimed-group CTAs per SM (0: unavailable)
   int ht_group_per_sm_bf16 = 0;
+  int ht_dense_per_sm_f32 = 0;    // the same with the shallow ring
+  int ht_dense_per_sm_bf16 = 0;
   int tk_stream_per_sm_f32 = 0;   // streaming Top-k candidate pass CTAs per SM
   int tk_stream_per_sm_bf16 = 0;
   int tk_group_per_sm_f32 = 0;    // Top-k candidate pass, claimed-group kernel CTAs per SM
@@ -233,7 +240,10 @@ cudaError_t launch_pdl(const void* fn, dim3 grid, uint32_t block, uint32_t smem,
 void count_launch();
 uint64_t wait_limit_ns();
 int64_t withheld_tile();
-int stream_kernel_mode();  // ef_test_set_stream_kernel: 0 by size, 1 static chunks, 2 claimed groups
+// ef_test_set_stream_kernel: 0 by size (and density), 1 static chunks, 2 claimed
+// groups, 3 claimed groups with the shallow ring (hard-threshold; the other
+// streaming passes treat it as 2)
+int stream_kernel_mode();
 
 // The streaming passes (hard-threshold, Top-k and layer-wise candidates) use
 // the claimed-group look-back kernel from this many tiles on (16.8 M
@@ -243,8 +253,13 @@ int stream_kernel_mode();  // ef_test_set_stream_kernel: 0 by size, 1 static chu
 constexpr uint32_t kGroupKernelMinTiles = 4096;
 inline bool use_group_kernel(uint32_t tiles) {
   const int mode = stream_kernel_mode();
-  return mode == 2 || (mode == 0 && tiles >= kGroupKernelMinTiles);
+  return mode >= 2 || (mode == 0 && tiles >= kGroupKernelMinTiles);
 }
+// Dense calls (the claimed-group hard-threshold kernel's last call on this
+// workspace sent at least this share of its coordinates, in 1/65536) run the
+// kernel with one ring stage fewer and the freed shared memory added to the
+// warps' pair buffers: fewer segments go through their global slots.
+constexpr uint32_t kDenseRingHint = 65536u / 12u;  // 8.3 %
 ScanCtx next_scan_ctx(Workspace& ws, uint32_t num_tiles);
 
 // ---- launchers (return the launch's cudaError_t) ----

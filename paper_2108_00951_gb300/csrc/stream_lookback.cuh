@@ -120,6 +120,8 @@ struct LbArgs {
   FF* err_parts;        // [groups] the groups' shares of it (used when err_out is set)
   uint32_t* slot_idx;   // [num_tiles * 16 * 256] a segment's pairs when its warp's buffer is
   float* slot_val;      // full: segment (tile, warp) at (tile * 16 + warp) * 256
+  uint32_t* density_out;  // optional (host-mapped): the call's pair count * 65536 / d, a hint
+                          // the host reads for later calls' choice of ring depth, or null
 };
 
 __device__ __forceinline__ uint32_t vld(const uint32_t& x) {
@@ -383,6 +385,8 @@ __global__ void __launch_bounds__(kLbThreads, 1)
           const uint32_t end = excl + total;
           *count_out = end < cap ? end : cap;
           if (la.tile_base) la.tile_base[T] = end;
+          if (la.density_out)
+            *la.density_out = static_cast<uint32_t>((static_cast<uint64_t>(end) << 16) / d);
         }
         if (la.err_out) {
           FF s{0.0f, 0.0f};

@@ -28,3 +28,16 @@ def stream_kernel(request):
         yield request.param
     finally:
         efs.ef_test_set_stream_kernel(0)
+
+
+@pytest.fixture(params=["chunks", "groups", "shallow"])
+def ht_stream_kernel(request):
+    """Runs a hard-threshold test with each of its streaming kernels: static
+    chunks, claimed groups, and claimed groups with the shallower ring and
+    larger pair buffers that dense calls use."""
+    import paper_2108_00951_gb300 as efs
+    efs.ef_test_set_stream_kernel({"chunks": 1, "groups": 2, "shallow": 3}[request.param])
+    try:
+        yield request.param
+    finally:
+        efs.ef_test_set_stream_kernel(0)

@@ -88,7 +88,7 @@ def _check(kind, g, e, gamma, arg, what, off=0):
     return gerr, want
 
 
-@pytest.mark.usefixtures("stream_kernel")
+@pytest.mark.usefixtures("ht_stream_kernel")
 @pytest.mark.parametrize("d", [1, 4097, 3 * 4096 + 17, 300_001])
 @pytest.mark.parametrize("off", [0, 1])
 def test_ht_error_norm(d, off):
@@ -97,7 +97,7 @@ def test_ht_error_norm(d, off):
         _check("ht", g, e, 0.1, lam, "ht d=%d off=%d lam=%g" % (d, off, lam), off=off)
 
 
-@pytest.mark.usefixtures("stream_kernel")
+@pytest.mark.usefixtures("ht_stream_kernel")
 def test_ht_error_norm_bf16():
     d = 100_003
     g, e = _inputs(d, 2)

@@ -46,7 +46,7 @@ def _check_same(gpu, ref, what):
 
 
 # ------------------------------------------------------------ hard-threshold
-@pytest.mark.usefixtures("stream_kernel")
+@pytest.mark.usefixtures("ht_stream_kernel")
 @pytest.mark.parametrize("bf16", [False, True])
 @pytest.mark.parametrize("d", RAGGED)
 def test_ht_random(d, bf16):
@@ -65,7 +65,7 @@ def test_ht_misaligned_bases(offs, bf16):
                 oracle.ef_hard_threshold(g, e, 0.1, 1.5e-3), "offsets %s" % (offs,))
 
 
-@pytest.mark.usefixtures("stream_kernel")
+@pytest.mark.usefixtures("ht_stream_kernel")
 def test_ht_adversarial_values():
     d = 3 * 4096 + 5
     rng = _rng("adv")
@@ -81,7 +81,7 @@ def test_ht_adversarial_values():
                     "adversarial lam=%g" % lam_)
 
 
-@pytest.mark.usefixtures("stream_kernel")
+@pytest.mark.usefixtures("ht_stream_kernel")
 def test_ht_fma_sensitive_values():
     # e = -round(gamma*g): a is the product's rounding error, which only a
     # single-rounding fma preserves
@@ -94,7 +94,7 @@ def test_ht_fma_sensitive_values():
                 "fma")
 
 
-@pytest.mark.usefixtures("stream_kernel")
+@pytest.mark.usefixtures("ht_stream_kernel")
 def test_ht_all_and_nothing_sent():
     d = 5 * 4096 + 1
     g, e = _inputs(d, 3)
@@ -114,7 +114,7 @@ def test_ht_zero_length():
     assert int(cnt.item()) == 0
 
 
-@pytest.mark.usefixtures("stream_kernel")
+@pytest.mark.usefixtures("ht_stream_kernel")
 @pytest.mark.parametrize("off", [0, 1])
 def test_ht_concurrent_streams(off):
     # calls on different streams use different workspaces and may overlap
@@ -220,6 +220,30 @@ def test_ht_balanced_chunks_over_calls():
     assert efs.ef_check_status() == efs.EF_OK
 
 
+def test_ht_ring_depth_follows_the_density_over_calls():
+    # from 4096 tiles on, the claimed-group kernel picks its ring depth from
+    # the density its earlier calls on this stream left in a hint word: sparse
+    # and dense calls in a row on one EF residual (the dense ones switch the
+    # next calls to the shallower ring, the sparse ones back), each equal to
+    # the oracle, the residual carried from call to call on both sides
+    d = 4096 * 4096 + 1237
+    rng = np.random.default_rng(29)
+    e_gpu, e_ref = gu.to_dev(np.zeros(d, np.float32)), np.zeros(d, np.float32)
+    idx = torch.empty(d, dtype=torch.int32, device=gu.DEV)
+    val = torch.empty(d, dtype=torch.float32, device=gu.DEV)
+    cnt = torch.zeros(1, dtype=torch.int32, device=gu.DEV)
+    for r, lam in enumerate([3e-3, 5e-4, 5e-4, 3e-3, 3e-3, 3e-2, 5e-4]):
+        g = (rng.standard_normal(d) * 1e-2).astype(np.float32)
+        efs.ef_hard_threshold(gu.g_device(g), e_gpu, 0.1, lam, idx, val, cnt)
+        ri, rv, e_ref = oracle.ef_hard_threshold(g, e_ref, 0.1, lam)
+        c = int(cnt.item())
+        assert c == ri.size, (r, c, ri.size)
+        gu.assert_bits(idx[:c].cpu().numpy().view(np.uint32), ri, "idx call %d" % r)
+        gu.assert_bits(val[:c].cpu().numpy(), rv, "val call %d" % r)
+        gu.assert_bits(e_gpu.cpu().numpy(), e_ref, "e' call %d" % r)
+    assert efs.ef_check_status() == efs.EF_OK
+
+
 # ---------------------------------------------------------------------- Top-k
 # ------------------------------------------- on-chip staging and its spill
 # The streaming compaction keeps each compute warp's first pairs of its CTA's
@@ -229,14 +253,14 @@ def test_ht_balanced_chunks_over_calls():
 SPILL_D = 3 * 2**20 + 4099
 
 
-@pytest.mark.usefixtures("stream_kernel")
+@pytest.mark.usefixtures("ht_stream_kernel")
 @pytest.mark.parametrize("bf16", [False, True])
 def test_ht_spill_everything_sent(bf16):
     g, e = _inputs(SPILL_D, 21, bf16=bf16)
     _check_same(gu.ht(g, e, 0.1, 0.0), oracle.ef_hard_threshold(g, e, 0.1, 0.0), "all sent")
 
 
-@pytest.mark.usefixtures("stream_kernel")
+@pytest.mark.usefixtures("ht_stream_kernel")
 def test_ht_spill_mixed_density():
     g, e = _inputs(SPILL_D, 22)
     g[: SPILL_D // 4] *= 1000.0  # a dense quarter (~96 % sent), the rest sends nothing
@@ -245,7 +269,7 @@ def test_ht_spill_mixed_density():
     _check_same((i, v, en), oracle.ef_hard_threshold(g, e, 0.1, 0.05), "mixed")
 
 
-@pytest.mark.usefixtures("stream_kernel")
+@pytest.mark.usefixtures("ht_stream_kernel")
 @pytest.mark.parametrize("out_off", [(1, 0), (2, 3), (3, 1)])
 def test_ht_misaligned_outputs(out_off):
     # the pairs are written with 16-byte stores matched to each output's own

@@ -59,7 +59,7 @@ def _ht_tiled(g, e, gamma, lam, g_off=0, e_off=0):
             tiles.cpu().numpy().view(np.uint32))
 
 
-@pytest.mark.usefixtures("stream_kernel")
+@pytest.mark.usefixtures("ht_stream_kernel")
 @pytest.mark.parametrize("bf16", [False, True])
 @pytest.mark.parametrize("d", SIZES)
 def test_hard_threshold_writes_the_tile_index(d, bf16):
@@ -74,7 +74,7 @@ def test_hard_threshold_writes_the_tile_index(d, bf16):
     assert efs.ef_check_status() == efs.EF_OK
 
 
-@pytest.mark.usefixtures("stream_kernel")
+@pytest.mark.usefixtures("ht_stream_kernel")
 @pytest.mark.parametrize("offs", [(0, 0), (1, 0)])
 def test_tile_index_with_the_error_norm(offs):
     # both optional outputs of ef_hard_threshold_tiled at once, on the
