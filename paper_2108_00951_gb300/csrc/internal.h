@@ -51,8 +51,10 @@ constexpr uint32_t kLwNone = 0, kLwWhole = 1, kLwSampled = 2, kLwAll = 3;
 constexpr uint32_t kLwSmemElems = 48u * 1024u;  // values one select CTA holds in shared memory
 constexpr uint32_t kLwWholeMax = 4096;          // segments at most this long: selected from e
 constexpr uint32_t kLwSampleGroups = 4096;      // groups of 4 coordinates sampled per CTA
-constexpr uint32_t kLwMaxParts = 16;            // sampling CTAs of one long segment, at most
-constexpr uint32_t kLwPartHistWords = kSampleBins + 32;  // merged histogram + arrival word
+constexpr uint32_t kLwMaxParts = 32;            // sampling CTAs of one long segment, at most
+constexpr int kLwSampleBits = 15;               // the sample histogram: top 15 bits of |a|
+constexpr uint32_t kLwSampleBins = 1u << kLwSampleBits;  // (1/128 of a binade each)
+constexpr uint32_t kLwPartHistWords = kLwSampleBins + 32;  // merged histogram + arrival word
 // Candidate bounds that admit nothing: the residual of the segment's
 // coordinates is then a, final in the streaming pass (kLwNoBound: segments
 // that send nothing), or decided by the select (kLwDeferred: short segments,
@@ -96,6 +98,7 @@ struct LwPlan {
   uint64_t d = 0;
   bool valid = false;
   uint32_t n_seg = 0, n_sampled = 0, n_select_ctas = 0, n_teams = 0, tiles = 0;
+  uint32_t n_part_hist = 0;  // merged sample histograms (segments sampled in parts), per copy
   uint64_t total_k = 0;
   std::vector<char> image;  // host image of the uploaded part
   char* dev = nullptr;

@@ -46,7 +46,8 @@ namespace {
 
 constexpr int kLwThreads = 1024;  // select CTAs
 constexpr uint32_t kLwSelectSmem = kLwSmemElems * sizeof(uint32_t);
-constexpr int kLwSampleShift = 31 - kSampleBits;  // magnitude bits below the sampled ones
+constexpr int kLwSampleShift = 31 - kLwSampleBits;  // magnitude bits below the sampled ones
+constexpr uint32_t kLwSampleSmem = kLwSampleBins * sizeof(uint32_t);  // the CTA's histogram
 constexpr int kLwStages = 4;
 
 __device__ __forceinline__ uint32_t mag_bits(float x) { return __float_as_uint(x) & 0x7fffffffu; }
@@ -72,7 +73,7 @@ __global__ void __launch_bounds__(kSampleThreads, 1)
     lw_sample_kernel(const GT* __restrict__ g, const float* __restrict__ e, float gamma,
                      const LwSeg* __restrict__ segs, const uint2* __restrict__ sampled,
                      uint32_t* mbound, uint32_t cand_cap, uint32_t* part_hist) {
-  __shared__ uint32_t s_hist[kSampleBins];
+  extern __shared__ uint32_t s_hist[];  // [kLwSampleBins]
   __shared__ uint32_t s_w[kSampleThreads / 32];
   __shared__ uint32_t s_bin, s_mass, s_last;
   const int tid = threadIdx.x;
@@ -83,7 +84,7 @@ __global__ void __launch_bounds__(kSampleThreads, 1)
   const uint32_t si = rec.x, part = rec.y & 0xffu, parts = (rec.y >> 8) & 0xffu,
                  slot = rec.y >> 16;
   LwSeg s = segs[si];
-  for (int b = tid; b < kSampleBins; b += kSampleThreads) s_hist[b] = 0;
+  for (uint32_t b = tid; b < kLwSampleBins; b += kSampleThreads) s_hist[b] = 0;
   uint64_t a0 = (static_cast<uint64_t>(s.lo) + 3u) & ~static_cast<uint64_t>(3);
   if (parts > 1) {
     const uint64_t avail = (static_cast<uint64_t>(s.hi) - a0) / 4;  // whole groups inside
@@ -124,37 +125,46 @@ __global__ void __launch_bounds__(kSampleThreads, 1)
   }
   __syncthreads();
   if (parts > 1) {
-    // add the part's histogram to the segment's merged one (after the wait:
-    // the previous call's last part left it at zero); the last part to
-    // arrive takes the merged histogram, leaves it at zero, and goes on
-    griddep_wait();
+    // add the part's histogram to the segment's merged one; the last part to
+    // arrive takes the merged histogram, leaves it at zero, and goes on. No
+    // wait first (the merge stays off the call's critical path): the copy of
+    // this call's parity (two alternate) was left at zero by the last
+    // sampling that used it, an earlier call's, and that grid is complete
+    // before this one starts: each call's select waits for its stream pass,
+    // which waits for the call's sampling, before it lets a later kernel start
     uint32_t* gh = part_hist + static_cast<size_t>(slot) * kLwPartHistWords;
-    for (int b = tid; b < kSampleBins; b += kSampleThreads)
+    for (uint32_t b = tid; b < kLwSampleBins; b += kSampleThreads)
       if (s_hist[b]) atomicAdd(&gh[b], s_hist[b]);
     __syncthreads();
     if (tid == 0) {
       __threadfence();
-      s_last = atomicAdd(&gh[kSampleBins], 1u) == parts - 1 ? 1u : 0u;
+      s_last = atomicAdd(&gh[kLwSampleBins], 1u) == parts - 1 ? 1u : 0u;
       if (s_last) __threadfence();  // the other parts' adds before the reads
     }
     __syncthreads();
     if (!s_last) return;
-    for (int b = tid; b < kSampleBins; b += kSampleThreads) {
-      s_hist[b] = __ldcg(&gh[b]);
-      gh[b] = 0;
+    constexpr int kBatch = 8;  // loads in flight per thread
+    for (uint32_t b0 = tid; b0 < kLwSampleBins; b0 += kBatch * kSampleThreads) {
+      uint32_t v[kBatch];
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) v[j] = __ldcg(&gh[b0 + j * kSampleThreads]);
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        s_hist[b0 + j * kSampleThreads] = v[j];
+        gh[b0 + j * kSampleThreads] = 0;
+      }
     }
-    if (tid == 0) gh[kSampleBins] = 0;
+    if (tid == 0) gh[kLwSampleBins] = 0;
     __syncthreads();
   }
-  // kPer consecutive bins per thread
-  constexpr int kPer = kSampleBins / kSampleThreads;
-  uint32_t c[kPer];
+  // kPer consecutive bins per thread, summed in a lane-rotated order (no
+  // two lanes of a warp on one bank)
+  constexpr int kPer = static_cast<int>(kLwSampleBins) / kSampleThreads;
+  static_assert(kPer == 32, "bins per thread: one per bank");
+  const int lane = tid & 31;
   uint32_t mine = 0;
 #pragma unroll
-  for (int i = 0; i < kPer; ++i) {
-    c[i] = s_hist[tid * kPer + i];
-    mine += c[i];
-  }
+  for (int i = 0; i < kPer; ++i) mine += s_hist[tid * kPer + ((i + lane) & (kPer - 1))];
   if (tid == 0) s_bin = 0xffffffffu;
   uint32_t m;  // sampled coordinates
   const uint32_t above = block_suffix_exclusive(mine, m, s_w);  // orders the reset
@@ -166,13 +176,15 @@ __global__ void __launch_bounds__(kSampleThreads, 1)
   // the products stay below 2^50).
   const uint64_t target = s.exact ? s.k : 3ull * s.k * m / (2ull * ds) + 32ull;
   if (target <= m && above < target && target - above <= mine) {
+    // the one thread whose bins hold the target walks them from the top
     uint64_t run = above;
-#pragma unroll
     for (int i = kPer - 1; i >= 0; --i) {
-      run += c[i];
-      if (run >= target && run - c[i] < target) {
+      const uint32_t c = s_hist[tid * kPer + i];
+      run += c;
+      if (run >= target) {
         s_bin = tid * kPer + i;
         s_mass = static_cast<uint32_t>(run);
+        break;
       }
     }
   }
@@ -835,6 +847,7 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t d, uint32_
   cudaError_t err = cudaSuccess;
   uint32_t* state = ws.topk_state(ws.topk_calls);
   uint32_t* other = ws.topk_state(ws.topk_calls + 1);
+  const uint32_t lw_parity = ws.topk_calls;
   ++ws.topk_calls;
   uint32_t* list_flags = state + kStListFlags / 4;
   uint32_t* list_idx = reinterpret_cast<uint32_t*>(ws.cand(0));
@@ -851,11 +864,13 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t d, uint32_
     if (p.n_sampled > 0) {
       const uint2* sampled = reinterpret_cast<const uint2*>(p.dev + p.off_samples);
       uint32_t cap = ws.cand_cap;
-      uint32_t* part_hist = reinterpret_cast<uint32_t*>(p.dev + p.off_part_hist);
+      // the merged histograms of the multi-part segments: two copies, by call parity
+      uint32_t* part_hist = reinterpret_cast<uint32_t*>(p.dev + p.off_part_hist) +
+                            static_cast<size_t>(lw_parity & 1u) * p.n_part_hist * kLwPartHistWords;
       void* sp[] = {(void*)&g, (void*)&e, (void*)&gamma, (void*)&segs, (void*)&sampled,
                     (void*)&mbound, (void*)&cap, (void*)&part_hist};
       err = launch_pdl(reinterpret_cast<const void*>(&lw_sample_kernel<GT>), p.n_sampled,
-                       kSampleThreads, 0, ws.stream, sp, false);
+                       kSampleThreads, kLwSampleSmem, ws.stream, sp, false);
       count_launch();
       if (err != cudaSuccess) return err;
     }
@@ -940,6 +955,13 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t d, uint32_
 
 void topk_layerwise_init_device(DeviceInfo& info) {
   int n = 0;
+  // the sampling kernel's histogram (dynamic shared memory); a failure here
+  // makes its launches fail, which the calls report
+  cudaFuncSetAttribute(lw_sample_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       kLwSampleSmem);
+  cudaFuncSetAttribute(lw_sample_kernel<uint16_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       kLwSampleSmem);
+  cudaGetLastError();
   if (cudaFuncSetAttribute(lw_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            kLwSelectSmem) != cudaSuccess ||
       cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, lw_select_kernel, kLwThreads,
@@ -996,12 +1018,16 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
       // than one CTA holds: the bound keeps 32 samples' slack, i.e.
       // 32 d_s / (4 groups) coordinates. Up to kLwMaxParts CTAs then sample
       // equal runs of it (kLwSampleGroups groups each) into one merged
-      // histogram, shrinking that slack.
+      // histogram, shrinking that slack: toward 3/4 of what one select CTA
+      // holds with the coordinates (half its shared memory) when the 1.5 k_s
+      // themselves fit there, else of what it holds as values alone.
       uint32_t parts = 1;
       if (!x.exact) {
-        const uint64_t need = 3ull * k / 2, fit = kLwSmemElems * 3ull / 4;
+        const uint64_t need = 3ull * k / 2;
+        const uint64_t fit = need < kLwSmemElems * 3ull / 8 ? kLwSmemElems * 3ull / 8
+                                                            : kLwSmemElems * 3ull / 4;
         const uint64_t slack = 32ull * ds / (4ull * x.groups);
-        if (need + slack > fit && need < fit / 2) {
+        if (need + slack > fit && need < fit) {
           const uint64_t want = (slack + (fit - need) - 1) / (fit - need);
           parts = static_cast<uint32_t>(std::min<uint64_t>(
               std::min<uint64_t>(want, kLwMaxParts), avail / kLwSampleGroups));
@@ -1130,7 +1156,7 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
   p.off_work_seg = take(sizeof(uint32_t) * work_seg.size());
   const size_t upload = off;
   p.off_teams = take(sizeof(LwTeamState) * n_teams);
-  p.off_part_hist = take(sizeof(uint32_t) * kLwPartHistWords * n_part_hist);
+  p.off_part_hist = take(2 * sizeof(uint32_t) * kLwPartHistWords * n_part_hist);
   const size_t zero_end = off;
   p.off_tile_base = take(sizeof(uint32_t) * (tiles + 1));
   p.total = off;
@@ -1175,6 +1201,7 @@ cudaError_t lw_prepare(Workspace& ws, const uint64_t* seg_end, const uint64_t* s
   p.d = d;
   p.n_seg = n_seg;
   p.n_sampled = n_sampled;
+  p.n_part_hist = n_part_hist;
   p.n_select_ctas = static_cast<uint32_t>(ctas.size());
   p.n_teams = n_teams;
   p.tiles = tiles;
