@@ -112,6 +112,7 @@ struct HtOp {
   static constexpr uint32_t kGBytes = kTileElems * sizeof(GT);
   static constexpr uint32_t kStageBytes = kGBytes + kTileElems * sizeof(float);
   static constexpr uint32_t kWarpStagePairs = 768;  // on-chip staged pairs per compute warp
+  static constexpr bool kKeepPairs = false;  // the message: read by the exchange, much later
   __device__ void prologue() const {}
   __device__ uint64_t initial_aux() const { return 0; }
 

@@ -62,6 +62,8 @@
 //   void prologue()                     every thread, once, at the start
 //   static constexpr uint32_t kPrefetchTiles;  tiles of the chunk pulled toward
 //   void prefetch(uint32_t tile)               L2 before the wait for the previous kernel
+//   static constexpr bool kKeepPairs;  the pairs are written with the L2
+//                                      evict-last policy (a later kernel of the call reads them)
 // Element layout: unit v of lane l of warp w covers the 4 coordinates from
 // tile * kTileElems + w * 256 + v * 128 + l * 4 (see stream_element_index).
 #pragma once
@@ -375,6 +377,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   griddep_launch_dependents();  // streaming is done: the next kernel may be scheduled
 
   // ------------------------------------------------------------- phase 2
+  const uint64_t keep_policy = Op::kKeepPairs ? l2_evict_last_policy() : 0ull;
   // the chunk's total (each compute warp contributes its own)
   uint32_t mine = lane == 0 && warp < kSWarps ? chunk_total : 0u;
   if (lane == 0) s_scratch[warp] = mine;
@@ -532,8 +535,12 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
           if (p0 + lane < cnt[u]) {
             const uint32_t q = dst[u] + p0 + lane;
             if (q < cap) {
-              idx_out[q] = xi[u];
-              val_out[q] = xv[u];
+              if constexpr (Op::kKeepPairs) {
+                st_pair_policy(idx_out + q, val_out + q, xi[u], xv[u], keep_policy);
+              } else {
+                idx_out[q] = xi[u];
+                val_out[q] = xv[u];
+              }
             } else {
               overflow = true;
             }

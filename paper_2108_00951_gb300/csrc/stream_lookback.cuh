@@ -412,6 +412,7 @@ __global__ void __launch_bounds__(kLbThreads, 1)
     // heads itself (lane w < 16: compute warp w's oldest unplaced pair).
     const int pw = warp - kLbPlaceWarp;
     constexpr int kPlaceThreads = 32 * kLbPlaceWarps;
+    const uint64_t keep_policy = Op::kKeepPairs ? l2_evict_last_policy() : 0ull;
     uint32_t head = 0;
     bool overflow = false;
     for (uint32_t seq = 0;; ++seq) {
@@ -471,8 +472,12 @@ __global__ void __launch_bounds__(kLbThreads, 1)
           }
           const uint32_t pos = dl + k;
           if (pos < cap) {
-            idx_out[pos] = xi;
-            val_out[pos] = xv;
+            if constexpr (Op::kKeepPairs) {
+              st_pair_policy(idx_out + pos, val_out + pos, xi, xv, keep_policy);
+            } else {
+              idx_out[pos] = xi;
+              val_out[pos] = xv;
+            }
           } else {
             overflow = true;
           }

@@ -98,6 +98,22 @@ __device__ __forceinline__ uint64_t l2_evict_first_policy() {
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
   return p;
 }
+// Kept in L2 ahead of streamed lines: small outputs that a later kernel of
+// the same call reads back (the candidate lists of the Top-k passes).
+__device__ __forceinline__ uint64_t l2_evict_last_policy() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+// One (index, value) pair written with an L2 cache policy.
+__device__ __forceinline__ void st_pair_policy(uint32_t* pi, float* pv, uint32_t xi, float xv,
+                                               uint64_t policy) {
+  asm volatile("st.global.L2::cache_hint.b32 [%0], %1, %2;" ::"l"(pi), "r"(xi), "l"(policy)
+               : "memory");
+  asm volatile("st.global.L2::cache_hint.b32 [%0], %1, %2;" ::"l"(pv), "r"(__float_as_uint(xv)),
+               "l"(policy)
+               : "memory");
+}
 __device__ __forceinline__ uint64_t l2_evict_normal_policy() {
   uint64_t p;
   asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(p));

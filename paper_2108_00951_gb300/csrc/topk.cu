@@ -101,6 +101,7 @@ struct TopkCandOp {
   static constexpr uint32_t kGBytes = kTileElems * sizeof(GT);
   static constexpr uint32_t kStageBytes = kGBytes + kTileElems * sizeof(float);
   static constexpr uint32_t kWarpStagePairs = 512;  // on-chip staged pairs per compute warp
+  static constexpr bool kKeepPairs = true;  // the candidate list: the select reads it next
   static constexpr int kSampleBins = efs::kSampleBins;
   static constexpr int kSampleShift = 31 - kSampleBits;  // key bits below the sampled ones
 

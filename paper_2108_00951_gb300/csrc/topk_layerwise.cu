@@ -218,6 +218,7 @@ struct LwCandOp {
   static constexpr uint32_t kGBytes = kTileElems * sizeof(GT);
   static constexpr uint32_t kStageBytes = kGBytes + kTileElems * sizeof(float);
   static constexpr uint32_t kWarpStagePairs = 512;  // on-chip staged pairs per compute warp
+  static constexpr bool kKeepPairs = true;  // the candidate list: the select reads it next
   __device__ void prologue() const { clear_state(other_state); }
   __device__ uint64_t initial_aux() const { return 0; }
 
