@@ -17,8 +17,6 @@ constexpr size_t kOffError = 8;         // uint32: latched device error bits
 constexpr size_t kOffBarArrive = 16;    // uint32: grid-barrier arrivals (zero after each barrier)
 constexpr size_t kOffTileClaim = 24;    // uint32[3]: work dispenser: handed out, CTAs finished,
                                         // groups resolved (zero between calls)
-constexpr size_t kOffTkLowerBound = 56; // uint64: sampled lower bound of the candidates' keys
-constexpr size_t kOffTkMode = 64;       // uint32: 0 candidates, 1 full array
 constexpr size_t kOffTkListCount = 72;  // uint32: candidates emitted by the streaming pass
 constexpr size_t kOffErrArrive = 80;    // uint32: arrivals of the e' norm pass (zero after it)
 constexpr size_t kOffStreamErr = 88;    // double: the streaming pass's share of ||e'||^2
@@ -31,6 +29,8 @@ constexpr size_t kStListFlags = 4;      // uint32: that pass's latched bits (ove
 constexpr size_t kStErrArrive = 8;      // uint32: select CTAs that published their ||e'||^2 share
 constexpr size_t kStSelect = 16;        // uint32[4]: short-list threshold published by CTA 0
 constexpr size_t kStCandCount = 32;     // uint32[6]: refine-level candidate counts
+constexpr size_t kStLowerBound = 64;    // uint64: sampled lower bound of the candidates' keys
+constexpr size_t kStMode = 72;          // uint32: 0 candidates, 1 full array
 constexpr size_t kStHist = 256;         // uint32[6][2048]: refine-level histograms
 constexpr int kHistLevels = 6;
 constexpr int kHistBins = 2048;

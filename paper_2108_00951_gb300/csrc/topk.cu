@@ -328,6 +328,14 @@ constexpr int kTkStages = 4;
 // derives the bound and publishes it with the mode. No CTA waits for
 // another, so the launch needs no co-residency; the streaming pass then has
 // no grid barrier and is a plain programmatic launch.
+// All of it runs before the wait for the previous kernel (the select of the
+// previous call, still running): the histogram, the arrival counter, the
+// bound and the mode live in this call's state block, which the previous
+// call's streaming pass zeroed and which that select does not read, and that
+// streaming pass completed before this grid could start (the select waited
+// for it before letting this kernel start). Only the last CTA waits, so the
+// grid completes after the previous kernel; the others leave their SMs to the
+// streaming pass, which may be scheduled from the start.
 template <typename GT>
 __global__ void __launch_bounds__(kStreamThreads)
     topk_sample_kernel(TopkCandOp<GT> op, uint32_t num_tiles) {
@@ -336,13 +344,14 @@ __global__ void __launch_bounds__(kStreamThreads)
   const uint32_t t_lo = static_cast<uint32_t>(static_cast<uint64_t>(c) * T / G);
   const uint32_t t_hi = static_cast<uint32_t>(static_cast<uint64_t>(c + 1) * T / G);
   for (int b = threadIdx.x; b < TopkCandOp<GT>::kSampleBins; b += blockDim.x) s_hist[b] = 0;
+  griddep_launch_dependents();  // the streaming pass waits for this whole grid
   __syncthreads();
   if (threadIdx.x < kComputeThreads && t_hi > t_lo) op.sample(t_lo, t_hi, threadIdx.x, s_hist);
   __syncthreads();
-  griddep_wait();  // the call's state block and the published words are free now
-  griddep_launch_dependents();
   op.merge(s_hist);
-  if (op.arrive_last()) op.choose();
+  if (!op.arrive_last()) return;
+  op.choose();
+  griddep_wait();  // this grid completes after the previous kernel
 }
 
 // Inputs the bulk copies cannot take (not 16-byte aligned): a = fmaf(γ,g,e)
@@ -898,8 +907,8 @@ cudaError_t launch_typed(const GT* g, float* e, float gamma, uint32_t k, uint32_
   args.list_val = reinterpret_cast<float*>(args.list_idx + ws.cand_cap);
   args.cand_count = state + kStCandCount / 4;
   args.cand_cap = ws.cand_cap;
-  args.lower_bound = ws.u64(kOffTkLowerBound);
-  args.mode = ws.u32(kOffTkMode);
+  args.lower_bound = reinterpret_cast<uint64_t*>(state + kStLowerBound / 4);
+  args.mode = state + kStMode / 4;
   args.sel = state + kStSelect / 4;
   args.list_count = ws.u32(kOffTkListCount);
   args.list_flags = state + kStListFlags / 4;
