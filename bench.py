@@ -244,14 +244,16 @@ def sources_hash(paths):
 
 def profiled_traffic(kernel_tag: str, workload: str):
     """DRAM bytes per launch from the committed ncu summary, if it was taken
-    on the current kernel sources; else None."""
+    on the current sources of the captured kernel (the entry's own source
+    list: the static-chunk and the claimed-group kernels differ); else None."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
             entry = json.load(f)[kernel_tag][workload]
+        sources = entry.get("sources", HT_KERNEL_SOURCES)
+        if entry.get("sources_sha256_16") != sources_hash(sources):
+            return None
     except Exception:
-        return None
-    if entry.get("sources_sha256_16") != sources_hash(HT_KERNEL_SOURCES):
         return None
     return entry.get("dram_bytes_per_launch")
 

@@ -233,6 +233,20 @@ __global__ void __launch_bounds__(kLbThreads, 1)
     ent[threadIdx.x].tag = 0xffffffffu;
   }
   __syncthreads();
+  // A dependent launch starts while the previous kernel's last groups are
+  // placed, a phase that leaves DRAM mostly idle: pull the first groups the
+  // CTAs will claim (about two each, claimed in CTA order) toward L2
+  // meanwhile. A prefetch is not a read of the data: L2 is the point of
+  // coherence, so the previous kernel's writes still land before the bulk
+  // copies read these lines. Whole tiles only.
+  if (threadIdx.x == 0 && Op::kPrefetchTiles > 0) {
+    const uint32_t full_tiles = d / kTileElems;
+    for (uint32_t r = 0; r < 2; ++r)
+      for (uint32_t j = 0; j < kLbGroupTiles; ++j) {
+        const uint32_t t = (blockIdx.x + r * gridDim.x) * kLbGroupTiles + j;
+        if (t < full_tiles) op.prefetch(t);
+      }
+  }
   // everything the previous kernels on the stream wrote (and the reset
   // group counter) is read only after this
   griddep_wait();
