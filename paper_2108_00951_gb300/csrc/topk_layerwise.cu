@@ -9,12 +9,14 @@
 //
 // Three launches, whatever the number of segments:
 //  1 sample   one CTA for each segment longer than kLwWholeMax with
-//             0 < k_s < d_s reads up to 4096 groups of 4 consecutive
-//             coordinates spread evenly over it (all of them when it holds no
-//             more), histograms the top 13 magnitude bits of a = fmaf(γ,g,e)
-//             in shared memory and picks the candidate bound: the bin holding
-//             k_s samples when every group was read, else about 1.5 times the
-//             needed mass above it.
+//             0 < k_s < d_s (up to kLwMaxParts for a long one with a small
+//             k_s, each over an equal run of it, their histograms merged)
+//             reads up to 4096 groups of 4 consecutive coordinates spread
+//             evenly over it (all of them when it holds no more), histograms
+//             the top 15 magnitude bits of a = fmaf(γ,g,e) in shared memory
+//             and picks the candidate bound: the bin holding k_s samples when
+//             every group was read, else about 1.5 times the needed mass
+//             above it.
 //  2 stream   the streaming compaction (stream_compact.cuh, or from 4096
 //             tiles on stream_lookback.cuh): a = fmaf(γ,g,e)
 //             is written over e (12 B per coordinate, the algorithmic bytes)
@@ -53,7 +55,9 @@ constexpr int kLwStages = 4;
 __device__ __forceinline__ uint32_t mag_bits(float x) { return __float_as_uint(x) & 0x7fffffffu; }
 
 // ------------------------------------------------------------- 1 sample
-// One CTA per sampled segment, one round of loads: thread t reads groups
+// One CTA per sampled segment or part of one (a part: an equal run of the
+// segment's aligned groups, sampled the same way; the parts' histograms are
+// merged in global memory), one round of loads: thread t reads groups
 // t, t + 1024, t + 2048, t + 3072 of the segment's G <= 4096 groups of 4
 // consecutive coordinates starting at multiples of 4 (one 16-byte load each
 // of e and of an fp32 g, 8 bytes of a bf16 g). Group q starts at
@@ -62,10 +66,11 @@ __device__ __forceinline__ uint32_t mag_bits(float x) { return __float_as_uint(x
 // aligned groups the segment holds (so the last group stays inside it);
 // G == A samples every one.
 //
-// Programmatic dependent launch: the loads and the histogram may run while
-// the previous kernel on the stream finishes (a sample read before that
-// kernel's writes only changes the bound, which is a filter); the bound is
-// written after the wait, so no earlier reader of it sees the new one.
+// Programmatic dependent launch: the loads, the histogram and the parts'
+// merge may run while the previous kernel on the stream finishes (a sample
+// read before that kernel's writes only changes the bound, which is a
+// filter); the bound is written after the wait, so no earlier reader of it
+// sees the new one.
 constexpr int kSampleThreads = 1024;
 
 template <typename GT>
