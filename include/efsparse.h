@@ -65,15 +65,17 @@
  * DIFFERENT streams never share a workspace and may run concurrently; calls
  * on the same stream are ordered by the stream.
  *
- * Concurrency: the streaming kernels' CTAs wait (bounded) only for
- * lower-numbered CTAs of the same launch, which the device dispatches first;
- * kernels that wait on every CTA of their grid (the Top-k select, the
- * layer-wise select with teams) are cooperative launches. If kernels on other
- * streams or other processes (MPS) hold SMs long enough that a CTA cannot
- * start within the bound (2 s), the call fails with EF_ERR_TIMEOUT (reported
- * by ef_check_status); it never hangs and never returns a wrong result. The
+ * Concurrency: below 4096 tiles (16,777,216 coordinates) the streaming
+ * kernel's CTAs wait (bounded) only for lower-numbered CTAs of the same
+ * launch, which the device dispatches first; kernels that wait on every CTA
+ * of their grid (the Top-k select, the layer-wise select with teams) are
+ * cooperative launches. If kernels on other streams or other processes (MPS)
+ * hold SMs long enough that a CTA cannot start within the bound (2 s), the
+ * call fails with EF_ERR_TIMEOUT (reported by ef_check_status); it never
+ * hangs and never returns a wrong result. From 4096 tiles on, the streaming
+ * kernel's CTAs claim groups of tiles in the order they start, and the
  * one-tile-per-CTA path (misaligned g or e, ef_hard_threshold_noalloc) takes
- * its tiles in the order CTAs start and needs no co-residency.
+ * its tiles the same way: neither needs co-residency.
  */
 #ifndef EFSPARSE_H
 #define EFSPARSE_H
